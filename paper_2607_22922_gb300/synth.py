@@ -1,0 +1,312 @@
+"""Seeded synthetic workloads for the iFVS query path (inputs only).
+
+This module draws the inputs of the query path — a PQ index (codebook and
+uint8 codes), attribute columns, queries with predicates at a target
+selectivity, the conditioning parameters (memory bank, W, hash seeds) and
+per-query w_z — and nothing else.  It holds none of the method's arithmetic:
+no distances, no look-up tables, no filtering, no top-k.  The oracle and the
+GPU path both read what it returns.
+
+The paper measures on SIFT1M / SIFT10M with a 16 x 8 PQ (§3.1, §3.2) and
+trained conditioning weights; neither the datasets nor the weights exist
+here, so every workload below is drawn from a seeded mixture with the same
+shapes.  The index is generated in PQ space: per-subspace codewords are drawn
+around mixture centres, every mixture component has a prototype code, a row
+keeps each prototype code with probability 1 - rho and otherwise takes a
+uniform codeword, and the row's raw vector is its reconstruction plus
+residual noise (raw vectors are only drawn when a test needs exact L2).
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+
+import numpy as np
+
+# Predicate records: n_clauses int32, reserved int32, 4 x {col int32, op
+# int32, lo int64, hi int64} — 104 bytes, the layout of the C interface.
+CLAUSE_DTYPE = np.dtype([("col", "<i4"), ("op", "<i4"), ("lo", "<i8"), ("hi", "<i8")])
+PREDICATE_DTYPE = np.dtype([("n_clauses", "<i4"), ("reserved", "<i4"), ("c", CLAUSE_DTYPE, (4,))])
+OP_EQ, OP_RANGE, OP_GE, OP_LT, OP_GT, OP_LE = 0, 1, 2, 3, 4, 5
+
+# w_z at which softplus(w_z) = 1 (the paper's initial state w_f = 1).
+WZ_IDENTITY = math.log(math.e - 1.0)
+
+
+@dataclasses.dataclass(frozen=True)
+class AttrSpec:
+    kind: str          # "uniform" | "cluster10" | "zipf"
+    lo: int
+    hi: int            # exclusive upper bound of the value range
+    dtype: str = "int32"
+    zipf_s: float = 1.1
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    N: int
+    D: int
+    M: int
+    K: int
+    clusters: int
+    kind: str                  # "gauss" | "sift" | "gist" | "deep"
+    attrs: tuple
+    nq: int
+    k: int
+    sels: tuple
+    batch: int = 0             # queries per search call (0 = all)
+    conjunctive: bool = False  # category = c AND date range
+    rho: float = 0.5           # probability that a row leaves its prototype code
+    B: int = 4096              # memory-bank rows
+    h: int = 2                 # hash functions
+    r: int = 8                 # adjustment rank
+    seed: int = 0x1F5
+
+    @property
+    def ds(self) -> int:
+        return self.D // self.M
+
+
+WORKLOADS = {
+    "gmm10k-d128-m16": Workload(
+        "gmm10k-d128-m16", 10_000, 128, 16, 256, 32, "gauss",
+        (AttrSpec("uniform", 0, 1000),), 100, 10, (0.01, 0.1, 0.5), seed=0x1F5),
+    "sift1m-d128-m16": Workload(
+        "sift1m-d128-m16", 1_000_000, 128, 16, 256, 256, "sift",
+        (AttrSpec("uniform", 0, 3650),), 10_000, 10, (0.001, 0.01, 0.1, 0.5, 1.0),
+        seed=0x1F6),
+    "gist1m-d960-m120": Workload(
+        "gist1m-d960-m120", 1_000_000, 960, 120, 256, 512, "gist",
+        (AttrSpec("cluster10", 0, 5120),), 1_000, 10, (0.01, 0.1, 0.5), seed=0x1F7),
+    "deep10m-d96-m12": Workload(
+        "deep10m-d96-m12", 10_000_000, 96, 12, 256, 1024, "deep",
+        (AttrSpec("uniform", 0, 3650), AttrSpec("zipf", 0, 100, "int16")), 10_000, 10,
+        (0.0001, 0.001, 0.01, 0.1, 0.5), conjunctive=True, seed=0x1F8),
+    "gmm100m-d128-m16": Workload(
+        "gmm100m-d128-m16", 100_000_000, 128, 16, 256, 4096, "gauss",
+        (AttrSpec("uniform", 0, 1_000_000),), 10_000, 100, (0.001, 0.01, 0.1, 1.0),
+        batch=1024, seed=0x1F9),
+}
+
+
+def scaled(w: Workload, N: int | None = None, nq: int | None = None, **kw) -> Workload:
+    """The same recipe at a smaller size (parity cases the oracle finishes)."""
+    d = dict(kw)
+    if N is not None:
+        d["N"] = N
+    if nq is not None:
+        d["nq"] = nq
+    return dataclasses.replace(w, **d)
+
+
+# ------------------------------------------------------------------ index
+
+@dataclasses.dataclass
+class Index:
+    w: Workload
+    codebook: np.ndarray        # [M][K][ds] float32
+    codes: np.ndarray           # [N][M] uint8
+    attrs: list                 # list of int32 / int16 arrays of length N
+    cluster: np.ndarray         # [N] int32 mixture component of each row
+    prototypes: np.ndarray      # [clusters][M] uint8
+    centres: np.ndarray         # [clusters][D] float32
+    noise_sigma: float
+
+
+def _centres(w: Workload, rng) -> np.ndarray:
+    if w.kind == "gauss":
+        c = rng.standard_normal((w.clusters, w.D))
+    elif w.kind == "sift":
+        c = np.clip(rng.normal(30.0, 25.0, (w.clusters, w.D)), 0.0, 255.0)
+    elif w.kind == "gist":
+        c = np.abs(rng.standard_normal((w.clusters, w.D)))
+        c /= np.linalg.norm(c, axis=1, keepdims=True)
+    elif w.kind == "deep":
+        c = rng.standard_normal((w.clusters, w.D))
+        c /= np.linalg.norm(c, axis=1, keepdims=True)
+    else:
+        raise ValueError(w.kind)
+    return c.astype(np.float32)
+
+
+def _spread(w: Workload) -> tuple:
+    """(codeword jitter, residual noise) per kind, in data units."""
+    return {"gauss": (0.3, 0.15), "sift": (12.0, 6.0), "gist": (0.01, 0.006),
+            "deep": (0.03, 0.015)}[w.kind]
+
+
+def _post(w: Workload, x: np.ndarray) -> np.ndarray:
+    if w.kind == "sift":
+        return np.clip(np.rint(x), 0.0, 255.0).astype(np.float32)
+    if w.kind == "gist":
+        x = np.abs(x)
+        return (x / np.maximum(np.linalg.norm(x, axis=-1, keepdims=True), 1e-12)).astype(np.float32)
+    if w.kind == "deep":
+        return (x / np.maximum(np.linalg.norm(x, axis=-1, keepdims=True), 1e-12)).astype(np.float32)
+    return x.astype(np.float32)
+
+
+def make_index(w: Workload, chunk: int = 4_000_000) -> Index:
+    """Codebook, codes, attribute columns (deterministic in ``w.seed``)."""
+    rng = np.random.default_rng(w.seed)
+    centres = _centres(w, rng)
+    jitter, noise = _spread(w)
+    owner = rng.integers(0, w.clusters, size=(w.M, w.K))
+    cb = np.empty((w.M, w.K, w.ds), dtype=np.float32)
+    for m in range(w.M):
+        sub = centres[owner[m], m * w.ds:(m + 1) * w.ds]
+        cb[m] = sub + jitter * rng.standard_normal(sub.shape)
+    if w.kind == "sift":
+        cb = np.clip(cb, 0.0, 255.0)
+    elif w.kind == "gist":
+        cb = np.abs(cb)
+    prototypes = rng.integers(0, w.K, size=(w.clusters, w.M), dtype=np.uint8)
+
+    codes = np.empty((w.N, w.M), dtype=np.uint8)
+    cluster = np.empty(w.N, dtype=np.int32)
+    keep_thresh = int(round((1.0 - w.rho) * 256))
+    for s in range(0, w.N, chunk):
+        e = min(w.N, s + chunk)
+        crng = np.random.default_rng([w.seed, 1, s])
+        cl = crng.integers(0, w.clusters, size=e - s, dtype=np.int32)
+        keep = crng.integers(0, 256, size=(e - s, w.M), dtype=np.uint16) < keep_thresh
+        rnd = crng.integers(0, w.K, size=(e - s, w.M), dtype=np.uint8)
+        codes[s:e] = np.where(keep, prototypes[cl], rnd)
+        cluster[s:e] = cl
+
+    attrs = []
+    for ai, spec in enumerate(w.attrs):
+        arng = np.random.default_rng([w.seed, 2, ai])
+        if spec.kind == "uniform":
+            a = arng.integers(spec.lo, spec.hi, size=w.N, dtype=np.int64)
+        elif spec.kind == "cluster10":
+            a = cluster.astype(np.int64) * 10 + arng.integers(0, 10, size=w.N)
+        elif spec.kind == "zipf":
+            p = zipf_probs(spec.hi - spec.lo, spec.zipf_s)
+            a = spec.lo + arng.choice(len(p), size=w.N, p=p)
+        else:
+            raise ValueError(spec.kind)
+        attrs.append(a.astype(np.int16 if spec.dtype == "int16" else np.int32))
+    return Index(w, cb, codes, attrs, cluster, prototypes, centres, noise)
+
+
+def zipf_probs(n: int, s: float) -> np.ndarray:
+    """P(value v) ∝ (v + 1)^-s for v in [0, n) (value 0 is the most common)."""
+    p = 1.0 / np.arange(1, n + 1, dtype=np.float64) ** s
+    return p / p.sum()
+
+
+def raw_vectors(ix: Index, start: int = 0, stop: int | None = None) -> np.ndarray:
+    """Raw vectors of rows [start, stop): reconstruction + residual noise."""
+    w = ix.w
+    stop = w.N if stop is None else stop
+    out = np.empty((stop - start, w.D), dtype=np.float32)
+    block = 1 << 16
+    for s in range(start - start % block, stop, block):
+        e = s + block
+        rng = np.random.default_rng([w.seed, 3, s])
+        noise = rng.standard_normal((block, w.D)).astype(np.float32) * ix.noise_sigma
+        a, b = max(s, start), min(e, stop)
+        if a >= b:
+            continue
+        codes = ix.codes[a:b]
+        rec = ix.codebook[np.arange(w.M)[None, :], codes]          # [n][M][ds] gather
+        x = rec.reshape(b - a, w.D) + noise[a - s:b - s]
+        out[a - start:b - start] = _post(w, x)
+    return out
+
+
+# ---------------------------------------------------------------- queries
+
+@dataclasses.dataclass
+class Queries:
+    q: np.ndarray          # [nq][D] float32
+    preds: np.ndarray      # [nq] PREDICATE_DTYPE
+    wz: np.ndarray         # [nq][D] float32
+    sel: float             # target selectivity of the bin
+
+
+def empty_predicates(n: int) -> np.ndarray:
+    return np.zeros(n, dtype=PREDICATE_DTYPE)
+
+
+def set_clause(pred, i, col, op, lo, hi=0):
+    pred["c"][i]["col"] = col
+    pred["c"][i]["op"] = op
+    pred["c"][i]["lo"] = lo
+    pred["c"][i]["hi"] = hi
+
+
+def make_queries(ix: Index, sel: float, nq: int | None = None, salt: int = 0,
+                 wz_sigma: float = 0.2) -> Queries:
+    """Queries drawn from the index's mixture, each with a predicate whose
+    target selectivity is ``sel``, plus per-query w_z around the identity."""
+    w = ix.w
+    nq = w.nq if nq is None else nq
+    rng = np.random.default_rng([w.seed, 4, int(round(sel * 1e6)), salt])
+    cl = rng.integers(0, w.clusters, size=nq)
+    keep = rng.random((nq, w.M)) < (1.0 - w.rho)
+    rnd = rng.integers(0, w.K, size=(nq, w.M))
+    codes = np.where(keep, ix.prototypes[cl], rnd).astype(np.int64)
+    rec = ix.codebook[np.arange(w.M)[None, :], codes].reshape(nq, w.D)
+    q = _post(w, rec + ix.noise_sigma * rng.standard_normal((nq, w.D)))
+
+    preds = empty_predicates(nq)
+    if w.conjunctive:
+        date, cat = w.attrs[0], w.attrs[1]
+        p = zipf_probs(cat.hi - cat.lo, cat.zipf_s)
+        cum = np.cumsum(p)
+        span = date.hi - date.lo
+        for i in range(nq):
+            if sel <= p[0]:
+                ok = np.nonzero(p >= sel)[0]
+                c = int(ok[rng.integers(0, len(ok))])
+                width = int(min(span, max(1, round(sel / p[c] * span))))
+                lo = date.lo + int(rng.integers(0, span - width + 1))
+                preds[i]["n_clauses"] = 2
+                set_clause(preds[i], 0, 1, OP_EQ, cat.lo + c)
+                set_clause(preds[i], 1, 0, OP_RANGE, lo, lo + width)
+            else:
+                c = int(np.searchsorted(cum, sel))
+                c = min(c, len(p) - 1)
+                width = int(min(span, max(1, round(sel / cum[c] * span))))
+                lo = date.lo + int(rng.integers(0, span - width + 1))
+                preds[i]["n_clauses"] = 2
+                set_clause(preds[i], 0, 1, OP_LE, cat.lo + c)
+                set_clause(preds[i], 1, 0, OP_RANGE, lo, lo + width)
+    else:
+        a = w.attrs[0]
+        span = a.hi - a.lo
+        width = int(min(span, max(1, round(sel * span))))
+        los = a.lo + rng.integers(0, span - width + 1, size=nq)
+        preds["n_clauses"] = 1
+        preds["c"][:, 0]["col"] = 0
+        preds["c"][:, 0]["op"] = OP_RANGE
+        preds["c"][:, 0]["lo"] = los
+        preds["c"][:, 0]["hi"] = los + width
+    wz = (WZ_IDENTITY + wz_sigma * rng.standard_normal((nq, w.D))).astype(np.float32)
+    return Queries(q.astype(np.float32), preds, wz, sel)
+
+
+# ------------------------------------------------------------ conditioning
+
+@dataclasses.dataclass
+class Conditioning:
+    bank: np.ndarray       # [B][M*r] float32
+    W: np.ndarray          # [M][r][K][ds] float32
+    seeds: np.ndarray      # [h] uint64
+
+
+def make_conditioning(ix: Index, scale: float = 0.05) -> Conditioning:
+    """Stand-in values for the trained memory bank and W (the paper's trained
+    weights are not available): bank ~ N(0, 1/h) so alpha ~ N(0, 1); W ~
+    N(0, (scale * codeword spread of the subspace)^2)."""
+    w = ix.w
+    rng = np.random.default_rng([w.seed, 5])
+    bank = (rng.standard_normal((w.B, w.M * w.r)) / math.sqrt(w.h)).astype(np.float32)
+    spread = ix.codebook.reshape(w.M, -1).std(axis=1).astype(np.float64)
+    W = rng.standard_normal((w.M, w.r, w.K, w.ds)) * (scale * spread)[:, None, None, None]
+    seeds = rng.integers(0, 2**63, size=w.h, dtype=np.int64).astype(np.uint64)
+    seeds ^= np.uint64(0x9E3779B97F4A7C15)
+    return Conditioning(bank, W.astype(np.float32), seeds)
