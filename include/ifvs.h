@@ -1,0 +1,251 @@
+/*
+ * ifvs.h — C ABI of the GB300 query path of iFVS (instance-optimised
+ * filtered vector search, arXiv 2607.22922).
+ *
+ * The library answers filtered k-nearest-neighbour queries over a fixed
+ * PQ-encoded dataset (the query form of Listing 1, §1: a conjunctive
+ * predicate on relational attribute columns, then ORDER BY distance LIMIT k)
+ * with the three stages of §2:
+ *   Filter  every row's attributes are tested against the predicate, giving
+ *           the candidate pool P as a pass bitmap;
+ *   Rank    the query- and predicate-conditioned codebook
+ *           C_iFVS = C_PQ + Delta, Delta = alpha . W, alpha = the sum of the h
+ *           memory-bank rows that <q, f> hashes to, and the filter weights
+ *           w_f = softplus(w_z) give each candidate the score of §2, which the
+ *           library evaluates as the equivalent weighted ADC distance
+ *           dist(v) = sum_m LUT[m][code_v[m]],
+ *           LUT[m][k] = sum_t w_f[m ds + t] (q[m ds + t] - C_iFVS[m][k][t])^2
+ *           (score(v) = sum w q^2 - dist(v): descending score is ascending
+ *           distance);
+ *   Select  the k candidates with the smallest (dist, row id).
+ *
+ * Every step runs in the library's CUDA kernels for sm_103a; there is no CPU
+ * fallback.  All calls are synchronous: they return once their outputs are
+ * written.  No call keeps a pointer to caller memory after it returns.
+ *
+ * Errors: every call returns an ifvs_status.  On error the outputs are
+ * unspecified and ifvs_last_error() (thread-local) describes the cause.
+ * Nothing aborts the process and nothing throws across the ABI.
+ *
+ * Thread safety: an index may be used by one thread at a time; different
+ * indexes may be used concurrently.
+ */
+#ifndef IFVS_H
+#define IFVS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define IFVS_MAX_CLAUSES 4
+#define IFVS_MAX_ATTRS 4
+#define IFVS_MAX_K 256      /* largest k (and rerank depth R) per query  */
+#define IFVS_MAX_M 128      /* largest number of PQ subspaces            */
+#define IFVS_N_STAGES 8
+
+typedef struct ifvs_index ifvs_index;
+
+typedef enum {
+    IFVS_OK = 0,
+    IFVS_ERR_ARG = -1,          /* invalid argument (message says which)      */
+    IFVS_ERR_OOM = -2,          /* device allocation failed                   */
+    IFVS_ERR_CUDA = -3,         /* a CUDA runtime call or kernel failed       */
+    IFVS_ERR_STATE = -4,        /* e.g. search before ifvs_load_codebooks     */
+    IFVS_ERR_UNSUPPORTED = -5   /* shape outside the supported range          */
+} ifvs_status;
+
+/* Clause operators (Listing 1 uses = and >; all are intervals on integers):
+ *   EQ    a == lo        RANGE lo <= a < hi     GE  a >= lo
+ *   LT    a <  lo        GT    a >  lo          LE  a <= lo
+ * Comparisons are exact on the column's integer values (int64 semantics). */
+enum { IFVS_OP_EQ = 0, IFVS_OP_RANGE = 1, IFVS_OP_GE = 2, IFVS_OP_LT = 3,
+       IFVS_OP_GT = 4, IFVS_OP_LE = 5 };
+
+/* Attribute column element types. */
+enum { IFVS_ATTR_I32 = 0, IFVS_ATTR_I16 = 1 };
+
+typedef struct {
+    int32_t col;   /* attribute column, 0 <= col < n_attrs */
+    int32_t op;    /* IFVS_OP_*                            */
+    int64_t lo;
+    int64_t hi;    /* used by IFVS_OP_RANGE only           */
+} ifvs_clause;     /* 24 bytes */
+
+/* A predicate is the conjunction (AND) of its first n_clauses clauses;
+ * n_clauses = 0 passes every row.  104 bytes. */
+typedef struct {
+    int32_t n_clauses;
+    int32_t reserved;   /* must be 0 */
+    ifvs_clause c[IFVS_MAX_CLAUSES];
+} ifvs_predicate;
+
+/* Flags of ifvs_search_params.flags and of ifvs_load_index(flags). */
+#define IFVS_F_DEVICE_IO    0x1u  /* array arguments are device pointers on
+                                     the index's device                       */
+#define IFVS_F_STAGE_TIMING 0x2u  /* time every kernel launch with CUDA events
+                                     on the launching stream (ifvs_stage_times) */
+#define IFVS_F_PLAIN_PQ     0x4u  /* ignore the memory bank: Delta = 0 (plain PQ
+                                     ADC, baseline Pre_IndexPQ_ADC of §3.2)   */
+
+typedef struct {
+    uint32_t flags;     /* IFVS_F_*                                            */
+    int32_t rerank;     /* R > 0: re-rank the R best ADC candidates by exact fp32
+                           L2 on the raw vectors (needs vectors at load), then
+                           keep k (k <= R <= IFVS_MAX_K).  0: off.              */
+    int32_t sub_batch;  /* queries per filter/scan pass; bounds the bitmap
+                           workspace to sub_batch * ceil(N/1024) * 128 bytes.
+                           0: automatic (at most 1024).                        */
+    int32_t reserved;   /* must be 0 */
+    void* stream;       /* cudaStream_t to run on; NULL: the index's stream   */
+} ifvs_search_params;
+
+/* Stages reported by ifvs_stage_times (index into its arrays). */
+enum {
+    IFVS_STAGE_PREDICATE = 0,  /* predicate validation + canonical intervals  */
+    IFVS_STAGE_FILTER = 1,     /* Filter: attribute columns -> pass bitmaps   */
+    IFVS_STAGE_CONDITION = 2,  /* fingerprint, alpha, w_f                     */
+    IFVS_STAGE_LUT = 3,        /* Delta, C_iFVS and the weighted ADC tables    */
+    IFVS_STAGE_SCAN = 4,       /* Rank: code scan + per-CTA top-k             */
+    IFVS_STAGE_MERGE = 5,      /* Select: merge of the per-CTA top-k lists    */
+    IFVS_STAGE_RERANK = 6,     /* exact fp32 rerank                           */
+    IFVS_STAGE_LAYOUT = 7      /* bitmap layout conversions                   */
+};
+
+/*
+ * ifvs_load_index — copy a PQ-encoded dataset to the device.
+ *   out         receives the new index (free with ifvs_free)
+ *   device      CUDA device ordinal
+ *   codes       [N][M] uint8, row-major: code of row i in subspace m (§1:
+ *               subspace m covers dimensions [m ds, (m+1) ds)); every code
+ *               must be < K
+ *   N           rows, 1 <= N < 2^32 - 1024
+ *   M, K        subspaces (1..IFVS_MAX_M) and codewords per subspace (1..256)
+ *   attr_cols   n_attrs pointers to columns of N elements (int32 or int16 as
+ *               attr_types says); n_attrs in 0..IFVS_MAX_ATTRS
+ *   vectors     [N][D] float32 raw vectors for the exact rerank, or NULL
+ *   D           vector dimension (a multiple of M)
+ *   flags       IFVS_F_DEVICE_IO: codes, columns and vectors are device
+ *               pointers on `device`
+ * The library copies everything; the caller keeps ownership of its buffers.
+ * Codes are stored re-laid out for the scan (rows padded to a multiple of
+ * 1024; each row's codes rotated so that a warp's 32 lanes read 32 distinct
+ * shared-memory banks).
+ */
+int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int64_t N,
+                    int32_t M, int32_t K, const void* const* attr_cols,
+                    const int32_t* attr_types, int32_t n_attrs, const float* vectors,
+                    int32_t D, uint32_t flags);
+
+/*
+ * ifvs_load_codebooks — the base codebook and the conditioning model (§2).
+ *   C_pq        [M][K][ds] float32 base codebook C_PQ (ds = D / M)
+ *   bank        [B][M r] float32 memory bank (row b viewed as alpha's M x r
+ *               layout), or NULL: Delta = 0 for every query
+ *   B, h, r     bank rows, hash functions per query, adjustment rank
+ *   W           [M][r][K][ds] float32 adjustment directions (NULL iff bank is)
+ *   hash_seeds  [h] uint64: hash i of <q, f> is
+ *               splitmix64_finalizer(fnv1a64(key) XOR hash_seeds[i]) mod B,
+ *               key = the float32 bits of q (little-endian), n_clauses
+ *               (int32) and each clause's col, op (int32), lo, hi (int64)
+ * Host pointers; copied.  May be called again to replace the model.
+ */
+int ifvs_load_codebooks(ifvs_index* ix, const float* C_pq, int32_t ds, const float* bank,
+                        int64_t B, int32_t h, int32_t r, const float* W,
+                        const uint64_t* hash_seeds);
+
+/*
+ * ifvs_search_batch — the whole query path (Filter, Rank, Select of §2) for
+ * nq queries.
+ *   queries   [nq][D] float32
+ *   preds     [nq] predicates
+ *   nq        >= 0 (0 returns at once)
+ *   k         1..IFVS_MAX_K results per query
+ *   wz        [nq][D] float32 predicate encodings w_z (w_f = softplus(w_z)),
+ *             or NULL: w_f = 1 exactly (the paper's initial state)
+ *   p         options, or NULL for defaults (host I/O, index stream)
+ *   ids       [nq][k] int64 out: row ids by ascending (dist, id); -1 pads
+ *             when fewer than k rows pass
+ *   dists     [nq][k] float32 out: weighted ADC distances (or exact L2 after
+ *             a rerank); +inf pads
+ *   npass     [nq] int64 out: |P| per query, or NULL
+ * Array arguments are host memory unless p->flags has IFVS_F_DEVICE_IO.
+ */
+int ifvs_search_batch(ifvs_index* ix, const float* queries, const ifvs_predicate* preds,
+                      int64_t nq, int32_t k, const float* wz, const ifvs_search_params* p,
+                      int64_t* ids, float* dists, int64_t* npass);
+
+/*
+ * ifvs_filter — stage 1 alone (§2 Filter).
+ *   bitmaps  [nq][ceil(N/32)] uint32 out: bit (i % 32) of word i / 32 is set
+ *            iff row i passes (bits beyond N are 0)
+ *   npass    [nq] int64 out, or NULL
+ */
+int ifvs_filter(ifvs_index* ix, const ifvs_predicate* preds, int64_t nq,
+                const ifvs_search_params* p, uint32_t* bitmaps, int64_t* npass);
+
+/*
+ * ifvs_condition — the conditioning and table build of §2 alone.  Every
+ * output may be NULL.
+ *   bank_idx  [nq][h] uint32 out: the h bank rows <q, f> hashes to
+ *   alpha     [nq][M r] float32 out: sum of those rows
+ *   wf        [nq][D] float32 out: softplus(w_z) (or 1)
+ *   C_ifvs    [nq][M][K][ds] float32 out: C_PQ + alpha . W
+ *   lut       [nq][M][K] float32 out: weighted ADC tables
+ */
+int ifvs_condition(ifvs_index* ix, const float* queries, const ifvs_predicate* preds,
+                   int64_t nq, const float* wz, const ifvs_search_params* p,
+                   uint32_t* bank_idx, float* alpha, float* wf, float* C_ifvs, float* lut);
+
+/*
+ * ifvs_scan_topk — Rank and Select from given tables and bitmaps.
+ *   lut      [nq][M][K] float32 weighted ADC tables
+ *   bitmaps  [nq][ceil(N/32)] uint32 pass bitmaps in the layout ifvs_filter
+ *            writes
+ *   ids, dists as for ifvs_search_batch
+ */
+int ifvs_scan_topk(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, int64_t nq,
+                   int32_t k, const ifvs_search_params* p, int64_t* ids, float* dists);
+
+/*
+ * ifvs_rerank — exact fp32 L2 (the Pre_IndexFlatL2 distance of §3.2) of
+ * candidate rows, then the k best by (dist, id).
+ *   cand  [nq][R] int64 candidate row ids; -1 entries are skipped
+ *   needs raw vectors given to ifvs_load_index
+ */
+int ifvs_rerank(ifvs_index* ix, const float* queries, const int64_t* cand, int64_t nq,
+                int32_t R, int32_t k, const ifvs_search_params* p, int64_t* ids,
+                float* dists);
+
+/*
+ * ifvs_stage_times — device time (ms, from CUDA events recorded on the
+ * launching stream around each launch) and launch counts per stage,
+ * accumulated over calls made with IFVS_F_STAGE_TIMING.  Either array may be
+ * NULL; reset != 0 zeroes the counters after reading.
+ */
+int ifvs_stage_times(ifvs_index* ix, double* ms, int64_t* launches, int32_t reset);
+
+/*
+ * ifvs_canonical_predicate — host-side helper exposing how a predicate is
+ * reduced to one closed interval [lo, lo + width_m1] per attribute column
+ * (clauses on the same column intersect).  Column c passes every value when
+ * lo[c] is the type's minimum and width_m1[c] the type's span minus one.
+ * *empty = 1 when no row can pass.  Returns IFVS_ERR_ARG for an invalid
+ * predicate.
+ */
+int ifvs_canonical_predicate(const ifvs_predicate* p, const int32_t* attr_types,
+                             int32_t n_attrs, int32_t* lo, uint32_t* width_m1, int32_t* empty);
+
+/* ifvs_index_info — out[0..7] = N, M, K, D, ds, n_attrs, has codebooks,
+ * device bytes held. */
+int ifvs_index_info(const ifvs_index* ix, int64_t* out);
+
+void ifvs_free(ifvs_index* ix);
+const char* ifvs_last_error(void);
+const char* ifvs_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* IFVS_H */

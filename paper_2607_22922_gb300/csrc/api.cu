@@ -1,0 +1,886 @@
+// Host side of the C ABI declared in include/ifvs.h: argument checks,
+// device memory of the index and its grow-only workspace, the launch
+// sequence of the query path per sub-batch, and per-stage CUDA-event timing.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <new>
+#include <utility>
+#include <vector>
+
+#include "internal.cuh"
+
+using namespace ifvs;
+
+namespace {
+
+thread_local char g_err[768] = "";
+
+int set_err(int code, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what, int line) {
+    cudaGetLastError();  // clear a sticky launch error where possible
+    return set_err(e == cudaErrorMemoryAllocation ? IFVS_ERR_OOM : IFVS_ERR_CUDA,
+                   "%s failed: %s (api.cu:%d)", what, cudaGetErrorString(e), line);
+}
+
+#define CUDA_TRY(x)                                                  \
+    do {                                                             \
+        cudaError_t e_ = (x);                                        \
+        if (e_ != cudaSuccess) return cuda_fail(e_, #x, __LINE__);   \
+    } while (0)
+
+#define TRY(x)               \
+    do {                     \
+        int rc_ = (x);       \
+        if (rc_ != 0) return rc_; \
+    } while (0)
+
+struct DevBuf {
+    void* p = nullptr;
+    size_t cap = 0;
+    template <class T> T* as() const { return reinterpret_cast<T*>(p); }
+};
+
+int ensure(DevBuf& b, size_t bytes) {
+    if (bytes == 0) bytes = 16;
+    if (bytes <= b.cap) return 0;
+    if (b.p) cudaFree(b.p);
+    b.p = nullptr;
+    b.cap = 0;
+    cudaError_t e = cudaMalloc(&b.p, bytes);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        b.p = nullptr;
+        return set_err(IFVS_ERR_OOM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+    }
+    b.cap = bytes;
+    return 0;
+}
+
+void release(DevBuf& b) {
+    if (b.p) cudaFree(b.p);
+    b.p = nullptr;
+    b.cap = 0;
+}
+
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+int64_t round_up(int64_t a, int64_t b) { return (a + b - 1) / b * b; }
+
+}  // namespace
+
+struct ifvs_index {
+    int device = 0;
+    int num_sms = 0;
+    int max_smem = 0;
+    cudaStream_t stream = nullptr;
+    int64_t N = 0, n_blocks = 0, n_rows_pad = 0;
+    int M = 0, K = 0, D = 0, ds = 0, row_bytes = 0, tab_words = 0;
+    int n_attrs = 0;
+    int32_t types[IFVS_MAX_ATTRS] = {0, 0, 0, 0};
+    void* d_attr[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
+    uint8_t* d_codes = nullptr;
+    float* d_vec = nullptr;
+    bool has_cb = false;
+    float* d_cpq = nullptr;
+    float* d_bank = nullptr;
+    float* d_W = nullptr;
+    uint64_t* d_seeds = nullptr;
+    int64_t B = 0;
+    int h = 0, r = 0;
+    size_t bytes = 0;
+    // workspace
+    DevBuf w_q, w_wz, w_preds, w_canon, w_err, w_bm, w_rows, w_npass, w_idx, w_alpha, w_wf,
+        w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist;
+    // timing
+    double stage_ms[IFVS_N_STAGES] = {0};
+    int64_t stage_launches[IFVS_N_STAGES] = {0};
+    std::vector<cudaEvent_t> ev_free;
+    std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> pending;
+
+    AttrCols cols() const {
+        AttrCols c;
+        for (int i = 0; i < IFVS_MAX_ATTRS; ++i) {
+            c.col[i] = d_attr[i];
+            c.type[i] = types[i];
+        }
+        c.n = n_attrs;
+        return c;
+    }
+    cudaEvent_t event() {
+        if (!ev_free.empty()) {
+            cudaEvent_t e = ev_free.back();
+            ev_free.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+        return e;
+    }
+    void collect() {
+        for (auto& pr : pending) {
+            float ms = 0.f;
+            if (cudaEventElapsedTime(&ms, pr.second.first, pr.second.second) == cudaSuccess)
+                stage_ms[pr.first] += ms;
+            ev_free.push_back(pr.second.first);
+            ev_free.push_back(pr.second.second);
+        }
+        pending.clear();
+        cudaGetLastError();
+    }
+};
+
+namespace {
+
+void free_index(ifvs_index* ix) {
+    if (!ix) return;
+    DeviceGuard g(ix->device);
+    if (ix->stream) cudaStreamSynchronize(ix->stream);
+    for (int i = 0; i < IFVS_MAX_ATTRS; ++i)
+        if (ix->d_attr[i]) cudaFree(ix->d_attr[i]);
+    void* ptrs[] = {ix->d_codes, ix->d_vec, ix->d_cpq, ix->d_bank, ix->d_W, ix->d_seeds};
+    for (void* p : ptrs)
+        if (p) cudaFree(p);
+    DevBuf* bufs[] = {&ix->w_q, &ix->w_wz, &ix->w_preds, &ix->w_canon, &ix->w_err, &ix->w_bm,
+                      &ix->w_rows, &ix->w_npass, &ix->w_idx, &ix->w_alpha, &ix->w_wf,
+                      &ix->w_lut, &ix->w_cifvs, &ix->w_part, &ix->w_ids, &ix->w_dists,
+                      &ix->w_cand, &ix->w_cdist};
+    for (DevBuf* b : bufs) release(*b);
+    for (auto& pr : ix->pending) {
+        ix->ev_free.push_back(pr.second.first);
+        ix->ev_free.push_back(pr.second.second);
+    }
+    for (cudaEvent_t e : ix->ev_free)
+        if (e) cudaEventDestroy(e);
+    if (ix->stream) cudaStreamDestroy(ix->stream);
+    delete ix;
+}
+
+int dev_alloc(ifvs_index* ix, void** p, size_t bytes) {
+    cudaError_t e = cudaMalloc(p, bytes ? bytes : 16);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        *p = nullptr;
+        return set_err(IFVS_ERR_OOM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+    }
+    ix->bytes += bytes;
+    return 0;
+}
+
+// Records a CUDA event pair around one launch on the launching stream when
+// timing is on; counts launches per stage always.
+struct Stage {
+    ifvs_index* ix;
+    cudaStream_t s;
+    bool on;
+    int stage;
+    cudaEvent_t a = nullptr;
+    Stage(ifvs_index* ix_, cudaStream_t s_, bool on_, int st) : ix(ix_), s(s_), on(on_), stage(st) {
+        if (on) {
+            a = ix->event();
+            if (a) cudaEventRecord(a, s);
+        }
+    }
+    cudaError_t end(cudaError_t launch_err) {
+        ix->stage_launches[stage] += 1;
+        if (on && a) {
+            cudaEvent_t b = ix->event();
+            if (b) {
+                cudaEventRecord(b, s);
+                ix->pending.push_back({stage, {a, b}});
+            } else {
+                ix->ev_free.push_back(a);
+            }
+        }
+        return launch_err;
+    }
+};
+
+struct Opts {
+    bool dio = false, timing = false, plain = false;
+    int R = 0;
+    int64_t sub_batch = 0;
+    cudaStream_t stream = nullptr;
+};
+
+int parse_opts(const ifvs_search_params* p, Opts* o) {
+    if (!p) return 0;
+    if (p->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING | IFVS_F_PLAIN_PQ))
+        return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", p->flags);
+    if (p->reserved != 0) return set_err(IFVS_ERR_ARG, "ifvs_search_params.reserved must be 0");
+    if (p->rerank < 0 || p->rerank > IFVS_MAX_K)
+        return set_err(IFVS_ERR_ARG, "rerank depth %d outside 0..%d", p->rerank, IFVS_MAX_K);
+    if (p->sub_batch < 0) return set_err(IFVS_ERR_ARG, "sub_batch must be >= 0");
+    o->dio = p->flags & IFVS_F_DEVICE_IO;
+    o->timing = p->flags & IFVS_F_STAGE_TIMING;
+    o->plain = p->flags & IFVS_F_PLAIN_PQ;
+    o->R = p->rerank;
+    o->sub_batch = p->sub_batch;
+    o->stream = reinterpret_cast<cudaStream_t>(p->stream);
+    return 0;
+}
+
+int64_t pick_sub_batch(const ifvs_index* ix, const Opts& o, int64_t nq) {
+    if (o.sub_batch > 0) return o.sub_batch < nq ? o.sub_batch : nq;
+    // bound the lane-major bitmaps to ~16 GiB and the batch to 1024 queries
+    const int64_t per_q = ix->n_blocks * 128;
+    int64_t sb = (int64_t(16) << 30) / (per_q > 0 ? per_q : 1);
+    if (sb > 1024) sb = 1024;
+    if (sb < 1) sb = 1;
+    return sb < nq ? sb : nq;
+}
+
+ScanShape scan_shape(const ifvs_index* ix, int64_t n, int kk) {
+    ScanShape sh;
+    sh.n_blocks = ix->n_blocks;
+    sh.M = ix->M;
+    sh.K = ix->K;
+    sh.row_bytes = ix->row_bytes;
+    sh.tab_words = ix->tab_words;
+    const size_t smem = scan_smem_bytes(ix->tab_words, scan_kp(kk));
+    int64_t per_sm = (int64_t)(ix->max_smem > 0 ? 233472 : 233472) / (int64_t)(smem + 1024);
+    if (per_sm < 1) per_sm = 1;
+    if (per_sm > 2) per_sm = 2;  // launch bound of the scan kernel
+    const int64_t resident = (int64_t)ix->num_sms * per_sm;
+    int64_t chunks = (resident * 8 + n - 1) / n;
+    int64_t max_chunks = ix->n_blocks / 16;
+    if (max_chunks < 1) max_chunks = 1;
+    const int64_t key_cap = 32768 / kk;  // bounds the merge's input per query
+    if (max_chunks > key_cap) max_chunks = key_cap > 0 ? key_cap : 1;
+    if (max_chunks > 65535) max_chunks = 65535;
+    if (chunks > max_chunks) chunks = max_chunks;
+    if (chunks < 1) chunks = 1;
+    sh.blocks_per_chunk = (ix->n_blocks + chunks - 1) / chunks;
+    sh.n_chunks = (int)((ix->n_blocks + sh.blocks_per_chunk - 1) / sh.blocks_per_chunk);
+    return sh;
+}
+
+// The query path for one sub-batch of n queries whose inputs are on the
+// device.  Writes k ids / dists per query to out_ids / out_dists (device)
+// and the pass counts to npass_u64 (device, zeroed here).
+int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
+             const ifvs_predicate* dp, const float* dwz, int64_t n, int k, int64_t* out_ids,
+             float* out_dists, unsigned long long* npass_u64) {
+    const int kk = o.R > 0 ? o.R : k;
+    const int Mr = ix->M * ix->r;
+    const bool cond = !o.plain && ix->d_bank != nullptr;
+    TRY(ensure(ix->w_canon, sizeof(CanonPred) * n));
+    TRY(ensure(ix->w_bm, (size_t)n * ix->n_blocks * 32 * 4));
+    TRY(ensure(ix->w_idx, sizeof(uint32_t) * n * (ix->h > 0 ? ix->h : 1)));
+    TRY(ensure(ix->w_alpha, sizeof(float) * n * (Mr > 0 ? Mr : 1)));
+    TRY(ensure(ix->w_wf, sizeof(float) * n * ix->D));
+    TRY(ensure(ix->w_lut, sizeof(float) * n * ix->M * ix->K));
+    const ScanShape sh = scan_shape(ix, n, kk);
+    TRY(ensure(ix->w_part, sizeof(uint64_t) * n * sh.n_chunks * kk));
+    if (o.R > 0) {
+        TRY(ensure(ix->w_cand, sizeof(int64_t) * n * kk));
+        TRY(ensure(ix->w_cdist, sizeof(float) * n * kk));
+    }
+    CUDA_TRY(cudaMemsetAsync(npass_u64, 0, sizeof(unsigned long long) * n, s));
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_PREDICATE);
+        CUDA_TRY(st.end(launch_canonicalize(dp, n, ix->cols(), ix->w_canon.as<CanonPred>(),
+                                            ix->w_err.as<int>(), s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);
+        CUDA_TRY(st.end(launch_filter(ix->cols(), ix->N, ix->n_blocks, ix->w_canon.as<CanonPred>(),
+                                      n, ix->w_bm.as<uint32_t>(), npass_u64, ix->num_sms, s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_CONDITION);
+        CUDA_TRY(st.end(launch_condition(dq, dp, n, ix->D, ix->d_seeds, ix->h, ix->B,
+                                         cond ? ix->d_bank : nullptr, Mr, dwz,
+                                         ix->w_idx.as<uint32_t>(), ix->w_alpha.as<float>(),
+                                         ix->w_wf.as<float>(), s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_LUT);
+        CUDA_TRY(st.end(launch_lut(ix->d_cpq, ix->d_W, cond ? ix->w_alpha.as<float>() : nullptr,
+                                   dq, ix->w_wf.as<float>(), n, ix->M, ix->K, ix->ds, ix->r,
+                                   ix->w_lut.as<float>(), nullptr, ix->num_sms, s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
+        CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_lut.as<float>(), ix->w_bm.as<uint32_t>(), n,
+                                    kk, sh, ix->w_part.as<uint64_t>(), s)));
+    }
+    int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;
+    float* m_dists = o.R > 0 ? ix->w_cdist.as<float>() : out_dists;
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_MERGE);
+        CUDA_TRY(st.end(launch_merge(ix->w_part.as<uint64_t>(), n, sh.n_chunks, kk, m_ids, m_dists, s)));
+    }
+    if (o.R > 0) {
+        Stage st(ix, s, o.timing, IFVS_STAGE_RERANK);
+        CUDA_TRY(st.end(launch_rerank(ix->d_vec, ix->N, ix->D, dq, m_ids, n, o.R, k, out_ids,
+                                      out_dists, s)));
+    }
+    return 0;
+}
+
+int check_index(const ifvs_index* ix, bool need_cb) {
+    if (!ix) return set_err(IFVS_ERR_ARG, "index is NULL");
+    if (need_cb && !ix->has_cb)
+        return set_err(IFVS_ERR_STATE, "ifvs_load_codebooks has not been called on this index");
+    return 0;
+}
+
+// Stage inputs of one sub-batch on the device (copies unless device I/O).
+int stage_inputs(ifvs_index* ix, cudaStream_t s, const Opts& o, int64_t q0, int64_t n,
+                 const float* queries, const ifvs_predicate* preds, const float* wz,
+                 const float** dq, const ifvs_predicate** dp, const float** dwz) {
+    const int D = ix->D;
+    if (o.dio) {
+        if (dq) *dq = queries ? queries + q0 * D : nullptr;
+        if (dp) *dp = preds ? preds + q0 : nullptr;
+        if (dwz) *dwz = wz ? wz + q0 * D : nullptr;
+        return 0;
+    }
+    if (dq) {
+        *dq = nullptr;
+        if (queries) {
+            TRY(ensure(ix->w_q, sizeof(float) * n * D));
+            CUDA_TRY(cudaMemcpyAsync(ix->w_q.p, queries + q0 * D, sizeof(float) * n * D,
+                                     cudaMemcpyHostToDevice, s));
+            *dq = ix->w_q.as<float>();
+        }
+    }
+    if (dp) {
+        *dp = nullptr;
+        if (preds) {
+            TRY(ensure(ix->w_preds, sizeof(ifvs_predicate) * n));
+            CUDA_TRY(cudaMemcpyAsync(ix->w_preds.p, preds + q0, sizeof(ifvs_predicate) * n,
+                                     cudaMemcpyHostToDevice, s));
+            *dp = ix->w_preds.as<ifvs_predicate>();
+        }
+    }
+    if (dwz) {
+        *dwz = nullptr;
+        if (wz) {
+            TRY(ensure(ix->w_wz, sizeof(float) * n * D));
+            CUDA_TRY(cudaMemcpyAsync(ix->w_wz.p, wz + q0 * D, sizeof(float) * n * D,
+                                     cudaMemcpyHostToDevice, s));
+            *dwz = ix->w_wz.as<float>();
+        }
+    }
+    return 0;
+}
+
+int copy_out(cudaStream_t s, bool dio, void* dst, const void* src, size_t bytes) {
+    if (bytes == 0) return 0;
+    CUDA_TRY(cudaMemcpyAsync(dst, src, bytes, dio ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, s));
+    return 0;
+}
+
+// Synchronise, fold the timing events, and report a malformed predicate.
+int finish(ifvs_index* ix, cudaStream_t s, bool check_preds) {
+    CUDA_TRY(cudaStreamSynchronize(s));
+    ix->collect();
+    if (check_preds) {
+        int err = 0;
+        CUDA_TRY(cudaMemcpy(&err, ix->w_err.p, sizeof(int), cudaMemcpyDeviceToHost));
+        if (err) return set_err(IFVS_ERR_ARG, "a predicate is malformed (n_clauses outside 0..4, "
+                                              "reserved != 0, column out of range or unknown operator)");
+    }
+    return 0;
+}
+
+int reset_err_flag(ifvs_index* ix, cudaStream_t s) {
+    TRY(ensure(ix->w_err, sizeof(int)));
+    CUDA_TRY(cudaMemsetAsync(ix->w_err.p, 0, sizeof(int), s));
+    return 0;
+}
+
+}  // namespace
+
+// ============================================================== C ABI
+
+extern "C" {
+
+const char* ifvs_last_error(void) { return g_err; }
+
+const char* ifvs_version(void) { return "ifvs-gb300 0.1 (sm_103a)"; }
+
+int ifvs_canonical_predicate(const ifvs_predicate* p, const int32_t* attr_types, int32_t n_attrs,
+                             int32_t* lo, uint32_t* width_m1, int32_t* empty) {
+    if (!p || (n_attrs > 0 && !attr_types) || n_attrs < 0 || n_attrs > IFVS_MAX_ATTRS)
+        return set_err(IFVS_ERR_ARG, "invalid arguments");
+    int32_t t[IFVS_MAX_ATTRS] = {0, 0, 0, 0};
+    for (int i = 0; i < n_attrs; ++i) t[i] = attr_types[i];
+    CanonPred c;
+    int rc = canonicalize(*p, t, n_attrs, &c);
+    for (int i = 0; i < n_attrs; ++i) {
+        if (lo) lo[i] = c.lo[i];
+        if (width_m1) width_m1[i] = c.wm1[i];
+    }
+    if (empty) *empty = c.empty;
+    if (rc != 0) return set_err(IFVS_ERR_ARG, "malformed predicate");
+    return IFVS_OK;
+}
+
+int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int64_t N, int32_t M,
+                    int32_t K, const void* const* attr_cols, const int32_t* attr_types,
+                    int32_t n_attrs, const float* vectors, int32_t D, uint32_t flags) {
+    if (!out) return set_err(IFVS_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (!codes) return set_err(IFVS_ERR_ARG, "codes is NULL");
+    if (N < 1 || N > (int64_t)0xFFFFFFFFLL - 2048)
+        return set_err(IFVS_ERR_ARG, "N = %lld outside 1..2^32-2049", (long long)N);
+    if (M < 1 || M > IFVS_MAX_M) return set_err(IFVS_ERR_UNSUPPORTED, "M = %d outside 1..%d", M, IFVS_MAX_M);
+    if (K < 1 || K > 256) return set_err(IFVS_ERR_UNSUPPORTED, "K = %d outside 1..256", K);
+    if (n_attrs < 0 || n_attrs > IFVS_MAX_ATTRS)
+        return set_err(IFVS_ERR_ARG, "n_attrs = %d outside 0..%d", n_attrs, IFVS_MAX_ATTRS);
+    if (n_attrs > 0 && (!attr_cols || !attr_types)) return set_err(IFVS_ERR_ARG, "attribute arrays are NULL");
+    for (int i = 0; i < n_attrs; ++i) {
+        if (!attr_cols[i]) return set_err(IFVS_ERR_ARG, "attribute column %d is NULL", i);
+        if (attr_types[i] != IFVS_ATTR_I32 && attr_types[i] != IFVS_ATTR_I16)
+            return set_err(IFVS_ERR_ARG, "attribute column %d has unknown type %d", i, attr_types[i]);
+    }
+    if (D < 0 || (D > 0 && D % M != 0)) return set_err(IFVS_ERR_ARG, "D = %d is not a multiple of M = %d", D, M);
+    if (vectors && D == 0) return set_err(IFVS_ERR_ARG, "raw vectors need D > 0");
+    if (flags & ~IFVS_F_DEVICE_IO) return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", flags);
+    const bool dio = flags & IFVS_F_DEVICE_IO;
+
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) {
+        cudaGetLastError();
+        return set_err(IFVS_ERR_CUDA, "no CUDA device is available");
+    }
+    if (device < 0 || device >= ndev) return set_err(IFVS_ERR_ARG, "device %d outside 0..%d", device, ndev - 1);
+    DeviceGuard g(device);
+    if (!g.ok) return set_err(IFVS_ERR_CUDA, "cudaSetDevice(%d) failed", device);
+
+    ifvs_index* ix = new (std::nothrow) ifvs_index();
+    if (!ix) return set_err(IFVS_ERR_OOM, "host allocation failed");
+    ix->device = device;
+    int rc = 0;
+    auto fail = [&](int code) {
+        free_index(ix);
+        return code;
+    };
+    if (cudaDeviceGetAttribute(&ix->num_sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&ix->max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, device) != cudaSuccess)
+        return fail(cuda_fail(cudaGetLastError(), "cudaDeviceGetAttribute", __LINE__));
+    if (cudaStreamCreateWithFlags(&ix->stream, cudaStreamNonBlocking) != cudaSuccess)
+        return fail(cuda_fail(cudaGetLastError(), "cudaStreamCreateWithFlags", __LINE__));
+    ix->N = N;
+    ix->M = M;
+    ix->K = K;
+    ix->D = D;
+    ix->ds = D > 0 ? D / M : 0;
+    ix->n_blocks = (N + kBlockRows - 1) / kBlockRows;
+    ix->n_rows_pad = ix->n_blocks * kBlockRows;
+    ix->row_bytes = (int)round_up(M, 4);
+    ix->tab_words = (int)round_up(M + 31, 32);
+    if (scan_smem_bytes(ix->tab_words, 256) > (size_t)ix->max_smem)
+        return fail(set_err(IFVS_ERR_UNSUPPORTED, "M = %d needs %zu bytes of shared memory (device: %d)",
+                            M, scan_smem_bytes(ix->tab_words, 256), ix->max_smem));
+    cudaStream_t s = ix->stream;
+    const cudaMemcpyKind h2d = dio ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+
+    // codes -> rotated rows
+    void* tmp = nullptr;
+    const uint8_t* src = codes;
+    if (!dio) {
+        if ((rc = dev_alloc(ix, &tmp, (size_t)N * M))) return fail(rc);
+        ix->bytes -= (size_t)N * M;
+        if (cudaMemcpyAsync(tmp, codes, (size_t)N * M, cudaMemcpyHostToDevice, s) != cudaSuccess) {
+            cudaFree(tmp);
+            return fail(cuda_fail(cudaGetLastError(), "cudaMemcpyAsync(codes)", __LINE__));
+        }
+        src = (const uint8_t*)tmp;
+    }
+    void* dcodes = nullptr;
+    if ((rc = dev_alloc(ix, &dcodes, (size_t)ix->n_rows_pad * ix->row_bytes))) {
+        if (tmp) cudaFree(tmp);
+        return fail(rc);
+    }
+    ix->d_codes = (uint8_t*)dcodes;
+    if ((rc = ensure(ix->w_err, sizeof(int)))) {
+        if (tmp) cudaFree(tmp);
+        return fail(rc);
+    }
+    cudaMemsetAsync(ix->w_err.p, 0, sizeof(int), s);
+    cudaError_t e = launch_relayout_codes(src, N, M, K, ix->row_bytes, ix->n_rows_pad, ix->d_codes,
+                                          ix->w_err.as<int>(), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (tmp) cudaFree(tmp);
+    if (e != cudaSuccess) return fail(cuda_fail(e, "code re-layout", __LINE__));
+    int bad = 0;
+    if (cudaMemcpy(&bad, ix->w_err.p, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return fail(cuda_fail(cudaGetLastError(), "cudaMemcpy(flag)", __LINE__));
+    if (bad) return fail(set_err(IFVS_ERR_ARG, "a code is >= K = %d", K));
+
+    // attribute columns, padded with zeros to n_rows_pad
+    ix->n_attrs = n_attrs;
+    for (int i = 0; i < n_attrs; ++i) {
+        ix->types[i] = attr_types[i];
+        const size_t es = attr_types[i] == IFVS_ATTR_I16 ? 2 : 4;
+        if ((rc = dev_alloc(ix, &ix->d_attr[i], es * ix->n_rows_pad))) return fail(rc);
+        if (cudaMemsetAsync(ix->d_attr[i], 0, es * ix->n_rows_pad, s) != cudaSuccess ||
+            cudaMemcpyAsync(ix->d_attr[i], attr_cols[i], es * N, h2d, s) != cudaSuccess)
+            return fail(cuda_fail(cudaGetLastError(), "attribute copy", __LINE__));
+    }
+    if (vectors) {
+        void* v = nullptr;
+        if ((rc = dev_alloc(ix, &v, sizeof(float) * N * D))) return fail(rc);
+        ix->d_vec = (float*)v;
+        if (cudaMemcpyAsync(v, vectors, sizeof(float) * N * D, h2d, s) != cudaSuccess)
+            return fail(cuda_fail(cudaGetLastError(), "vector copy", __LINE__));
+    }
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return fail(cuda_fail(e, "index upload", __LINE__));
+    *out = ix;
+    return IFVS_OK;
+}
+
+int ifvs_load_codebooks(ifvs_index* ix, const float* C_pq, int32_t ds, const float* bank, int64_t B,
+                        int32_t h, int32_t r, const float* W, const uint64_t* hash_seeds) {
+    TRY(check_index(ix, false));
+    if (!C_pq) return set_err(IFVS_ERR_ARG, "C_pq is NULL");
+    if (ds < 1) return set_err(IFVS_ERR_ARG, "ds = %d must be >= 1", ds);
+    if (ix->D > 0 && ix->D != ix->M * ds)
+        return set_err(IFVS_ERR_ARG, "ds = %d does not match D = %d and M = %d", ds, ix->D, ix->M);
+    if (bank) {
+        if (B < 1 || B > 0xFFFFFFFFLL) return set_err(IFVS_ERR_ARG, "B = %lld outside 1..2^32-1", (long long)B);
+        if (h < 1 || h > 64) return set_err(IFVS_ERR_ARG, "h = %d outside 1..64", h);
+        if (r < 1 || r > 256) return set_err(IFVS_ERR_ARG, "r = %d outside 1..256", r);
+        if (!W || !hash_seeds) return set_err(IFVS_ERR_ARG, "W and hash_seeds are required with a bank");
+    }
+    DeviceGuard g(ix->device);
+    cudaStream_t s = ix->stream;
+    CUDA_TRY(cudaStreamSynchronize(s));
+    void* old[] = {ix->d_cpq, ix->d_bank, ix->d_W, ix->d_seeds};
+    for (void* p : old)
+        if (p) cudaFree(p);
+    ix->d_cpq = nullptr;
+    ix->d_bank = nullptr;
+    ix->d_W = nullptr;
+    ix->d_seeds = nullptr;
+    ix->has_cb = false;
+    ix->ds = ds;
+    ix->D = ix->M * ds;
+    const size_t ncb = (size_t)ix->M * ix->K * ds;
+    void* p = nullptr;
+    TRY(dev_alloc(ix, &p, sizeof(float) * ncb));
+    ix->d_cpq = (float*)p;
+    CUDA_TRY(cudaMemcpyAsync(p, C_pq, sizeof(float) * ncb, cudaMemcpyHostToDevice, s));
+    if (bank) {
+        ix->B = B;
+        ix->h = h;
+        ix->r = r;
+        TRY(dev_alloc(ix, &p, sizeof(float) * (size_t)B * ix->M * r));
+        ix->d_bank = (float*)p;
+        CUDA_TRY(cudaMemcpyAsync(p, bank, sizeof(float) * (size_t)B * ix->M * r, cudaMemcpyHostToDevice, s));
+        TRY(dev_alloc(ix, &p, sizeof(float) * ncb * r));
+        ix->d_W = (float*)p;
+        CUDA_TRY(cudaMemcpyAsync(p, W, sizeof(float) * ncb * r, cudaMemcpyHostToDevice, s));
+        TRY(dev_alloc(ix, &p, sizeof(uint64_t) * h));
+        ix->d_seeds = (uint64_t*)p;
+        CUDA_TRY(cudaMemcpyAsync(p, hash_seeds, sizeof(uint64_t) * h, cudaMemcpyHostToDevice, s));
+    } else {
+        ix->B = 0;
+        ix->h = 0;
+        ix->r = 0;
+    }
+    CUDA_TRY(cudaStreamSynchronize(s));
+    ix->has_cb = true;
+    return IFVS_OK;
+}
+
+int ifvs_search_batch(ifvs_index* ix, const float* queries, const ifvs_predicate* preds, int64_t nq,
+                      int32_t k, const float* wz, const ifvs_search_params* p, int64_t* ids,
+                      float* dists, int64_t* npass) {
+    TRY(check_index(ix, true));
+    Opts o;
+    TRY(parse_opts(p, &o));
+    if (nq < 0) return set_err(IFVS_ERR_ARG, "nq < 0");
+    if (k < 1 || k > IFVS_MAX_K) return set_err(IFVS_ERR_ARG, "k = %d outside 1..%d", k, IFVS_MAX_K);
+    if (o.R > 0 && o.R < k) return set_err(IFVS_ERR_ARG, "rerank depth %d is below k = %d", o.R, k);
+    if (o.R > 0 && !ix->d_vec) return set_err(IFVS_ERR_STATE, "rerank needs raw vectors at load time");
+    if (nq == 0) return IFVS_OK;
+    if (!queries || !preds || !ids || !dists) return set_err(IFVS_ERR_ARG, "an array argument is NULL");
+    DeviceGuard g(ix->device);
+    cudaStream_t s = o.stream ? o.stream : ix->stream;
+    const int64_t sb = pick_sub_batch(ix, o, nq);
+    TRY(reset_err_flag(ix, s));
+    TRY(ensure(ix->w_npass, sizeof(unsigned long long) * sb));
+    if (!o.dio) {
+        TRY(ensure(ix->w_ids, sizeof(int64_t) * sb * k));
+        TRY(ensure(ix->w_dists, sizeof(float) * sb * k));
+    }
+    for (int64_t q0 = 0; q0 < nq; q0 += sb) {
+        const int64_t n = sb < nq - q0 ? sb : nq - q0;
+        const float *dq, *dwz;
+        const ifvs_predicate* dp;
+        TRY(stage_inputs(ix, s, o, q0, n, queries, preds, wz, &dq, &dp, &dwz));
+        int64_t* oid = o.dio ? ids + q0 * k : ix->w_ids.as<int64_t>();
+        float* odi = o.dio ? dists + q0 * k : ix->w_dists.as<float>();
+        TRY(run_path(ix, s, o, dq, dp, dwz, n, k, oid, odi, ix->w_npass.as<unsigned long long>()));
+        if (!o.dio) {
+            TRY(copy_out(s, false, ids + q0 * k, oid, sizeof(int64_t) * n * k));
+            TRY(copy_out(s, false, dists + q0 * k, odi, sizeof(float) * n * k));
+        }
+        if (npass) TRY(copy_out(s, o.dio, npass + q0, ix->w_npass.p, sizeof(int64_t) * n));
+        if (!o.dio && q0 + sb < nq) CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    return finish(ix, s, true);
+}
+
+int ifvs_filter(ifvs_index* ix, const ifvs_predicate* preds, int64_t nq, const ifvs_search_params* p,
+                uint32_t* bitmaps, int64_t* npass) {
+    TRY(check_index(ix, false));
+    Opts o;
+    TRY(parse_opts(p, &o));
+    if (nq < 0) return set_err(IFVS_ERR_ARG, "nq < 0");
+    if (nq == 0) return IFVS_OK;
+    if (!preds || !bitmaps) return set_err(IFVS_ERR_ARG, "an array argument is NULL");
+    DeviceGuard g(ix->device);
+    cudaStream_t s = o.stream ? o.stream : ix->stream;
+    const int64_t sb = pick_sub_batch(ix, o, nq);
+    const int64_t wrows = (ix->N + 31) / 32;
+    TRY(reset_err_flag(ix, s));
+    TRY(ensure(ix->w_npass, sizeof(unsigned long long) * sb));
+    TRY(ensure(ix->w_canon, sizeof(CanonPred) * sb));
+    TRY(ensure(ix->w_bm, (size_t)sb * ix->n_blocks * 128));
+    if (!o.dio) TRY(ensure(ix->w_rows, (size_t)sb * wrows * 4));
+    for (int64_t q0 = 0; q0 < nq; q0 += sb) {
+        const int64_t n = sb < nq - q0 ? sb : nq - q0;
+        const ifvs_predicate* dp;
+        TRY(stage_inputs(ix, s, o, q0, n, nullptr, preds, nullptr, nullptr, &dp, nullptr));
+        CUDA_TRY(cudaMemsetAsync(ix->w_npass.p, 0, sizeof(unsigned long long) * n, s));
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_PREDICATE);
+            CUDA_TRY(st.end(launch_canonicalize(dp, n, ix->cols(), ix->w_canon.as<CanonPred>(),
+                                                ix->w_err.as<int>(), s)));
+        }
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);
+            CUDA_TRY(st.end(launch_filter(ix->cols(), ix->N, ix->n_blocks, ix->w_canon.as<CanonPred>(), n,
+                                          ix->w_bm.as<uint32_t>(), ix->w_npass.as<unsigned long long>(),
+                                          ix->num_sms, s)));
+        }
+        uint32_t* rows = o.dio ? bitmaps + q0 * wrows : ix->w_rows.as<uint32_t>();
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_LAYOUT);
+            CUDA_TRY(st.end(launch_bitmap_layout(ix->w_bm.as<uint32_t>(), rows, n, ix->n_blocks, wrows,
+                                                 true, s)));
+        }
+        if (!o.dio) TRY(copy_out(s, false, bitmaps + q0 * wrows, rows, sizeof(uint32_t) * n * wrows));
+        if (npass) TRY(copy_out(s, o.dio, npass + q0, ix->w_npass.p, sizeof(int64_t) * n));
+        if (q0 + sb < nq) CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    return finish(ix, s, true);
+}
+
+int ifvs_condition(ifvs_index* ix, const float* queries, const ifvs_predicate* preds, int64_t nq,
+                   const float* wz, const ifvs_search_params* p, uint32_t* bank_idx, float* alpha,
+                   float* wf, float* C_ifvs, float* lut) {
+    TRY(check_index(ix, true));
+    Opts o;
+    TRY(parse_opts(p, &o));
+    if (nq < 0) return set_err(IFVS_ERR_ARG, "nq < 0");
+    if (nq == 0) return IFVS_OK;
+    if (!queries || !preds) return set_err(IFVS_ERR_ARG, "queries / preds is NULL");
+    DeviceGuard g(ix->device);
+    cudaStream_t s = o.stream ? o.stream : ix->stream;
+    const bool cond = !o.plain && ix->d_bank != nullptr;
+    const int Mr = ix->M * ix->r;
+    const int64_t sb = nq < 1024 ? nq : 1024;
+    TRY(reset_err_flag(ix, s));
+    TRY(ensure(ix->w_canon, sizeof(CanonPred) * sb));
+    TRY(ensure(ix->w_idx, sizeof(uint32_t) * sb * (ix->h > 0 ? ix->h : 1)));
+    TRY(ensure(ix->w_alpha, sizeof(float) * sb * (Mr > 0 ? Mr : 1)));
+    TRY(ensure(ix->w_wf, sizeof(float) * sb * ix->D));
+    TRY(ensure(ix->w_lut, sizeof(float) * sb * ix->M * ix->K));
+    if (C_ifvs) TRY(ensure(ix->w_cifvs, sizeof(float) * sb * ix->M * ix->K * ix->ds));
+    for (int64_t q0 = 0; q0 < nq; q0 += sb) {
+        const int64_t n = sb < nq - q0 ? sb : nq - q0;
+        const float *dq, *dwz;
+        const ifvs_predicate* dp;
+        TRY(stage_inputs(ix, s, o, q0, n, queries, preds, wz, &dq, &dp, &dwz));
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_PREDICATE);
+            CUDA_TRY(st.end(launch_canonicalize(dp, n, ix->cols(), ix->w_canon.as<CanonPred>(),
+                                                ix->w_err.as<int>(), s)));
+        }
+        if (!cond) {
+            CUDA_TRY(cudaMemsetAsync(ix->w_idx.p, 0, sizeof(uint32_t) * n * (ix->h > 0 ? ix->h : 1), s));
+            CUDA_TRY(cudaMemsetAsync(ix->w_alpha.p, 0, sizeof(float) * n * (Mr > 0 ? Mr : 1), s));
+        }
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_CONDITION);
+            CUDA_TRY(st.end(launch_condition(dq, dp, n, ix->D, ix->d_seeds, ix->h, ix->B,
+                                             cond ? ix->d_bank : nullptr, Mr, dwz,
+                                             ix->w_idx.as<uint32_t>(), ix->w_alpha.as<float>(),
+                                             ix->w_wf.as<float>(), s)));
+        }
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_LUT);
+            CUDA_TRY(st.end(launch_lut(ix->d_cpq, ix->d_W, cond ? ix->w_alpha.as<float>() : nullptr, dq,
+                                       ix->w_wf.as<float>(), n, ix->M, ix->K, ix->ds, ix->r,
+                                       ix->w_lut.as<float>(), C_ifvs ? ix->w_cifvs.as<float>() : nullptr,
+                                       ix->num_sms, s)));
+        }
+        if (bank_idx && ix->h > 0)
+            TRY(copy_out(s, o.dio, bank_idx + q0 * ix->h, ix->w_idx.p, sizeof(uint32_t) * n * ix->h));
+        if (alpha && Mr > 0) TRY(copy_out(s, o.dio, alpha + q0 * Mr, ix->w_alpha.p, sizeof(float) * n * Mr));
+        if (wf) TRY(copy_out(s, o.dio, wf + q0 * ix->D, ix->w_wf.p, sizeof(float) * n * ix->D));
+        if (lut)
+            TRY(copy_out(s, o.dio, lut + q0 * ix->M * ix->K, ix->w_lut.p, sizeof(float) * n * ix->M * ix->K));
+        if (C_ifvs)
+            TRY(copy_out(s, o.dio, C_ifvs + q0 * ix->M * ix->K * ix->ds, ix->w_cifvs.p,
+                         sizeof(float) * n * ix->M * ix->K * ix->ds));
+        if (q0 + sb < nq) CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    return finish(ix, s, true);
+}
+
+int ifvs_scan_topk(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, int64_t nq, int32_t k,
+                   const ifvs_search_params* p, int64_t* ids, float* dists) {
+    TRY(check_index(ix, false));
+    Opts o;
+    TRY(parse_opts(p, &o));
+    if (nq < 0) return set_err(IFVS_ERR_ARG, "nq < 0");
+    if (k < 1 || k > IFVS_MAX_K) return set_err(IFVS_ERR_ARG, "k = %d outside 1..%d", k, IFVS_MAX_K);
+    if (nq == 0) return IFVS_OK;
+    if (!lut || !bitmaps || !ids || !dists) return set_err(IFVS_ERR_ARG, "an array argument is NULL");
+    DeviceGuard g(ix->device);
+    cudaStream_t s = o.stream ? o.stream : ix->stream;
+    const int64_t sb = pick_sub_batch(ix, o, nq);
+    const int64_t wrows = (ix->N + 31) / 32;
+    const size_t lut_n = (size_t)ix->M * ix->K;
+    TRY(ensure(ix->w_bm, (size_t)sb * ix->n_blocks * 128));
+    if (!o.dio) {
+        TRY(ensure(ix->w_rows, (size_t)sb * wrows * 4));
+        TRY(ensure(ix->w_lut, sizeof(float) * sb * lut_n));
+        TRY(ensure(ix->w_ids, sizeof(int64_t) * sb * k));
+        TRY(ensure(ix->w_dists, sizeof(float) * sb * k));
+    }
+    for (int64_t q0 = 0; q0 < nq; q0 += sb) {
+        const int64_t n = sb < nq - q0 ? sb : nq - q0;
+        const float* dl = lut + q0 * lut_n;
+        const uint32_t* drows = bitmaps + q0 * wrows;
+        if (!o.dio) {
+            CUDA_TRY(cudaMemcpyAsync(ix->w_lut.p, dl, sizeof(float) * n * lut_n, cudaMemcpyHostToDevice, s));
+            CUDA_TRY(cudaMemcpyAsync(ix->w_rows.p, drows, sizeof(uint32_t) * n * wrows, cudaMemcpyHostToDevice, s));
+            dl = ix->w_lut.as<float>();
+            drows = ix->w_rows.as<uint32_t>();
+        }
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_LAYOUT);
+            CUDA_TRY(st.end(launch_bitmap_layout(drows, ix->w_bm.as<uint32_t>(), n, ix->n_blocks, wrows,
+                                                 false, s)));
+        }
+        const ScanShape sh = scan_shape(ix, n, k);
+        TRY(ensure(ix->w_part, sizeof(uint64_t) * n * sh.n_chunks * k));
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
+            CUDA_TRY(st.end(launch_scan(ix->d_codes, dl, ix->w_bm.as<uint32_t>(), n, k, sh,
+                                        ix->w_part.as<uint64_t>(), s)));
+        }
+        int64_t* oid = o.dio ? ids + q0 * k : ix->w_ids.as<int64_t>();
+        float* odi = o.dio ? dists + q0 * k : ix->w_dists.as<float>();
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_MERGE);
+            CUDA_TRY(st.end(launch_merge(ix->w_part.as<uint64_t>(), n, sh.n_chunks, k, oid, odi, s)));
+        }
+        if (!o.dio) {
+            TRY(copy_out(s, false, ids + q0 * k, oid, sizeof(int64_t) * n * k));
+            TRY(copy_out(s, false, dists + q0 * k, odi, sizeof(float) * n * k));
+            CUDA_TRY(cudaStreamSynchronize(s));
+        }
+    }
+    return finish(ix, s, false);
+}
+
+int ifvs_rerank(ifvs_index* ix, const float* queries, const int64_t* cand, int64_t nq, int32_t R,
+                int32_t k, const ifvs_search_params* p, int64_t* ids, float* dists) {
+    TRY(check_index(ix, false));
+    Opts o;
+    TRY(parse_opts(p, &o));
+    if (!ix->d_vec) return set_err(IFVS_ERR_STATE, "rerank needs raw vectors at load time");
+    if (ix->D <= 0) return set_err(IFVS_ERR_STATE, "vector dimension unknown");
+    if (nq < 0) return set_err(IFVS_ERR_ARG, "nq < 0");
+    if (R < 1 || R > IFVS_MAX_K) return set_err(IFVS_ERR_ARG, "R = %d outside 1..%d", R, IFVS_MAX_K);
+    if (k < 1 || k > R) return set_err(IFVS_ERR_ARG, "k = %d outside 1..R", k);
+    if (nq == 0) return IFVS_OK;
+    if (!queries || !cand || !ids || !dists) return set_err(IFVS_ERR_ARG, "an array argument is NULL");
+    DeviceGuard g(ix->device);
+    cudaStream_t s = o.stream ? o.stream : ix->stream;
+    const float* dq = queries;
+    const int64_t* dc = cand;
+    int64_t* oid = ids;
+    float* odi = dists;
+    if (!o.dio) {
+        TRY(ensure(ix->w_q, sizeof(float) * nq * ix->D));
+        TRY(ensure(ix->w_cand, sizeof(int64_t) * nq * R));
+        TRY(ensure(ix->w_ids, sizeof(int64_t) * nq * k));
+        TRY(ensure(ix->w_dists, sizeof(float) * nq * k));
+        CUDA_TRY(cudaMemcpyAsync(ix->w_q.p, queries, sizeof(float) * nq * ix->D, cudaMemcpyHostToDevice, s));
+        CUDA_TRY(cudaMemcpyAsync(ix->w_cand.p, cand, sizeof(int64_t) * nq * R, cudaMemcpyHostToDevice, s));
+        dq = ix->w_q.as<float>();
+        dc = ix->w_cand.as<int64_t>();
+        oid = ix->w_ids.as<int64_t>();
+        odi = ix->w_dists.as<float>();
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_RERANK);
+        CUDA_TRY(st.end(launch_rerank(ix->d_vec, ix->N, ix->D, dq, dc, nq, R, k, oid, odi, s)));
+    }
+    if (!o.dio) {
+        TRY(copy_out(s, false, ids, oid, sizeof(int64_t) * nq * k));
+        TRY(copy_out(s, false, dists, odi, sizeof(float) * nq * k));
+    }
+    return finish(ix, s, false);
+}
+
+int ifvs_stage_times(ifvs_index* ix, double* ms, int64_t* launches, int32_t reset) {
+    TRY(check_index(ix, false));
+    for (int i = 0; i < IFVS_N_STAGES; ++i) {
+        if (ms) ms[i] = ix->stage_ms[i];
+        if (launches) launches[i] = ix->stage_launches[i];
+        if (reset) {
+            ix->stage_ms[i] = 0.0;
+            ix->stage_launches[i] = 0;
+        }
+    }
+    return IFVS_OK;
+}
+
+int ifvs_index_info(const ifvs_index* ix, int64_t* out) {
+    if (!ix || !out) return set_err(IFVS_ERR_ARG, "NULL argument");
+    out[0] = ix->N;
+    out[1] = ix->M;
+    out[2] = ix->K;
+    out[3] = ix->D;
+    out[4] = ix->ds;
+    out[5] = ix->n_attrs;
+    out[6] = ix->has_cb ? 1 : 0;
+    out[7] = (int64_t)ix->bytes;
+    return IFVS_OK;
+}
+
+void ifvs_free(ifvs_index* ix) { free_index(ix); }
+
+}  // extern "C"

@@ -1,0 +1,176 @@
+// Stage 1 of §2 (Filter): every row's attribute values are tested against
+// the query's predicate (the conjunctive form of Listing 1), giving the
+// candidate pool P as a pass bitmap.
+//
+// One warp owns one 1024-row block: lane l holds the 32 attribute values of
+// rows b*1024 + 32*j + l (j = 0..31), loaded with 32 coalesced 128-byte
+// column reads, and then evaluates every query of its group against them,
+// so the columns are read once per query group.  The lane's 32 pass bits
+// form its word of the lane-major bitmap directly (no ballot needed), one
+// 128-byte store per warp and query.  Popcounts go through a warp reduction
+// into npass.
+#include "internal.cuh"
+
+namespace ifvs {
+
+__global__ void k_canonicalize(const ifvs_predicate* __restrict__ preds, int64_t nq,
+                               AttrCols cols, CanonPred* __restrict__ out, int* __restrict__ err) {
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= nq) return;
+    ifvs_predicate p = preds[i];
+    CanonPred c;
+    if (canonicalize(p, cols.type, cols.n, &c) != 0) atomicOr(err, 1);
+    out[i] = c;
+}
+
+cudaError_t launch_canonicalize(const ifvs_predicate* preds, int64_t nq, AttrCols cols,
+                                CanonPred* out, int* err, cudaStream_t s) {
+    if (nq <= 0) return cudaSuccess;
+    int threads = 128;
+    int64_t blocks = (nq + threads - 1) / threads;
+    k_canonicalize<<<(unsigned)blocks, threads, 0, s>>>(preds, nq, cols, out, err);
+    return cudaGetLastError();
+}
+
+template <int NA>
+__global__ void __launch_bounds__(kThreads) k_filter(AttrCols cols, int64_t N, int64_t n_blocks,
+                                                     const CanonPred* __restrict__ canon,
+                                                     int64_t nq, int q_per_cta,
+                                                     uint32_t* __restrict__ bm,
+                                                     unsigned long long* __restrict__ npass) {
+    const int lane = threadIdx.x & 31;
+    const int64_t b = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
+    if (b >= n_blocks) return;
+    const int64_t q0 = (int64_t)blockIdx.y * q_per_cta;
+    const int64_t q1 = min(nq, q0 + (int64_t)q_per_cta);
+    const int64_t row0 = b * kBlockRows + lane;
+
+    // rows beyond N: their bits stay 0 (the columns are padded, so the
+    // loads themselves stay inside the allocation)
+    uint32_t valid = 0xFFFFFFFFu;
+    if (b * kBlockRows + kBlockRows > N) {
+        valid = 0;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) valid |= (uint32_t)(row0 + 32 * j < N) << j;
+    }
+
+    int32_t v[NA][32];
+#pragma unroll
+    for (int c = 0; c < NA; ++c) {
+        if (cols.type[c] == IFVS_ATTR_I16) {
+            const int16_t* col = (const int16_t*)cols.col[c] + row0;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[c][j] = __ldg(col + 32 * j);
+        } else {
+            const int32_t* col = (const int32_t*)cols.col[c] + row0;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[c][j] = __ldg(col + 32 * j);
+        }
+    }
+
+    const int64_t words = n_blocks * 32;
+    for (int64_t q = q0; q < q1; ++q) {
+        const CanonPred* cp = canon + q;
+        uint32_t m = 0;
+        if (!cp->empty) {
+            m = valid;
+            const uint32_t used = cp->used;
+#pragma unroll
+            for (int c = 0; c < NA; ++c) {
+                if (used >> c & 1u) {
+                    const int32_t lo = cp->lo[c];
+                    const uint32_t wm1 = cp->wm1[c];
+                    uint32_t mc = 0;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        mc |= (uint32_t)((uint32_t)(v[c][j] - lo) <= wm1) << j;
+                    m &= mc;
+                }
+            }
+        }
+        bm[q * words + b * 32 + lane] = m;
+        unsigned cnt = __reduce_add_sync(0xFFFFFFFFu, (unsigned)__popc(m));
+        if (lane == 0 && cnt) atomicAdd(npass + q, (unsigned long long)cnt);
+    }
+}
+
+cudaError_t launch_filter(AttrCols cols, int64_t N, int64_t n_blocks, const CanonPred* canon,
+                          int64_t nq, uint32_t* bm, unsigned long long* npass, int num_sms,
+                          cudaStream_t s) {
+    if (nq <= 0) return cudaSuccess;
+    const int64_t tiles = (n_blocks + kWarps - 1) / kWarps;
+    // enough CTAs to fill the GPU a few times over; each CTA walks a group
+    // of queries so that a column tile is read once per group
+    const int64_t target = (int64_t)num_sms * 8;
+    int64_t groups = (target + tiles - 1) / tiles;
+    if (groups < 1) groups = 1;
+    if (groups > nq) groups = nq;
+    if (groups > 65535) groups = 65535;
+    const int64_t qpc = (nq + groups - 1) / groups;
+    groups = (nq + qpc - 1) / qpc;
+    dim3 grid((unsigned)tiles, (unsigned)groups);
+    int na = cols.n < 1 ? 1 : cols.n;
+    switch (na) {
+        case 1: k_filter<1><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, nq, (int)qpc, bm, npass); break;
+        case 2: k_filter<2><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, nq, (int)qpc, bm, npass); break;
+        case 3: k_filter<3><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, nq, (int)qpc, bm, npass); break;
+        default: k_filter<4><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, nq, (int)qpc, bm, npass); break;
+    }
+    return cudaGetLastError();
+}
+
+// ---- layout conversion ---------------------------------------------------
+
+// Transpose the 32x32 bit matrix held one row per lane (lane l, bit j =
+// element (l, j)) so that lane l ends up with column l.  Five butterfly
+// stages swap the off-diagonal s x s sub-blocks for s = 16, 8, 4, 2, 1.
+__device__ __forceinline__ uint32_t transpose32(uint32_t x, int lane) {
+    const uint32_t masks[5] = {0x0000FFFFu, 0x00FF00FFu, 0x0F0F0F0Fu, 0x33333333u, 0x55555555u};
+#pragma unroll
+    for (int i = 0; i < 5; ++i) {
+        const int s = 16 >> i;
+        const uint32_t mk = masks[i];
+        const uint32_t y = __shfl_xor_sync(0xFFFFFFFFu, x, s);
+        x = (lane & s) ? ((x & ~mk) | ((y >> s) & mk)) : ((x & mk) | ((y & mk) << s));
+    }
+    return x;
+}
+
+__global__ void k_bitmap_layout(const uint32_t* __restrict__ src, uint32_t* __restrict__ dst,
+                                int64_t nq, int64_t n_blocks, int64_t n_words_rows,
+                                bool to_rows) {
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (gw >= nq * n_blocks) return;
+    const int64_t q = gw / n_blocks, b = gw - q * n_blocks;
+    const int64_t lm = q * n_blocks * 32 + b * 32 + lane;
+    const int64_t ri = b * 32 + lane;
+    const int64_t rows_off = q * n_words_rows + ri;
+    uint32_t x;
+    if (to_rows) {
+        x = src[lm];
+    } else {
+        x = ri < n_words_rows ? src[rows_off] : 0u;
+    }
+    // lane-major word (b, l) bit j == row-ordered word (b*32 + j) bit l
+    x = transpose32(x, lane);
+    if (to_rows) {
+        if (ri < n_words_rows) dst[rows_off] = x;
+    } else {
+        dst[lm] = x;
+    }
+}
+
+cudaError_t launch_bitmap_layout(const uint32_t* src, uint32_t* dst, int64_t nq,
+                                 int64_t n_blocks, int64_t n_words_rows, bool to_rows,
+                                 cudaStream_t s) {
+    if (nq <= 0) return cudaSuccess;
+    const int64_t warps = nq * n_blocks;
+    const int threads = 256;
+    const int64_t blocks = (warps * 32 + threads - 1) / threads;
+    k_bitmap_layout<<<(unsigned)blocks, threads, 0, s>>>(src, dst, nq, n_blocks, n_words_rows,
+                                                        to_rows);
+    return cudaGetLastError();
+}
+
+}  // namespace ifvs

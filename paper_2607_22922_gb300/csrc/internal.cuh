@@ -1,0 +1,149 @@
+// Internal declarations of the iFVS GB300 library (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ifvs.h"
+
+namespace ifvs {
+
+// A bitmap block covers 1024 rows: 32 lane-words of 32 bits.  In the
+// device ("lane-major") layout, word (b * 32 + l) bit j is row
+// b * 1024 + 32 * j + l, so lane l of a warp owns rows congruent to l mod 32
+// and reads its 32 pass bits of a block in one coalesced 128-byte load.
+constexpr int kBlockRows = 1024;
+constexpr int kWarps = 8;          // warps per CTA in the scan and filter
+constexpr int kThreads = kWarps * 32;
+
+// One predicate reduced to a closed interval per attribute column:
+// row passes iff for every column c, (uint32)(a_c - lo[c]) <= wm1[c].
+struct CanonPred {
+    int32_t lo[IFVS_MAX_ATTRS];
+    uint32_t wm1[IFVS_MAX_ATTRS];
+    uint32_t used;     // bit c: column c is constrained
+    int32_t empty;     // 1: no row can pass
+    int32_t invalid;   // 1: malformed predicate
+    int32_t pad;
+};
+
+// Reduce a predicate to per-column intervals (clauses on one column
+// intersect).  Returns 0, or -1 when the predicate is malformed.
+__host__ __device__ inline int canonicalize(const ifvs_predicate& p, const int32_t* types,
+                                            int n_attrs, CanonPred* out) {
+    int64_t lo[IFVS_MAX_ATTRS], hi[IFVS_MAX_ATTRS];
+    out->used = 0;
+    out->empty = 0;
+    out->invalid = 0;
+    out->pad = 0;
+    for (int c = 0; c < IFVS_MAX_ATTRS; ++c) {
+        bool i16 = c < n_attrs && types[c] == IFVS_ATTR_I16;
+        lo[c] = i16 ? -32768 : -2147483648LL;
+        hi[c] = i16 ? 32767 : 2147483647LL;
+    }
+    int bad = (p.n_clauses < 0 || p.n_clauses > IFVS_MAX_CLAUSES || p.reserved != 0);
+    int nc = bad ? 0 : p.n_clauses;
+    for (int i = 0; i < nc; ++i) {
+        const ifvs_clause& cl = p.c[i];
+        if (cl.col < 0 || cl.col >= n_attrs) { bad = 1; break; }
+        int64_t a, b;
+        const int64_t kMin = (-9223372036854775807LL - 1), kMax = 9223372036854775807LL;
+        bool none = false;
+        switch (cl.op) {
+            case IFVS_OP_EQ: a = cl.lo; b = cl.lo; break;
+            case IFVS_OP_RANGE:
+                a = cl.lo;
+                if (cl.hi == kMin) { none = true; b = kMin; } else { b = cl.hi - 1; }
+                break;
+            case IFVS_OP_GE: a = cl.lo; b = kMax; break;
+            case IFVS_OP_LT:
+                a = kMin;
+                if (cl.lo == kMin) { none = true; b = kMin; } else { b = cl.lo - 1; }
+                break;
+            case IFVS_OP_GT:
+                b = kMax;
+                if (cl.lo == kMax) { none = true; a = kMax; } else { a = cl.lo + 1; }
+                break;
+            case IFVS_OP_LE: a = kMin; b = cl.lo; break;
+            default: bad = 1; a = 0; b = 0; break;
+        }
+        if (bad) break;
+        if (none) { out->empty = 1; continue; }
+        if (a > lo[cl.col]) lo[cl.col] = a;
+        if (b < hi[cl.col]) hi[cl.col] = b;
+        out->used |= 1u << cl.col;
+    }
+    for (int c = 0; c < IFVS_MAX_ATTRS; ++c) {
+        if (lo[c] > hi[c]) {
+            out->empty = 1;
+            out->lo[c] = 0;
+            out->wm1[c] = 0;
+        } else {
+            out->lo[c] = (int32_t)lo[c];
+            out->wm1[c] = (uint32_t)(hi[c] - lo[c]);
+        }
+    }
+    if (bad) { out->invalid = 1; out->empty = 1; return -1; }
+    return 0;
+}
+
+struct AttrCols {
+    const void* col[IFVS_MAX_ATTRS];
+    int32_t type[IFVS_MAX_ATTRS];
+    int32_t n;
+};
+
+// ---- kernel launchers (one per translation unit) -----------------------
+// Every launcher returns the cudaError_t of its launch.
+
+// predicates -> canonical intervals; *err |= 1 for any malformed predicate
+cudaError_t launch_canonicalize(const ifvs_predicate* preds, int64_t nq, AttrCols cols,
+                                CanonPred* out, int* err, cudaStream_t s);
+
+// Filter: lane-major pass bitmaps [nq][n_blocks * 32] + popcounts (added to npass)
+cudaError_t launch_filter(AttrCols cols, int64_t N, int64_t n_blocks, const CanonPred* canon,
+                          int64_t nq, uint32_t* bm, unsigned long long* npass, int num_sms,
+                          cudaStream_t s);
+
+// 32x32 bit transposes between the lane-major layout and the row-ordered
+// layout of the ABI ([nq][ceil(N/32)]).  to_rows = true: lane-major -> rows.
+cudaError_t launch_bitmap_layout(const uint32_t* src, uint32_t* dst, int64_t nq,
+                                 int64_t n_blocks, int64_t n_words_rows, bool to_rows,
+                                 cudaStream_t s);
+
+// fingerprint + alpha (when bank != nullptr) and w_f
+cudaError_t launch_condition(const float* q, const ifvs_predicate* preds, int64_t nq, int D,
+                             const uint64_t* seeds, int h, int64_t B, const float* bank, int Mr,
+                             const float* wz, uint32_t* idx, float* alpha, float* wf,
+                             cudaStream_t s);
+
+// Delta, C_iFVS (optional output) and the weighted ADC tables
+cudaError_t launch_lut(const float* cpq, const float* W, const float* alpha, const float* q,
+                       const float* wf, int64_t nq, int M, int K, int ds, int r,
+                       float* lut, float* cifvs, int num_sms, cudaStream_t s);
+
+struct ScanShape {
+    int64_t n_blocks;      // bitmap blocks (rows padded to n_blocks * 1024)
+    int M, K;
+    int row_bytes;         // code row stride in bytes (M rounded up to 4)
+    int tab_words;         // LUT table stride in words per codeword
+    int64_t blocks_per_chunk;
+    int n_chunks;
+};
+size_t scan_smem_bytes(int tab_words, int kp);
+int scan_kp(int k);
+// Rank: per (query, chunk) CTA, the k best keys (dist bits << 32 | row) of
+// the chunk's passing rows -> partials [nq][n_chunks][k]
+cudaError_t launch_scan(const uint8_t* codes, const float* lut, const uint32_t* bm, int64_t nq,
+                        int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s);
+// Select: merge [nq][n_lists][k] partial keys -> ids / dists
+cudaError_t launch_merge(const uint64_t* partials, int64_t nq, int n_lists, int k,
+                         int64_t* ids, float* dists, cudaStream_t s);
+// exact fp32 rerank of cand [nq][R] -> k best
+cudaError_t launch_rerank(const float* X, int64_t N, int D, const float* q, const int64_t* cand,
+                          int64_t nq, int R, int k, int64_t* ids, float* dists, cudaStream_t s);
+// codes [N][M] -> rotated rows [n_rows_pad][row_bytes]; *bad = 1 if a code >= K
+cudaError_t launch_relayout_codes(const uint8_t* src, int64_t N, int M, int K, int row_bytes,
+                                  int64_t n_rows_pad, uint8_t* dst, int* bad, cudaStream_t s);
+
+}  // namespace ifvs
