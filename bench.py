@@ -1,0 +1,486 @@
+#!/usr/bin/env python3
+"""Benchmark of the iFVS query path: QPS at recall@k per selectivity bin.
+
+Workload: gmm100m-d128-m16 — 10^8 PQ-coded rows (M = 16 subspaces x 8
+dimensions, K = 256, uint8 codes, 1.6 GB), one int32 attribute uniform in
+[0, 10^6), queries in batches of 1024 with range predicates at 0.1 %, 1 %,
+10 % and 100 % selectivity, k = 100, conditioned codebooks (memory bank
+B = 4096, h = 2, r = 8) and per-query w_z.  A step is one batch of 1024
+queries through the whole path (filter, fingerprint, alpha, w_f, Delta,
+C_iFVS, tables, scan, top-k merge); steps cycle through the four bins.
+
+Printed (rank 0): one JSON line with the value (queries per second over
+all ranks, inputs resident on the device), e2e (the same through the C ABI
+with pinned host buffers), per-bin QPS and recall@k, the scan kernel's
+roofline figures, clocks sampled during the timed region, and the oracle
+timed on host cores as a reported CPU baseline.
+
+``--impl reference`` times the oracle instead (the plain C CPU program of
+the method), on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD = "gmm100m-d128-m16"
+CPU_SAMPLE_ROWS = 10_000_000
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=16)
+    ap.add_argument("--warmup", type=int, default=4)
+    ap.add_argument("--impl", default="ifvs", choices=["ifvs", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--rows", type=int, default=0, help="override N (smaller runs)")
+    ap.add_argument("--recall-queries", type=int, default=16, help="per bin; 0 = skip")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--out", default="", help="also write the JSON line to this file")
+    return ap.parse_args()
+
+
+def workload(args):
+    from paper_2607_22922_gb300 import synth
+    w = synth.WORKLOADS[args.workload]
+    if args.rows:
+        w = synth.scaled(w, N=args.rows)
+    return w
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def dist_init(world, device):
+    if world <= 1:
+        return None
+    import torch
+    import torch.distributed as dist
+    backend = "nccl" if torch.cuda.is_available() else "gloo"
+    kw = {"device_id": device} if backend == "nccl" else {}
+    try:
+        dist.init_process_group(backend=backend, **kw)
+    except TypeError:
+        dist.init_process_group(backend=backend)
+    return dist
+
+
+def reduce_max(dist, x, device):
+    """Max of a float over ranks (identity for one rank)."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist, device=None):
+    if dist is not None:
+        if device is not None and dist.get_backend() == "nccl":
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons (every 200 ms)."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id=None):
+        self.proc = None
+        self.gpu_id = gpu_id
+
+    def start(self):
+        cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+               "-lms", "200"]
+        if self.gpu_id:
+            cmd[1:1] = ["-i", str(self.gpu_id)]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        mhz, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                mhz.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not mhz:
+            return None
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": max(mx),
+                "samples": len(mhz), "reasons": sorted(reasons)}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def scan_traffic():
+    """DRAM bytes per scan launch from the committed ncu summary, valid only
+    while the scan kernel's source is unchanged."""
+    p = os.path.join(ROOT, "profiles", "scan_traffic.json")
+    src = os.path.join(ROOT, "paper_2607_22922_gb300", "csrc", "scan.cu")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    if d.get("scan_cu_sha256") != sha:
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------ CPU baseline
+
+def cpu_baseline(w, ix, cond, batches, max_seconds=30.0):
+    """The oracle as it stands, single-threaded, on one query per bin over the
+    first CPU_SAMPLE_ROWS rows; per-query time scaled by N / rows."""
+    import oracle
+    rows = min(CPU_SAMPLE_ROWS, w.N)
+    codes = ix.codes[:rows]
+    attrs = [a[:rows] for a in ix.attrs]
+    t_total, nq = 0.0, 0
+    for qs in batches:
+        t0 = time.perf_counter()
+        oracle.search(codes, attrs, ix.codebook, qs.q[:1], qs.preds[:1], w.k, bank=cond.bank,
+                      W=cond.W, seeds=cond.seeds, wz=qs.wz[:1])
+        t_total += (time.perf_counter() - t0) * (w.N / rows)
+        nq += 1
+        if t_total > max_seconds * (w.N / rows):
+            break
+    return {"value": nq / t_total, "unit": "queries/s", "cores": 1, "kind": "oracle",
+            "sample": "1 query per selectivity bin (%d bins) over the first %d of %d rows, "
+                      "time scaled by N/rows" % (nq, rows, w.N)}
+
+
+# ------------------------------------------------------------ recall
+
+def recall_at_k(w, ix, batches, ids_by_bin, nsample, device):
+    """recall@k of the returned ids against the exact filtered top-k (§3.1)
+    over the raw vectors, for the first ``nsample`` queries of each bin."""
+    import torch
+    from paper_2607_22922_gb300 import synth
+    block = 1 << 22
+    cb = torch.from_numpy(ix.codebook).to(device)
+    attr = ix.attrs[0]
+    qs_all = torch.cat([torch.from_numpy(b.q[:nsample]) for b in batches]).to(device).double()
+    lo = np.concatenate([b.preds["c"][:nsample, 0]["lo"] for b in batches])
+    hi = np.concatenate([b.preds["c"][:nsample, 0]["hi"] for b in batches])
+    nq = qs_all.shape[0]
+    best_d = torch.full((nq, w.k), float("inf"), dtype=torch.float64, device=device)
+    best_i = torch.full((nq, w.k), -1, dtype=torch.int64, device=device)
+    lo_t = torch.from_numpy(lo).to(device)
+    hi_t = torch.from_numpy(hi).to(device)
+    qn = (qs_all * qs_all).sum(1, keepdim=True)
+    for s in range(0, w.N, block):
+        e = min(w.N, s + block)
+        x = synth.raw_vectors_torch(ix, s, e, device, cb).double()
+        d = qn + (x * x).sum(1)[None, :] - 2.0 * qs_all @ x.T
+        a = torch.from_numpy(attr[s:e].astype(np.int64)).to(device)
+        ok = (a[None, :] >= lo_t[:, None]) & (a[None, :] < hi_t[:, None])
+        d = torch.where(ok, d, torch.full_like(d, float("inf")))
+        kk = min(w.k, e - s)
+        dv, di = torch.topk(d, kk, dim=1, largest=False)
+        di = di + s
+        cd = torch.cat([best_d, dv], 1)
+        ci = torch.cat([best_i, di], 1)
+        o = torch.argsort(cd, dim=1, stable=True)[:, :w.k]
+        best_d = torch.gather(cd, 1, o)
+        best_i = torch.gather(ci, 1, o)
+        best_i = torch.where(torch.isinf(best_d), torch.full_like(best_i, -1), best_i)
+    gt = best_i.cpu().numpy()
+    out = {}
+    for b, (qs, ids) in enumerate(zip(batches, ids_by_bin)):
+        r = []
+        for i in range(nsample):
+            g = gt[b * nsample + i]
+            valid = g[g >= 0]
+            if len(valid) == 0:
+                continue
+            r.append(len(np.intersect1d(valid, ids[i])) / len(valid))
+        out[qs.sel] = float(np.mean(r)) if r else None
+    return out
+
+
+# ------------------------------------------------------------ arms
+
+def run_ifvs(args):
+    import torch
+    world, rank, local = dist_env()
+    if not torch.cuda.is_available():
+        raise SystemExit("no CUDA device: the benchmark needs a GPU")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    dist = dist_init(world, device)
+    from paper_2607_22922_gb300 import build, synth
+    if rank == 0 or world == 1:
+        build.build()
+    barrier(dist, device)
+    build.build()
+    from paper_2607_22922_gb300 import ifvs
+
+    w = workload(args)
+    t0 = time.time()
+    ix = synth.make_index(w)
+    cond = synth.make_conditioning(ix)
+    batches = [synth.make_queries(ix, s, nq=w.batch, salt=rank) for s in w.sels]
+    t_gen = time.time() - t0
+    g = ifvs.Index(ix.codes, ix.attrs, device=local)
+    g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
+
+    stream = torch.cuda.Stream(device=device)
+    sptr = stream.cuda_stream
+    nb = len(batches)
+    dev_in, dev_out = [], []
+    for qs in batches:
+        dev_in.append((torch.from_numpy(qs.q).to(device),
+                       torch.from_numpy(qs.preds.view(np.uint8).copy()).to(device),
+                       torch.from_numpy(qs.wz).to(device)))
+        n = len(qs.q)
+        dev_out.append((torch.empty((n, w.k), dtype=torch.int64, device=device),
+                        torch.empty((n, w.k), dtype=torch.float32, device=device),
+                        torch.empty(n, dtype=torch.int64, device=device)))
+    torch.cuda.synchronize()
+    flags = ifvs.IFVS_F_DEVICE_IO | ifvs.IFVS_F_STAGE_TIMING
+
+    def step(i):
+        b = i % nb
+        q, p, wz = dev_in[b]
+        oi, od, on = dev_out[b]
+        ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on,
+                               flags=flags, stream=sptr)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    g.stage_times(reset=True)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    gpu_uuid = None
+    try:
+        gpu_uuid = torch.cuda.get_device_properties(device).uuid
+        gpu_uuid = "GPU-" + str(gpu_uuid) if gpu_uuid is not None else None
+    except Exception:
+        gpu_uuid = None
+    clocks = Clocks(gpu_uuid)
+    barrier(dist, device)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    with torch.cuda.stream(stream):
+        ev[0].record(stream)
+        for i in range(args.steps):
+            step(args.warmup + i)
+            ev[i + 1].record(stream)
+    torch.cuda.synchronize()
+    barrier(dist, device)
+    clk = clocks.stop()
+    step_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)]
+    total_ms = ev[0].elapsed_time(ev[-1])
+    max_ms = reduce_max(dist, total_ms, device)
+    stages = g.stage_times(reset=True)
+    launches = sum(v[1] for v in stages.values())
+
+    # per-bin figures and the scan roofline (algorithmic bytes: passing rows'
+    # codes + the bin's lane-major bitmap, per query)
+    per_bin = {}
+    n_blocks = (w.N + 1023) // 1024
+    scan_bytes = 0.0
+    for b, qs in enumerate(batches):
+        ms_b = [step_ms[i] for i in range(args.steps) if (args.warmup + i) % nb == b]
+        npass = dev_out[b][2].cpu().numpy()
+        nsteps_b = len(ms_b)
+        scan_bytes += nsteps_b * float((npass * w.M).sum() + len(npass) * n_blocks * 128)
+        per_bin[str(qs.sel)] = {
+            "qps": (len(qs.q) * nsteps_b) / (sum(ms_b) / 1000.0) if ms_b else None,
+            "ms_per_batch": float(np.mean(ms_b)) if ms_b else None,
+            "mean_selectivity": float(npass.mean() / w.N)}
+    scan_ms, scan_n = stages["scan"]
+    hbm_peak, peak_kind = measured_peaks()
+    achieved = (scan_bytes / scan_n) / (scan_ms / scan_n / 1000.0) / 1e9 if scan_n else None
+    traffic = scan_traffic()
+    roofline = {"kernel": "k_scan", "bound": "hbm", "achieved": achieved, "peak": hbm_peak,
+                "unit": "GB/s", "frac": achieved / hbm_peak if achieved else None,
+                "traffic": traffic, "peak_kind": peak_kind + " (hbm copy, burst)",
+                "avg_launch_ms": scan_ms / scan_n if scan_n else None,
+                "algorithmic_bytes_per_launch": scan_bytes / scan_n if scan_n else None}
+    share = {k: v[0] for k, v in stages.items()}
+
+    # end to end through the C ABI with pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        host_in, host_out = [], []
+        for qs in batches:
+            n = len(qs.q)
+            hq = torch.from_numpy(qs.q).pin_memory()
+            hp = torch.from_numpy(qs.preds.view(np.uint8).copy()).pin_memory()
+            hw = torch.from_numpy(qs.wz).pin_memory()
+            host_in.append((hq.numpy(), hp.numpy().view(synth.PREDICATE_DTYPE), hw.numpy(), (hq, hp, hw)))
+            ho = (torch.empty((n, w.k), dtype=torch.int64).pin_memory(),
+                  torch.empty((n, w.k), dtype=torch.float32).pin_memory(),
+                  torch.empty(n, dtype=torch.int64).pin_memory())
+            host_out.append((ho[0].numpy(), ho[1].numpy(), ho[2].numpy(), ho))
+
+        def hstep(i):
+            b = i % nb
+            q, p, wz, _ = host_in[b]
+            oi, od, on, _ = host_out[b]
+            ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr)
+
+        for i in range(args.warmup):
+            hstep(i)
+        barrier(dist, device)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            hstep(args.warmup + i)
+        torch.cuda.synchronize()
+        e_ms = (time.perf_counter() - t0) * 1000.0
+        barrier(dist, device)
+        e_ms = reduce_max(dist, e_ms, device)
+        nq_b = w.batch
+        e2e = {"value": world * args.steps * nq_b / (e_ms / 1000.0), "unit": "queries/s",
+               "h2d_bytes_per_step": nq_b * (w.D * 4 * 2 + 104),
+               "d2h_bytes_per_step": nq_b * (w.k * 12 + 8)}
+
+    # recall@k (outside the timed regions)
+    recall = None
+    if args.recall_queries > 0 and rank == 0:
+        ids_by_bin = [dev_out[b][0].cpu().numpy()[:args.recall_queries] for b in range(nb)]
+        recall = recall_at_k(w, ix, batches, ids_by_bin, args.recall_queries, device)
+        for s, r in recall.items():
+            per_bin[str(s)]["recall@%d" % w.k] = r
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, ix, cond, batches)
+
+    value = world * args.steps * w.batch / (max_ms / 1000.0)
+    line = {
+        "metric": "QPS at recall@%d per selectivity bin (code-scan HBM GB/s vs peak)" % w.k,
+        "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": max_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32 (uint8 codes)",
+        "data": "synthetic (seeded Gaussian-mixture PQ index; paper datasets and trained weights absent)",
+        "config": {"workload": w.name, "N": w.N, "D": w.D, "M": w.M, "K": w.K, "k": w.k,
+                   "batch": w.batch, "bins": list(w.sels), "B": w.B, "h": w.h, "r": w.r,
+                   "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (%.1f GB codes + %.1f GB attributes)"
+                         % (w.N * w.M / 1e9, w.N * 4 / 1e9)},
+        "bins": per_bin, "roofline": roofline, "stage_ms": share, "gpu_launches": launches,
+        "clocks": clk, "e2e": e2e, "cpu_baseline": cpu, "setup_s": round(t_gen, 1),
+    }
+    if rank == 0:
+        s = json.dumps(line)
+        print(s, flush=True)
+        if args.out:
+            with open(args.out, "w") as f:
+                f.write(s + "\n")
+    g.close()
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    """The oracle as it stands on the host cores, each step one query of the
+    next bin over the first CPU_SAMPLE_ROWS rows, time scaled by N / rows."""
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2607_22922_gb300 import synth
+    import oracle
+    oracle.build()
+    w = workload(args)
+    rows = min(CPU_SAMPLE_ROWS, w.N)
+    ws = synth.scaled(w, N=rows)        # the same rows as the first `rows` of the workload
+    ix = synth.make_index(ws)
+    cond = synth.make_conditioning(ix)
+    batches = [synth.make_queries(ix, s, nq=8) for s in w.sels]
+    scale = w.N / rows
+
+    def step(i):
+        qs = batches[i % len(batches)]
+        j = (i // len(batches)) % len(qs.q)
+        oracle.search(ix.codes, ix.attrs, ix.codebook, qs.q[j:j + 1], qs.preds[j:j + 1], w.k,
+                      bank=cond.bank, W=cond.W, seeds=cond.seeds, wz=qs.wz[j:j + 1])
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(args.warmup + i)
+    sec = (time.perf_counter() - t0) * scale
+    value = args.steps / sec
+    sample = ("1 query per step cycling through the %d bins, over the first %d of %d rows; "
+              "time scaled by N/rows" % (len(batches), rows, w.N))
+    line = {
+        "impl": "reference",
+        "metric": "QPS at recall@%d per selectivity bin (code-scan HBM GB/s vs peak)" % w.k,
+        "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": sec * 1000.0 / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": w.name, "N": w.N, "k": w.k,
+                                        "batch": 1, "bins": list(w.sels)},
+        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ifvs(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -146,15 +146,23 @@ def ifvs_load_index(codes, attrs, vectors=None, D=0, device=0, K=256, device_io=
 
 
 def ifvs_load_codebooks(ix, C_pq, bank=None, h=0, r=0, W=None, hash_seeds=None):
+    info = ifvs_index_info(ix)
     C_pq = _host(C_pq, np.float32)
     M, K, ds = C_pq.shape
+    if (M, K) != (info["M"], info["K"]):
+        raise ValueError("C_pq is %s; the index has M = %d, K = %d" % (C_pq.shape, info["M"], info["K"]))
     bank = _host(bank, np.float32)
     W = _host(W, np.float32)
     seeds = _host(hash_seeds, np.uint64)
     B = 0 if bank is None else bank.shape[0]
     if bank is not None:
+        if W is None or seeds is None:
+            raise ValueError("W and hash_seeds are required with a bank")
         h = len(seeds)
         r = W.shape[1]
+        if W.shape != (M, r, K, ds) or bank.ndim != 2 or bank.shape[1] != M * r:
+            raise ValueError("bank %s / W %s do not match M = %d, K = %d, ds = %d"
+                             % (bank.shape, W.shape, M, K, ds))
     _check(_lib.ifvs_load_codebooks(ix, _ptr(C_pq), ds, _ptr(bank), B, h, r, _ptr(W), _ptr(seeds)))
 
 

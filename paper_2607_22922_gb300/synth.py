@@ -217,6 +217,35 @@ def raw_vectors(ix: Index, start: int = 0, stop: int | None = None) -> np.ndarra
     return out
 
 
+def raw_vectors_torch(ix: Index, start: int, stop: int, device, codebook_t=None):
+    """Raw vectors of rows [start, stop) drawn on a torch device: the same
+    recipe as ``raw_vectors`` (reconstruction + residual noise) with torch's
+    generator, seeded per 2^22-row block, for datasets too large for the host.
+    Rows must not straddle a block boundary (callers walk whole blocks)."""
+    import torch
+    w = ix.w
+    block = 1 << 22
+    if start // block != (stop - 1) // block:
+        raise ValueError("rows must lie in one 2^22-row block")
+    cb = codebook_t if codebook_t is not None else torch.from_numpy(ix.codebook).to(device)
+    codes = torch.from_numpy(ix.codes[start:stop]).to(device).long()
+    m = torch.arange(w.M, device=device)[None, :]
+    rec = cb[m, codes].reshape(stop - start, w.D)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(w.seed) * 1_000_003 + start // block)
+    noise = torch.randn((block, w.D), generator=gen, device=device, dtype=torch.float32)
+    off = start % block
+    x = rec + ix.noise_sigma * noise[off:off + (stop - start)]
+    if w.kind == "sift":
+        x = torch.clamp(torch.round(x), 0.0, 255.0)
+    elif w.kind == "gist":
+        x = x.abs()
+        x = x / x.norm(dim=1, keepdim=True).clamp_min(1e-12)
+    elif w.kind == "deep":
+        x = x / x.norm(dim=1, keepdim=True).clamp_min(1e-12)
+    return x
+
+
 # ---------------------------------------------------------------- queries
 
 @dataclasses.dataclass

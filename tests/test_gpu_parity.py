@@ -134,7 +134,7 @@ def _small(ifvs, N, M=16, K=256, ds=2, seed=0, attrs=None, dup_rows=False, vecto
         attrs = [rng.integers(0, 100, N).astype(np.int32)]
     Cpq = rng.standard_normal((M, K, ds)).astype(np.float32)
     X = rng.standard_normal((N, M * ds)).astype(np.float32) if vectors else None
-    g = ifvs.Index(codes, attrs, vectors=X, D=M * ds)
+    g = ifvs.Index(codes, attrs, vectors=X, D=M * ds, K=K)
     g.load_codebooks(Cpq)
     return g, codes, attrs, Cpq, X
 
