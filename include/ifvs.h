@@ -209,6 +209,31 @@ int ifvs_scan_topk(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, in
                    int32_t k, const ifvs_search_params* p, int64_t* ids, float* dists);
 
 /*
+ * ifvs_scan_topk_static — ifvs_scan_topk without any device allocation.
+ * The paper has no counterpart: this entry point exists for callers that
+ * must not allocate device memory while serving queries — code whose device
+ * memory belongs to another allocator (a framework's caching pool), or
+ * latency-critical loops that allocate nothing after start-up, because
+ * cudaMalloc / cudaFree can synchronise the whole device.
+ *   lut, bitmaps, ids, dists  device pointers, shapes as for ifvs_scan_topk
+ *   stream                    cudaStream_t to enqueue on (NULL: legacy stream)
+ * The call only enqueues work on `stream` and returns; results are ready
+ * when the stream reaches them.  Its scratch is a file-scope device array of
+ * IFVS_STATIC_SCRATCH_BYTES that every GPU running the library holds until
+ * the process exits; queries are processed in sub-batches that fit it.
+ * Sizes beyond it (one query's lane-major bitmap, N / 8 bytes rounded up to
+ * 128-byte blocks, plus k keys, above the array) return
+ * IFVS_ERR_UNSUPPORTED.  The first call on a device looks up the array's
+ * device address (cudaGetSymbolAddress); make that first call before any
+ * stream capture.  All calls share the array: calls whose work overlaps on
+ * the GPU (different streams, or threads without ordering) race.  No
+ * cudaMalloc, cudaFree or allocating library routine is called.
+ */
+#define IFVS_STATIC_SCRATCH_BYTES (32u << 20)
+int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, int64_t nq,
+                          int32_t k, void* stream, int64_t* ids, float* dists);
+
+/*
  * ifvs_rerank — exact fp32 L2 (the Pre_IndexFlatL2 distance of §3.2) of
  * candidate rows, then the k best by (dist, id).
  *   cand  [nq][R] int64 candidate row ids; -1 entries are skipped

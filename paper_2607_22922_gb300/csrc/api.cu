@@ -413,6 +413,30 @@ int reset_err_flag(ifvs_index* ix, cudaStream_t s) {
 
 }  // namespace
 
+// ============================================================== internal
+
+int ifvs::index_view(const ifvs_index* ix, IndexView* out) {
+    if (!ix) return set_err(IFVS_ERR_ARG, "index is NULL");
+    out->device = ix->device;
+    out->num_sms = ix->num_sms;
+    out->N = ix->N;
+    out->n_blocks = ix->n_blocks;
+    out->M = ix->M;
+    out->K = ix->K;
+    out->row_bytes = ix->row_bytes;
+    out->tab_words = ix->tab_words;
+    out->codes = ix->d_codes;
+    return 0;
+}
+
+int ifvs::report_error(int code, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
 // ============================================================== C ABI
 
 extern "C" {

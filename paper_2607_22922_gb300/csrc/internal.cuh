@@ -146,4 +146,16 @@ cudaError_t launch_rerank(const float* X, int64_t N, int D, const float* q, cons
 cudaError_t launch_relayout_codes(const uint8_t* src, int64_t N, int M, int K, int row_bytes,
                                   int64_t n_rows_pad, uint8_t* dst, int* bad, cudaStream_t s);
 
+// Read-only view of a loaded index, for entry points defined outside api.cu.
+struct IndexView {
+    int device;
+    int num_sms;
+    int64_t N, n_blocks;
+    int M, K, row_bytes, tab_words;
+    const uint8_t* codes;
+};
+int index_view(const ifvs_index* ix, IndexView* out);
+// Sets the thread-local message of ifvs_last_error and returns `code`.
+int report_error(int code, const char* fmt, ...);
+
 }  // namespace ifvs

@@ -53,6 +53,7 @@ def _load():
         "ifvs_condition": (C.c_int, [P, P, P, I64, P, P, P, P, P, P, P]),
         "ifvs_scan_topk": (C.c_int, [P, P, P, I64, I32, P, P, P]),
         "ifvs_rerank": (C.c_int, [P, P, P, I64, I32, I32, P, P, P]),
+        "ifvs_scan_topk_static": (C.c_int, [P, P, P, I64, I32, P, P, P]),
         "ifvs_stage_times": (C.c_int, [P, P, P, I32]),
         "ifvs_canonical_predicate": (C.c_int, [P, P, I32, P, P, P]),
         "ifvs_index_info": (C.c_int, [P, P]),
@@ -226,6 +227,16 @@ def ifvs_scan_topk(ix, lut, bitmaps, k, flags=0, sub_batch=0):
     p = _params(flags, 0, sub_batch)
     _check(_lib.ifvs_scan_topk(ix, _ptr(lut), _ptr(bitmaps), nq, k, C.byref(p), _ptr(ids),
                                _ptr(dists)))
+    return ids, dists
+
+
+def ifvs_scan_topk_static(ix, lut, bitmaps, k, ids, dists, stream=None):
+    """Device tensors only (lut [nq][M][K] float32, bitmaps [nq][ceil(N/32)]
+    uint32, ids [nq][k] int64, dists [nq][k] float32); enqueues on ``stream``
+    and returns without synchronising.  Uses no device allocation."""
+    nq = int(lut.shape[0])
+    _check(_lib.ifvs_scan_topk_static(ix, _ptr(lut), _ptr(bitmaps), nq, k, stream, _ptr(ids),
+                                      _ptr(dists)))
     return ids, dists
 
 
