@@ -50,6 +50,7 @@ def parse():
     ap.add_argument("--recall-queries", type=int, default=16, help="per bin; 0 = skip")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--chunk-blocks", type=int, default=0, help="scan chunk size in 1024-row blocks (0 = auto)")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
     return ap.parse_args()
 
@@ -294,7 +295,7 @@ def run_ifvs(args):
         q, p, wz = dev_in[b]
         oi, od, on = dev_out[b]
         ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on,
-                               flags=flags, stream=sptr)
+                               flags=flags, stream=sptr, chunk_blocks=args.chunk_blocks)
 
     for i in range(args.warmup):
         step(i)
@@ -370,7 +371,8 @@ def run_ifvs(args):
             b = i % nb
             q, p, wz, _ = host_in[b]
             oi, od, on, _ = host_out[b]
-            ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr)
+            ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr,
+                                   chunk_blocks=args.chunk_blocks)
 
         for i in range(args.warmup):
             hstep(i)

@@ -97,7 +97,9 @@ typedef struct {
     int32_t sub_batch;  /* queries per filter/scan pass; bounds the bitmap
                            workspace to sub_batch * ceil(N/1024) * 128 bytes.
                            0: automatic (at most 1024).                        */
-    int32_t reserved;   /* must be 0 */
+    int32_t chunk_blocks; /* rows per scan CTA in units of 1024 (0: automatic);
+                           a tuning knob: CTAs of different queries that walk
+                           the same chunk together share its codes in L2     */
     void* stream;       /* cudaStream_t to run on; NULL: the index's stream   */
 } ifvs_search_params;
 
@@ -222,7 +224,8 @@ int ifvs_scan_topk(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, in
  * IFVS_STATIC_SCRATCH_BYTES that every GPU running the library holds until
  * the process exits; queries are processed in sub-batches that fit it.
  * Sizes beyond it (one query's lane-major bitmap, N / 8 bytes rounded up to
- * 128-byte blocks, plus k keys, above the array) return
+ * 128-byte blocks, plus its 64 KB scan table (160 KB for M > 33) and k keys,
+ * above the array) return
  * IFVS_ERR_UNSUPPORTED.  The first call on a device looks up the array's
  * device address (cudaGetSymbolAddress); make that first call before any
  * stream capture.  All calls share the array: calls whose work overlaps on

@@ -110,7 +110,7 @@ struct ifvs_index {
     size_t bytes = 0;
     // workspace
     DevBuf w_q, w_wz, w_preds, w_canon, w_err, w_bm, w_rows, w_npass, w_idx, w_alpha, w_wf,
-        w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist;
+        w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist, w_tab;
     // timing
     double stage_ms[IFVS_N_STAGES] = {0};
     int64_t stage_launches[IFVS_N_STAGES] = {0};
@@ -163,7 +163,7 @@ void free_index(ifvs_index* ix) {
     DevBuf* bufs[] = {&ix->w_q, &ix->w_wz, &ix->w_preds, &ix->w_canon, &ix->w_err, &ix->w_bm,
                       &ix->w_rows, &ix->w_npass, &ix->w_idx, &ix->w_alpha, &ix->w_wf,
                       &ix->w_lut, &ix->w_cifvs, &ix->w_part, &ix->w_ids, &ix->w_dists,
-                      &ix->w_cand, &ix->w_cdist};
+                      &ix->w_cand, &ix->w_cdist, &ix->w_tab};
     for (DevBuf* b : bufs) release(*b);
     for (auto& pr : ix->pending) {
         ix->ev_free.push_back(pr.second.first);
@@ -219,6 +219,7 @@ struct Opts {
     bool dio = false, timing = false, plain = false;
     int R = 0;
     int64_t sub_batch = 0;
+    int64_t chunk_blocks = 0;
     cudaStream_t stream = nullptr;
 };
 
@@ -226,7 +227,7 @@ int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (!p) return 0;
     if (p->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING | IFVS_F_PLAIN_PQ))
         return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", p->flags);
-    if (p->reserved != 0) return set_err(IFVS_ERR_ARG, "ifvs_search_params.reserved must be 0");
+    if (p->chunk_blocks < 0) return set_err(IFVS_ERR_ARG, "chunk_blocks must be >= 0");
     if (p->rerank < 0 || p->rerank > IFVS_MAX_K)
         return set_err(IFVS_ERR_ARG, "rerank depth %d outside 0..%d", p->rerank, IFVS_MAX_K);
     if (p->sub_batch < 0) return set_err(IFVS_ERR_ARG, "sub_batch must be >= 0");
@@ -235,6 +236,7 @@ int parse_opts(const ifvs_search_params* p, Opts* o) {
     o->plain = p->flags & IFVS_F_PLAIN_PQ;
     o->R = p->rerank;
     o->sub_batch = p->sub_batch;
+    o->chunk_blocks = p->chunk_blocks;
     o->stream = reinterpret_cast<cudaStream_t>(p->stream);
     return 0;
 }
@@ -249,19 +251,20 @@ int64_t pick_sub_batch(const ifvs_index* ix, const Opts& o, int64_t nq) {
     return sb < nq ? sb : nq;
 }
 
-ScanShape scan_shape(const ifvs_index* ix, int64_t n, int kk) {
+ScanShape scan_shape(const ifvs_index* ix, int64_t n, int kk, int64_t chunk_blocks) {
     ScanShape sh;
     sh.n_blocks = ix->n_blocks;
     sh.M = ix->M;
     sh.K = ix->K;
     sh.row_bytes = ix->row_bytes;
     sh.tab_words = ix->tab_words;
-    const size_t smem = scan_smem_bytes(ix->tab_words, scan_kp(kk));
-    int64_t per_sm = (int64_t)(ix->max_smem > 0 ? 233472 : 233472) / (int64_t)(smem + 1024);
-    if (per_sm < 1) per_sm = 1;
-    if (per_sm > 2) per_sm = 2;  // launch bound of the scan kernel
-    const int64_t resident = (int64_t)ix->num_sms * per_sm;
+    const int64_t resident = (int64_t)ix->num_sms * scan_ctas_per_sm(ix->tab_words, scan_kp(kk));
     int64_t chunks = (resident * 8 + n - 1) / n;
+    // the CTAs that walk a chunk together share it through L2: keep a
+    // chunk's codes within about the L2 size (128 MB)
+    const int64_t l2_blocks = ((int64_t)128 << 20) / ((int64_t)kBlockRows * ix->row_bytes);
+    const int64_t by_l2 = (ix->n_blocks + l2_blocks - 1) / l2_blocks;
+    if (chunks < by_l2) chunks = by_l2;
     int64_t max_chunks = ix->n_blocks / 16;
     if (max_chunks < 1) max_chunks = 1;
     const int64_t key_cap = 32768 / kk;  // bounds the merge's input per query
@@ -269,6 +272,10 @@ ScanShape scan_shape(const ifvs_index* ix, int64_t n, int kk) {
     if (max_chunks > 65535) max_chunks = 65535;
     if (chunks > max_chunks) chunks = max_chunks;
     if (chunks < 1) chunks = 1;
+    if (chunk_blocks > 0) {
+        chunks = (ix->n_blocks + chunk_blocks - 1) / chunk_blocks;
+        if (chunks > 65535) chunks = 65535;
+    }
     sh.blocks_per_chunk = (ix->n_blocks + chunks - 1) / chunks;
     sh.n_chunks = (int)((ix->n_blocks + sh.blocks_per_chunk - 1) / sh.blocks_per_chunk);
     return sh;
@@ -289,7 +296,8 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
     TRY(ensure(ix->w_alpha, sizeof(float) * n * (Mr > 0 ? Mr : 1)));
     TRY(ensure(ix->w_wf, sizeof(float) * n * ix->D));
     TRY(ensure(ix->w_lut, sizeof(float) * n * ix->M * ix->K));
-    const ScanShape sh = scan_shape(ix, n, kk);
+    TRY(ensure(ix->w_tab, sizeof(float) * n * 256 * ix->tab_words));
+    const ScanShape sh = scan_shape(ix, n, kk, o.chunk_blocks);
     TRY(ensure(ix->w_part, sizeof(uint64_t) * n * sh.n_chunks * kk));
     if (o.R > 0) {
         TRY(ensure(ix->w_cand, sizeof(int64_t) * n * kk));
@@ -320,8 +328,13 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
                                    ix->w_lut.as<float>(), nullptr, ix->num_sms, s)));
     }
     {
+        Stage st(ix, s, o.timing, IFVS_STAGE_LUT);
+        CUDA_TRY(st.end(launch_tables(ix->w_lut.as<float>(), n, ix->M, ix->K, ix->tab_words,
+                                      ix->w_tab.as<float>(), s)));
+    }
+    {
         Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
-        CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_lut.as<float>(), ix->w_bm.as<uint32_t>(), n,
+        CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_tab.as<float>(), ix->w_bm.as<uint32_t>(), n,
                                     kk, sh, ix->w_part.as<uint64_t>(), s)));
     }
     int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;
@@ -335,6 +348,17 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
         CUDA_TRY(st.end(launch_rerank(ix->d_vec, ix->N, ix->D, dq, m_ids, n, o.R, k, out_ids,
                                       out_dists, s)));
     }
+    return 0;
+}
+
+// The scan keeps the table and per-warp lists of the next power of two >= k
+// in shared memory; large M leaves room for smaller k only.
+int check_scan_fits(const ifvs_index* ix, int kk) {
+    const size_t need = scan_smem_bytes(ix->tab_words, scan_kp(kk));
+    if (need > (size_t)ix->max_smem)
+        return set_err(IFVS_ERR_UNSUPPORTED,
+                       "k = %d with M = %d needs %zu bytes of shared memory per CTA (device: %d)",
+                       kk, ix->M, need, ix->max_smem);
     return 0;
 }
 
@@ -516,9 +540,9 @@ int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int6
     ix->n_rows_pad = ix->n_blocks * kBlockRows;
     ix->row_bytes = (int)round_up(M, 4);
     ix->tab_words = (int)round_up(M + 31, 32);
-    if (scan_smem_bytes(ix->tab_words, 256) > (size_t)ix->max_smem)
+    if (scan_smem_bytes(ix->tab_words, scan_kp(1)) > (size_t)ix->max_smem)
         return fail(set_err(IFVS_ERR_UNSUPPORTED, "M = %d needs %zu bytes of shared memory (device: %d)",
-                            M, scan_smem_bytes(ix->tab_words, 256), ix->max_smem));
+                            M, scan_smem_bytes(ix->tab_words, scan_kp(1)), ix->max_smem));
     cudaStream_t s = ix->stream;
     const cudaMemcpyKind h2d = dio ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
 
@@ -642,6 +666,7 @@ int ifvs_search_batch(ifvs_index* ix, const float* queries, const ifvs_predicate
     if (k < 1 || k > IFVS_MAX_K) return set_err(IFVS_ERR_ARG, "k = %d outside 1..%d", k, IFVS_MAX_K);
     if (o.R > 0 && o.R < k) return set_err(IFVS_ERR_ARG, "rerank depth %d is below k = %d", o.R, k);
     if (o.R > 0 && !ix->d_vec) return set_err(IFVS_ERR_STATE, "rerank needs raw vectors at load time");
+    TRY(check_scan_fits(ix, o.R > 0 ? o.R : k));
     if (nq == 0) return IFVS_OK;
     if (!queries || !preds || !ids || !dists) return set_err(IFVS_ERR_ARG, "an array argument is NULL");
     DeviceGuard g(ix->device);
@@ -787,6 +812,7 @@ int ifvs_scan_topk(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, in
     TRY(parse_opts(p, &o));
     if (nq < 0) return set_err(IFVS_ERR_ARG, "nq < 0");
     if (k < 1 || k > IFVS_MAX_K) return set_err(IFVS_ERR_ARG, "k = %d outside 1..%d", k, IFVS_MAX_K);
+    TRY(check_scan_fits(ix, k));
     if (nq == 0) return IFVS_OK;
     if (!lut || !bitmaps || !ids || !dists) return set_err(IFVS_ERR_ARG, "an array argument is NULL");
     DeviceGuard g(ix->device);
@@ -816,12 +842,17 @@ int ifvs_scan_topk(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, in
             CUDA_TRY(st.end(launch_bitmap_layout(drows, ix->w_bm.as<uint32_t>(), n, ix->n_blocks, wrows,
                                                  false, s)));
         }
-        const ScanShape sh = scan_shape(ix, n, k);
+        const ScanShape sh = scan_shape(ix, n, k, o.chunk_blocks);
         TRY(ensure(ix->w_part, sizeof(uint64_t) * n * sh.n_chunks * k));
+        TRY(ensure(ix->w_tab, sizeof(float) * n * 256 * ix->tab_words));
+        {
+            Stage st(ix, s, o.timing, IFVS_STAGE_LUT);
+            CUDA_TRY(st.end(launch_tables(dl, n, ix->M, ix->K, ix->tab_words, ix->w_tab.as<float>(), s)));
+        }
         {
             Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
-            CUDA_TRY(st.end(launch_scan(ix->d_codes, dl, ix->w_bm.as<uint32_t>(), n, k, sh,
-                                        ix->w_part.as<uint64_t>(), s)));
+            CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_tab.as<float>(), ix->w_bm.as<uint32_t>(), n, k,
+                                        sh, ix->w_part.as<uint64_t>(), s)));
         }
         int64_t* oid = o.dio ? ids + q0 * k : ix->w_ids.as<int64_t>();
         float* odi = o.dio ? dists + q0 * k : ix->w_dists.as<float>();

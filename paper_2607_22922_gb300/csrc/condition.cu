@@ -199,4 +199,39 @@ cudaError_t launch_lut(const float* cpq, const float* W, const float* alpha, con
     return cudaGetLastError();
 }
 
+// ---- scan tables -------------------------------------------------------------
+//
+// The scan keeps each query's table in shared memory as 256 rows (one per
+// codeword) of S words, word w of row c = LUT[w mod M][c] for w < M + 31
+// (zero above).  This kernel writes that layout once per query so that every
+// scan CTA fetches it with coalesced 16-byte loads.  Grid: query x 32-codeword
+// tile; the tile passes through shared memory padded to 33 words per row so
+// that both the coalesced reads and the rotated writes are conflict-free.
+__global__ void __launch_bounds__(256) k_tables(const float* __restrict__ lut, int M, int K, int S,
+                                                float* __restrict__ tab) {
+    __shared__ float st[IFVS_MAX_M * 33];
+    const int64_t q = blockIdx.x;
+    const int c0 = blockIdx.y * 32;
+    const float* src = lut + q * (int64_t)M * K;
+    for (int i = threadIdx.x; i < M * 32; i += blockDim.x) {
+        const int m = i >> 5, cc = i & 31, c = c0 + cc;
+        st[m * 33 + cc] = c < K ? src[(int64_t)m * K + c] : 0.f;
+    }
+    __syncthreads();
+    float* dst = tab + q * (int64_t)256 * S + (int64_t)c0 * S;
+    const int wu = M + 31;
+    for (int i = threadIdx.x; i < 32 * S; i += blockDim.x) {
+        const int cc = i / S, w = i - cc * S;
+        dst[i] = w < wu ? st[(w % M) * 33 + cc] : 0.f;
+    }
+}
+
+cudaError_t launch_tables(const float* lut, int64_t nq, int M, int K, int S, float* tab,
+                          cudaStream_t s) {
+    if (nq <= 0) return cudaSuccess;
+    dim3 grid((unsigned)nq, 8);
+    k_tables<<<grid, 256, 0, s>>>(lut, M, K, S, tab);
+    return cudaGetLastError();
+}
+
 }  // namespace ifvs

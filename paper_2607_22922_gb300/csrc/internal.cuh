@@ -122,6 +122,11 @@ cudaError_t launch_lut(const float* cpq, const float* W, const float* alpha, con
                        const float* wf, int64_t nq, int M, int K, int ds, int r,
                        float* lut, float* cifvs, int num_sms, cudaStream_t s);
 
+// weighted ADC tables [nq][M][K] -> the scan's shared-memory layout
+// [nq][256][S] (S = tab_words)
+cudaError_t launch_tables(const float* lut, int64_t nq, int M, int K, int S, float* tab,
+                          cudaStream_t s);
+
 struct ScanShape {
     int64_t n_blocks;      // bitmap blocks (rows padded to n_blocks * 1024)
     int M, K;
@@ -131,10 +136,13 @@ struct ScanShape {
     int n_chunks;
 };
 size_t scan_smem_bytes(int tab_words, int kp);
+// CTAs of the scan resident per SM for this table stride and list size
+int scan_ctas_per_sm(int tab_words, int kp);
 int scan_kp(int k);
 // Rank: per (query, chunk) CTA, the k best keys (dist bits << 32 | row) of
-// the chunk's passing rows -> partials [nq][n_chunks][k]
-cudaError_t launch_scan(const uint8_t* codes, const float* lut, const uint32_t* bm, int64_t nq,
+// the chunk's passing rows -> partials [nq][n_chunks][k]; `tab` holds the
+// tables written by launch_tables
+cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm, int64_t nq,
                         int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s);
 // Select: merge [nq][n_lists][k] partial keys -> ids / dists
 cudaError_t launch_merge(const uint64_t* partials, int64_t nq, int n_lists, int k,

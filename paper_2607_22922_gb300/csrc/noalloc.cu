@@ -57,8 +57,11 @@ int scratch_address(int dev, unsigned char** out) {
 // GPU about eight times over, at least 16 blocks per chunk, at most 32768
 // keys per query for the merge).
 int64_t chunks_for(const IndexView& v, int64_t n, int k) {
-    const int64_t resident = (int64_t)v.num_sms * 2;
+    const int64_t resident = (int64_t)v.num_sms * scan_ctas_per_sm(v.tab_words, scan_kp(k));
     int64_t c = (resident * 8 + n - 1) / n;
+    const int64_t l2_blocks = ((int64_t)128 << 20) / ((int64_t)kBlockRows * v.row_bytes);
+    const int64_t by_l2 = (v.n_blocks + l2_blocks - 1) / l2_blocks;
+    if (c < by_l2) c = by_l2;
     int64_t cap = v.n_blocks / 16;
     if (cap < 1) cap = 1;
     if (cap > 32768 / k) cap = 32768 / k > 0 ? 32768 / k : 1;
@@ -70,7 +73,8 @@ int64_t chunks_for(const IndexView& v, int64_t n, int k) {
 
 size_t footprint(const IndexView& v, int64_t n, int64_t chunks, int k) {
     const size_t bm = (size_t)n * v.n_blocks * 128;
-    return bm + (size_t)n * chunks * k * sizeof(uint64_t);
+    const size_t tab = (size_t)n * 256 * v.tab_words * sizeof(float);
+    return bm + tab + (size_t)n * chunks * k * sizeof(uint64_t);
 }
 
 }  // namespace
@@ -88,7 +92,7 @@ extern "C" int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uin
     if (k < 1 || k > IFVS_MAX_K) return report_error(IFVS_ERR_ARG, "k = %d outside 1..%d", k, IFVS_MAX_K);
     if (nq == 0) return IFVS_OK;
     if (!lut || !bitmaps || !ids || !dists) return report_error(IFVS_ERR_ARG, "an array argument is NULL");
-    // one query must fit: its lane-major bitmap and one list of k keys
+    // one query must fit: its lane-major bitmap, its table and one list of k keys
     if (footprint(v, 1, 1, k) > kScratchBytes)
         return report_error(IFVS_ERR_UNSUPPORTED,
                             "N = %lld needs %zu bytes of scratch per query; the static scratch "
@@ -117,7 +121,9 @@ extern "C" int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uin
         int64_t chunks = chunks_for(v, n, k);
         while (chunks > 1 && footprint(v, n, chunks, k) > kScratchBytes) chunks = (chunks + 1) / 2;
         uint32_t* bm = reinterpret_cast<uint32_t*>(base);
-        uint64_t* part = reinterpret_cast<uint64_t*>(base + (size_t)n * v.n_blocks * 128);
+        float* tab = reinterpret_cast<float*>(base + (size_t)n * v.n_blocks * 128);
+        uint64_t* part = reinterpret_cast<uint64_t*>(base + (size_t)n * v.n_blocks * 128 +
+                                                     (size_t)n * 256 * v.tab_words * sizeof(float));
         ScanShape sh;
         sh.n_blocks = v.n_blocks;
         sh.M = v.M;
@@ -127,7 +133,8 @@ extern "C" int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uin
         sh.blocks_per_chunk = (v.n_blocks + chunks - 1) / chunks;
         sh.n_chunks = (int)((v.n_blocks + sh.blocks_per_chunk - 1) / sh.blocks_per_chunk);
         cudaError_t e = launch_bitmap_layout(bitmaps + q0 * wrows, bm, n, v.n_blocks, wrows, false, s);
-        if (e == cudaSuccess) e = launch_scan(v.codes, lut + q0 * lut_n, bm, n, k, sh, part, s);
+        if (e == cudaSuccess) e = launch_tables(lut + q0 * lut_n, n, v.M, v.K, v.tab_words, tab, s);
+        if (e == cudaSuccess) e = launch_scan(v.codes, tab, bm, n, k, sh, part, s);
         if (e == cudaSuccess) e = launch_merge(part, n, sh.n_chunks, k, ids + q0 * k, dists + q0 * k, s);
         if (e != cudaSuccess) {
             cudaGetLastError();

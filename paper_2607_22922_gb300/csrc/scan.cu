@@ -3,36 +3,62 @@
 // form of the printed score), and each CTA keeps the k smallest
 // (dist, row id) of its chunk exactly.
 //
-// Work split: CTA (query q, chunk c) — blockIdx.x runs over queries so that
-// the CTAs resident together share the same code chunk through L2.  Inside
-// a CTA, warp w walks bitmap blocks c0 + w, c0 + w + 8, ...; lane l of a warp
-// owns rows b*1024 + 32*j + l (the lane-major bitmap gives it its 32 pass
-// bits in one load) and reads a row's codes with one 16-byte load (M = 16).
+// Work split.  CTA (query q, chunk c), 16 warps; blockIdx.x runs over the
+// queries so that the CTAs resident together walk the same code chunk and
+// share it through L2.  Warp w of the CTA owns bitmap blocks c0 + w,
+// c0 + w + 16, ...; lane l owns, in each of them, the 32 rows
+// b*1024 + 32*j + l, whose pass bits form its lane-major bitmap word.
 //
-// LUT placement: the scan issues one shared-memory load per code byte, so
-// bank conflicts decide its speed.  The table of query q is stored as 256
-// rows (one per codeword) of S words, S a multiple of 32, word w of row c
-// holding LUT[w mod M][c] for w < M + 31.  Row i's codes are stored rotated
-// by rot(i) = (i mod 32) mod M, so lane l (i = l mod 32) reads at step s the
-// code of subspace (l + s) mod M and finds its entry at word l + s of that
-// codeword's row: bank (l + s) mod 32, distinct across the warp for any
-// codes.  For M = 16 the row stride is 256 bytes and the byte address is
-// formed by one byte permute: code * 256 + 4 * l (+ 4 * s as an immediate).
+// LUT placement.  The scan issues one shared-memory load per code byte, so
+// bank conflicts set its speed.  The table of query q is stored as 256 rows
+// (one per codeword) of S words, S a multiple of 32, word w of row c holding
+// LUT[w mod M][c] for w < M + 31.  Row i's codes are stored rotated by
+// (i mod 32) mod M, so the lane that owns row i (lane i mod 32) reads at
+// step s the code of subspace (l + s) mod M and finds its entry at word
+// l + s of that codeword's row: bank (l + s) mod 32, distinct across the
+// warp whatever the codes.  For M = 16 the row stride is 256 bytes and the
+// address is one byte permute, code * 256 + 4l, with the table base and the
+// step 4s in the load's immediate offset (the table starts the CTA's dynamic
+// shared memory, whose address the kernel checks).
 //
-// Top-k: each warp keeps a sorted list of its KP best keys and a candidate
-// area of KP slots in shared memory; a key (dist bits << 32 | row) enters
-// the area when it is below the warp's current k-th key, and a full area is
-// merged by a warp bitonic sort.  Keys are unique (row ids are), so the
-// result is exact and independent of timing.  At the end warp 0 merges the
-// other warps' lists and writes the CTA's k keys.
+// Compaction.  Each lane visits only its own passing rows, so it keeps its
+// residue class and the conflict-free banks at any selectivity.  The warp's
+// bitmap words sit in a ring of 8 blocks in shared memory (lane l's word in
+// bank l); lanes advance through the ring at their own pace, four rows per
+// round, and the ring is refilled by halves, from words prefetched into
+// registers, once every lane has left the older half.  When every lane
+// holds a full word of the same block the warp takes the block in lockstep
+// without per-row bit handling.
+//
+// Top-k.  Each warp keeps a sorted list of its KP best keys and a candidate
+// area of KP slots; a key (dist bits << 32 | row) enters the area when it
+// is below the warp's current k-th key, and a full area is merged by a warp
+// bitonic sort.  Keys are unique (row ids are), so the result is exact and
+// independent of scheduling.  At the end warp 0 merges the other warps'
+// lists and writes the CTA's k keys.
 #include "internal.cuh"
 
 namespace ifvs {
 
+constexpr int kScanWarps = 16;
+constexpr int kScanThreads = kScanWarps * 32;
+constexpr int kRing = 8;          // bitmap words per lane in the ring
+constexpr int kHalf = kRing / 2;
+constexpr int kU = 4;             // rows per lane per round
+
 int scan_kp(int k) { return k <= 32 ? 32 : (k <= 64 ? 64 : (k <= 128 ? 128 : 256)); }
 
 size_t scan_smem_bytes(int tab_words, int kp) {
-    return (size_t)256 * tab_words * 4 + (size_t)kWarps * 2 * kp * 8;
+    return (size_t)256 * tab_words * 4 + (size_t)kScanWarps * 2 * kp * 8 +
+           (size_t)kScanWarps * kRing * 32 * 4;
+}
+
+int scan_ctas_per_sm(int tab_words, int kp) {
+    const size_t per_cta = scan_smem_bytes(tab_words, kp) + 1024;
+    const int by_smem = (int)((size_t)233472 / per_cta);
+    const int by_threads = 2048 / kScanThreads;
+    int n = by_smem < by_threads ? by_smem : by_threads;
+    return n < 1 ? 1 : n;
 }
 
 __device__ __forceinline__ void warp_sort(uint64_t* a, int n, int lane) {
@@ -87,52 +113,272 @@ struct WarpTopK {
     }
 };
 
-__device__ __forceinline__ uint4 ldg_nc_v4(const uint8_t* p) {
+// L2 policies: code rows are read by every query of a batch (keep them, so
+// the CTAs that walk the same chunk share them); bitmap words are read once.
+__device__ __forceinline__ uint64_t policy_evict_last() {
+    uint64_t pol;
+    asm("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+__device__ __forceinline__ uint4 ldg_nc_v4(const uint8_t* p, uint64_t pol) {
     uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+    asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
+                 : "l"(p), "l"(pol));
     return v;
 }
 
-// 16 look-ups of one M = 16 row (row stride of the table: 256 bytes)
-__device__ __forceinline__ float lookup16(const uint4 c, const char* tab, uint32_t lane4) {
-    const uint32_t w[4] = {c.x, c.y, c.z, c.w};
-    float acc0 = 0.f, acc1 = 0.f;
-#pragma unroll
-    for (int s = 0; s < 16; ++s) {
-        // bytes: [4*lane, code, 0, 0] -> code * 256 + 4 * lane
-        const uint32_t off = __byte_perm(w[s >> 2], lane4, 0x5504u | ((uint32_t)(s & 3) << 4));
-        const float v = *reinterpret_cast<const float*>(tab + off + 4 * s);
-        if (s & 1) acc1 += v; else acc0 += v;
-    }
-    return acc0 + acc1;
+__device__ __forceinline__ uint32_t ldg_nc_u32(const uint32_t* p, uint64_t pol) {
+    uint32_t v;
+    asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.u32 %0, [%1], %2;"
+                 : "=r"(v) : "l"(p), "l"(pol));
+    return v;
 }
 
-constexpr int kU = 4;   // rows per lane in flight
+template <int IMM>
+__device__ __forceinline__ float lds_imm(uint32_t addr) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1+%2];" : "=f"(v) : "r"(addr), "n"(IMM));
+    return v;
+}
 
-template <int KP, bool M16>
-__global__ void __launch_bounds__(kThreads, 2)
-k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ luts,
-       const uint32_t* __restrict__ bm, int64_t nq, int k, ScanShape sh,
-       uint64_t* __restrict__ partials) {
-    extern __shared__ __align__(16) uint8_t smem[];
+// Two packed fp32 additions at once (Blackwell f32x2 pipe).
+__device__ __forceinline__ uint64_t add_f32x2(uint64_t acc, float a, float b) {
+    uint64_t r;
+    asm("{\n\t.reg .b64 t;\n\tmov.b64 t, {%1, %2};\n\tadd.rn.f32x2 %0, %3, t;\n\t}"
+        : "=l"(r) : "f"(a), "f"(b), "l"(acc));
+    return r;
+}
+
+__device__ __forceinline__ void unpack_f32x2(uint64_t v, float& a, float& b) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+
+// Shared address at which the dynamic shared memory of a CTA begins on this
+// architecture (after the 1 KB the hardware reserves); the kernel checks it.
+constexpr uint32_t kDynSmemBase = 0x400u;
+
+// Distances of two M = 16 rows (codes ca, cb).  One byte permute forms
+// code * 256 + 4 * lane; FAST (table at kDynSmemBase): the table base and
+// the step go into the load's immediate offset; otherwise the base is added.
+template <bool FAST>
+__device__ __forceinline__ void lookup16x2(const uint4 ca, const uint4 cb, uint32_t tb,
+                                           uint32_t base, float& da, float& db) {
+    const uint32_t wa[4] = {ca.x, ca.y, ca.z, ca.w};
+    const uint32_t wb[4] = {cb.x, cb.y, cb.z, cb.w};
+    uint64_t acc = 0ull;
+#pragma unroll
+    for (int s = 0; s < 16; ++s) {
+        const uint32_t sel = 0x5504u | ((uint32_t)(s & 3) << 4);
+        uint32_t oa = __byte_perm(wa[s >> 2], tb, sel);
+        uint32_t ob = __byte_perm(wb[s >> 2], tb, sel);
+        if (!FAST) {
+            oa += base;
+            ob += base;
+        }
+        constexpr uint32_t B0 = FAST ? kDynSmemBase : 0u;
+        float va, vb;
+        switch (s) {
+#define IFVS_LDS_CASE(S)                  \
+    case S:                               \
+        va = lds_imm<B0 + 4 * S>(oa);     \
+        vb = lds_imm<B0 + 4 * S>(ob);     \
+        break;
+            IFVS_LDS_CASE(0) IFVS_LDS_CASE(1) IFVS_LDS_CASE(2) IFVS_LDS_CASE(3)
+            IFVS_LDS_CASE(4) IFVS_LDS_CASE(5) IFVS_LDS_CASE(6) IFVS_LDS_CASE(7)
+            IFVS_LDS_CASE(8) IFVS_LDS_CASE(9) IFVS_LDS_CASE(10) IFVS_LDS_CASE(11)
+            IFVS_LDS_CASE(12) IFVS_LDS_CASE(13) IFVS_LDS_CASE(14) IFVS_LDS_CASE(15)
+#undef IFVS_LDS_CASE
+            default: va = 0.f; vb = 0.f; break;
+        }
+        acc = add_f32x2(acc, va, vb);
+    }
+    unpack_f32x2(acc, da, db);
+}
+
+// Distance of one row for any M (runtime loop; row_bytes a multiple of 4).
+__device__ __forceinline__ float lookup_any(const uint8_t* rp, bool pass, int M, int S,
+                                            const float* tab, int lane) {
+    float acc = 0.f;
+    for (int w = 0; w * 4 < M; ++w) {
+        const uint32_t wd = pass ? __ldg(reinterpret_cast<const uint32_t*>(rp) + w) : 0u;
+#pragma unroll
+        for (int bb = 0; bb < 4; ++bb) {
+            const int s = 4 * w + bb;
+            if (s < M) acc += tab[(int)((wd >> (8 * bb)) & 0xFFu) * S + lane + s];
+        }
+    }
+    return acc;
+}
+
+template <int KP, bool M16, bool FAST>
+__device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
+                                           const uint32_t* __restrict__ bmq, const ScanShape& sh,
+                                           int64_t b0, int64_t b1, const float* tab,
+                                           uint32_t* ring, WarpTopK<KP>& tk, int lane, int warp) {
     const int M = M16 ? 16 : sh.M;
     const int S = M16 ? 64 : sh.tab_words;
-    const int K = sh.K;
+    const int row_bytes = sh.row_bytes;
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
+    const uint32_t tb = 4u * (uint32_t)lane;
+
+    const uint64_t keep = policy_evict_last();
+    const int64_t first = b0 + warp;
+    const int T = first < b1 ? (int)((b1 - first + kScanWarps - 1) / kScanWarps) : 0;
+    auto word_addr = [&](int t) { return bmq + (first + (int64_t)t * kScanWarps) * 32 + lane; };
+
+    // ring: words of the blocks t in [F - kRing, F) in slot t % kRing
+    int F = T < kRing ? T : kRing;
+#pragma unroll
+    for (int i = 0; i < kRing; ++i)
+        if (i < F) ring[i * 32 + lane] = ldg_nc_u32(word_addr(i), policy_evict_first());
+    uint32_t pf[kHalf];
+    int npf = T - F < kHalf ? T - F : kHalf;
+#pragma unroll
+    for (int i = 0; i < kHalf; ++i) pf[i] = i < npf ? ldg_nc_u32(word_addr(F + i), policy_evict_first()) : 0u;
+    __syncwarp();
+    int pos = 0;
+    uint32_t cur = F > 0 ? ring[lane] : 0u;
+
+    for (;;) {
+        const int slow = (int)__reduce_min_sync(0xFFFFFFFFu, (unsigned)pos);
+        if (npf > 0 && slow >= F - kHalf) {
+#pragma unroll
+            for (int i = 0; i < kHalf; ++i)
+                if (i < npf) ring[((F + i) % kRing) * 32 + lane] = pf[i];
+            F += npf;
+            npf = T - F < kHalf ? T - F : kHalf;
+            const uint64_t once = policy_evict_first();
+#pragma unroll
+            for (int i = 0; i < kHalf; ++i) pf[i] = i < npf ? ldg_nc_u32(word_addr(F + i), once) : 0u;
+            __syncwarp();
+        }
+        // lanes whose word is used up move on before the mode is chosen
+        while (cur == 0u && pos + 1 < F) {
+            ++pos;
+            cur = ring[(pos % kRing) * 32 + lane];
+        }
+        const bool dense = __all_sync(0xFFFFFFFFu, cur == 0xFFFFFFFFu) &&
+                           __reduce_min_sync(0xFFFFFFFFu, (unsigned)pos) ==
+                               __reduce_max_sync(0xFFFFFFFFu, (unsigned)pos);
+        if (dense) {
+            // every lane holds all 32 rows of the same block: lockstep rows
+            const uint32_t rb = (uint32_t)((first + (int64_t)pos * kScanWarps) * kBlockRows) + lane;
+#pragma unroll 1
+            for (int j0 = 0; j0 < 32; j0 += kU) {
+                uint32_t row[kU];
+#pragma unroll
+                for (int u = 0; u < kU; ++u) row[u] = rb + 32u * (uint32_t)(j0 + u);
+                if constexpr (M16) {
+                    uint4 c[kU];
+#pragma unroll
+                    for (int u = 0; u < kU; ++u) c[u] = ldg_nc_v4(codes + (size_t)row[u] * 16, keep);
+                    float d[kU];
+#pragma unroll
+                    for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, base, d[u], d[u + 1]);
+                    uint64_t key[kU];
+                    bool want = false;
+#pragma unroll
+                    for (int u = 0; u < kU; ++u) {
+                        key[u] = ((uint64_t)__float_as_uint(d[u]) << 32) | row[u];
+                        want |= key[u] < tk.thr;
+                    }
+                    if (__any_sync(0xFFFFFFFFu, want)) {
+#pragma unroll
+                        for (int u = 0; u < kU; ++u) tk.offer(key[u], key[u] < tk.thr, lane);
+                    }
+                } else {
+#pragma unroll 1
+                    for (int u = 0; u < kU; ++u) {
+                        const float d = lookup_any(codes + (size_t)row[u] * row_bytes, true, M, S, tab, lane);
+                        const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | row[u];
+                        tk.offer(key, key < tk.thr, lane);
+                    }
+                }
+            }
+            cur = 0u;
+            continue;
+        }
+        // up to kU passing rows of this lane
+        uint32_t row[kU];
+        unsigned valid = 0u;
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            while (cur == 0u && pos + 1 < F) {
+                ++pos;
+                cur = ring[(pos % kRing) * 32 + lane];
+            }
+            row[u] = 0u;
+            if (cur != 0u) {
+                const int j = __ffs(cur) - 1;
+                cur &= cur - 1u;
+                row[u] = (uint32_t)((first + (int64_t)pos * kScanWarps) * kBlockRows) + 32u * (uint32_t)j + lane;
+                valid |= 1u << u;
+            }
+        }
+        if (__ballot_sync(0xFFFFFFFFu, valid != 0u) == 0u) {
+            if (F >= T) break;   // every word loaded and consumed
+            continue;            // lanes wait for the next refill
+        }
+        if constexpr (M16) {
+            uint4 c[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u)
+                c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)row[u] * 16, keep) : make_uint4(0, 0, 0, 0);
+            float d[kU];
+#pragma unroll
+            for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, base, d[u], d[u + 1]);
+            uint64_t key[kU];
+            bool want = false;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                key[u] = ((uint64_t)__float_as_uint(d[u]) << 32) | row[u];
+                want |= (valid >> u & 1u) && key[u] < tk.thr;
+            }
+            if (__any_sync(0xFFFFFFFFu, want)) {
+#pragma unroll
+                for (int u = 0; u < kU; ++u) tk.offer(key[u], (valid >> u & 1u) && key[u] < tk.thr, lane);
+            }
+        } else {
+#pragma unroll 1
+            for (int u = 0; u < kU; ++u) {
+                const bool pass = valid >> u & 1u;
+                const float d = lookup_any(codes + (size_t)row[u] * row_bytes, pass, M, S, tab, lane);
+                const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | row[u];
+                tk.offer(key, pass && key < tk.thr, lane);
+            }
+        }
+    }
+}
+
+template <int KP, bool M16, int MINB>
+__global__ void __launch_bounds__(kScanThreads, MINB)
+k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
+       const uint32_t* __restrict__ bm, int64_t nq, int k, ScanShape sh,
+       uint64_t* __restrict__ partials) {
+    extern __shared__ __align__(256) uint8_t smem[];
+    const int S = M16 ? 64 : sh.tab_words;
     float* tab = reinterpret_cast<float*>(smem);
     uint64_t* tkbuf = reinterpret_cast<uint64_t*>(smem + (size_t)256 * S * 4);
+    uint32_t* ringbase = reinterpret_cast<uint32_t*>(smem + (size_t)256 * S * 4 +
+                                                     (size_t)kScanWarps * 2 * KP * 8);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t q = blockIdx.x;
     const int chunk = blockIdx.y;
 
-    // 1) the query's table, replicated and rotated (see the file comment)
-    const float* lut = luts + q * (int64_t)M * K;
-    const int wu = M + 31;
-    for (int e = threadIdx.x; e < 256 * wu; e += kThreads) {
-        const int c = e / wu, w = e - c * wu;
-        const int m = w % M;
-        tab[c * S + w] = c < K ? __ldg(lut + (int64_t)m * K + c) : 0.f;
+    // 1) the query's table, replicated and rotated (see the file comment),
+    //    as written by k_tables: a straight 16-byte-wide copy
+    {
+        const float4* src = reinterpret_cast<const float4*>(tables + q * (int64_t)256 * S);
+        float4* dst = reinterpret_cast<float4*>(tab);
+        for (int i = threadIdx.x; i < 64 * S; i += kScanThreads) dst[i] = __ldg(src + i);
     }
     WarpTopK<KP> tk;
     tk.init(tkbuf + warp * 2 * KP, k, lane);
@@ -142,96 +388,71 @@ k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ luts,
     const int64_t b0 = (int64_t)chunk * sh.blocks_per_chunk;
     const int64_t b1 = min(sh.n_blocks, b0 + sh.blocks_per_chunk);
     const uint32_t* bmq = bm + q * sh.n_blocks * 32;
-    const uint32_t lane4 = (uint32_t)lane * 4u;
-    const char* tabc = reinterpret_cast<const char*>(tab);
-    const int row_bytes = sh.row_bytes;
-
-    for (int64_t b = b0 + warp; b < b1; b += kWarps) {
-        const uint32_t mword = __ldg(bmq + b * 32 + lane);
-        if (__ballot_sync(0xFFFFFFFFu, mword != 0u) == 0u) continue;
-        const int64_t rbase = b * kBlockRows + lane;
-        for (int j0 = 0; j0 < 32; j0 += kU) {
-            const uint32_t bits = (mword >> j0) & ((1u << kU) - 1u);
-            if (__ballot_sync(0xFFFFFFFFu, bits != 0u) == 0u) continue;
-            if (M16) {
-                uint4 c[kU];
-#pragma unroll
-                for (int u = 0; u < kU; ++u) {
-                    const int64_t row = rbase + 32 * (j0 + u);
-                    c[u] = (bits >> u & 1u) ? ldg_nc_v4(codes + row * 16) : make_uint4(0, 0, 0, 0);
-                }
-#pragma unroll
-                for (int u = 0; u < kU; ++u) {
-                    const int64_t row = rbase + 32 * (j0 + u);
-                    const float d = lookup16(c[u], tabc, lane4);
-                    const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | (uint64_t)(uint32_t)row;
-                    tk.offer(key, (bits >> u & 1u) && key < tk.thr, lane);
-                }
-            } else {
-#pragma unroll 1
-                for (int u = 0; u < kU; ++u) {
-                    const int64_t row = rbase + 32 * (j0 + u);
-                    const bool pass = bits >> u & 1u;
-                    const uint8_t* rp = codes + row * row_bytes;
-                    float acc = 0.f;
-                    for (int w = 0; w * 4 < M; ++w) {
-                        const uint32_t wd = pass ? __ldg(reinterpret_cast<const uint32_t*>(rp) + w) : 0u;
-#pragma unroll
-                        for (int bb = 0; bb < 4; ++bb) {
-                            const int s = 4 * w + bb;
-                            if (s < M) acc += tab[(int)((wd >> (8 * bb)) & 0xFFu) * S + lane + s];
-                        }
-                    }
-                    const uint64_t key = ((uint64_t)__float_as_uint(acc) << 32) | (uint64_t)(uint32_t)row;
-                    tk.offer(key, pass && key < tk.thr, lane);
-                }
-            }
-        }
+    uint32_t* ring = ringbase + warp * kRing * 32;
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
+    const bool fast = base == kDynSmemBase;
+    if constexpr (M16) {
+        if (fast)
+            scan_chunk<KP, true, true>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
+        else
+            scan_chunk<KP, true, false>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
+    } else {
+        scan_chunk<KP, false, false>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
     }
 
-    // 3) merge the warps' lists; warp 0 writes the CTA's k best keys
+    // 3) merge the warps' lists pairwise (4 levels); warp 0 writes the
+    //    CTA's k best keys
     tk.flush(lane);
-    __syncthreads();
-    if (warp == 0) {
-        for (int w = 1; w < kWarps; ++w) {
-            const uint64_t* other = tkbuf + w * 2 * KP;
+#pragma unroll 1
+    for (int step = 1; step < kScanWarps; step <<= 1) {
+        __syncthreads();
+        if ((warp & (2 * step - 1)) == 0) {
+            const uint64_t* other = tkbuf + (warp + step) * 2 * KP;
             for (int i = lane; i < k; i += 32) tk.buf[KP + i] = other[i];
             __syncwarp();
             tk.flush(lane);
         }
+    }
+    if (warp == 0) {
         uint64_t* out = partials + (q * sh.n_chunks + chunk) * (int64_t)k;
         for (int i = lane; i < k; i += 32) out[i] = tk.buf[i];
     }
 }
 
+template <int KP, bool M16, int MINB>
+static cudaError_t launch_one(const uint8_t* codes, const float* tab, const uint32_t* bm,
+                              int64_t nq, int k, const ScanShape& sh, uint64_t* partials,
+                              size_t smem, cudaStream_t s) {
+    cudaError_t e = cudaFuncSetAttribute(k_scan<KP, M16, MINB>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
+    k_scan<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(codes, tab, bm, nq, k, sh, partials);
+    return cudaGetLastError();
+}
+
 template <int KP>
-static cudaError_t launch_scan_kp(const uint8_t* codes, const float* lut, const uint32_t* bm,
+static cudaError_t launch_scan_kp(const uint8_t* codes, const float* tab, const uint32_t* bm,
                                   int64_t nq, int k, const ScanShape& sh, uint64_t* partials,
                                   cudaStream_t s) {
     const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
     const size_t smem = scan_smem_bytes(sh.tab_words, KP);
-    dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
-    cudaError_t e;
     if (m16) {
-        e = cudaFuncSetAttribute(k_scan<KP, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        k_scan<KP, true><<<grid, kThreads, smem, s>>>(codes, lut, bm, nq, k, sh, partials);
-    } else {
-        e = cudaFuncSetAttribute(k_scan<KP, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        k_scan<KP, false><<<grid, kThreads, smem, s>>>(codes, lut, bm, nq, k, sh, partials);
+        if (scan_ctas_per_sm(sh.tab_words, KP) >= 2)
+            return launch_one<KP, true, 2>(codes, tab, bm, nq, k, sh, partials, smem, s);
+        return launch_one<KP, true, 1>(codes, tab, bm, nq, k, sh, partials, smem, s);
     }
-    return cudaGetLastError();
+    return launch_one<KP, false, 1>(codes, tab, bm, nq, k, sh, partials, smem, s);
 }
 
-cudaError_t launch_scan(const uint8_t* codes, const float* lut, const uint32_t* bm, int64_t nq,
+cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm, int64_t nq,
                         int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s) {
     if (nq <= 0) return cudaSuccess;
     switch (scan_kp(k)) {
-        case 32: return launch_scan_kp<32>(codes, lut, bm, nq, k, sh, partials, s);
-        case 64: return launch_scan_kp<64>(codes, lut, bm, nq, k, sh, partials, s);
-        case 128: return launch_scan_kp<128>(codes, lut, bm, nq, k, sh, partials, s);
-        default: return launch_scan_kp<256>(codes, lut, bm, nq, k, sh, partials, s);
+        case 32: return launch_scan_kp<32>(codes, tab, bm, nq, k, sh, partials, s);
+        case 64: return launch_scan_kp<64>(codes, tab, bm, nq, k, sh, partials, s);
+        case 128: return launch_scan_kp<128>(codes, tab, bm, nq, k, sh, partials, s);
+        default: return launch_scan_kp<256>(codes, tab, bm, nq, k, sh, partials, s);
     }
 }
 
