@@ -32,21 +32,48 @@ cudaError_t launch_canonicalize(const ifvs_predicate* preds, int64_t nq, AttrCol
     return cudaGetLastError();
 }
 
+// Fail bits of 8 rows against one interval, shifted into `fail` (row j0 + 7
+// first, so that after four calls bit j is row j).  For each row:
+// off = v - lo (mod 2^32); the carry out of off + ~wm1 is 1 exactly when
+// off > wm1, i.e. when the row fails; addc shifts the carry in.  The carry
+// never leaves the asm block.
+__device__ __forceinline__ uint32_t fail8(uint32_t fail, const int32_t* v, int32_t lo, uint32_t nwm1) {
+    asm("{\n\t.reg .u32 t;\n\t"
+        "sub.u32 t, %8, %9;\n\tadd.cc.u32 t, t, %10;\n\taddc.u32 %0, %0, %0;\n\t"
+        "sub.u32 t, %7, %9;\n\tadd.cc.u32 t, t, %10;\n\taddc.u32 %0, %0, %0;\n\t"
+        "sub.u32 t, %6, %9;\n\tadd.cc.u32 t, t, %10;\n\taddc.u32 %0, %0, %0;\n\t"
+        "sub.u32 t, %5, %9;\n\tadd.cc.u32 t, t, %10;\n\taddc.u32 %0, %0, %0;\n\t"
+        "sub.u32 t, %4, %9;\n\tadd.cc.u32 t, t, %10;\n\taddc.u32 %0, %0, %0;\n\t"
+        "sub.u32 t, %3, %9;\n\tadd.cc.u32 t, t, %10;\n\taddc.u32 %0, %0, %0;\n\t"
+        "sub.u32 t, %2, %9;\n\tadd.cc.u32 t, t, %10;\n\taddc.u32 %0, %0, %0;\n\t"
+        "sub.u32 t, %1, %9;\n\tadd.cc.u32 t, t, %10;\n\taddc.u32 %0, %0, %0;\n\t"
+        "}"
+        : "+r"(fail)
+        : "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+          "r"(lo), "r"(nwm1));
+    return fail;
+}
+
+constexpr int kFilterQ = 256;   // queries staged in shared memory at a time
+
 template <int NA>
 __global__ void __launch_bounds__(kThreads) k_filter(AttrCols cols, int64_t N, int64_t n_blocks,
                                                      const CanonPred* __restrict__ canon,
                                                      int64_t nq, int q_per_cta,
                                                      uint32_t* __restrict__ bm,
                                                      unsigned long long* __restrict__ npass) {
+    __shared__ int2 s_iv[kFilterQ][NA];      // (lo, ~wm1) per query and column
+    __shared__ uint32_t s_keep[kFilterQ];    // 0 for a predicate no row can pass
+    __shared__ uint32_t s_used[kFilterQ];
     const int lane = threadIdx.x & 31;
     const int64_t b = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
-    if (b >= n_blocks) return;
+    const bool live = b < n_blocks;
     const int64_t q0 = (int64_t)blockIdx.y * q_per_cta;
     const int64_t q1 = min(nq, q0 + (int64_t)q_per_cta);
-    const int64_t row0 = b * kBlockRows + lane;
+    const int64_t row0 = (live ? b : 0) * kBlockRows + lane;
 
-    // rows beyond N: their bits stay 0 (the columns are padded, so the
-    // loads themselves stay inside the allocation)
+    // rows beyond N keep their bits at 0 (columns are padded, so the loads
+    // themselves stay inside the allocation)
     uint32_t valid = 0xFFFFFFFFu;
     if (b * kBlockRows + kBlockRows > N) {
         valid = 0;
@@ -69,28 +96,36 @@ __global__ void __launch_bounds__(kThreads) k_filter(AttrCols cols, int64_t N, i
     }
 
     const int64_t words = n_blocks * 32;
-    for (int64_t q = q0; q < q1; ++q) {
-        const CanonPred* cp = canon + q;
-        uint32_t m = 0;
-        if (!cp->empty) {
-            m = valid;
-            const uint32_t used = cp->used;
+    for (int64_t g0 = q0; g0 < q1; g0 += kFilterQ) {
+        const int ng = (int)min((int64_t)kFilterQ, q1 - g0);
+        __syncthreads();
+        for (int i = threadIdx.x; i < ng; i += blockDim.x) {
+            const CanonPred cp = canon[g0 + i];
+#pragma unroll
+            for (int c = 0; c < NA; ++c) s_iv[i][c] = make_int2(cp.lo[c], (int32_t)~cp.wm1[c]);
+            s_keep[i] = cp.empty ? 0u : 0xFFFFFFFFu;
+            s_used[i] = cp.used;
+        }
+        __syncthreads();
+        if (!live) continue;
+        for (int i = 0; i < ng; ++i) {
+            uint32_t m = valid & s_keep[i];
+            const uint32_t used = s_used[i];
 #pragma unroll
             for (int c = 0; c < NA; ++c) {
-                if (used >> c & 1u) {
-                    const int32_t lo = cp->lo[c];
-                    const uint32_t wm1 = cp->wm1[c];
-                    uint32_t mc = 0;
+                if (NA == 1 || (used >> c & 1u)) {
+                    const int2 iv = s_iv[i][c];
+                    uint32_t fail = 0;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        mc |= (uint32_t)((uint32_t)(v[c][j] - lo) <= wm1) << j;
-                    m &= mc;
+                    for (int j8 = 24; j8 >= 0; j8 -= 8) fail = fail8(fail, &v[c][j8], iv.x, (uint32_t)iv.y);
+                    m &= ~fail;
                 }
             }
+            const int64_t q = g0 + i;
+            bm[q * words + b * 32 + lane] = m;
+            const unsigned cnt = __reduce_add_sync(0xFFFFFFFFu, (unsigned)__popc(m));
+            if (lane == 0 && cnt) atomicAdd(npass + q, (unsigned long long)cnt);
         }
-        bm[q * words + b * 32 + lane] = m;
-        unsigned cnt = __reduce_add_sync(0xFFFFFFFFu, (unsigned)__popc(m));
-        if (lane == 0 && cnt) atomicAdd(npass + q, (unsigned long long)cnt);
     }
 }
 
