@@ -3,10 +3,10 @@
 // form of the printed score), and each CTA keeps the k smallest
 // (dist, row id) of its chunk exactly.
 //
-// Work split.  CTA (query q, chunk c), 16 warps; blockIdx.x runs over the
+// Work split.  CTA (query q, chunk c), 8 warps; blockIdx.x runs over the
 // queries so that the CTAs resident together walk the same code chunk and
 // share it through L2.  Warp w of the CTA owns bitmap blocks c0 + w,
-// c0 + w + 16, ...; lane l owns, in each of them, the 32 rows
+// c0 + w + 8, ...; lane l owns, in each of them, the 32 rows
 // b*1024 + 32*j + l, whose pass bits form its lane-major bitmap word.
 //
 // LUT placement.  The scan issues one shared-memory load per code byte, so
@@ -23,8 +23,8 @@
 //
 // Compaction.  Each lane visits only its own passing rows, so it keeps its
 // residue class and the conflict-free banks at any selectivity.  The warp's
-// bitmap words sit in a ring of 8 blocks in shared memory (lane l's word in
-// bank l); lanes advance through the ring at their own pace, four rows per
+// bitmap words sit in a ring of 16 blocks in shared memory (lane l's word in
+// bank l); lanes advance through the ring at their own pace, eight rows per
 // round, and the ring is refilled by halves, from words prefetched into
 // registers, once every lane has left the older half.  When every lane
 // holds a full word of the same block the warp takes the block in lockstep
@@ -34,17 +34,30 @@
 // area of KP slots; a key (dist bits << 32 | row) enters the area when it
 // is below the warp's current k-th key, and a full area is merged by a warp
 // bitonic sort.  Keys are unique (row ids are), so the result is exact and
-// independent of scheduling.  At the end warp 0 merges the other warps'
-// lists and writes the CTA's k keys.
+// independent of scheduling.  At the end the warps' lists are merged
+// pairwise and warp 0 writes the CTA's k keys.
+//
+// The tile constants (warps per CTA, ring depth, rows per round) were chosen
+// by measurement on the 10^8-row workload; the macros below only exist to
+// rebuild variants for such sweeps.
 #include "internal.cuh"
 
 namespace ifvs {
 
-constexpr int kScanWarps = 16;
+#ifndef IFVS_SCAN_WARPS
+#define IFVS_SCAN_WARPS 8
+#endif
+#ifndef IFVS_SCAN_RING
+#define IFVS_SCAN_RING 16
+#endif
+#ifndef IFVS_SCAN_ROWS
+#define IFVS_SCAN_ROWS 8
+#endif
+constexpr int kScanWarps = IFVS_SCAN_WARPS;
 constexpr int kScanThreads = kScanWarps * 32;
-constexpr int kRing = 8;          // bitmap words per lane in the ring
+constexpr int kRing = IFVS_SCAN_RING;    // bitmap words per lane in the ring
 constexpr int kHalf = kRing / 2;
-constexpr int kU = 4;             // rows per lane per round
+constexpr int kU = IFVS_SCAN_ROWS;       // rows per lane per round (even)
 
 int scan_kp(int k) { return k <= 32 ? 32 : (k <= 64 ? 64 : (k <= 128 ? 128 : 256)); }
 
@@ -438,7 +451,11 @@ static cudaError_t launch_scan_kp(const uint8_t* codes, const float* tab, const 
     const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
     const size_t smem = scan_smem_bytes(sh.tab_words, KP);
     if (m16) {
+#ifndef IFVS_SCAN_ONE_CTA
         if (scan_ctas_per_sm(sh.tab_words, KP) >= 2)
+#else
+        if (false)
+#endif
             return launch_one<KP, true, 2>(codes, tab, bm, nq, k, sh, partials, smem, s);
         return launch_one<KP, true, 1>(codes, tab, bm, nq, k, sh, partials, smem, s);
     }
