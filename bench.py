@@ -94,6 +94,12 @@ def reduce_max(dist, x, device):
     return float(t.item())
 
 
+def whole_job_qps(world, steps, batch, max_ms):
+    """Queries per second of the whole job: every rank ran `steps` batches of
+    `batch` queries; the job took the slowest rank's time."""
+    return world * steps * batch / (max_ms / 1000.0)
+
+
 def barrier(dist, device=None):
     if dist is not None:
         if device is not None and dist.get_backend() == "nccl":
@@ -386,7 +392,7 @@ def run_ifvs(args):
         barrier(dist, device)
         e_ms = reduce_max(dist, e_ms, device)
         nq_b = w.batch
-        e2e = {"value": world * args.steps * nq_b / (e_ms / 1000.0), "unit": "queries/s",
+        e2e = {"value": whole_job_qps(world, args.steps, nq_b, e_ms), "unit": "queries/s",
                "h2d_bytes_per_step": nq_b * (w.D * 4 * 2 + 104),
                "d2h_bytes_per_step": nq_b * (w.k * 12 + 8)}
 
@@ -402,7 +408,7 @@ def run_ifvs(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, ix, cond, batches)
 
-    value = world * args.steps * w.batch / (max_ms / 1000.0)
+    value = whole_job_qps(world, args.steps, w.batch, max_ms)
     line = {
         "metric": "QPS at recall@%d per selectivity bin (code-scan HBM GB/s vs peak)" % w.k,
         "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
