@@ -49,8 +49,13 @@ _lib = None
 def lib():
     global _lib
     if _lib is None:
-        build()
-        L = C.CDLL(_SO)
+        # IFVS_ORACLE_SO points the wrapper at another build of oracle.c (the
+        # mutation test loads copies with planted mistakes this way)
+        so = os.environ.get("IFVS_ORACLE_SO")
+        if not so:
+            build()
+            so = _SO
+        L = C.CDLL(so)
         P, I32_, I64, U64, D = C.c_void_p, C.c_int32, C.c_int64, C.c_uint64, C.c_double
         sig = {
             "orc_row_passes": (C.c_int, [P, P, I32_, I64, P]),

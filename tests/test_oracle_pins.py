@@ -400,6 +400,9 @@ def test_recall_values(orc):
     assert orc.recall(np.array([1, 2, 3, 4]), np.array([4, 9, 1, 8])) == 0.5
     assert orc.recall(np.array([1, -1, -1]), np.array([1, -1, -1])) == 1.0
     assert orc.recall(np.array([5, 6]), np.array([7, 8])) == 0.0
+    # padded ground truth: only its valid ids count
+    assert orc.recall(np.array([1, 2, 3]), np.array([1, -1, -1])) == 1.0
+    assert orc.recall(np.array([7, 2, 3]), np.array([1, 2, -1])) == 0.5
 
 
 # ------------------------------------------------------------ PQ construction
@@ -415,6 +418,22 @@ def test_kmeans_objective_non_increasing_and_encode_is_argmin(orc):
         np.testing.assert_array_equal(codes[:, m], d.argmin(axis=1))
     rec = np.stack([orc.reconstruct(Cq, c) for c in codes[:5]])
     np.testing.assert_array_equal(rec[:, :4], Cq[0][codes[:5, 0]])
+
+
+def test_encode_ties_go_to_the_smaller_codeword(orc):
+    # codewords 1 and 3 coincide; points on them must take codeword 1
+    Cq = np.zeros((1, 4, 2))
+    Cq[0] = [[5.0, 5.0], [1.0, 2.0], [9.0, 9.0], [1.0, 2.0]]
+    X = np.array([[1.0, 2.0], [1.25, 2.0], [9.0, 9.0]], np.float32)
+    np.testing.assert_array_equal(orc.pq_encode(X, Cq)[:, 0], [1, 1, 2])
+
+
+def test_exact_distance_closed_form(orc):
+    X = np.array([[0, 0, 0], [1, 2, 2], [3, 0, 4]], np.float32)
+    gi, gd = orc.exact_topk(X, np.zeros(3, np.float32), None, 3)
+    assert list(gi) == [0, 1, 2] and list(gd) == [0.0, 9.0, 25.0]
+    ri, rd = orc.rerank(X, np.zeros(3, np.float32), np.array([2, -1, 1]), 2)
+    assert list(ri) == [1, 2] and list(rd) == [9.0, 25.0]
 
 
 def test_kmeans_exact_when_codewords_cover_distinct_points(orc):
