@@ -60,6 +60,9 @@ def workload(args):
     w = synth.WORKLOADS[args.workload]
     if args.rows:
         w = synth.scaled(w, N=args.rows)
+    if w.batch <= 0:
+        # workloads whose recipe names no batch size run 1024-query steps
+        w = synth.scaled(w, batch=min(w.nq, 1024))
     return w
 
 
@@ -398,7 +401,7 @@ def run_ifvs(args):
 
     # recall@k (outside the timed regions)
     recall = None
-    if args.recall_queries > 0 and rank == 0:
+    if args.recall_queries > 0 and rank == 0 and not w.conjunctive:
         ids_by_bin = [dev_out[b][0].cpu().numpy()[:args.recall_queries] for b in range(nb)]
         recall = recall_at_k(w, ix, batches, ids_by_bin, args.recall_queries, device)
         for s, r in recall.items():
