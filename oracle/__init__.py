@@ -82,6 +82,8 @@ def lib():
             "orc_pq_encode": (None, [P, I64, I32_, I32_, I32_, P, P]),
             "orc_reconstruct": (None, [P, P, I32_, I32_, I32_, P]),
             "orc_sdc": (D, [P, P, P, I32_, I32_, I32_]),
+            "orc_pq_encode_f32": (None, [P, I64, I32_, I32_, I32_, P, P, P]),
+            "orc_lloyd_step": (None, [P, I64, I32_, I32_, I32_, P, P, P, P]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -355,3 +357,27 @@ def sdc(Cf, cq, cv):
     Cf = _c(Cf, np.float64)
     M, K, ds = Cf.shape
     return float(lib().orc_sdc(_p(Cf), _p(_c(cq, np.uint8)), _p(_c(cv, np.uint8)), M, K, ds))
+
+
+def pq_encode_f32(X, Cpq):
+    """Argmin encoding decided in float32 (fixed order, no fused multiply-add)."""
+    X = _c(X, np.float32)
+    Cpq = _c(Cpq, np.float32)
+    M, K, ds = Cpq.shape
+    codes = np.zeros((X.shape[0], M), dtype=np.uint8)
+    dmin = np.zeros((X.shape[0], M), dtype=np.float32)
+    lib().orc_pq_encode_f32(_p(X), X.shape[0], X.shape[1], M, K, _p(Cpq), _p(codes), _p(dmin))
+    return codes, dmin
+
+
+def lloyd_step(X, C_in):
+    """One Lloyd iteration per subspace from float32 centroids."""
+    X = _c(X, np.float32)
+    C_in = _c(C_in, np.float32)
+    M, K, ds = C_in.shape
+    C_out = np.zeros_like(C_in)
+    codes = np.zeros((X.shape[0], M), dtype=np.uint8)
+    obj = np.zeros(M, dtype=np.float64)
+    lib().orc_lloyd_step(_p(X), X.shape[0], X.shape[1], M, K, _p(C_in), _p(C_out), _p(codes),
+                         _p(obj))
+    return C_out, codes, obj

@@ -487,3 +487,76 @@ double orc_sdc(const double* C, const uint8_t* cq, const uint8_t* cv, int32_t M,
         }
     return s;
 }
+
+/* ------------------------------------------------------------------ */
+/* Encoding and Lloyd iterations decided in float32 (see oracle.h).  With
+ * -ffp-contract=off each expression below is one float32 rounding. */
+
+static float sq_dist_sub_f32(const float* x, const float* c, int32_t ds) {
+    float s = 0.0f;
+    for (int32_t t = 0; t < ds; ++t) {
+        float diff = x[t] - c[t];
+        float sq = diff * diff;
+        s = s + sq;
+    }
+    return s;
+}
+
+void orc_pq_encode_f32(const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
+                       const float* C, uint8_t* codes, float* dmin) {
+    int32_t ds = D / M;
+    for (int64_t i = 0; i < n; ++i)
+        for (int32_t m = 0; m < M; ++m) {
+            const float* x = X + i * D + m * ds;
+            const float* Cm = C + (int64_t)m * K * ds;
+            int32_t best = 0;
+            float bd = sq_dist_sub_f32(x, Cm, ds);
+            for (int32_t c = 1; c < K; ++c) {
+                float d = sq_dist_sub_f32(x, Cm + (int64_t)c * ds, ds);
+                if (d < bd) {
+                    bd = d;
+                    best = c;
+                }
+            }
+            codes[i * M + m] = (uint8_t)best;
+            if (dmin) dmin[i * M + m] = bd;
+        }
+}
+
+void orc_lloyd_step(const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
+                    const float* C_in, float* C_out, uint8_t* codes, double* objective) {
+    int32_t ds = D / M;
+    float* dmin = (float*)malloc(sizeof(float) * (size_t)(n > 0 ? n : 1) * M);
+    double* sum = (double*)malloc(sizeof(double) * (size_t)K * ds);
+    int64_t* cnt = (int64_t*)malloc(sizeof(int64_t) * (size_t)K);
+    orc_pq_encode_f32(X, n, D, M, K, C_in, codes, dmin);
+    for (int32_t m = 0; m < M; ++m) {
+        double obj = 0.0;
+        for (int64_t t = 0; t < (int64_t)K * ds; ++t) sum[t] = 0.0;
+        for (int32_t c = 0; c < K; ++c) cnt[c] = 0;
+        for (int64_t i = 0; i < n; ++i) {
+            int32_t c = codes[i * M + m];
+            cnt[c]++;
+            obj += (double)dmin[i * M + m];
+            for (int32_t t = 0; t < ds; ++t) sum[(int64_t)c * ds + t] += (double)X[i * D + m * ds + t];
+        }
+        if (objective) objective[m] = obj;
+        float* Co = C_out + (int64_t)m * K * ds;
+        const float* Ci = C_in + (int64_t)m * K * ds;
+        for (int32_t c = 0; c < K; ++c)
+            for (int32_t t = 0; t < ds; ++t)
+                Co[(int64_t)c * ds + t] = cnt[c] > 0 ? (float)(sum[(int64_t)c * ds + t] / (double)cnt[c])
+                                                     : Ci[(int64_t)c * ds + t];
+        for (int32_t c = 0; c < K; ++c)
+            if (cnt[c] == 0 && n > 0) {
+                int64_t far = 0;
+                for (int64_t i = 1; i < n; ++i)
+                    if (dmin[i * M + m] > dmin[far * M + m]) far = i;
+                for (int32_t t = 0; t < ds; ++t) Co[(int64_t)c * ds + t] = X[far * D + m * ds + t];
+                dmin[far * M + m] = 0.0f;
+            }
+    }
+    free(dmin);
+    free(sum);
+    free(cnt);
+}

@@ -132,6 +132,21 @@ void orc_pq_encode(const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
 void orc_reconstruct(const double* C, const uint8_t* code_row, int32_t M, int32_t K,
                      int32_t ds, double* x);
 
+/* The same encoding decided in float32, the precision of the GPU encoder:
+ * per codeword, s = 0; for t ascending: s = s + (x_t - c_t) * (x_t - c_t),
+ * each operation rounded to float32 (no fused multiply-add); argmin, ties to
+ * the smallest codeword.  dmin (optional, [n][M]) receives the minimum. */
+void orc_pq_encode_f32(const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
+                       const float* C, uint8_t* codes, float* dmin);
+/* One Lloyd iteration per subspace from float32 centroids C_in: assignment by
+ * orc_pq_encode_f32; each non-empty cluster's new centroid is the fp64 mean
+ * of its members rounded to float32; then every empty cluster, in increasing
+ * order, takes the member point farthest from its centroid (largest float32
+ * distance, ties to the smallest row), whose distance is then set to 0.
+ * objective [M] (optional) = sum of the float32 minimum distances (fp64). */
+void orc_lloyd_step(const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
+                    const float* C_in, float* C_out, uint8_t* codes, double* objective);
+
 /* Symmetric distance (baseline Pre_IndexPQ_SDC, §3.2): the query is encoded
  * first; dist = sum_m ||C[m][cq[m]] - C[m][cv[m]]||^2. */
 double orc_sdc(const double* C, const uint8_t* cq, const uint8_t* cv, int32_t M, int32_t K,

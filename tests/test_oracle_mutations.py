@@ -50,11 +50,17 @@ MUTATIONS = {
                                     "if (i < 0 || i >= N) continue;\n        double s = 0.0;\n        for (int32_t d = 0; d < D; ++d) {\n            double diff = (double)q[d] - (double)X[i * D + d];\n            s += fabs(diff);"),
     "k-means mean off by one": ("C[(int64_t)c * ds + t] = sum[(int64_t)c * ds + t] / (double)cnt[c];",
                                 "C[(int64_t)c * ds + t] = sum[(int64_t)c * ds + t] / (double)(cnt[c] + 1);"),
-    "encode ties to the larger codeword": ("            if (d < bd) {\n                    bd = d;\n                    best = c;\n                }\n            }\n            codes[i * M + m] = (uint8_t)best;",
-                                           "            if (d <= bd) {\n                    bd = d;\n                    best = c;\n                }\n            }\n            codes[i * M + m] = (uint8_t)best;"),
+    "encode ties to the larger codeword": ("            if (d < bd) {\n                    bd = d;\n                    best = c;\n                }\n            }\n            codes[i * M + m] = (uint8_t)best;\n        }\n}",
+                                           "            if (d <= bd) {\n                    bd = d;\n                    best = c;\n                }\n            }\n            codes[i * M + m] = (uint8_t)best;\n        }\n}"),
     "SDC wrong codeword": ("double diff = C[((int64_t)m * K + cq[m]) * ds + t] - C[((int64_t)m * K + cv[m]) * ds + t];",
                            "double diff = C[((int64_t)m * K + cq[m]) * ds + t] - C[((int64_t)m * K + cq[m]) * ds + t];"),
     "recall counts invalid ids": ("if (gt[j] < 0) continue;", "if (gt[j] < -1) continue;"),
+    "f32 encode fused multiply-add": ("float sq = diff * diff;\n        s = s + sq;", "s = fmaf(diff, diff, s);"),
+    "f32 encode ties to the larger": ("                if (d < bd) {\n                    bd = d;\n                    best = c;\n                }\n            }\n            codes[i * M + m] = (uint8_t)best;\n            if (dmin)",
+                                      "                if (d <= bd) {\n                    bd = d;\n                    best = c;\n                }\n            }\n            codes[i * M + m] = (uint8_t)best;\n            if (dmin)"),
+    "Lloyd keeps the old centroid": ("Co[(int64_t)c * ds + t] = cnt[c] > 0 ? (float)(sum[(int64_t)c * ds + t] / (double)cnt[c])",
+                                     "Co[(int64_t)c * ds + t] = cnt[c] > 0 ? Ci[(int64_t)c * ds + t]"),
+    "Lloyd reseeds with the nearest point": ("if (dmin[i * M + m] > dmin[far * M + m]) far = i;", "if (dmin[i * M + m] < dmin[far * M + m]) far = i;"),
 }
 
 

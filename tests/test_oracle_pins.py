@@ -453,3 +453,77 @@ def test_sdc_properties(orc):
     assert orc.sdc(Cq, a, b) == orc.sdc(Cq, b, a)
     ra, rb = orc.reconstruct(Cq, a), orc.reconstruct(Cq, b)
     assert abs(orc.sdc(Cq, a, b) - cdist(ra[None], rb[None], "sqeuclidean")[0, 0]) < 1e-12
+
+
+# ------------------------------------------------------------ float32 encoding, Lloyd step
+
+def test_encode_f32_agrees_with_fp64_away_from_ties(orc):
+    rng = np.random.default_rng(21)
+    X = rng.standard_normal((800, 16)).astype(np.float32)
+    Cq = rng.standard_normal((2, 64, 8)).astype(np.float32)
+    c32, d32 = orc.pq_encode_f32(X, Cq)
+    c64 = orc.pq_encode(X, Cq.astype(np.float64))
+    for m in range(2):
+        d = cdist(X[:, m * 8:(m + 1) * 8].astype(np.float64), Cq[m].astype(np.float64), "sqeuclidean")
+        srt = np.sort(d, axis=1)
+        clear = (srt[:, 1] - srt[:, 0]) > 1e-5 * srt[:, 1]
+        np.testing.assert_array_equal(c32[clear, m], c64[clear, m])
+        np.testing.assert_allclose(d32[:, m], srt[:, 0], rtol=2e-6)
+    assert clear.mean() > 0.99
+
+
+def test_encode_f32_rounds_every_operation(orc):
+    """x = (2^-12, 1 + 2^-12) against the zero codeword: the squares are
+    2^-24 and 1 + 2^-11 + 2^-24; rounding the second square to float32 (a
+    tie, to even) gives 1 + 2^-11, and adding 2^-24 ties back to 1 + 2^-11.
+    A fused multiply-add would give 1 + 2^-11 + 2^-23 instead."""
+    X = np.array([[2.0 ** -12, 1.0 + 2.0 ** -12]], np.float32)
+    Cq = np.zeros((1, 1, 2), np.float32)
+    _, dmin = orc.pq_encode_f32(X, Cq)
+    assert float(dmin[0, 0]) == 1.0 + 2.0 ** -11
+
+
+def test_encode_f32_ties_to_smaller_codeword(orc):
+    Cq = np.array([[[5, 5], [1, 2], [9, 9], [1, 2]]], np.float32)
+    X = np.array([[1.0, 2.0], [1.25, 2.0], [9.0, 9.0]], np.float32)
+    codes, dmin = orc.pq_encode_f32(X, Cq)
+    assert list(codes[:, 0]) == [1, 1, 2] and list(dmin[:, 0]) == [0.0, 0.0625, 0.0]
+
+
+def test_lloyd_step_is_the_member_mean(orc):
+    rng = np.random.default_rng(22)
+    X = rng.standard_normal((500, 8)).astype(np.float32)
+    C0 = X[rng.choice(500, 16, replace=False)].reshape(16, 2, 4).transpose(1, 0, 2).copy()
+    C1, codes, obj = orc.lloyd_step(X, C0)
+    c_ref, d_ref = orc.pq_encode_f32(X, C0)
+    np.testing.assert_array_equal(codes, c_ref)
+    np.testing.assert_allclose(obj, d_ref.astype(np.float64).sum(axis=0), rtol=1e-12)
+    for m in range(2):
+        sub = X[:, m * 4:(m + 1) * 4].astype(np.float64)
+        cnt = np.bincount(codes[:, m], minlength=16)
+        for k in range(16):
+            if cnt[k]:
+                np.testing.assert_array_equal(C1[m, k], sub[codes[:, m] == k].mean(axis=0).astype(np.float32))
+
+
+def test_lloyd_step_reseeds_empty_codeword_with_farthest_point(orc):
+    X = np.array([[0.0], [1.0], [10.0], [10.5]], np.float32)
+    C0 = np.array([[[0.0], [10.0], [1000.0]]], np.float32)   # codeword 2 gets nobody
+    C1, codes, obj = orc.lloyd_step(X, C0)
+    assert list(codes[:, 0]) == [0, 0, 1, 1]
+    # means 0.5 and 10.25; the farthest point is row 1 or row 3 (distance
+    # 1.0 vs 0.25): row 1 (x = 1.0) becomes codeword 2
+    np.testing.assert_array_equal(C1[0, :, 0], [0.5, 10.25, 1.0])
+    assert obj[0] == 0.0 + 1.0 + 0.0 + 0.25
+
+
+def test_lloyd_steps_do_not_increase_the_objective(orc):
+    rng = np.random.default_rng(23)
+    X = (rng.standard_normal((600, 8)) + rng.integers(0, 4, (600, 1)) * 3).astype(np.float32)
+    C = X[:12].reshape(12, 2, 4).transpose(1, 0, 2).copy()
+    last = None
+    for _ in range(6):
+        C, _, obj = orc.lloyd_step(X, C)
+        if last is not None:
+            assert (obj <= last * (1 + 1e-6)).all()
+        last = obj
