@@ -247,6 +247,37 @@ int ifvs_rerank(ifvs_index* ix, const float* queries, const int64_t* cand, int64
                 float* dists);
 
 /*
+ * ifvs_pq_encode — PQ encoding of raw vectors (the offline step before the
+ * query path: §1's product quantisation, 16 x 8 in §3.2), on `device`.
+ *   X       [n][D] float32; subspace m covers dimensions [m ds, (m+1) ds)
+ *   C_pq    [M][K][ds] float32 codebook
+ *   codes   [n][M] uint8 out: argmin over codewords of the float32 squared
+ *           distance s = s + (x_t - c_t)^2 accumulated for t ascending with
+ *           every operation rounded on its own; ties to the smallest codeword
+ *   dmin    [n][M] float32 out (that minimum), or NULL
+ *   flags   IFVS_F_DEVICE_IO: all arrays are device pointers
+ */
+int ifvs_pq_encode(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
+                   const float* C_pq, uint8_t* codes, float* dmin, uint32_t flags);
+
+/*
+ * ifvs_pq_train — `iters` Lloyd iterations per subspace from C_init
+ * (k-means training of the PQ codebook).  Each iteration assigns every row
+ * as ifvs_pq_encode does, then replaces each codeword used by at least one
+ * row by the fp64 mean of its rows rounded to float32; each unused
+ * codeword, in increasing order, takes the row farthest from its codeword
+ * (largest distance, ties to the smallest row), whose distance then counts
+ * as 0.
+ *   C_init     [M][K][ds] float32 start (e.g. K distinct sample rows)
+ *   C_out      [M][K][ds] float32 out
+ *   objective  [iters][M] fp64 out (sum of the assignment's minimum
+ *              distances at each iteration, before its update), or NULL
+ */
+int ifvs_pq_train(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
+                  int32_t iters, const float* C_init, float* C_out, double* objective,
+                  uint32_t flags);
+
+/*
  * ifvs_stage_times — device time (ms, from CUDA events recorded on the
  * launching stream around each launch) and launch counts per stage,
  * accumulated over calls made with IFVS_F_STAGE_TIMING.  Either array may be

@@ -5,6 +5,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
 #include <new>
 #include <utility>
 #include <vector>
@@ -908,6 +909,153 @@ int ifvs_rerank(ifvs_index* ix, const float* queries, const int64_t* cand, int64
         TRY(copy_out(s, false, dists, odi, sizeof(float) * nq * k));
     }
     return finish(ix, s, false);
+}
+
+// ---- PQ construction ----------------------------------------------------------
+
+namespace {
+
+struct PqArgs {
+    int device = 0, num_sms = 0;
+    cudaStream_t s = nullptr;
+    std::vector<void*> owned;
+    ~PqArgs() {
+        if (s) cudaStreamSynchronize(s);
+        for (void* p : owned) cudaFree(p);
+        if (s) cudaStreamDestroy(s);
+    }
+    int alloc(void** p, size_t bytes) {
+        cudaError_t e = cudaMalloc(p, bytes ? bytes : 16);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            *p = nullptr;
+            return set_err(IFVS_ERR_OOM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+        }
+        owned.push_back(*p);
+        return 0;
+    }
+    // device copy of a host input (or the pointer itself with device I/O)
+    int input(const void* host, size_t bytes, bool dio, const void** out) {
+        if (dio) {
+            *out = host;
+            return 0;
+        }
+        void* p = nullptr;
+        TRY(alloc(&p, bytes));
+        CUDA_TRY(cudaMemcpyAsync(p, host, bytes, cudaMemcpyHostToDevice, s));
+        *out = p;
+        return 0;
+    }
+};
+
+int pq_check(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
+             uint32_t flags, PqArgs* a) {
+    if (n < 0) return set_err(IFVS_ERR_ARG, "n < 0");
+    if (n > 0 && !X) return set_err(IFVS_ERR_ARG, "X is NULL");
+    if (n > (int64_t)0xFFFFFFFFLL) return set_err(IFVS_ERR_ARG, "n = %lld above 2^32 - 1", (long long)n);
+    if (M < 1 || D < M || D % M != 0) return set_err(IFVS_ERR_ARG, "D = %d must be a positive multiple of M = %d", D, M);
+    if (K < 1 || K > 256) return set_err(IFVS_ERR_UNSUPPORTED, "K = %d outside 1..256", K);
+    if ((size_t)K * (D / M) * sizeof(double) + (size_t)K * 8 > 200 * 1024)
+        return set_err(IFVS_ERR_UNSUPPORTED, "K x ds too large for the shared-memory codebook");
+    if (flags & ~IFVS_F_DEVICE_IO) return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", flags);
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) {
+        cudaGetLastError();
+        return set_err(IFVS_ERR_CUDA, "no CUDA device is available");
+    }
+    if (device < 0 || device >= ndev) return set_err(IFVS_ERR_ARG, "device %d outside 0..%d", device, ndev - 1);
+    a->device = device;
+    CUDA_TRY(cudaDeviceGetAttribute(&a->num_sms, cudaDevAttrMultiProcessorCount, device));
+    CUDA_TRY(cudaStreamCreateWithFlags(&a->s, cudaStreamNonBlocking));
+    return 0;
+}
+
+}  // namespace
+
+extern "C" int ifvs_pq_encode(int32_t device, const float* X, int64_t n, int32_t D, int32_t M,
+                              int32_t K, const float* C_pq, uint8_t* codes, float* dmin,
+                              uint32_t flags) {
+    if (!C_pq || (n > 0 && !codes)) return set_err(IFVS_ERR_ARG, "C_pq / codes is NULL");
+    DeviceGuard g(device);
+    PqArgs a;
+    TRY(pq_check(device, X, n, D, M, K, flags, &a));
+    if (n == 0) return IFVS_OK;
+    const bool dio = flags & IFVS_F_DEVICE_IO;
+    const int ds = D / M;
+    const void *dX, *dC;
+    TRY(a.input(X, sizeof(float) * n * D, dio, &dX));
+    TRY(a.input(C_pq, sizeof(float) * M * K * ds, dio, &dC));
+    uint8_t* dcodes = codes;
+    float* ddmin = dmin;
+    if (!dio) {
+        void* p;
+        TRY(a.alloc(&p, (size_t)n * M));
+        dcodes = (uint8_t*)p;
+        ddmin = nullptr;
+        if (dmin) {
+            TRY(a.alloc(&p, sizeof(float) * n * M));
+            ddmin = (float*)p;
+        }
+    }
+    CUDA_TRY(launch_pq_assign((const float*)dX, n, D, M, K, (const float*)dC, dcodes, ddmin, a.s));
+    if (!dio) {
+        CUDA_TRY(cudaMemcpyAsync(codes, dcodes, (size_t)n * M, cudaMemcpyDeviceToHost, a.s));
+        if (dmin) CUDA_TRY(cudaMemcpyAsync(dmin, ddmin, sizeof(float) * n * M, cudaMemcpyDeviceToHost, a.s));
+    }
+    CUDA_TRY(cudaStreamSynchronize(a.s));
+    return IFVS_OK;
+}
+
+extern "C" int ifvs_pq_train(int32_t device, const float* X, int64_t n, int32_t D, int32_t M,
+                             int32_t K, int32_t iters, const float* C_init, float* C_out,
+                             double* objective, uint32_t flags) {
+    if (!C_init || !C_out) return set_err(IFVS_ERR_ARG, "C_init / C_out is NULL");
+    if (iters < 0) return set_err(IFVS_ERR_ARG, "iters < 0");
+    DeviceGuard g(device);
+    PqArgs a;
+    TRY(pq_check(device, X, n, D, M, K, flags, &a));
+    const bool dio = flags & IFVS_F_DEVICE_IO;
+    const int ds = D / M;
+    const size_t cb_bytes = sizeof(float) * (size_t)M * K * ds;
+    const void *dX = nullptr, *dC0;
+    if (n > 0) TRY(a.input(X, sizeof(float) * n * D, dio, &dX));
+    TRY(a.input(C_init, cb_bytes, dio, &dC0));
+    void *cA, *cB, *codes, *dmin, *sums, *counts, *best, *obj;
+    TRY(a.alloc(&cA, cb_bytes));
+    TRY(a.alloc(&cB, cb_bytes));
+    TRY(a.alloc(&codes, (size_t)(n > 0 ? n : 1) * M));
+    TRY(a.alloc(&dmin, sizeof(float) * (size_t)(n > 0 ? n : 1) * M));
+    TRY(a.alloc(&sums, sizeof(double) * (size_t)M * K * ds));
+    TRY(a.alloc(&counts, sizeof(unsigned long long) * (size_t)M * K));
+    TRY(a.alloc(&best, sizeof(unsigned long long)));
+    TRY(a.alloc(&obj, sizeof(double) * M));
+    CUDA_TRY(cudaMemcpyAsync(cA, dC0, cb_bytes, cudaMemcpyDeviceToDevice, a.s));
+    std::vector<unsigned long long> cnt((size_t)M * K);
+    for (int it = 0; it < iters && n > 0; ++it) {
+        CUDA_TRY(launch_pq_assign((const float*)dX, n, D, M, K, (const float*)cA, (uint8_t*)codes,
+                                  (float*)dmin, a.s));
+        if (objective) {
+            CUDA_TRY(launch_pq_objective((const float*)dmin, n, M, (double*)obj, a.num_sms, a.s));
+            CUDA_TRY(cudaMemcpyAsync(objective + (size_t)it * M, obj, sizeof(double) * M,
+                                     dio ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, a.s));
+        }
+        CUDA_TRY(launch_pq_update((const float*)dX, n, D, M, K, (const uint8_t*)codes, (double*)sums,
+                                  (unsigned long long*)counts, (const float*)cA, (float*)cB,
+                                  a.num_sms, a.s));
+        CUDA_TRY(cudaMemcpyAsync(cnt.data(), counts, sizeof(unsigned long long) * cnt.size(),
+                                 cudaMemcpyDeviceToHost, a.s));
+        CUDA_TRY(cudaStreamSynchronize(a.s));
+        for (int m = 0; m < M; ++m)
+            for (int c = 0; c < K; ++c)
+                if (cnt[(size_t)m * K + c] == 0)
+                    CUDA_TRY(launch_pq_reseed((const float*)dX, n, D, M, K, m, c,
+                                              (unsigned long long*)best, (float*)cB, (float*)dmin,
+                                              a.num_sms, a.s));
+        std::swap(cA, cB);
+    }
+    CUDA_TRY(cudaMemcpyAsync(C_out, cA, cb_bytes, dio ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, a.s));
+    CUDA_TRY(cudaStreamSynchronize(a.s));
+    return IFVS_OK;
 }
 
 int ifvs_stage_times(ifvs_index* ix, double* ms, int64_t* launches, int32_t reset) {

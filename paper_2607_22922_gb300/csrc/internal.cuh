@@ -154,6 +154,21 @@ cudaError_t launch_rerank(const float* X, int64_t N, int D, const float* q, cons
 cudaError_t launch_relayout_codes(const uint8_t* src, int64_t N, int M, int K, int row_bytes,
                                   int64_t n_rows_pad, uint8_t* dst, int* bad, cudaStream_t s);
 
+// ---- PQ construction (csrc/pq.cu) --------------------------------------
+// codes [n][M] and optional dmin [n][M] (float32 argmin, fixed order)
+cudaError_t launch_pq_assign(const float* X, int64_t n, int D, int M, int K, const float* C,
+                             uint8_t* codes, float* dmin, cudaStream_t s);
+// Lloyd update: fp64 means of the members (sums [M][K][ds], counts [M][K])
+cudaError_t launch_pq_update(const float* X, int64_t n, int D, int M, int K, const uint8_t* codes,
+                             double* sums, unsigned long long* counts, const float* C_in,
+                             float* C_out, int num_sms, cudaStream_t s);
+// empty codeword c of subspace m <- the farthest row (best: 8-byte scratch)
+cudaError_t launch_pq_reseed(const float* X, int64_t n, int D, int M, int K, int m, int c,
+                             unsigned long long* best, float* C_out, float* dmin, int num_sms,
+                             cudaStream_t s);
+cudaError_t launch_pq_objective(const float* dmin, int64_t n, int M, double* objective, int num_sms,
+                                cudaStream_t s);
+
 // Read-only view of a loaded index, for entry points defined outside api.cu.
 struct IndexView {
     int device;

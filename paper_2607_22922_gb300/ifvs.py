@@ -54,6 +54,8 @@ def _load():
         "ifvs_scan_topk": (C.c_int, [P, P, P, I64, I32, P, P, P]),
         "ifvs_rerank": (C.c_int, [P, P, P, I64, I32, I32, P, P, P]),
         "ifvs_scan_topk_static": (C.c_int, [P, P, P, I64, I32, P, P, P]),
+        "ifvs_pq_encode": (C.c_int, [I32, P, I64, I32, I32, I32, P, P, P, U32]),
+        "ifvs_pq_train": (C.c_int, [I32, P, I64, I32, I32, I32, I32, P, P, P, U32]),
         "ifvs_stage_times": (C.c_int, [P, P, P, I32]),
         "ifvs_canonical_predicate": (C.c_int, [P, P, I32, P, P, P]),
         "ifvs_index_info": (C.c_int, [P, P]),
@@ -238,6 +240,31 @@ def ifvs_scan_topk_static(ix, lut, bitmaps, k, ids, dists, stream=None):
     _check(_lib.ifvs_scan_topk_static(ix, _ptr(lut), _ptr(bitmaps), nq, k, stream, _ptr(ids),
                                       _ptr(dists)))
     return ids, dists
+
+
+def ifvs_pq_encode(X, C_pq, device=0, want_dmin=False):
+    """codes [n][M] uint8 (and dmin [n][M] float32) for host arrays."""
+    X = _host(X, np.float32)
+    C_pq = _host(C_pq, np.float32)
+    n, D = X.shape
+    M, K, ds = C_pq.shape
+    codes = np.empty((n, M), np.uint8)
+    dmin = np.empty((n, M), np.float32) if want_dmin else None
+    _check(_lib.ifvs_pq_encode(device, _ptr(X), n, D, M, K, _ptr(C_pq), _ptr(codes), _ptr(dmin), 0))
+    return (codes, dmin) if want_dmin else codes
+
+
+def ifvs_pq_train(X, C_init, iters, device=0):
+    """Lloyd iterations from C_init [M][K][ds]; returns (C_out, objective [iters][M])."""
+    X = _host(X, np.float32)
+    C_init = _host(C_init, np.float32)
+    n, D = X.shape
+    M, K, ds = C_init.shape
+    C_out = np.empty_like(C_init)
+    obj = np.empty((max(iters, 1), M), np.float64)
+    _check(_lib.ifvs_pq_train(device, _ptr(X), n, D, M, K, iters, _ptr(C_init), _ptr(C_out),
+                              _ptr(obj), 0))
+    return C_out, obj[:iters]
 
 
 def ifvs_rerank(ix, queries, cand, k, flags=0):

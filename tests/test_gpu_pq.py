@@ -1,0 +1,88 @@
+"""PQ construction on the GPU vs the oracle: the encoder decides in float32
+with the oracle's fixed operation order, so codes and minimum distances are
+compared bit for bit; a Lloyd iteration's new centroids (fp64 means rounded
+to float32, summed in another order) within one float32 ulp."""
+import numpy as np
+import pytest
+
+from paper_2607_22922_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ifvs():
+    from paper_2607_22922_gb300 import build
+    build.build()
+    from paper_2607_22922_gb300 import ifvs as mod
+    return mod
+
+
+def _data(w, n, seed):
+    ix = synth.make_index(synth.scaled(w, N=n))
+    X = synth.raw_vectors(ix)
+    rng = np.random.default_rng(seed)
+    C0 = X[rng.choice(n, w.K, replace=False)].reshape(w.K, w.M, w.ds).transpose(1, 0, 2).copy()
+    return X, C0
+
+
+CASES = [("gmm10k-d128-m16", 20_011), ("sift1m-d128-m16", 30_007), ("deep10m-d96-m12", 12_345),
+         ("gist1m-d960-m120", 3_001)]
+
+
+@pytest.mark.parametrize("name,n", CASES)
+def test_encode_bit_exact(ifvs, orc, name, n):
+    X, C0 = _data(synth.WORKLOADS[name], n, 1)
+    codes, dmin = ifvs.ifvs_pq_encode(X, C0, want_dmin=True)
+    rc, rd = orc.pq_encode_f32(X, C0)
+    np.testing.assert_array_equal(codes, rc)
+    np.testing.assert_array_equal(dmin, rd)
+
+
+def test_encode_ragged_and_small_codebooks(ifvs, orc):
+    rng = np.random.default_rng(4)
+    for n, M, K, ds in ((1, 1, 1, 1), (33, 3, 5, 3), (257, 4, 16, 2), (1000, 2, 256, 12)):
+        X = rng.standard_normal((n, M * ds)).astype(np.float32)
+        C = rng.standard_normal((M, K, ds)).astype(np.float32)
+        C[:, -1] = C[:, 0]                       # duplicate codeword: ties go to 0
+        codes, dmin = ifvs.ifvs_pq_encode(X, C, want_dmin=True)
+        rc, rd = orc.pq_encode_f32(X, C)
+        np.testing.assert_array_equal(codes, rc)
+        np.testing.assert_array_equal(dmin, rd)
+
+
+def _ulp_close(a, b):
+    a = np.asarray(a, np.float32)
+    b = np.asarray(b, np.float32)
+    return np.abs(a.astype(np.float64) - b.astype(np.float64)) <= np.spacing(np.maximum(np.abs(a), np.abs(b)))
+
+
+@pytest.mark.parametrize("name,n", CASES[:3])
+def test_one_lloyd_step(ifvs, orc, name, n):
+    X, C0 = _data(synth.WORKLOADS[name], n, 2)
+    C1, obj = ifvs.ifvs_pq_train(X, C0, 1)
+    R1, _, robj = orc.lloyd_step(X, C0)
+    assert _ulp_close(C1, R1).all()
+    np.testing.assert_allclose(obj[0], robj, rtol=1e-12)
+
+
+def test_empty_codewords_take_the_farthest_points(ifvs, orc):
+    rng = np.random.default_rng(5)
+    X = rng.standard_normal((4000, 16)).astype(np.float32)
+    C0 = rng.standard_normal((2, 64, 8)).astype(np.float32)
+    C0[:, 40:] += 100.0                          # 24 codewords per subspace attract nobody
+    C1, _ = ifvs.ifvs_pq_train(X, C0, 1)
+    R1, codes, _ = orc.lloyd_step(X, C0)
+    assert (np.bincount(codes[:, 0], minlength=64)[40:] == 0).all()
+    assert _ulp_close(C1, R1).all()
+
+
+def test_lloyd_iterations_track_the_oracle(ifvs, orc):
+    X, C = _data(synth.WORKLOADS["gmm10k-d128-m16"], 8_000, 3)
+    G, gobj = ifvs.ifvs_pq_train(X, C, 5)
+    R = C
+    for it in range(5):
+        R, _, robj = orc.lloyd_step(X, R)
+        np.testing.assert_allclose(gobj[it], robj, rtol=1e-9)
+    assert (np.diff(gobj, axis=0) <= 1e-6 * gobj[:-1]).all()
+    assert _ulp_close(G, R).mean() > 0.999
