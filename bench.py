@@ -52,6 +52,11 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--chunk-blocks", type=int, default=0, help="scan chunk size in 1024-row blocks (0 = auto)")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
+    ap.add_argument("--mode", default="search", choices=["search", "pq"],
+                    help="search: the query path; pq: PQ encoding + Lloyd training of the index")
+    ap.add_argument("--pq-rows", type=int, default=1 << 24, help="rows encoded per step (--mode pq)")
+    ap.add_argument("--pq-train-rows", type=int, default=1 << 20, help="Lloyd sample rows (--mode pq)")
+    ap.add_argument("--pq-iters", type=int, default=25, help="Lloyd iterations (--mode pq)")
     return ap.parse_args()
 
 
@@ -171,19 +176,23 @@ def measured_peaks():
     return 6800.0, "fallback"
 
 
-def scan_traffic():
-    """DRAM bytes per scan launch from the committed ncu summary, valid only
-    while the scan kernel's source is unchanged."""
-    p = os.path.join(ROOT, "profiles", "scan_traffic.json")
-    src = os.path.join(ROOT, "paper_2607_22922_gb300", "csrc", "scan.cu")
+def kernel_traffic(summary, source):
+    """DRAM bytes per launch from a committed ncu summary, valid only while
+    the kernel's source file is unchanged."""
+    p = os.path.join(ROOT, "profiles", summary)
+    src = os.path.join(ROOT, "paper_2607_22922_gb300", "csrc", source)
     if not os.path.exists(p):
         return None
     with open(p) as f:
         d = json.load(f)
     sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
-    if d.get("scan_cu_sha256") != sha:
+    if d.get(source.replace(".", "_") + "_sha256") != sha:
         return None
     return d.get("dram_bytes_per_launch")
+
+
+def scan_traffic():
+    return kernel_traffic("scan_traffic.json", "scan.cu")
 
 
 # ------------------------------------------------------------ CPU baseline
@@ -437,6 +446,159 @@ def run_ifvs(args):
         dist.destroy_process_group()
 
 
+def run_pq(args):
+    """PQ construction (the offline step before the query path): a step
+    encodes one slice of raw vectors against the workload's codebook with
+    one kernel; Lloyd training on a sample is timed beside it."""
+    import torch
+    world, rank, local = dist_env()
+    if not torch.cuda.is_available():
+        raise SystemExit("no CUDA device: the benchmark needs a GPU")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    dist = dist_init(world, device)
+    from paper_2607_22922_gb300 import build, synth
+    if rank == 0 or world == 1:
+        build.build()
+    barrier(dist, device)
+    build.build()
+    from paper_2607_22922_gb300 import ifvs
+
+    w = workload(args)
+    rows = min(args.pq_rows, w.N)
+    t0 = time.time()
+    ix = synth.make_index(synth.scaled(w, N=rows))
+    cb = torch.from_numpy(ix.codebook).to(device)
+    block = 1 << 22
+    X = torch.empty((rows, w.D), dtype=torch.float32, device=device)
+    for s0 in range(0, rows, block):
+        s1 = min(rows, s0 + block)
+        X[s0:s1] = synth.raw_vectors_torch(ix, s0, s1, device, cb)
+    codes = torch.empty((rows, w.M), dtype=torch.uint8, device=device)
+    torch.cuda.synchronize()
+    t_gen = time.time() - t0
+    stream = torch.cuda.Stream(device=device)
+    sptr = stream.cuda_stream
+    dio = ifvs.IFVS_F_DEVICE_IO
+
+    def step():
+        ifvs.ifvs_pq_encode(X, cb, device=local, codes=codes, flags=dio, stream=sptr)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    clocks = Clocks()
+    barrier(dist, device)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    with torch.cuda.stream(stream):
+        ev[0].record(stream)
+        for i in range(args.steps):
+            step()
+            ev[i + 1].record(stream)
+    torch.cuda.synchronize()
+    barrier(dist, device)
+    clk = clocks.stop()
+    total_ms = ev[0].elapsed_time(ev[-1])
+    max_ms = reduce_max(dist, total_ms, device)
+    launch_ms = total_ms / args.steps
+
+    # roofline: three rounded float32 operations (sub, mul, add) per row,
+    # codeword and dimension; the FP32 pipes of 152 SMs x 128 lanes at the
+    # SM clock (one operation per lane per cycle)
+    props = torch.cuda.get_device_properties(device)
+    sms = props.multi_processor_count
+    mhz = (clk or {}).get("sm_max_mhz") or 2070.0
+    ops = 3.0 * rows * w.K * w.D
+    achieved = ops / (launch_ms / 1000.0) / 1e12
+    peak = sms * 128 * mhz * 1e6 / 1e12
+    roofline = {"kernel": "k_pq_assign", "bound": "alu", "achieved": achieved, "peak": peak,
+                "unit": "TFLOP/s", "frac": achieved / peak,
+                "traffic": kernel_traffic("pq_encode_traffic.json", "pq.cu"),
+                "peak_kind": "derived: %d SMs x 128 FP32 lanes x %.0f MHz (max SM clock)" % (sms, mhz),
+                "avg_launch_ms": launch_ms, "algorithmic_flop_per_launch": ops,
+                "algorithmic_bytes_per_launch": rows * (w.D * 4 + w.M)}
+
+    # Lloyd training on a sample (device I/O, 25 iterations by default)
+    n_tr = min(args.pq_train_rows, rows)
+    rng = np.random.default_rng(7)
+    pick = torch.from_numpy(np.sort(rng.choice(n_tr, w.K, replace=False))).to(device)
+    C0 = X[:n_tr][pick].reshape(w.K, w.M, w.ds).permute(1, 0, 2).contiguous()
+    C1 = torch.empty_like(C0)
+    obj = torch.empty((args.pq_iters, w.M), dtype=torch.float64, device=device)
+    ifvs.ifvs_pq_train(X[:n_tr], C0, 1, device=local, C_out=C1, objective=obj[:1], flags=dio,
+                       stream=sptr)
+    torch.cuda.synchronize()
+    t1 = time.perf_counter()
+    ifvs.ifvs_pq_train(X[:n_tr], C0, args.pq_iters, device=local, C_out=C1, objective=obj,
+                       flags=dio, stream=sptr)
+    torch.cuda.synchronize()
+    tr_s = time.perf_counter() - t1
+    o = obj.sum(1).cpu().numpy()
+    lloyd = {"rows": n_tr, "iters": args.pq_iters, "seconds": tr_s,
+             "ms_per_iter": tr_s * 1000.0 / max(1, args.pq_iters),
+             "objective_first": float(o[0]), "objective_last": float(o[-1]),
+             "objective_non_increasing": bool((np.diff(o) <= 1e-9 * np.abs(o[:-1])).all())}
+
+    # end to end: host vectors (pinned) in, host codes out, through the C ABI
+    e2e = None
+    if not args.no_e2e:
+        hX = X.cpu().pin_memory()
+        hXn = hX.numpy()
+        ifvs.ifvs_pq_encode(hXn, ix.codebook, device=local)
+        barrier(dist, device)
+        torch.cuda.synchronize()
+        t1 = time.perf_counter()
+        for _ in range(args.steps):
+            ifvs.ifvs_pq_encode(hXn, ix.codebook, device=local)
+        e_ms = (time.perf_counter() - t1) * 1000.0
+        barrier(dist, device)
+        e_ms = reduce_max(dist, e_ms, device)
+        e2e = {"value": world * args.steps * rows / (e_ms / 1000.0), "unit": "rows/s",
+               "h2d_bytes_per_step": rows * w.D * 4 + w.M * w.K * w.ds * 4,
+               "d2h_bytes_per_step": rows * w.M}
+        del hX
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        sample = 20_000
+        Xs = X[:sample].cpu().numpy()
+        t1 = time.perf_counter()
+        done = 0
+        while time.perf_counter() - t1 < 10.0:
+            oracle.pq_encode_f32(Xs, ix.codebook)
+            done += sample
+        sec = time.perf_counter() - t1
+        cpu = {"value": done / sec, "unit": "rows/s", "cores": 1, "kind": "oracle",
+               "sample": "float32 encode of the first %d rows, repeated for >= 10 s" % sample}
+
+    line = {
+        "metric": "PQ encode throughput (rows/s)", "value": world * args.steps * rows / (max_ms / 1000.0),
+        "unit": "rows/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": max_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded Gaussian-mixture vectors)",
+        "config": {"workload": "%s raw vectors, PQ encode in %d-row slices" % (w.name, rows),
+                   "rows_per_step": rows, "D": w.D, "M": w.M, "K": w.K,
+                   "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (%.1f GB per step)" % (rows * w.D * 4 / 1e9)},
+        "roofline": roofline, "lloyd": lloyd, "gpu_launches": args.steps, "clocks": clk,
+        "e2e": e2e, "cpu_baseline": cpu, "setup_s": round(t_gen, 1),
+    }
+    if rank == 0:
+        s = json.dumps(line)
+        print(s, flush=True)
+        if args.out:
+            with open(args.out, "w") as f:
+                f.write(s + "\n")
+    if dist is not None:
+        dist.destroy_process_group()
+
+
 def run_reference(args):
     """The oracle as it stands on the host cores, each step one query of the
     next bin over the first CPU_SAMPLE_ROWS rows, time scaled by N / rows."""
@@ -489,6 +651,8 @@ def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.mode == "pq":
+        run_pq(args)
     else:
         run_ifvs(args)
 

@@ -256,9 +256,15 @@ int ifvs_rerank(ifvs_index* ix, const float* queries, const int64_t* cand, int64
  *           every operation rounded on its own; ties to the smallest codeword
  *   dmin    [n][M] float32 out (that minimum), or NULL
  *   flags   IFVS_F_DEVICE_IO: all arrays are device pointers
+ *   stream  cudaStream_t for the work, or NULL (a stream of the call's own)
+ * With IFVS_F_DEVICE_IO and a non-NULL stream the call allocates nothing,
+ * only enqueues one kernel and returns; otherwise it returns when the
+ * results are written.  Errors: IFVS_ERR_ARG (NULL pointer, n < 0 or
+ * above 2^32 - 1, D not a multiple of M, unknown flag), IFVS_ERR_UNSUPPORTED
+ * (K outside 1..256, K x ds x 8 bytes above 200 KB), IFVS_ERR_OOM, IFVS_ERR_CUDA.
  */
 int ifvs_pq_encode(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
-                   const float* C_pq, uint8_t* codes, float* dmin, uint32_t flags);
+                   const float* C_pq, uint8_t* codes, float* dmin, uint32_t flags, void* stream);
 
 /*
  * ifvs_pq_train — `iters` Lloyd iterations per subspace from C_init
@@ -272,10 +278,14 @@ int ifvs_pq_encode(int32_t device, const float* X, int64_t n, int32_t D, int32_t
  *   C_out      [M][K][ds] float32 out
  *   objective  [iters][M] fp64 out (sum of the assignment's minimum
  *              distances at each iteration, before its update), or NULL
+ *   stream     cudaStream_t for the work, or NULL (a stream of the call's own)
+ * The call returns when C_out (and objective) are written; it reads the
+ * per-codeword counts back to the host once per iteration.  Errors as
+ * ifvs_pq_encode, plus IFVS_ERR_ARG for iters < 0.
  */
 int ifvs_pq_train(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
                   int32_t iters, const float* C_init, float* C_out, double* objective,
-                  uint32_t flags);
+                  uint32_t flags, void* stream);
 
 /*
  * ifvs_stage_times — device time (ms, from CUDA events recorded on the

@@ -8,6 +8,7 @@ resource usage (registers, spills, shared memory).
 from __future__ import annotations
 
 import concurrent.futures as cf
+import fcntl
 import os
 import shutil
 import subprocess
@@ -48,7 +49,18 @@ def _stale(target, deps):
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
+    """Compiles stale objects and relinks; concurrent callers (test workers)
+    serialise on a lock file so that none links a half-written object."""
     os.makedirs(OBJDIR, exist_ok=True)
+    with open(os.path.join(OBJDIR, ".lock"), "w") as lk:
+        fcntl.flock(lk, fcntl.LOCK_EX)
+        try:
+            return _build_locked(force, verbose)
+        finally:
+            fcntl.flock(lk, fcntl.LOCK_UN)
+
+
+def _build_locked(force: bool, verbose: bool) -> str:
     exe = nvcc()
     common = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                      "-I", INCLUDE, "-I", CSRC]
@@ -57,13 +69,17 @@ def build(force: bool = False, verbose: bool = False) -> str:
     hdrs = _deps()
     jobs = []
     for src in sources():
-        obj = os.path.join(OBJDIR, os.path.basename(src)[:-3] + ".o")
-        if force or verbose or _stale(obj, [src] + hdrs):
-            jobs.append([exe] + common + ["-c", src, "-o", obj])
+        name = os.path.basename(src)
+        obj = os.path.join(OBJDIR, name[:-3] + ".o")
+        if force or verbose or _stale(obj, [src] + hdrs + [os.path.abspath(__file__)]):
+            jobs.append(([exe] + common + ["-c", src, "-o", obj + ".tmp"], obj))
     objs = [os.path.join(OBJDIR, os.path.basename(s)[:-3] + ".o") for s in sources()]
 
-    def run(cmd):
+    def run(job):
+        cmd, obj = job
         p = subprocess.run(cmd, capture_output=True, text=True)
+        if p.returncode == 0:
+            os.replace(obj + ".tmp", obj)
         return cmd, p
 
     if jobs:

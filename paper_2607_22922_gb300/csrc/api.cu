@@ -918,11 +918,12 @@ namespace {
 struct PqArgs {
     int device = 0, num_sms = 0;
     cudaStream_t s = nullptr;
+    bool own_stream = false;
     std::vector<void*> owned;
     ~PqArgs() {
-        if (s) cudaStreamSynchronize(s);
+        if (s && (own_stream || !owned.empty())) cudaStreamSynchronize(s);
         for (void* p : owned) cudaFree(p);
-        if (s) cudaStreamDestroy(s);
+        if (s && own_stream) cudaStreamDestroy(s);
     }
     int alloc(void** p, size_t bytes) {
         cudaError_t e = cudaMalloc(p, bytes ? bytes : 16);
@@ -949,7 +950,7 @@ struct PqArgs {
 };
 
 int pq_check(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
-             uint32_t flags, PqArgs* a) {
+             uint32_t flags, void* stream, PqArgs* a) {
     if (n < 0) return set_err(IFVS_ERR_ARG, "n < 0");
     if (n > 0 && !X) return set_err(IFVS_ERR_ARG, "X is NULL");
     if (n > (int64_t)0xFFFFFFFFLL) return set_err(IFVS_ERR_ARG, "n = %lld above 2^32 - 1", (long long)n);
@@ -966,7 +967,12 @@ int pq_check(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, in
     if (device < 0 || device >= ndev) return set_err(IFVS_ERR_ARG, "device %d outside 0..%d", device, ndev - 1);
     a->device = device;
     CUDA_TRY(cudaDeviceGetAttribute(&a->num_sms, cudaDevAttrMultiProcessorCount, device));
-    CUDA_TRY(cudaStreamCreateWithFlags(&a->s, cudaStreamNonBlocking));
+    if (stream) {
+        a->s = (cudaStream_t)stream;
+    } else {
+        CUDA_TRY(cudaStreamCreateWithFlags(&a->s, cudaStreamNonBlocking));
+        a->own_stream = true;
+    }
     return 0;
 }
 
@@ -974,11 +980,11 @@ int pq_check(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, in
 
 extern "C" int ifvs_pq_encode(int32_t device, const float* X, int64_t n, int32_t D, int32_t M,
                               int32_t K, const float* C_pq, uint8_t* codes, float* dmin,
-                              uint32_t flags) {
+                              uint32_t flags, void* stream) {
     if (!C_pq || (n > 0 && !codes)) return set_err(IFVS_ERR_ARG, "C_pq / codes is NULL");
     DeviceGuard g(device);
     PqArgs a;
-    TRY(pq_check(device, X, n, D, M, K, flags, &a));
+    TRY(pq_check(device, X, n, D, M, K, flags, stream, &a));
     if (n == 0) return IFVS_OK;
     const bool dio = flags & IFVS_F_DEVICE_IO;
     const int ds = D / M;
@@ -1002,18 +1008,18 @@ extern "C" int ifvs_pq_encode(int32_t device, const float* X, int64_t n, int32_t
         CUDA_TRY(cudaMemcpyAsync(codes, dcodes, (size_t)n * M, cudaMemcpyDeviceToHost, a.s));
         if (dmin) CUDA_TRY(cudaMemcpyAsync(dmin, ddmin, sizeof(float) * n * M, cudaMemcpyDeviceToHost, a.s));
     }
-    CUDA_TRY(cudaStreamSynchronize(a.s));
+    if (a.own_stream || !dio) CUDA_TRY(cudaStreamSynchronize(a.s));
     return IFVS_OK;
 }
 
 extern "C" int ifvs_pq_train(int32_t device, const float* X, int64_t n, int32_t D, int32_t M,
                              int32_t K, int32_t iters, const float* C_init, float* C_out,
-                             double* objective, uint32_t flags) {
+                             double* objective, uint32_t flags, void* stream) {
     if (!C_init || !C_out) return set_err(IFVS_ERR_ARG, "C_init / C_out is NULL");
     if (iters < 0) return set_err(IFVS_ERR_ARG, "iters < 0");
     DeviceGuard g(device);
     PqArgs a;
-    TRY(pq_check(device, X, n, D, M, K, flags, &a));
+    TRY(pq_check(device, X, n, D, M, K, flags, stream, &a));
     const bool dio = flags & IFVS_F_DEVICE_IO;
     const int ds = D / M;
     const size_t cb_bytes = sizeof(float) * (size_t)M * K * ds;

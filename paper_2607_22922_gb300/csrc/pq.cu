@@ -3,7 +3,8 @@
 //
 // k_pq_assign: one thread per row; the whole codebook of the current
 // subspace sits in shared memory and every lane of a warp reads the same
-// codeword (broadcast).  The distance to a codeword is accumulated in
+// codeword (broadcast); two codewords are measured at once with packed
+// float32 differences and squares.  The distance to a codeword is accumulated in
 // float32 in a fixed order — s = s + (x_t - c_t)^2 for t ascending, every
 // operation rounded on its own (no fused multiply-add) — and the argmin
 // keeps the smallest codeword on ties, so the codes are bit-exact with the
@@ -22,34 +23,119 @@ namespace ifvs {
 
 constexpr int kPqThreads = 256;
 
+// packed float32 pairs: each half is rounded on its own, as two scalar
+// operations with the same rounding would be (explicit .rn: never fused)
+__device__ __forceinline__ unsigned long long f2_sub(unsigned long long a, unsigned long long b) {
+    unsigned long long d;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ unsigned long long f2_mul(unsigned long long a, unsigned long long b) {
+    unsigned long long d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ unsigned long long f2_dup(float x) {
+    unsigned long long d;
+    asm("mov.b64 %0, {%1, %1};" : "=l"(d) : "f"(x));
+    return d;
+}
+__device__ __forceinline__ void f2_split(unsigned long long v, float& lo, float& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+
+// Codewords 2p and 2p+1 of one subspace are interleaved in shared memory as
+// [p][t][2], so one 16-byte broadcast load gives both codewords' values at
+// t and t+1; an odd K keeps its last codeword in plain [t] order after the
+// pairs.  Differences and squares of both codewords run packed; the two
+// sums stay scalar: a packed multiply feeding a packed add is compiled into
+// a fused multiply-add (one rounding instead of two) even with explicit
+// .rn, volatile asm and -fmad=false, which would change the float32 sums.
+// The first term needs no add (0 + sq = sq exactly).
+template <int DS>
+__device__ __forceinline__ void pair_dist(const float* __restrict__ cbp,
+                                          const unsigned long long (&xx)[DS], float& s0,
+                                          float& s1) {
+    static_assert(DS % 2 == 0, "pairs of dimensions");
+    const ulonglong2* c = reinterpret_cast<const ulonglong2*>(cbp);
+#pragma unroll
+    for (int t = 0; t < DS; t += 2) {
+        const ulonglong2 cc = c[t / 2];
+        const unsigned long long d0 = f2_sub(xx[t], cc.x);
+        const unsigned long long d1 = f2_sub(xx[t + 1], cc.y);
+        float a0, b0, a1, b1;
+        f2_split(f2_mul(d0, d0), a0, b0);
+        f2_split(f2_mul(d1, d1), a1, b1);
+        if (t == 0) {
+            s0 = a0;
+            s1 = b0;
+        } else {
+            s0 = __fadd_rn(s0, a0);
+            s1 = __fadd_rn(s1, b0);
+        }
+        s0 = __fadd_rn(s0, a1);
+        s1 = __fadd_rn(s1, b1);
+    }
+}
+
 template <int DS>
 __global__ void __launch_bounds__(kPqThreads) k_pq_assign(const float* __restrict__ X, int64_t n,
                                                           int D, int M, int K,
                                                           const float* __restrict__ C,
                                                           uint8_t* __restrict__ codes,
                                                           float* __restrict__ dmin) {
-    extern __shared__ __align__(16) float cb[];   // K * DS floats of one subspace
+    extern __shared__ __align__(16) float cb[];   // K * DS floats of one subspace, pairs interleaved
     const int64_t i = (int64_t)blockIdx.x * kPqThreads + threadIdx.x;
+    const int KP = K >> 1;
     for (int m = 0; m < M; ++m) {
         __syncthreads();
-        for (int e = threadIdx.x; e < K * DS; e += kPqThreads) cb[e] = C[(int64_t)m * K * DS + e];
+        for (int e = threadIdx.x; e < K * DS; e += kPqThreads) {
+            const int k = e / DS, t = e - k * DS;
+            const int dst = k < 2 * KP ? ((k >> 1) * DS + t) * 2 + (k & 1) : e;
+            cb[dst] = C[(int64_t)m * K * DS + e];
+        }
         __syncthreads();
         if (i >= n) continue;
-        float x[DS];
+        unsigned long long xx[DS];
 #pragma unroll
-        for (int t = 0; t < DS; ++t) x[t] = __ldg(X + i * D + m * DS + t);
+        for (int t = 0; t < DS; ++t) xx[t] = f2_dup(__ldg(X + i * D + m * DS + t));
         float best = 0.f;
         int bk = 0;
-        for (int k = 0; k < K; ++k) {
+        if (KP > 0) {
+            float s0, s1;
+            pair_dist<DS>(cb, xx, s0, s1);
+            best = s0;
+            if (s1 < best) {
+                best = s1;
+                bk = 1;
+            }
+        }
+#pragma unroll 4
+        for (int p = 1; p < KP; ++p) {
+            float s0, s1;
+            pair_dist<DS>(cb + p * DS * 2, xx, s0, s1);
+            if (s0 < best) {
+                best = s0;
+                bk = 2 * p;
+            }
+            if (s1 < best) {
+                best = s1;
+                bk = 2 * p + 1;
+            }
+        }
+        if (K & 1) {
+            const float* c = cb + (K - 1) * DS;
             float s = 0.f;
 #pragma unroll
             for (int t = 0; t < DS; ++t) {
-                const float d = __fsub_rn(x[t], cb[k * DS + t]);
+                float x, unused;
+                f2_split(xx[t], x, unused);
+                const float d = __fsub_rn(x, c[t]);
                 s = __fadd_rn(s, __fmul_rn(d, d));
             }
-            if (k == 0 || s < best) {
+            if (KP == 0 || s < best) {
                 best = s;
-                bk = k;
+                bk = K - 1;
             }
         }
         codes[i * M + m] = (uint8_t)bk;

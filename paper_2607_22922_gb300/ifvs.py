@@ -54,8 +54,8 @@ def _load():
         "ifvs_scan_topk": (C.c_int, [P, P, P, I64, I32, P, P, P]),
         "ifvs_rerank": (C.c_int, [P, P, P, I64, I32, I32, P, P, P]),
         "ifvs_scan_topk_static": (C.c_int, [P, P, P, I64, I32, P, P, P]),
-        "ifvs_pq_encode": (C.c_int, [I32, P, I64, I32, I32, I32, P, P, P, U32]),
-        "ifvs_pq_train": (C.c_int, [I32, P, I64, I32, I32, I32, I32, P, P, P, U32]),
+        "ifvs_pq_encode": (C.c_int, [I32, P, I64, I32, I32, I32, P, P, P, U32, P]),
+        "ifvs_pq_train": (C.c_int, [I32, P, I64, I32, I32, I32, I32, P, P, P, U32, P]),
         "ifvs_stage_times": (C.c_int, [P, P, P, I32]),
         "ifvs_canonical_predicate": (C.c_int, [P, P, I32, P, P, P]),
         "ifvs_index_info": (C.c_int, [P, P]),
@@ -242,29 +242,46 @@ def ifvs_scan_topk_static(ix, lut, bitmaps, k, ids, dists, stream=None):
     return ids, dists
 
 
-def ifvs_pq_encode(X, C_pq, device=0, want_dmin=False):
-    """codes [n][M] uint8 (and dmin [n][M] float32) for host arrays."""
-    X = _host(X, np.float32)
-    C_pq = _host(C_pq, np.float32)
-    n, D = X.shape
-    M, K, ds = C_pq.shape
-    codes = np.empty((n, M), np.uint8)
-    dmin = np.empty((n, M), np.float32) if want_dmin else None
-    _check(_lib.ifvs_pq_encode(device, _ptr(X), n, D, M, K, _ptr(C_pq), _ptr(codes), _ptr(dmin), 0))
-    return (codes, dmin) if want_dmin else codes
+def ifvs_pq_encode(X, C_pq, device=0, want_dmin=False, codes=None, dmin=None, flags=0,
+                   stream=None):
+    """Host mode (default): numpy in, codes [n][M] uint8 (and dmin [n][M]
+    float32) out.  With IFVS_F_DEVICE_IO in ``flags``, X, C_pq, ``codes``
+    (and ``dmin``, if wanted) are preallocated device tensors; with a stream
+    the call only enqueues the kernel."""
+    dio = bool(flags & IFVS_F_DEVICE_IO)
+    if not dio:
+        X = _host(X, np.float32)
+        C_pq = _host(C_pq, np.float32)
+    n, D = int(X.shape[0]), int(X.shape[1])
+    M, K, ds = (int(v) for v in C_pq.shape)
+    if not dio:
+        codes = np.empty((n, M), np.uint8)
+        dmin = np.empty((n, M), np.float32) if want_dmin else None
+    elif codes is None:
+        raise ValueError("device I/O needs a preallocated codes tensor")
+    _check(_lib.ifvs_pq_encode(device, _ptr(X), n, D, M, K, _ptr(C_pq), _ptr(codes), _ptr(dmin),
+                               flags, stream))
+    return (codes, dmin) if (want_dmin or dmin is not None) else codes
 
 
-def ifvs_pq_train(X, C_init, iters, device=0):
-    """Lloyd iterations from C_init [M][K][ds]; returns (C_out, objective [iters][M])."""
-    X = _host(X, np.float32)
-    C_init = _host(C_init, np.float32)
-    n, D = X.shape
-    M, K, ds = C_init.shape
-    C_out = np.empty_like(C_init)
-    obj = np.empty((max(iters, 1), M), np.float64)
+def ifvs_pq_train(X, C_init, iters, device=0, C_out=None, objective=None, flags=0, stream=None):
+    """Lloyd iterations from C_init [M][K][ds]; returns (C_out, objective
+    [iters][M]).  With IFVS_F_DEVICE_IO, X, C_init, ``C_out`` and ``objective``
+    (or None) are device tensors."""
+    dio = bool(flags & IFVS_F_DEVICE_IO)
+    if not dio:
+        X = _host(X, np.float32)
+        C_init = _host(C_init, np.float32)
+    n, D = int(X.shape[0]), int(X.shape[1])
+    M, K, ds = (int(v) for v in C_init.shape)
+    if not dio:
+        C_out = np.empty_like(C_init)
+        objective = np.empty((max(iters, 1), M), np.float64)
+    elif C_out is None:
+        raise ValueError("device I/O needs a preallocated C_out tensor")
     _check(_lib.ifvs_pq_train(device, _ptr(X), n, D, M, K, iters, _ptr(C_init), _ptr(C_out),
-                              _ptr(obj), 0))
-    return C_out, obj[:iters]
+                              _ptr(objective), flags, stream))
+    return C_out, (objective[:iters] if objective is not None else None)
 
 
 def ifvs_rerank(ix, queries, cand, k, flags=0):

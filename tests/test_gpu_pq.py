@@ -86,3 +86,27 @@ def test_lloyd_iterations_track_the_oracle(ifvs, orc):
         np.testing.assert_allclose(gobj[it], robj, rtol=1e-9)
     assert (np.diff(gobj, axis=0) <= 1e-6 * gobj[:-1]).all()
     assert _ulp_close(G, R).mean() > 0.999
+
+
+def test_device_io_on_a_caller_stream(ifvs, orc):
+    import torch
+    X, C0 = _data(synth.WORKLOADS["gmm10k-d128-m16"], 9_999, 6)
+    dev = torch.device("cuda", 0)
+    s = torch.cuda.Stream(device=dev)
+    Xd, Cd = torch.from_numpy(X).to(dev), torch.from_numpy(C0).to(dev)
+    codes = torch.empty((len(X), C0.shape[0]), dtype=torch.uint8, device=dev)
+    dmin = torch.empty((len(X), C0.shape[0]), dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+    ifvs.ifvs_pq_encode(Xd, Cd, codes=codes, dmin=dmin, flags=ifvs.IFVS_F_DEVICE_IO,
+                        stream=s.cuda_stream)
+    s.synchronize()
+    rc, rd = orc.pq_encode_f32(X, C0)
+    np.testing.assert_array_equal(codes.cpu().numpy(), rc)
+    np.testing.assert_array_equal(dmin.cpu().numpy(), rd)
+    C1 = torch.empty_like(Cd)
+    obj = torch.empty((2, C0.shape[0]), dtype=torch.float64, device=dev)
+    ifvs.ifvs_pq_train(Xd, Cd, 2, C_out=C1, objective=obj, flags=ifvs.IFVS_F_DEVICE_IO,
+                       stream=s.cuda_stream)
+    H1, hobj = ifvs.ifvs_pq_train(X, C0, 2)
+    np.testing.assert_array_equal(C1.cpu().numpy(), H1)
+    np.testing.assert_array_equal(obj.cpu().numpy(), hobj)
