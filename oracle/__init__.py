@@ -84,6 +84,13 @@ def lib():
             "orc_sdc": (D, [P, P, P, I32_, I32_, I32_]),
             "orc_pq_encode_f32": (None, [P, I64, I32_, I32_, I32_, P, P, P]),
             "orc_lloyd_step": (None, [P, I64, I32_, I32_, I32_, P, P, P, P]),
+            "orc_train_loss": (D, [P, I32_, I32_, I32_, P, P, I64, I32_, I32_, P, P, P, P, P,
+                                   I64, P, I32_, I32_, D, D, P, P, P]),
+            "orc_mine_negatives": (C.c_int, [P, I64, I32_, I32_, I32_, P, P, I32_, P, P, I64,
+                                             I32_, I32_, P, P, P, P, P, I64, P, I32_, I32_, P]),
+            "orc_train_step": (C.c_int, [P, I64, I32_, I32_, I32_, P, P, I32_, P, P, I64, I32_,
+                                         I32_, P, P, P, P, P, I64, P, I32_, I32_, D, D, D, P, P,
+                                         P, P, P]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -381,3 +388,74 @@ def lloyd_step(X, C_in):
     lib().orc_lloyd_step(_p(X), X.shape[0], X.shape[1], M, K, _p(C_in), _p(C_out), _p(codes),
                          _p(obj))
     return C_out, codes, obj
+
+
+# ---------------------------------------------------------------- learning (§2 "Learning")
+
+def _train_common(codes, C_pq, bank, W, seeds, wz, queries, preds):
+    codes = _c(codes, np.uint8)
+    C_pq = _c(C_pq, np.float32)
+    M = codes.shape[1]
+    _, K, ds = C_pq.shape
+    D = M * ds
+    queries = _c(queries, np.float32).reshape(-1, D)
+    return (codes, C_pq, _c(bank, np.float32), _c(W, np.float32), _c(seeds, np.uint64),
+            _c(wz, np.float32).reshape(D), queries, _preds(preds), M, K, ds, D)
+
+
+def train_loss(codes, C_pq, bank, W, seeds, wz, queries, preds, cand, P, tau, lam,
+               grads=True):
+    """Loss of the queries with candidate lists cand [nq][V] (positives first,
+    P of them; -1 = absent) and one shared w_z [D]; with ``grads`` also
+    dL/dbank [B][M r], dL/dW [M][r][K][ds], dL/dw_z [D] (fp64)."""
+    codes, C_pq, bank, W, seeds, wz, queries, preds, M, K, ds, D = _train_common(
+        codes, C_pq, bank, W, seeds, wz, queries, preds)
+    cand = _c(cand, np.int64)
+    nq, V = cand.shape
+    B, Mr = bank.shape
+    r = W.shape[1]
+    gb = np.zeros((B, Mr)) if grads else None
+    gW = np.zeros(W.shape) if grads else None
+    gz = np.zeros(D) if grads else None
+    L = lib().orc_train_loss(_p(codes), M, K, ds, _p(C_pq), _p(bank), B, len(seeds), r, _p(W),
+                             _p(seeds), _p(wz), _p(queries), _p(preds), nq, _p(cand), P, V,
+                             float(tau), float(lam), _p(gb), _p(gW), _p(gz))
+    return (L, gb, gW, gz) if grads else L
+
+
+def mine_negatives(codes, cols, C_pq, bank, W, seeds, wz, queries, preds, pos, n_neg):
+    """Per query the n_neg best non-positive rows of the pool (-1 padded)."""
+    codes, C_pq, bank, W, seeds, wz, queries, preds, M, K, ds, D = _train_common(
+        codes, C_pq, bank, W, seeds, wz, queries, preds)
+    pos = _c(pos, np.int64)
+    nq, P = pos.shape
+    cs = _Cols(cols)
+    neg = np.zeros((nq, n_neg), np.int64)
+    rc = lib().orc_mine_negatives(_p(codes), codes.shape[0], M, K, ds, cs.ptrs, _p(cs.types),
+                                  cs.n, _p(C_pq), _p(bank), bank.shape[0], len(seeds),
+                                  W.shape[1], _p(W), _p(seeds), _p(wz), _p(queries), _p(preds),
+                                  nq, _p(pos), P, n_neg, _p(neg))
+    if rc != 0:
+        raise ValueError("invalid predicate")
+    return neg
+
+
+def train_step(codes, cols, C_pq, bank, W, seeds, wz, queries, preds, pos, n_neg, tau, lam, lr):
+    """Mining, loss, gradient and one SGD step; returns (loss, bank', W',
+    w_z', negatives)."""
+    codes, C_pq, bank, W, seeds, wz, queries, preds, M, K, ds, D = _train_common(
+        codes, C_pq, bank, W, seeds, wz, queries, preds)
+    pos = _c(pos, np.int64)
+    nq, P = pos.shape
+    cs = _Cols(cols)
+    b2, W2, z2 = np.empty_like(bank), np.empty_like(W), np.empty_like(wz)
+    neg = np.zeros((nq, n_neg), np.int64)
+    loss = np.zeros(1)
+    rc = lib().orc_train_step(_p(codes), codes.shape[0], M, K, ds, cs.ptrs, _p(cs.types), cs.n,
+                              _p(C_pq), _p(bank), bank.shape[0], len(seeds), W.shape[1], _p(W),
+                              _p(seeds), _p(wz), _p(queries), _p(preds), nq, _p(pos), P, n_neg,
+                              float(tau), float(lam), float(lr), _p(b2), _p(W2), _p(z2), _p(neg),
+                              _p(loss))
+    if rc != 0:
+        raise ValueError("invalid predicate")
+    return float(loss[0]), b2, W2, z2, neg

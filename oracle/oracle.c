@@ -560,3 +560,217 @@ void orc_lloyd_step(const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
     free(sum);
     free(cnt);
 }
+
+/* ------------------------------------------------------------------ */
+/* Learning C_iFVS and w_f: §2 "Learning".  The paper fixes the initial
+ * state (alpha = 0, i.e. a zero bank, and w_f = 1), the positives (the
+ * query's ground-truth rows), the hard negatives (the highest-scoring rows of
+ * the pool that are not ground truth, under the current parameters), an
+ * anchor term that keeps C_iFVS close to C_PQ, and which parameters move
+ * (bank, W, w_f; C_PQ and the codes stay fixed).  Readings for what it
+ * leaves open:
+ *   score = -dist (the printed score minus sum w q^2, a per-query constant
+ *   that no softmax sees);
+ *   per positive g of a query, softmax cross-entropy of g against the
+ *   query's negatives N at temperature tau,
+ *     l_g = dist_g / tau + log( exp(-dist_g / tau) + sum_{n in N} exp(-dist_n / tau) ),
+ *   averaged over the query's positives, plus lambda * ||Delta||^2 summed
+ *   over all M K ds entries (= ||C_iFVS - C_PQ||^2);
+ *   L = the mean of that over the queries;
+ *   w_f = softplus(w_z) with one learned w_z [D] for all queries (the
+ *   predicate Transformer that would give w_z per predicate is not given);
+ *   optimiser: plain SGD, theta <- theta - lr * dL/dtheta. */
+
+static double sigmoid(double x) {
+    if (x >= 0) return 1.0 / (1.0 + exp(-x));
+    double e = exp(x);
+    return e / (1.0 + e);
+}
+
+double orc_train_loss(const uint8_t* codes, int32_t M, int32_t K, int32_t ds,
+                      const float* C_pq, const float* bank, int64_t B, int32_t h, int32_t r,
+                      const float* W, const uint64_t* seeds, const float* wz,
+                      const float* queries, const orc_predicate* preds, int64_t nq,
+                      const int64_t* cand, int32_t P, int32_t V, double tau, double lambda,
+                      double* g_bank, double* g_W, double* g_wz) {
+    const int32_t D = M * ds, Mr = M * r;
+    const int64_t nC = (int64_t)M * K * ds, nW = (int64_t)M * r * K * ds;
+    uint32_t* idx = (uint32_t*)malloc(sizeof(uint32_t) * (size_t)h);
+    double* alpha = (double*)malloc(sizeof(double) * (size_t)Mr);
+    double* wf = (double*)malloc(sizeof(double) * (size_t)D);
+    double* C = (double*)malloc(sizeof(double) * (size_t)nC);
+    double* delta = (double*)malloc(sizeof(double) * (size_t)nC);
+    double* lut = (double*)malloc(sizeof(double) * (size_t)M * K);
+    double* dist = (double*)malloc(sizeof(double) * (size_t)(V > 0 ? V : 1));
+    double* gam = (double*)malloc(sizeof(double) * (size_t)(V > 0 ? V : 1));
+    double* gC = (double*)malloc(sizeof(double) * (size_t)nC);
+    double* gw = (double*)malloc(sizeof(double) * (size_t)D);
+    double* galpha = (double*)malloc(sizeof(double) * (size_t)Mr);
+    const int grads = (g_bank != NULL && g_W != NULL && g_wz != NULL);
+    if (grads) {
+        for (int64_t e = 0; e < B * Mr; ++e) g_bank[e] = 0.0;
+        for (int64_t e = 0; e < nW; ++e) g_W[e] = 0.0;
+        for (int32_t d = 0; d < D; ++d) g_wz[d] = 0.0;
+    }
+    orc_filter_weights(wz, D, wf);
+    double L = 0.0;
+    for (int64_t qi = 0; qi < nq; ++qi) {
+        const float* q = queries + qi * D;
+        const int64_t* cq = cand + qi * V;
+        orc_fingerprint(q, D, &preds[qi], seeds, h, B, idx);
+        orc_alpha(bank, B, Mr, idx, h, alpha);
+        /* Delta[m][k][t] = sum_j alpha[m][j] W[m][j][k][t]; C = C_PQ + Delta */
+        for (int32_t m = 0; m < M; ++m)
+            for (int32_t k = 0; k < K; ++k)
+                for (int32_t t = 0; t < ds; ++t) {
+                    double s = 0.0;
+                    for (int32_t j = 0; j < r; ++j)
+                        s += alpha[m * r + j] * (double)W[(((int64_t)m * r + j) * K + k) * ds + t];
+                    delta[((int64_t)m * K + k) * ds + t] = s;
+                }
+        orc_condition(C_pq, alpha, W, M, K, ds, r, C);
+        orc_lut(q, C, wf, M, K, ds, lut);
+        for (int32_t v = 0; v < V; ++v) {
+            dist[v] = cq[v] >= 0 ? orc_adc(lut, codes + cq[v] * M, M, K) : 0.0;
+            gam[v] = 0.0;
+        }
+        /* positive term: softmax cross-entropy of each positive against N */
+        int32_t npos = 0;
+        double lpos = 0.0;
+        for (int32_t g = 0; g < P; ++g) {
+            if (cq[g] < 0) continue;
+            ++npos;
+            double dmin = dist[g];
+            for (int32_t n = P; n < V; ++n)
+                if (cq[n] >= 0 && dist[n] < dmin) dmin = dist[n];
+            double Z = exp(-(dist[g] - dmin) / tau);
+            for (int32_t n = P; n < V; ++n)
+                if (cq[n] >= 0) Z += exp(-(dist[n] - dmin) / tau);
+            lpos += dist[g] / tau - dmin / tau + log(Z);
+            /* d l_g / d dist_g = (1 - p_g) / tau;  d l_g / d dist_n = -p_n / tau */
+            gam[g] += (1.0 - exp(-(dist[g] - dmin) / tau) / Z) / tau;
+            for (int32_t n = P; n < V; ++n)
+                if (cq[n] >= 0) gam[n] -= exp(-(dist[n] - dmin) / tau) / Z / tau;
+        }
+        if (npos > 0) {
+            lpos /= npos;
+            for (int32_t v = 0; v < V; ++v) gam[v] /= npos;
+        }
+        double anchor = 0.0;
+        for (int64_t e = 0; e < nC; ++e) anchor += delta[e] * delta[e];
+        L += (lpos + lambda * anchor) / (double)nq;
+        if (!grads) continue;
+        /* dL_q/dC at the candidates' codewords and dL_q/dw_f */
+        for (int64_t e = 0; e < nC; ++e) gC[e] = 0.0;
+        for (int32_t d = 0; d < D; ++d) gw[d] = 0.0;
+        for (int32_t v = 0; v < V; ++v) {
+            if (cq[v] < 0) continue;
+            const uint8_t* code = codes + cq[v] * M;
+            for (int32_t m = 0; m < M; ++m)
+                for (int32_t t = 0; t < ds; ++t) {
+                    const int64_t e = ((int64_t)m * K + code[m]) * ds + t;
+                    const double diff = (double)q[m * ds + t] - C[e];
+                    gC[e] += gam[v] * (-2.0 * wf[m * ds + t] * diff);
+                    gw[m * ds + t] += gam[v] * diff * diff;
+                }
+        }
+        /* dL_q/dDelta = dL_q/dC + 2 lambda Delta; chain rule through Delta = alpha . W */
+        for (int32_t e = 0; e < Mr; ++e) galpha[e] = 0.0;
+        for (int32_t m = 0; m < M; ++m)
+            for (int32_t k = 0; k < K; ++k)
+                for (int32_t t = 0; t < ds; ++t) {
+                    const int64_t e = ((int64_t)m * K + k) * ds + t;
+                    const double gD = gC[e] + 2.0 * lambda * delta[e];
+                    for (int32_t j = 0; j < r; ++j) {
+                        const int64_t w = (((int64_t)m * r + j) * K + k) * ds + t;
+                        galpha[m * r + j] += gD * (double)W[w];
+                        g_W[w] += alpha[m * r + j] * gD / (double)nq;
+                    }
+                }
+        /* alpha = sum of the fetched bank rows: each fetch receives dL/dalpha */
+        for (int32_t i = 0; i < h; ++i)
+            for (int32_t e = 0; e < Mr; ++e) g_bank[(int64_t)idx[i] * Mr + e] += galpha[e] / (double)nq;
+        /* w_f = softplus(w_z): dw_f/dw_z = sigmoid(w_z) */
+        for (int32_t d = 0; d < D; ++d) g_wz[d] += gw[d] * sigmoid((double)wz[d]) / (double)nq;
+    }
+    free(idx);
+    free(alpha);
+    free(wf);
+    free(C);
+    free(delta);
+    free(lut);
+    free(dist);
+    free(gam);
+    free(gC);
+    free(gw);
+    free(galpha);
+    return L;
+}
+
+int orc_mine_negatives(const uint8_t* codes, int64_t N, int32_t M, int32_t K, int32_t ds,
+                       const void* const* cols, const int32_t* types, int32_t n_attrs,
+                       const float* C_pq, const float* bank, int64_t B, int32_t h, int32_t r,
+                       const float* W, const uint64_t* seeds, const float* wz,
+                       const float* queries, const orc_predicate* preds, int64_t nq,
+                       const int64_t* pos, int32_t P, int32_t n_neg, int64_t* neg) {
+    const int32_t D = M * ds, kk = P + n_neg;
+    float* wzq = (float*)calloc((size_t)(nq > 0 ? nq : 1) * D, sizeof(float));
+    int64_t* ids = (int64_t*)malloc(sizeof(int64_t) * (size_t)(nq > 0 ? nq : 1) * (kk > 0 ? kk : 1));
+    double* dd = (double*)malloc(sizeof(double) * (size_t)(nq > 0 ? nq : 1) * (kk > 0 ? kk : 1));
+    for (int64_t qi = 0; qi < nq; ++qi)
+        for (int32_t d = 0; d < D; ++d) wzq[qi * D + d] = wz[d];
+    int rc = orc_search(codes, N, M, K, ds, cols, types, n_attrs, C_pq, bank, B, h, r, W, seeds,
+                        queries, preds, wzq, nq, kk, ids, dd, NULL, NULL, NULL, NULL, NULL);
+    /* the best n_neg of the pool that are not positives: at most P of the
+     * top P + n_neg can be positives, so the rest of that list suffices */
+    for (int64_t qi = 0; qi < nq && rc == 0; ++qi) {
+        int32_t got = 0;
+        for (int32_t j = 0; j < kk && got < n_neg; ++j) {
+            const int64_t id = ids[qi * kk + j];
+            if (id < 0) break;
+            int is_pos = 0;
+            for (int32_t g = 0; g < P; ++g)
+                if (pos[qi * P + g] == id) is_pos = 1;
+            if (!is_pos) neg[qi * n_neg + got++] = id;
+        }
+        for (; got < n_neg; ++got) neg[qi * n_neg + got] = -1;
+    }
+    free(wzq);
+    free(ids);
+    free(dd);
+    return rc;
+}
+
+int orc_train_step(const uint8_t* codes, int64_t N, int32_t M, int32_t K, int32_t ds,
+                   const void* const* cols, const int32_t* types, int32_t n_attrs,
+                   const float* C_pq, const float* bank, int64_t B, int32_t h, int32_t r,
+                   const float* W, const uint64_t* seeds, const float* wz,
+                   const float* queries, const orc_predicate* preds, int64_t nq,
+                   const int64_t* pos, int32_t P, int32_t n_neg, double tau, double lambda,
+                   double lr, float* bank_out, float* W_out, float* wz_out, int64_t* neg,
+                   double* loss) {
+    const int32_t D = M * ds, V = P + n_neg;
+    const int64_t nB = B * M * r, nW = (int64_t)M * r * K * ds;
+    int64_t* cand = (int64_t*)malloc(sizeof(int64_t) * (size_t)(nq > 0 ? nq : 1) * (V > 0 ? V : 1));
+    double* gb = (double*)malloc(sizeof(double) * (size_t)nB);
+    double* gW = (double*)malloc(sizeof(double) * (size_t)nW);
+    double* gz = (double*)malloc(sizeof(double) * (size_t)D);
+    int rc = orc_mine_negatives(codes, N, M, K, ds, cols, types, n_attrs, C_pq, bank, B, h, r, W,
+                                seeds, wz, queries, preds, nq, pos, P, n_neg, neg);
+    if (rc == 0) {
+        for (int64_t qi = 0; qi < nq; ++qi) {
+            for (int32_t g = 0; g < P; ++g) cand[qi * V + g] = pos[qi * P + g];
+            for (int32_t n = 0; n < n_neg; ++n) cand[qi * V + P + n] = neg[qi * n_neg + n];
+        }
+        *loss = orc_train_loss(codes, M, K, ds, C_pq, bank, B, h, r, W, seeds, wz, queries, preds,
+                               nq, cand, P, V, tau, lambda, gb, gW, gz);
+        for (int64_t e = 0; e < nB; ++e) bank_out[e] = (float)((double)bank[e] - lr * gb[e]);
+        for (int64_t e = 0; e < nW; ++e) W_out[e] = (float)((double)W[e] - lr * gW[e]);
+        for (int32_t d = 0; d < D; ++d) wz_out[d] = (float)((double)wz[d] - lr * gz[d]);
+    }
+    free(cand);
+    free(gb);
+    free(gW);
+    free(gz);
+    return rc;
+}

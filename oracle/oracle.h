@@ -17,7 +17,9 @@
  *   §2, stage 1 Filter    predicate over every row's attributes -> pool P
  *   §2, stage 2 Rank      score(v) = sum_m sum_d [2 w q C - w C^2]
  *   §2, stage 3 Select    top-k by score
- *   §2, "Learning"        alpha = 0, w_f = 1 reduces to plain PQ
+ *   §2, "Learning"        alpha = 0, w_f = 1 reduces to plain PQ; the
+ *                         training of bank, W and w_f (positives, mined
+ *                         hard negatives, anchor to C_PQ)
  *   §3.1                  exact filtered ground truth over passing rows
  *   §3.2 B1               Pre_IndexFlatL2 / Pre_IndexFlatL2_PQ /
  *                         Pre_IndexPQ_ADC / Pre_IndexPQ_SDC
@@ -151,6 +153,38 @@ void orc_lloyd_step(const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
  * first; dist = sum_m ||C[m][cq[m]] - C[m][cv[m]]||^2. */
 double orc_sdc(const double* C, const uint8_t* cq, const uint8_t* cv, int32_t M, int32_t K,
                int32_t ds);
+
+/* Learning C_iFVS and w_f (§2 "Learning"); the readings are stated in
+ * oracle.c.  orc_train_loss: the loss of nq queries whose candidate lists
+ * cand [nq][V] hold the positives first (P of them) and then the negatives
+ * (id -1 = absent), with one shared w_z [D] (non-NULL); if g_bank [B][M r],
+ * g_W [M][r][K][ds] and g_wz [D] are all non-NULL they receive dL/d(bank,
+ * W, w_z). */
+double orc_train_loss(const uint8_t* codes, int32_t M, int32_t K, int32_t ds,
+                      const float* C_pq, const float* bank, int64_t B, int32_t h, int32_t r,
+                      const float* W, const uint64_t* seeds, const float* wz,
+                      const float* queries, const orc_predicate* preds, int64_t nq,
+                      const int64_t* cand, int32_t P, int32_t V, double tau, double lambda,
+                      double* g_bank, double* g_W, double* g_wz);
+/* Hard negatives: per query the n_neg rows of the pool with the smallest
+ * current distance that are not among its P positives (pos [nq][P], -1 =
+ * absent), ties to the smaller row; -1 where the pool runs out. */
+int orc_mine_negatives(const uint8_t* codes, int64_t N, int32_t M, int32_t K, int32_t ds,
+                       const void* const* cols, const int32_t* types, int32_t n_attrs,
+                       const float* C_pq, const float* bank, int64_t B, int32_t h, int32_t r,
+                       const float* W, const uint64_t* seeds, const float* wz,
+                       const float* queries, const orc_predicate* preds, int64_t nq,
+                       const int64_t* pos, int32_t P, int32_t n_neg, int64_t* neg);
+/* One training step: mine negatives, loss and gradient, then plain SGD on
+ * bank, W and w_z (new values rounded to float32 into the *_out arrays). */
+int orc_train_step(const uint8_t* codes, int64_t N, int32_t M, int32_t K, int32_t ds,
+                   const void* const* cols, const int32_t* types, int32_t n_attrs,
+                   const float* C_pq, const float* bank, int64_t B, int32_t h, int32_t r,
+                   const float* W, const uint64_t* seeds, const float* wz,
+                   const float* queries, const orc_predicate* preds, int64_t nq,
+                   const int64_t* pos, int32_t P, int32_t n_neg, double tau, double lambda,
+                   double lr, float* bank_out, float* W_out, float* wz_out, int64_t* neg,
+                   double* loss);
 
 #ifdef __cplusplus
 }

@@ -3,7 +3,7 @@
 Each case plants one mistake in a copy of oracle/oracle.c (a dropped term, a
 wrong sign, index or bound, a transposed operand, a changed constant, a
 reversed tie rule), builds it, and runs tests/test_oracle_pins.py against
-it: at least one pin must fail.  Nothing here touches the GPU path.
+it (and tests/test_oracle_train_pins.py): at least one pin must fail.  Nothing here touches the GPU path.
 """
 import os
 import shutil
@@ -61,6 +61,24 @@ MUTATIONS = {
     "Lloyd keeps the old centroid": ("Co[(int64_t)c * ds + t] = cnt[c] > 0 ? (float)(sum[(int64_t)c * ds + t] / (double)cnt[c])",
                                      "Co[(int64_t)c * ds + t] = cnt[c] > 0 ? Ci[(int64_t)c * ds + t]"),
     "Lloyd reseeds with the nearest point": ("if (dmin[i * M + m] > dmin[far * M + m]) far = i;", "if (dmin[i * M + m] < dmin[far * M + m]) far = i;"),
+    'train: negatives pushed the wrong way': ('if (cq[n] >= 0) gam[n] -= exp(-(dist[n] - dmin) / tau) / Z / tau;',
+                                              'if (cq[n] >= 0) gam[n] += exp(-(dist[n] - dmin) / tau) / Z / tau;'),
+    'train: anchor gradient halved': ('const double gD = gC[e] + 2.0 * lambda * delta[e];',
+                                      'const double gD = gC[e] + lambda * delta[e];'),
+    'train: w_z gradient without the sigmoid': ('g_wz[d] += gw[d] * sigmoid((double)wz[d]) / (double)nq;',
+                                                'g_wz[d] += gw[d] / (double)nq;'),
+    'train: positives summed, not averaged': ('lpos /= npos;',
+                                              'lpos /= 1;'),
+    'train: mining keeps positives': ('if (!is_pos) neg[qi * n_neg + got++] = id;',
+                                      'neg[qi * n_neg + got++] = id;'),
+    'train: W gradient without alpha': ('g_W[w] += alpha[m * r + j] * gD / (double)nq;',
+                                        'g_W[w] += gD / (double)nq;'),
+    'train: codeword gradient sign': ('gC[e] += gam[v] * (-2.0 * wf[m * ds + t] * diff);',
+                                      'gC[e] += gam[v] * (2.0 * wf[m * ds + t] * diff);'),
+    'train: bank gradient to the first fetch only': ('for (int32_t i = 0; i < h; ++i)\n            for (int32_t e = 0; e < Mr; ++e) g_bank',
+                                                     'for (int32_t i = 0; i < 1; ++i)\n            for (int32_t e = 0; e < Mr; ++e) g_bank'),
+    'train: SGD ascends': ('bank_out[e] = (float)((double)bank[e] - lr * gb[e]);',
+                           'bank_out[e] = (float)((double)bank[e] + lr * gb[e]);'),
 }
 
 
@@ -84,6 +102,7 @@ def test_pins_catch_mutation(name, source, tmp_path):
                            "-o", so, str(d / "oracle.c"), "-lm"])
     env = dict(os.environ, IFVS_ORACLE_SO=so)
     p = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
-                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py"),
+                        os.path.join(ROOT, "tests", "test_oracle_train_pins.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert p.returncode != 0, "no pin caught the mutation '%s'" % name
