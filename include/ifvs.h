@@ -43,7 +43,7 @@ extern "C" {
 #define IFVS_MAX_ATTRS 4
 #define IFVS_MAX_K 256      /* largest k (and rerank depth R) per query  */
 #define IFVS_MAX_M 128      /* largest number of PQ subspaces            */
-#define IFVS_N_STAGES 8
+#define IFVS_N_STAGES 9
 
 typedef struct ifvs_index ifvs_index;
 
@@ -112,7 +112,8 @@ enum {
     IFVS_STAGE_SCAN = 4,       /* Rank: code scan + per-CTA top-k             */
     IFVS_STAGE_MERGE = 5,      /* Select: merge of the per-CTA top-k lists    */
     IFVS_STAGE_RERANK = 6,     /* exact fp32 rerank                           */
-    IFVS_STAGE_LAYOUT = 7      /* bitmap layout conversions                   */
+    IFVS_STAGE_LAYOUT = 7,     /* bitmap layout conversions                   */
+    IFVS_STAGE_TRAIN = 8       /* training: loss, gradient and SGD kernels    */
 };
 
 /*
@@ -286,6 +287,72 @@ int ifvs_pq_encode(int32_t device, const float* X, int64_t n, int32_t D, int32_t
 int ifvs_pq_train(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
                   int32_t iters, const float* C_init, float* C_out, double* objective,
                   uint32_t flags, void* stream);
+
+/*
+ * Training of the memory bank, W and w_f (§2 "Learning": at the start the
+ * bank is zero (alpha = 0) and w_f = 1; each query-predicate pair scores its
+ * ground-truth rows and hard negatives mined from its pool, i.e. the
+ * highest-scoring rows that are not ground truth under the current
+ * parameters; an anchor term keeps C_iFVS near C_PQ; gradients reach the
+ * bank, W and w_f while C_PQ and the codes stay fixed).  The paper leaves the
+ * loss, the regulariser weight and the optimiser open; this library reads
+ * them as: score = -dist; for each positive g of a query,
+ *   l_g = dist_g / tau + log( exp(-dist_g / tau) + sum_{n in N} exp(-dist_n / tau) )
+ * over the query's negatives N, averaged over its positives, plus
+ * lambda ||Delta||^2 (all M K ds entries); the loss L is the mean over the
+ * queries; one w_z [D] is learned for all queries (w_f = softplus(w_z); the
+ * predicate Transformer is not given); plain SGD.  Distances are float32
+ * terms summed in fp64; gradients are float32; every sum runs in a fixed
+ * order, so results are deterministic.  One call handles one mini-batch of
+ * at most 1024 queries; the index must hold a bank, W and seeds with
+ * r <= 32.
+ */
+typedef struct {
+    float tau;          /* softmax temperature, > 0                          */
+    float lambda;       /* anchor weight, >= 0                               */
+    float lr;           /* SGD step size, >= 0 (ifvs_train_step)             */
+    int32_t n_pos;      /* positives per query (P)                           */
+    int32_t n_neg;      /* negatives per query; 1 <= P + n_neg <= 512
+                           (<= IFVS_MAX_K when mined)                         */
+    uint32_t flags;     /* IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING            */
+    void* stream;       /* cudaStream_t, or NULL for the index's stream       */
+} ifvs_train_params;
+
+/*
+ * ifvs_train_grad — the loss and its gradient for given candidates, without
+ * mining and without an update.
+ *   queries [nq][D] float32, preds [nq], wz [D] the shared w_z
+ *   cand    [nq][P + n_neg] int64: the P positives, then the negatives
+ *           (-1 = absent; a query without valid positives adds only its
+ *           anchor term)
+ *   g_bank  [B][M r], g_W [M][r][K][ds], g_wz [D] float32 out (each may be
+ *           NULL); loss: the mean loss (host double) or NULL
+ * Returns when all outputs are written.  Errors: IFVS_ERR_ARG (parameters,
+ * nq > 1024, NULL arrays, malformed predicate), IFVS_ERR_STATE (no bank),
+ * IFVS_ERR_UNSUPPORTED (r > 32, shared memory), IFVS_ERR_OOM, IFVS_ERR_CUDA.
+ */
+int ifvs_train_grad(ifvs_index* ix, const float* queries, const ifvs_predicate* preds, int64_t nq,
+                    const float* wz, const int64_t* cand, const ifvs_train_params* tp,
+                    float* g_bank, float* g_W, float* g_wz, double* loss);
+
+/*
+ * ifvs_train_step — one SGD step on a mini-batch: mines each query's hard
+ * negatives with the query path (top P + n_neg under the current bank, W and
+ * w_z, positives removed, the first n_neg kept, -1 where the pool runs out),
+ * computes the loss and gradient as ifvs_train_grad, then updates the
+ * index's bank and W in place and wz [D] (in/out) by theta -= lr * dL/dtheta.
+ *   positives  [nq][P] int64 (-1 = absent)
+ *   negatives  [nq][n_neg] int64 out (the mined negatives) or NULL
+ * Errors as ifvs_train_grad.
+ */
+int ifvs_train_step(ifvs_index* ix, const float* queries, const ifvs_predicate* preds, int64_t nq,
+                    float* wz, const int64_t* positives, const ifvs_train_params* tp,
+                    int64_t* negatives, double* loss);
+
+/* ifvs_get_conditioning — copies the index's current bank [B][M r] and W
+ * [M][r][K][ds] (either may be NULL) to host memory, or to device memory
+ * with IFVS_F_DEVICE_IO in flags. */
+int ifvs_get_conditioning(ifvs_index* ix, float* bank, float* W, uint32_t flags);
 
 /*
  * ifvs_stage_times — device time (ms, from CUDA events recorded on the

@@ -8,6 +8,7 @@
 #include <algorithm>
 #include <new>
 #include <utility>
+#include <cmath>
 #include <vector>
 
 #include "internal.cuh"
@@ -112,6 +113,9 @@ struct ifvs_index {
     // workspace
     DevBuf w_q, w_wz, w_preds, w_canon, w_err, w_bm, w_rows, w_npass, w_idx, w_alpha, w_wf,
         w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist, w_tab;
+    // training workspace
+    DevBuf t_cand, t_pos, t_mined, t_mdist, t_gC, t_gw, t_loss, t_G, t_gW, t_galpha, t_gbank,
+        t_gwz, t_wz, t_neg;
     // timing
     double stage_ms[IFVS_N_STAGES] = {0};
     int64_t stage_launches[IFVS_N_STAGES] = {0};
@@ -164,7 +168,9 @@ void free_index(ifvs_index* ix) {
     DevBuf* bufs[] = {&ix->w_q, &ix->w_wz, &ix->w_preds, &ix->w_canon, &ix->w_err, &ix->w_bm,
                       &ix->w_rows, &ix->w_npass, &ix->w_idx, &ix->w_alpha, &ix->w_wf,
                       &ix->w_lut, &ix->w_cifvs, &ix->w_part, &ix->w_ids, &ix->w_dists,
-                      &ix->w_cand, &ix->w_cdist, &ix->w_tab};
+                      &ix->w_cand, &ix->w_cdist, &ix->w_tab, &ix->t_cand, &ix->t_pos,
+                      &ix->t_mined, &ix->t_mdist, &ix->t_gC, &ix->t_gw, &ix->t_loss, &ix->t_G,
+                      &ix->t_gW, &ix->t_galpha, &ix->t_gbank, &ix->t_gwz, &ix->t_wz, &ix->t_neg};
     for (DevBuf* b : bufs) release(*b);
     for (auto& pr : ix->pending) {
         ix->ev_free.push_back(pr.second.first);
@@ -424,6 +430,7 @@ int finish(ifvs_index* ix, cudaStream_t s, bool check_preds) {
     if (check_preds) {
         int err = 0;
         CUDA_TRY(cudaMemcpy(&err, ix->w_err.p, sizeof(int), cudaMemcpyDeviceToHost));
+        if (err & 2) return set_err(IFVS_ERR_ARG, "a candidate row id is outside -1..N-1");
         if (err) return set_err(IFVS_ERR_ARG, "a predicate is malformed (n_clauses outside 0..4, "
                                               "reserved != 0, column out of range or unknown operator)");
     }
@@ -433,6 +440,148 @@ int finish(ifvs_index* ix, cudaStream_t s, bool check_preds) {
 int reset_err_flag(ifvs_index* ix, cudaStream_t s) {
     TRY(ensure(ix->w_err, sizeof(int)));
     CUDA_TRY(cudaMemsetAsync(ix->w_err.p, 0, sizeof(int), s));
+    return 0;
+}
+
+// ---- training (§2 "Learning") ----------------------------------------
+
+int train_check(ifvs_index* ix, const ifvs_train_params* tp, int64_t nq, bool step, Opts* o) {
+    TRY(check_index(ix, true));
+    if (!tp) return set_err(IFVS_ERR_ARG, "training parameters are NULL");
+    if (!ix->d_bank) return set_err(IFVS_ERR_STATE, "training needs a memory bank, W and seeds (ifvs_load_codebooks)");
+    if (tp->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING))
+        return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", tp->flags);
+    if (!(tp->tau > 0.f) || !std::isfinite(tp->tau)) return set_err(IFVS_ERR_ARG, "tau must be finite and > 0");
+    if (!(tp->lambda >= 0.f) || !std::isfinite(tp->lambda)) return set_err(IFVS_ERR_ARG, "lambda must be finite and >= 0");
+    if (step && (!(tp->lr >= 0.f) || !std::isfinite(tp->lr))) return set_err(IFVS_ERR_ARG, "lr must be finite and >= 0");
+    const int V = tp->n_pos + tp->n_neg;
+    if (tp->n_pos < 0 || tp->n_neg < 0 || V < 1 || V > kTrainMaxV)
+        return set_err(IFVS_ERR_ARG, "n_pos = %d, n_neg = %d: need n_pos, n_neg >= 0 and 1 <= n_pos + n_neg <= %d",
+                       tp->n_pos, tp->n_neg, kTrainMaxV);
+    if (step && V > IFVS_MAX_K)
+        return set_err(IFVS_ERR_ARG, "mining n_pos + n_neg = %d rows per query exceeds %d", V, IFVS_MAX_K);
+    if (step) TRY(check_scan_fits(ix, V));
+    if (nq < 0 || nq > 1024) return set_err(IFVS_ERR_ARG, "nq = %lld outside 0..1024 (one mini-batch per call)", (long long)nq);
+    if (ix->r > kTrainMaxR) return set_err(IFVS_ERR_UNSUPPORTED, "training supports r <= %d (index: %d)", kTrainMaxR, ix->r);
+    if (train_query_smem(V, ix->M * ix->r) > (size_t)ix->max_smem)
+        return set_err(IFVS_ERR_UNSUPPORTED, "M r = %d with %d candidates exceeds shared memory", ix->M * ix->r, V);
+    o->dio = tp->flags & IFVS_F_DEVICE_IO;
+    o->timing = tp->flags & IFVS_F_STAGE_TIMING;
+    o->stream = reinterpret_cast<cudaStream_t>(tp->stream);
+    return 0;
+}
+
+// Stages queries, predicates and the shared w_z (a device copy in t_wz and a
+// per-query broadcast in w_wz), and validates the predicates.
+int train_stage(ifvs_index* ix, cudaStream_t s, const Opts& o, int64_t n, const float* queries,
+                const ifvs_predicate* preds, const float* wz, const float** dq,
+                const ifvs_predicate** dp) {
+    TRY(stage_inputs(ix, s, o, 0, n, queries, preds, nullptr, dq, dp, nullptr));
+    TRY(ensure(ix->t_wz, sizeof(float) * ix->D));
+    CUDA_TRY(cudaMemcpyAsync(ix->t_wz.p, wz, sizeof(float) * ix->D,
+                             o.dio ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s));
+    TRY(ensure(ix->w_wz, sizeof(float) * n * ix->D));
+    CUDA_TRY(launch_broadcast_wz(ix->t_wz.as<float>(), ix->D, n, ix->w_wz.as<float>(), s));
+    TRY(ensure(ix->w_canon, sizeof(CanonPred) * n));
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_PREDICATE);
+        CUDA_TRY(st.end(launch_canonicalize(*dp, n, ix->cols(), ix->w_canon.as<CanonPred>(),
+                                            ix->w_err.as<int>(), s)));
+    }
+    return 0;
+}
+
+// Loss and gradients of one mini-batch into the t_* buffers (gW, gbank, gwz).
+int train_gradient(ifvs_index* ix, cudaStream_t s, const Opts& o, const TrainQueryArgs& a) {
+    const int Mr = ix->M * ix->r, KD = ix->K * ix->ds;
+    const float inv_n = 1.f / (float)a.n;
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_train_gram(ix->d_W, ix->M, ix->r, KD, ix->t_G.as<float>(), s)));
+    }
+    CUDA_TRY(cudaMemsetAsync(a.gC, 0, sizeof(float) * (size_t)a.n * ix->M * KD, s));
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_train_query(a, s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_train_gW(a.alpha, a.gC, ix->d_W, a.n, ix->M, ix->r, KD, a.lambda, inv_n,
+                                        ix->t_gW.as<float>(), s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_train_galpha(a.gC, ix->d_W, ix->t_G.as<float>(), a.alpha, a.n, ix->M,
+                                            ix->r, KD, a.lambda, ix->t_galpha.as<float>(), s)));
+    }
+    CUDA_TRY(cudaMemsetAsync(ix->t_gbank.p, 0, sizeof(float) * (size_t)ix->B * Mr, s));
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_train_bank(ix->w_idx.as<uint32_t>(), a.n, ix->h, Mr,
+                                          ix->t_galpha.as<float>(), inv_n, ix->t_gbank.as<float>(), s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_train_wz(a.gw, a.n, ix->D, ix->t_wz.as<float>(), inv_n,
+                                        ix->t_gwz.as<float>(), s)));
+    }
+    return 0;
+}
+
+int train_buffers(ifvs_index* ix, int64_t n, int V) {
+    const int64_t Mr = (int64_t)ix->M * ix->r, KD = (int64_t)ix->K * ix->ds;
+    TRY(ensure(ix->t_gC, sizeof(float) * n * ix->M * KD));
+    TRY(ensure(ix->t_gw, sizeof(float) * n * ix->D));
+    TRY(ensure(ix->t_loss, sizeof(double) * n));
+    TRY(ensure(ix->t_G, sizeof(float) * ix->M * ix->r * ix->r));
+    TRY(ensure(ix->t_gW, sizeof(float) * ix->M * ix->r * KD));
+    TRY(ensure(ix->t_galpha, sizeof(float) * n * Mr));
+    TRY(ensure(ix->t_gbank, sizeof(float) * ix->B * Mr));
+    TRY(ensure(ix->t_gwz, sizeof(float) * ix->D));
+    TRY(ensure(ix->w_idx, sizeof(uint32_t) * n * ix->h));
+    TRY(ensure(ix->w_alpha, sizeof(float) * n * Mr));
+    TRY(ensure(ix->w_wf, sizeof(float) * n * ix->D));
+    (void)V;
+    return 0;
+}
+
+TrainQueryArgs train_args(ifvs_index* ix, const ifvs_train_params* tp, int64_t n, const float* dq) {
+    TrainQueryArgs a{};
+    a.codes = ix->d_codes;
+    a.row_bytes = ix->row_bytes;
+    a.M = ix->M;
+    a.K = ix->K;
+    a.ds = ix->ds;
+    a.D = ix->D;
+    a.r = ix->r;
+    a.C_pq = ix->d_cpq;
+    a.W = ix->d_W;
+    a.G = ix->t_G.as<float>();
+    a.q = dq;
+    a.wf = ix->w_wf.as<float>();
+    a.alpha = ix->w_alpha.as<float>();
+    a.P = tp->n_pos;
+    a.n_neg = tp->n_neg;
+    a.tau = tp->tau;
+    a.lambda = tp->lambda;
+    a.n = n;
+    a.N = ix->N;
+    a.err = ix->w_err.as<int>();
+    a.gC = ix->t_gC.as<float>();
+    a.gw = ix->t_gw.as<float>();
+    a.loss = ix->t_loss.as<double>();
+    return a;
+}
+
+// Mean of the per-query losses, summed in query order on the host.
+int train_loss_out(ifvs_index* ix, cudaStream_t s, int64_t n, double* loss) {
+    if (!loss) return 0;
+    std::vector<double> l((size_t)n);
+    CUDA_TRY(cudaMemcpyAsync(l.data(), ix->t_loss.p, sizeof(double) * n, cudaMemcpyDeviceToHost, s));
+    CUDA_TRY(cudaStreamSynchronize(s));
+    double t = 0.0;
+    for (double v : l) t += v;
+    *loss = t / (double)n;
     return 0;
 }
 
@@ -1061,6 +1210,136 @@ extern "C" int ifvs_pq_train(int32_t device, const float* X, int64_t n, int32_t 
     }
     CUDA_TRY(cudaMemcpyAsync(C_out, cA, cb_bytes, dio ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, a.s));
     CUDA_TRY(cudaStreamSynchronize(a.s));
+    return IFVS_OK;
+}
+
+int ifvs_train_grad(ifvs_index* ix, const float* queries, const ifvs_predicate* preds, int64_t nq,
+                    const float* wz, const int64_t* cand, const ifvs_train_params* tp, float* g_bank,
+                    float* g_W, float* g_wz, double* loss) {
+    Opts o;
+    TRY(train_check(ix, tp, nq, false, &o));
+    if (nq == 0) {
+        if (loss) *loss = 0.0;
+        return IFVS_OK;
+    }
+    if (!queries || !preds || !wz || !cand) return set_err(IFVS_ERR_ARG, "an input array is NULL");
+    DeviceGuard g(ix->device);
+    cudaStream_t s = o.stream ? o.stream : ix->stream;
+    const int V = tp->n_pos + tp->n_neg;
+    const int64_t Mr = (int64_t)ix->M * ix->r;
+    TRY(reset_err_flag(ix, s));
+    const float* dq;
+    const ifvs_predicate* dp;
+    TRY(train_stage(ix, s, o, nq, queries, preds, wz, &dq, &dp));
+    TRY(train_buffers(ix, nq, V));
+    const int64_t* dcand = cand;
+    if (!o.dio) {
+        TRY(ensure(ix->t_cand, sizeof(int64_t) * nq * V));
+        CUDA_TRY(cudaMemcpyAsync(ix->t_cand.p, cand, sizeof(int64_t) * nq * V, cudaMemcpyHostToDevice, s));
+        dcand = ix->t_cand.as<int64_t>();
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_CONDITION);
+        CUDA_TRY(st.end(launch_condition(dq, dp, nq, ix->D, ix->d_seeds, ix->h, ix->B, ix->d_bank,
+                                         (int)Mr, ix->w_wz.as<float>(), ix->w_idx.as<uint32_t>(),
+                                         ix->w_alpha.as<float>(), ix->w_wf.as<float>(), s)));
+    }
+    TrainQueryArgs a = train_args(ix, tp, nq, dq);
+    a.pos = dcand;
+    a.pos_stride = V;
+    a.negsrc = dcand + tp->n_pos;
+    a.neg_stride = V;
+    a.S = tp->n_neg;
+    a.exclude = 0;
+    TRY(train_gradient(ix, s, o, a));
+    const size_t nW = sizeof(float) * (size_t)ix->M * ix->r * ix->K * ix->ds;
+    if (g_bank) TRY(copy_out(s, o.dio, g_bank, ix->t_gbank.p, sizeof(float) * ix->B * Mr));
+    if (g_W) TRY(copy_out(s, o.dio, g_W, ix->t_gW.p, nW));
+    if (g_wz) TRY(copy_out(s, o.dio, g_wz, ix->t_gwz.p, sizeof(float) * ix->D));
+    TRY(train_loss_out(ix, s, nq, loss));
+    return finish(ix, s, true);
+}
+
+int ifvs_train_step(ifvs_index* ix, const float* queries, const ifvs_predicate* preds, int64_t nq,
+                    float* wz, const int64_t* positives, const ifvs_train_params* tp,
+                    int64_t* negatives, double* loss) {
+    Opts o;
+    TRY(train_check(ix, tp, nq, true, &o));
+    if (nq == 0) {
+        if (loss) *loss = 0.0;
+        return IFVS_OK;
+    }
+    if (!queries || !preds || !wz || (tp->n_pos > 0 && !positives))
+        return set_err(IFVS_ERR_ARG, "an input array is NULL");
+    DeviceGuard g(ix->device);
+    cudaStream_t s = o.stream ? o.stream : ix->stream;
+    const int P = tp->n_pos, kk = tp->n_pos + tp->n_neg;
+    const int64_t Mr = (int64_t)ix->M * ix->r;
+    TRY(reset_err_flag(ix, s));
+    const float* dq;
+    const ifvs_predicate* dp;
+    TRY(train_stage(ix, s, o, nq, queries, preds, wz, &dq, &dp));
+    TRY(train_buffers(ix, nq, kk));
+    const int64_t* dpos = positives;
+    if (!o.dio && P > 0) {
+        TRY(ensure(ix->t_pos, sizeof(int64_t) * nq * P));
+        CUDA_TRY(cudaMemcpyAsync(ix->t_pos.p, positives, sizeof(int64_t) * nq * P, cudaMemcpyHostToDevice, s));
+        dpos = ix->t_pos.as<int64_t>();
+    }
+    // hard negatives: the query path with the current bank, W and w_z, top n_pos + n_neg
+    TRY(ensure(ix->t_mined, sizeof(int64_t) * nq * kk));
+    TRY(ensure(ix->t_mdist, sizeof(float) * nq * kk));
+    TRY(ensure(ix->w_npass, sizeof(unsigned long long) * nq));
+    Opts mo = o;
+    mo.dio = true;
+    mo.plain = false;
+    mo.R = 0;
+    mo.sub_batch = 0;
+    mo.chunk_blocks = 0;
+    TRY(run_path(ix, s, mo, dq, dp, ix->w_wz.as<float>(), nq, kk, ix->t_mined.as<int64_t>(),
+                 ix->t_mdist.as<float>(), ix->w_npass.as<unsigned long long>()));
+    TRY(ensure(ix->t_neg, sizeof(int64_t) * nq * (tp->n_neg > 0 ? tp->n_neg : 1)));
+    TrainQueryArgs a = train_args(ix, tp, nq, dq);
+    a.pos = dpos;
+    a.pos_stride = P;
+    a.negsrc = ix->t_mined.as<int64_t>();
+    a.neg_stride = kk;
+    a.S = kk;
+    a.exclude = 1;
+    a.neg_out = ix->t_neg.as<int64_t>();
+    TRY(train_gradient(ix, s, o, a));
+    // plain SGD on the bank, W and the shared w_z
+    const int64_t nW = (int64_t)ix->M * ix->r * ix->K * ix->ds;
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_sgd(ix->d_bank, ix->t_gbank.as<float>(), ix->B * Mr, tp->lr, s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_sgd(ix->d_W, ix->t_gW.as<float>(), nW, tp->lr, s)));
+    }
+    {
+        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
+        CUDA_TRY(st.end(launch_sgd(ix->t_wz.as<float>(), ix->t_gwz.as<float>(), ix->D, tp->lr, s)));
+    }
+    TRY(copy_out(s, o.dio, wz, ix->t_wz.p, sizeof(float) * ix->D));
+    if (negatives && tp->n_neg > 0)
+        TRY(copy_out(s, o.dio, negatives, ix->t_neg.p, sizeof(int64_t) * nq * tp->n_neg));
+    TRY(train_loss_out(ix, s, nq, loss));
+    return finish(ix, s, true);
+}
+
+int ifvs_get_conditioning(ifvs_index* ix, float* bank, float* W, uint32_t flags) {
+    TRY(check_index(ix, true));
+    if (!ix->d_bank) return set_err(IFVS_ERR_STATE, "the index has no memory bank");
+    if (flags & ~IFVS_F_DEVICE_IO) return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", flags);
+    const bool dio = flags & IFVS_F_DEVICE_IO;
+    DeviceGuard g(ix->device);
+    cudaStream_t s = ix->stream;
+    const size_t nW = sizeof(float) * (size_t)ix->M * ix->r * ix->K * ix->ds;
+    if (bank) TRY(copy_out(s, dio, bank, ix->d_bank, sizeof(float) * ix->B * ix->M * ix->r));
+    if (W) TRY(copy_out(s, dio, W, ix->d_W, nW));
+    CUDA_TRY(cudaStreamSynchronize(s));
     return IFVS_OK;
 }
 

@@ -169,6 +169,54 @@ cudaError_t launch_pq_reseed(const float* X, int64_t n, int D, int M, int K, int
 cudaError_t launch_pq_objective(const float* dmin, int64_t n, int M, double* objective, int num_sms,
                                 cudaStream_t s);
 
+// ---- training of bank, W, w_f (csrc/train.cu) --------------------------
+constexpr int kTrainMaxR = 32;     // r per subspace handled by the gradient kernels
+constexpr int kTrainMaxV = 512;    // positives + negatives per query
+struct TrainQueryArgs {
+    const uint8_t* codes;          // index layout (rows rotated, row_bytes apart)
+    int row_bytes, M, K, ds, D, r;
+    const float* C_pq;             // [M][K][ds]
+    const float* W;                // [M][r][K][ds]
+    const float* G;                // [M][r][r] Gram matrices (written by the gradient launch)
+    const float* q;                // [n][D]
+    const float* wf;               // [n][D]
+    const float* alpha;            // [n][M r]
+    const int64_t* pos;            // positives, row q at pos + q * pos_stride, P of them
+    int64_t pos_stride;
+    int P;
+    const int64_t* negsrc;         // negative source, row q at negsrc + q * neg_stride, S entries
+    int64_t neg_stride;
+    int S, n_neg;
+    int exclude;                   // 1: mined list (skip positives, stop at -1); 0: take as given
+    float tau, lambda;
+    int64_t n;
+    int64_t N;                     // rows of the index: ids outside -1..N-1 are refused
+    int* err;                      // |= 2 when a candidate id is outside -1..N-1 (then treated as absent)
+    int64_t* neg_out;              // [n][n_neg] or null
+    float* gC;                     // [n][M][K][ds] scratch
+    float* gw;                     // [n][D] scratch: dL/dw_f per query
+    double* loss;                  // [n]
+};
+size_t train_query_smem(int V, int Mr);
+// G [M][r][r] = W[m] W[m]^T
+cudaError_t launch_train_gram(const float* W, int M, int r, int KD, float* G, cudaStream_t s);
+// per query: candidates, distances, softmax, loss, gC (zeroed by the caller), dL/dw_f
+cudaError_t launch_train_query(const TrainQueryArgs& a, cudaStream_t s);
+// gW [M][r][K ds] of the mean loss (written, not accumulated)
+cudaError_t launch_train_gW(const float* alpha, const float* gC, const float* W, int64_t n, int M, int r,
+                            int KD, float lambda, float inv_n, float* gW, cudaStream_t s);
+// galpha [n][M r] per query (not divided by n)
+cudaError_t launch_train_galpha(const float* gC, const float* W, const float* G, const float* alpha,
+                                int64_t n, int M, int r, int KD, float lambda, float* galpha,
+                                cudaStream_t s);
+// gbank rows fetched by the batch (other rows must be zeroed by the caller)
+cudaError_t launch_train_bank(const uint32_t* idx, int64_t n, int h, int Mr, const float* galpha,
+                              float inv_n, float* gbank, cudaStream_t s);
+cudaError_t launch_train_wz(const float* gw, int64_t n, int D, const float* wz, float inv_n, float* gwz,
+                            cudaStream_t s);
+cudaError_t launch_broadcast_wz(const float* wz, int D, int64_t n, float* out, cudaStream_t s);
+cudaError_t launch_sgd(float* theta, const float* g, int64_t n, float lr, cudaStream_t s);
+
 // Read-only view of a loaded index, for entry points defined outside api.cu.
 struct IndexView {
     int device;

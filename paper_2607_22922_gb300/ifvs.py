@@ -20,8 +20,8 @@ IFVS_OK, IFVS_ERR_ARG, IFVS_ERR_OOM, IFVS_ERR_CUDA, IFVS_ERR_STATE, IFVS_ERR_UNS
 IFVS_OP_EQ, IFVS_OP_RANGE, IFVS_OP_GE, IFVS_OP_LT, IFVS_OP_GT, IFVS_OP_LE = 0, 1, 2, 3, 4, 5
 IFVS_ATTR_I32, IFVS_ATTR_I16 = 0, 1
 IFVS_F_DEVICE_IO, IFVS_F_STAGE_TIMING, IFVS_F_PLAIN_PQ = 0x1, 0x2, 0x4
-IFVS_MAX_K, IFVS_MAX_M, IFVS_MAX_ATTRS, IFVS_N_STAGES = 256, 128, 4, 8
-STAGES = ("predicate", "filter", "condition", "lut", "scan", "merge", "rerank", "layout")
+IFVS_MAX_K, IFVS_MAX_M, IFVS_MAX_ATTRS, IFVS_N_STAGES = 256, 128, 4, 9
+STAGES = ("predicate", "filter", "condition", "lut", "scan", "merge", "rerank", "layout", "train")
 
 # ifvs_predicate: 104 bytes (n_clauses, reserved, 4 x {col, op, lo, hi})
 CLAUSE_DTYPE = np.dtype([("col", "<i4"), ("op", "<i4"), ("lo", "<i8"), ("hi", "<i8")])
@@ -37,6 +37,11 @@ class IfvsError(RuntimeError):
 class SearchParams(C.Structure):
     _fields_ = [("flags", C.c_uint32), ("rerank", C.c_int32), ("sub_batch", C.c_int32),
                 ("chunk_blocks", C.c_int32), ("stream", C.c_void_p)]
+
+
+class TrainParams(C.Structure):
+    _fields_ = [("tau", C.c_float), ("lam", C.c_float), ("lr", C.c_float), ("n_pos", C.c_int32),
+                ("n_neg", C.c_int32), ("flags", C.c_uint32), ("stream", C.c_void_p)]
 
 
 def _load():
@@ -56,6 +61,9 @@ def _load():
         "ifvs_scan_topk_static": (C.c_int, [P, P, P, I64, I32, P, P, P]),
         "ifvs_pq_encode": (C.c_int, [I32, P, I64, I32, I32, I32, P, P, P, U32, P]),
         "ifvs_pq_train": (C.c_int, [I32, P, I64, I32, I32, I32, I32, P, P, P, U32, P]),
+        "ifvs_train_grad": (C.c_int, [P, P, P, I64, P, P, P, P, P, P, P]),
+        "ifvs_train_step": (C.c_int, [P, P, P, I64, P, P, P, P, P]),
+        "ifvs_get_conditioning": (C.c_int, [P, P, P, U32]),
         "ifvs_stage_times": (C.c_int, [P, P, P, I32]),
         "ifvs_canonical_predicate": (C.c_int, [P, P, I32, P, P, P]),
         "ifvs_index_info": (C.c_int, [P, P]),
@@ -284,6 +292,63 @@ def ifvs_pq_train(X, C_init, iters, device=0, C_out=None, objective=None, flags=
     return C_out, (objective[:iters] if objective is not None else None)
 
 
+def _train_params(tau, lam, lr, n_pos, n_neg, flags, stream):
+    tp = TrainParams()
+    tp.tau, tp.lam, tp.lr = float(tau), float(lam), float(lr)
+    tp.n_pos, tp.n_neg = int(n_pos), int(n_neg)
+    tp.flags = flags
+    tp.stream = stream
+    return tp
+
+
+def ifvs_train_grad(ix, queries, preds, wz, cand, n_pos, tau, lam, B, Mr, W_shape, flags=0,
+                    stream=None, g_bank=None, g_W=None, g_wz=None):
+    """Loss and gradients (dL/dbank [B][Mr], dL/dW, dL/dw_z) of one mini-batch
+    for given candidates cand [nq][n_pos + n_neg] (positives first)."""
+    dio = bool(flags & IFVS_F_DEVICE_IO)
+    nq, V = int(cand.shape[0]), int(cand.shape[1])
+    if not dio:
+        queries = _host(queries, np.float32)
+        preds = np.ascontiguousarray(preds)
+        wz = _host(wz, np.float32)
+        cand = _host(cand, np.int64)
+        g_bank = np.empty((B, Mr), np.float32)
+        g_W = np.empty(W_shape, np.float32)
+        g_wz = np.empty(wz.shape[-1], np.float32)
+    tp = _train_params(tau, lam, 0.0, n_pos, V - n_pos, flags, stream)
+    loss = C.c_double(0.0)
+    _check(_lib.ifvs_train_grad(ix, _ptr(queries), _ptr(preds), nq, _ptr(wz), _ptr(cand),
+                                C.byref(tp), _ptr(g_bank), _ptr(g_W), _ptr(g_wz), C.byref(loss)))
+    return loss.value, g_bank, g_W, g_wz
+
+
+def ifvs_train_step(ix, queries, preds, wz, positives, n_neg, tau, lam, lr, flags=0, stream=None,
+                    negatives=None):
+    """One SGD step; updates the index's bank and W and ``wz`` in place.
+    Returns (loss, negatives [nq][n_neg])."""
+    dio = bool(flags & IFVS_F_DEVICE_IO)
+    nq, P = int(positives.shape[0]), int(positives.shape[1])
+    if not dio:
+        queries = _host(queries, np.float32)
+        preds = np.ascontiguousarray(preds)
+        positives = _host(positives, np.int64)
+        if not (isinstance(wz, np.ndarray) and wz.dtype == np.float32 and wz.flags.c_contiguous):
+            raise ValueError("wz must be a C-contiguous float32 array (updated in place)")
+        negatives = np.empty((nq, n_neg), np.int64)
+    tp = _train_params(tau, lam, lr, P, n_neg, flags, stream)
+    loss = C.c_double(0.0)
+    _check(_lib.ifvs_train_step(ix, _ptr(queries), _ptr(preds), nq, _ptr(wz), _ptr(positives),
+                                C.byref(tp), _ptr(negatives), C.byref(loss)))
+    return loss.value, negatives
+
+
+def ifvs_get_conditioning(ix, B, Mr, W_shape):
+    bank = np.empty((B, Mr), np.float32)
+    W = np.empty(W_shape, np.float32)
+    _check(_lib.ifvs_get_conditioning(ix, _ptr(bank), _ptr(W), 0))
+    return bank, W
+
+
 def ifvs_rerank(ix, queries, cand, k, flags=0):
     queries = _host(queries, np.float32)
     cand = _host(cand, np.int64)
@@ -333,12 +398,18 @@ class Index:
         self.h = ifvs_load_index(codes, attrs, vectors, D, device, K, device_io)
         self.N, self.M = int(codes.shape[0]), int(codes.shape[1])
         self.K = K
+        self._bank_shape = self._W_shape = None
 
     def load_codebooks(self, C_pq, bank=None, W=None, hash_seeds=None):
         ifvs_load_codebooks(self.h, C_pq, bank=bank, W=W, hash_seeds=hash_seeds)
         self.ds = int(np.asarray(C_pq).shape[2])
         self.r = 0 if W is None else int(np.asarray(W).shape[1])
         self.hh = 0 if hash_seeds is None else len(hash_seeds)
+        if bank is not None:
+            self._bank_shape = (int(bank.shape[0]), self.M * self.r)
+            self._W_shape = (self.M, self.r, self.K, self.ds)
+        else:
+            self._bank_shape = self._W_shape = None
         return self
 
     def search(self, queries, preds, k, wz=None, **kw):
@@ -356,6 +427,22 @@ class Index:
 
     def rerank(self, queries, cand, k, **kw):
         return ifvs_rerank(self.h, queries, cand, k, **kw)
+
+    def _cond_shapes(self):
+        if self._bank_shape is None:
+            raise IfvsError(IFVS_ERR_STATE, "no memory bank loaded")
+        return self._bank_shape, self._W_shape
+
+    def train_grad(self, queries, preds, wz, cand, n_pos, tau, lam, **kw):
+        (B, Mr), Ws = self._cond_shapes()
+        return ifvs_train_grad(self.h, queries, preds, wz, cand, n_pos, tau, lam, B, Mr, Ws, **kw)
+
+    def train_step(self, queries, preds, wz, positives, n_neg, tau, lam, lr, **kw):
+        return ifvs_train_step(self.h, queries, preds, wz, positives, n_neg, tau, lam, lr, **kw)
+
+    def conditioning(self):
+        (B, Mr), Ws = self._cond_shapes()
+        return ifvs_get_conditioning(self.h, B, Mr, Ws)
 
     def stage_times(self, reset=False):
         return ifvs_stage_times(self.h, reset)
