@@ -23,6 +23,7 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -36,6 +37,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 WORKLOAD = "gmm100m-d128-m16"
+TRAIN_WORKLOAD = "sift1m-d128-m16"
 CPU_SAMPLE_ROWS = 10_000_000
 
 
@@ -45,15 +47,23 @@ def parse():
     ap.add_argument("--steps", type=int, default=16)
     ap.add_argument("--warmup", type=int, default=4)
     ap.add_argument("--impl", default="ifvs", choices=["ifvs", "reference"])
-    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--workload", default=None,
+                    help="default: %s (search, pq), %s (train)" % (WORKLOAD, TRAIN_WORKLOAD))
     ap.add_argument("--rows", type=int, default=0, help="override N (smaller runs)")
     ap.add_argument("--recall-queries", type=int, default=16, help="per bin; 0 = skip")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--chunk-blocks", type=int, default=0, help="scan chunk size in 1024-row blocks (0 = auto)")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
-    ap.add_argument("--mode", default="search", choices=["search", "pq"],
-                    help="search: the query path; pq: PQ encoding + Lloyd training of the index")
+    ap.add_argument("--mode", default="search", choices=["search", "pq", "train"],
+                    help="search: the query path; pq: PQ encoding + Lloyd training of the index; "
+                         "train: SGD steps on the bank, W and w_z")
+    ap.add_argument("--train-neg", type=int, default=32, help="hard negatives per query (--mode train)")
+    ap.add_argument("--train-tau", type=float, default=8.0, help="softmax temperature (--mode train)")
+    ap.add_argument("--train-lambda", type=float, default=0.001, help="anchor weight (--mode train)")
+    ap.add_argument("--train-lr", type=float, default=5.0, help="SGD step for bank and W (--mode train)")
+    ap.add_argument("--train-lr-wz", type=float, default=0.0,
+                    help="SGD step for w_z (--mode train; 0 keeps the initial w_f = 1)")
     ap.add_argument("--pq-rows", type=int, default=1 << 24, help="rows encoded per step (--mode pq)")
     ap.add_argument("--pq-train-rows", type=int, default=1 << 20, help="Lloyd sample rows (--mode pq)")
     ap.add_argument("--pq-iters", type=int, default=25, help="Lloyd iterations (--mode pq)")
@@ -62,7 +72,8 @@ def parse():
 
 def workload(args):
     from paper_2607_22922_gb300 import synth
-    w = synth.WORKLOADS[args.workload]
+    name = args.workload or (TRAIN_WORKLOAD if args.mode == "train" else WORKLOAD)
+    w = synth.WORKLOADS[name]
     if args.rows:
         w = synth.scaled(w, N=args.rows)
     if w.batch <= 0:
@@ -220,22 +231,21 @@ def cpu_baseline(w, ix, cond, batches, max_seconds=30.0):
 
 # ------------------------------------------------------------ recall
 
-def recall_at_k(w, ix, batches, ids_by_bin, nsample, device):
-    """recall@k of the returned ids against the exact filtered top-k (§3.1)
-    over the raw vectors, for the first ``nsample`` queries of each bin."""
+def exact_topk_gpu(w, ix, q, preds, k, device):
+    """Exact filtered top-k (§3.1) over the raw vectors (drawn on the device
+    block by block) for range predicates on attribute 0, in fp64 with torch:
+    ids [nq][k] (-1 padded), outside any timed region."""
     import torch
     from paper_2607_22922_gb300 import synth
     block = 1 << 22
     cb = torch.from_numpy(ix.codebook).to(device)
     attr = ix.attrs[0]
-    qs_all = torch.cat([torch.from_numpy(b.q[:nsample]) for b in batches]).to(device).double()
-    lo = np.concatenate([b.preds["c"][:nsample, 0]["lo"] for b in batches])
-    hi = np.concatenate([b.preds["c"][:nsample, 0]["hi"] for b in batches])
+    qs_all = torch.from_numpy(np.ascontiguousarray(q)).to(device).double()
+    lo_t = torch.from_numpy(np.ascontiguousarray(preds["c"][:, 0]["lo"])).to(device)
+    hi_t = torch.from_numpy(np.ascontiguousarray(preds["c"][:, 0]["hi"])).to(device)
     nq = qs_all.shape[0]
-    best_d = torch.full((nq, w.k), float("inf"), dtype=torch.float64, device=device)
-    best_i = torch.full((nq, w.k), -1, dtype=torch.int64, device=device)
-    lo_t = torch.from_numpy(lo).to(device)
-    hi_t = torch.from_numpy(hi).to(device)
+    best_d = torch.full((nq, k), float("inf"), dtype=torch.float64, device=device)
+    best_i = torch.full((nq, k), -1, dtype=torch.int64, device=device)
     qn = (qs_all * qs_all).sum(1, keepdim=True)
     for s in range(0, w.N, block):
         e = min(w.N, s + block)
@@ -244,26 +254,36 @@ def recall_at_k(w, ix, batches, ids_by_bin, nsample, device):
         a = torch.from_numpy(attr[s:e].astype(np.int64)).to(device)
         ok = (a[None, :] >= lo_t[:, None]) & (a[None, :] < hi_t[:, None])
         d = torch.where(ok, d, torch.full_like(d, float("inf")))
-        kk = min(w.k, e - s)
+        kk = min(k, e - s)
         dv, di = torch.topk(d, kk, dim=1, largest=False)
         di = di + s
         cd = torch.cat([best_d, dv], 1)
         ci = torch.cat([best_i, di], 1)
-        o = torch.argsort(cd, dim=1, stable=True)[:, :w.k]
+        o = torch.argsort(cd, dim=1, stable=True)[:, :k]
         best_d = torch.gather(cd, 1, o)
         best_i = torch.gather(ci, 1, o)
         best_i = torch.where(torch.isinf(best_d), torch.full_like(best_i, -1), best_i)
-    gt = best_i.cpu().numpy()
+    return best_i.cpu().numpy()
+
+
+def recall_vs(gt, ids):
+    r = []
+    for g, i in zip(gt, ids):
+        valid = g[g >= 0]
+        if len(valid):
+            r.append(len(np.intersect1d(valid, i)) / len(valid))
+    return float(np.mean(r)) if r else None
+
+
+def recall_at_k(w, ix, batches, ids_by_bin, nsample, device):
+    """recall@k of the returned ids against the exact filtered top-k (§3.1)
+    over the raw vectors, for the first ``nsample`` queries of each bin."""
+    q = np.concatenate([b.q[:nsample] for b in batches])
+    preds = np.concatenate([b.preds[:nsample] for b in batches])
+    gt = exact_topk_gpu(w, ix, q, preds, w.k, device)
     out = {}
     for b, (qs, ids) in enumerate(zip(batches, ids_by_bin)):
-        r = []
-        for i in range(nsample):
-            g = gt[b * nsample + i]
-            valid = g[g >= 0]
-            if len(valid) == 0:
-                continue
-            r.append(len(np.intersect1d(valid, ids[i])) / len(valid))
-        out[qs.sel] = float(np.mean(r)) if r else None
+        out[qs.sel] = recall_vs(gt[b * nsample:(b + 1) * nsample], ids[:nsample])
     return out
 
 
@@ -599,6 +619,160 @@ def run_pq(args):
         dist.destroy_process_group()
 
 
+def run_train(args):
+    """Training of the bank, W and w_z (§2 "Learning"): each step is one
+    mini-batch of queries through ifvs_train_step (mining with the query
+    path, loss, gradient, SGD); steps cycle through the selectivity bins.
+    Positives are the exact filtered top-k over the raw vectors, computed
+    outside the timed region; the parameters start from the paper's initial
+    state (zero bank, w_f = 1)."""
+    import torch
+    world, rank, local = dist_env()
+    if not torch.cuda.is_available():
+        raise SystemExit("no CUDA device: the benchmark needs a GPU")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    dist = dist_init(world, device)
+    from paper_2607_22922_gb300 import build, synth
+    if rank == 0 or world == 1:
+        build.build()
+    barrier(dist, device)
+    build.build()
+    from paper_2607_22922_gb300 import ifvs
+
+    w = workload(args)
+    P, n_neg = w.k, args.train_neg
+    t0 = time.time()
+    ix = synth.make_index(w)
+    cond = synth.make_conditioning(ix)
+    batches = [synth.make_queries(ix, s, nq=w.batch, salt=rank) for s in w.sels]
+    gts = [exact_topk_gpu(w, ix, b.q, b.preds, P, device) for b in batches]
+    t_gen = time.time() - t0
+    bank0 = np.zeros_like(cond.bank)
+    wz0 = np.full(w.D, math.log(math.e - 1.0), np.float32)
+    g = ifvs.Index(ix.codes, ix.attrs, D=w.D, K=w.K, device=local)
+    g.load_codebooks(ix.codebook, bank=bank0, W=cond.W, hash_seeds=cond.seeds)
+
+    def recall_now(wz_host):
+        ids = []
+        for b in batches:
+            i, _, _ = g.search(b.q, b.preds, P, wz=np.tile(wz_host, (len(b.q), 1)))
+            ids.append(i)
+        return [recall_vs(gt, i) for gt, i in zip(gts, ids)]
+
+    rec0 = recall_now(wz0)
+    stream = torch.cuda.Stream(device=device)
+    sptr = stream.cuda_stream
+    nb = len(batches)
+    dev_in = [(torch.from_numpy(b.q).to(device),
+               torch.from_numpy(b.preds.view(np.uint8).copy()).to(device),
+               torch.from_numpy(gt).to(device)) for b, gt in zip(batches, gts)]
+    wz = torch.from_numpy(wz0.copy()).to(device)
+    neg = torch.empty((w.batch, n_neg), dtype=torch.int64, device=device)
+    flags = ifvs.IFVS_F_DEVICE_IO | ifvs.IFVS_F_STAGE_TIMING
+    losses = []
+
+    def step(i):
+        q, p, pos = dev_in[i % nb]
+        L, _ = ifvs.ifvs_train_step(g.h, q, p, wz, pos, n_neg, args.train_tau, args.train_lambda,
+                                    args.train_lr, flags=flags, stream=sptr, negatives=neg,
+                                    lr_wz=args.train_lr_wz)
+        losses.append(L)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    g.stage_times(reset=True)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    clocks = Clocks()
+    barrier(dist, device)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    with torch.cuda.stream(stream):
+        ev[0].record(stream)
+        for i in range(args.steps):
+            step(args.warmup + i)
+        ev[1].record(stream)
+    torch.cuda.synchronize()
+    barrier(dist, device)
+    clk = clocks.stop()
+    total_ms = ev[0].elapsed_time(ev[1])
+    max_ms = reduce_max(dist, total_ms, device)
+    stages = g.stage_times(reset=True)
+    launches = sum(v[1] for v in stages.values())
+    rec1 = recall_now(wz.cpu().numpy())
+
+    # end to end through the C ABI with host arrays (queries, predicates,
+    # positives and w_z in; w_z, negatives and the loss out)
+    e2e = None
+    if not args.no_e2e:
+        wzh = wz.cpu().numpy().copy()
+
+        def hstep(i):
+            b = batches[i % nb]
+            ifvs.ifvs_train_step(g.h, b.q, b.preds, wzh, gts[i % nb], n_neg, args.train_tau,
+                                 args.train_lambda, args.train_lr, stream=sptr,
+                                 lr_wz=args.train_lr_wz)
+
+        for i in range(args.warmup):
+            hstep(i)
+        barrier(dist, device)
+        torch.cuda.synchronize()
+        t1 = time.perf_counter()
+        for i in range(args.steps):
+            hstep(args.warmup + i)
+        torch.cuda.synchronize()
+        e_ms = reduce_max(dist, (time.perf_counter() - t1) * 1000.0, device)
+        e2e = {"value": whole_job_qps(world, args.steps, w.batch, e_ms), "unit": "queries/s",
+               "h2d_bytes_per_step": w.batch * (w.D * 4 + 104 + P * 8) + w.D * 4,
+               "d2h_bytes_per_step": w.batch * n_neg * 8 + w.D * 4 + w.batch * 8}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        b = batches[2 % nb]
+        nsamp = 4
+        t1 = time.perf_counter()
+        oracle.train_step(ix.codes, ix.attrs, ix.codebook, bank0, cond.W, cond.seeds, wz0,
+                          b.q[:nsamp], b.preds[:nsamp], gts[2 % nb][:nsamp], n_neg,
+                          args.train_tau, args.train_lambda, args.train_lr, args.train_lr_wz)
+        sec = time.perf_counter() - t1
+        cpu = {"value": nsamp / sec, "unit": "queries/s", "cores": 1, "kind": "oracle",
+               "sample": "one training step on %d queries of the %g bin (full N)" % (nsamp, b.sel)}
+
+    train_ms = stages["train"][0]
+    line = {
+        "metric": "training throughput (queries per second through ifvs_train_step)",
+        "value": whole_job_qps(world, args.steps, w.batch, max_ms), "unit": "queries/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": max_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32 (fp64 distance sums and softmax)",
+        "data": "synthetic (seeded Gaussian-mixture PQ index; paper datasets absent)",
+        "config": {"workload": "%s, SGD on bank/W/w_z, %d-query mini-batches" % (w.name, w.batch),
+                   "N": w.N, "D": w.D, "M": w.M, "K": w.K, "B": w.B, "h": w.h, "r": w.r,
+                   "n_pos": P, "n_neg": n_neg, "tau": args.train_tau, "lambda": args.train_lambda,
+                   "lr": args.train_lr, "lr_wz": args.train_lr_wz, "bins": list(w.sels),
+                   "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "codes (%.0f MB) fit in L2" % (w.N * w.M / 1e6)},
+        "stage_ms": {k: v[0] for k, v in stages.items()},
+        "train_share": train_ms / sum(v[0] for v in stages.values()),
+        "gpu_launches": launches, "clocks": clk, "e2e": e2e, "cpu_baseline": cpu,
+        "loss_first": losses[0], "loss_last": losses[-1],
+        "recall@%d_before" % P: rec0, "recall@%d_after" % P: rec1, "setup_s": round(t_gen, 1),
+    }
+    if rank == 0:
+        s = json.dumps(line)
+        print(s, flush=True)
+        if args.out:
+            with open(args.out, "w") as f:
+                f.write(s + "\n")
+    g.close()
+    if dist is not None:
+        dist.destroy_process_group()
+
+
 def run_reference(args):
     """The oracle as it stands on the host cores, each step one query of the
     next bin over the first CPU_SAMPLE_ROWS rows, time scaled by N / rows."""
@@ -653,6 +827,8 @@ def main():
         run_reference(args)
     elif args.mode == "pq":
         run_pq(args)
+    elif args.mode == "train":
+        run_train(args)
     else:
         run_ifvs(args)
 

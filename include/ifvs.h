@@ -301,7 +301,10 @@ int ifvs_pq_train(int32_t device, const float* X, int64_t n, int32_t D, int32_t 
  * over the query's negatives N, averaged over its positives, plus
  * lambda ||Delta||^2 (all M K ds entries); the loss L is the mean over the
  * queries; one w_z [D] is learned for all queries (w_f = softplus(w_z); the
- * predicate Transformer is not given); plain SGD.  Distances are float32
+ * predicate Transformer is not given); plain SGD, with a step size of its
+ * own for w_z (at a fixed temperature, shrinking every weight lowers this
+ * loss whenever positives trail hard negatives, so a jointly learned w_f
+ * can collapse toward 0).  Distances are float32
  * terms summed in fp64; gradients are float32; every sum runs in a fixed
  * order, so results are deterministic.  One call handles one mini-batch of
  * at most 1024 queries; the index must hold a bank, W and seeds with
@@ -310,7 +313,8 @@ int ifvs_pq_train(int32_t device, const float* X, int64_t n, int32_t D, int32_t 
 typedef struct {
     float tau;          /* softmax temperature, > 0                          */
     float lambda;       /* anchor weight, >= 0                               */
-    float lr;           /* SGD step size, >= 0 (ifvs_train_step)             */
+    float lr;           /* SGD step size for the bank and W, >= 0            */
+    float lr_wz;        /* SGD step size for w_z, >= 0 (0 keeps w_f fixed)   */
     int32_t n_pos;      /* positives per query (P)                           */
     int32_t n_neg;      /* negatives per query; 1 <= P + n_neg <= 512
                            (<= IFVS_MAX_K when mined)                         */
@@ -340,7 +344,8 @@ int ifvs_train_grad(ifvs_index* ix, const float* queries, const ifvs_predicate* 
  * negatives with the query path (top P + n_neg under the current bank, W and
  * w_z, positives removed, the first n_neg kept, -1 where the pool runs out),
  * computes the loss and gradient as ifvs_train_grad, then updates the
- * index's bank and W in place and wz [D] (in/out) by theta -= lr * dL/dtheta.
+ * index's bank and W in place (theta -= lr * dL/dtheta) and wz [D] (in/out,
+ * wz -= lr_wz * dL/dwz).
  *   positives  [nq][P] int64 (-1 = absent)
  *   negatives  [nq][n_neg] int64 out (the mined negatives) or NULL
  * Errors as ifvs_train_grad.

@@ -89,8 +89,8 @@ def lib():
             "orc_mine_negatives": (C.c_int, [P, I64, I32_, I32_, I32_, P, P, I32_, P, P, I64,
                                              I32_, I32_, P, P, P, P, P, I64, P, I32_, I32_, P]),
             "orc_train_step": (C.c_int, [P, I64, I32_, I32_, I32_, P, P, I32_, P, P, I64, I32_,
-                                         I32_, P, P, P, P, P, I64, P, I32_, I32_, D, D, D, P, P,
-                                         P, P, P]),
+                                         I32_, P, P, P, P, P, I64, P, I32_, I32_, D, D, D, D, P,
+                                         P, P, P, P]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -440,9 +440,11 @@ def mine_negatives(codes, cols, C_pq, bank, W, seeds, wz, queries, preds, pos, n
     return neg
 
 
-def train_step(codes, cols, C_pq, bank, W, seeds, wz, queries, preds, pos, n_neg, tau, lam, lr):
-    """Mining, loss, gradient and one SGD step; returns (loss, bank', W',
-    w_z', negatives)."""
+def train_step(codes, cols, C_pq, bank, W, seeds, wz, queries, preds, pos, n_neg, tau, lam, lr,
+               lr_wz=None):
+    """Mining, loss, gradient and one SGD step (step lr for bank and W, lr_wz
+    for w_z, default lr); returns (loss, bank', W', w_z', negatives)."""
+    lr_wz = lr if lr_wz is None else lr_wz
     codes, C_pq, bank, W, seeds, wz, queries, preds, M, K, ds, D = _train_common(
         codes, C_pq, bank, W, seeds, wz, queries, preds)
     pos = _c(pos, np.int64)
@@ -454,8 +456,8 @@ def train_step(codes, cols, C_pq, bank, W, seeds, wz, queries, preds, pos, n_neg
     rc = lib().orc_train_step(_p(codes), codes.shape[0], M, K, ds, cs.ptrs, _p(cs.types), cs.n,
                               _p(C_pq), _p(bank), bank.shape[0], len(seeds), W.shape[1], _p(W),
                               _p(seeds), _p(wz), _p(queries), _p(preds), nq, _p(pos), P, n_neg,
-                              float(tau), float(lam), float(lr), _p(b2), _p(W2), _p(z2), _p(neg),
-                              _p(loss))
+                              float(tau), float(lam), float(lr), float(lr_wz), _p(b2), _p(W2),
+                              _p(z2), _p(neg), _p(loss))
     if rc != 0:
         raise ValueError("invalid predicate")
     return float(loss[0]), b2, W2, z2, neg

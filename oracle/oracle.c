@@ -579,7 +579,10 @@ void orc_lloyd_step(const float* X, int64_t n, int32_t D, int32_t M, int32_t K,
  *   L = the mean of that over the queries;
  *   w_f = softplus(w_z) with one learned w_z [D] for all queries (the
  *   predicate Transformer that would give w_z per predicate is not given);
- *   optimiser: plain SGD, theta <- theta - lr * dL/dtheta. */
+ *   optimiser: plain SGD, theta <- theta - lr * dL/dtheta, with a step size
+ *   of its own for w_z (a jointly learned w_z can shrink every weight toward
+ *   0: at a fixed temperature that lowers the loss whenever positives trail
+ *   hard negatives, whatever it does to the ranking). */
 
 static double sigmoid(double x) {
     if (x >= 0) return 1.0 / (1.0 + exp(-x));
@@ -747,8 +750,8 @@ int orc_train_step(const uint8_t* codes, int64_t N, int32_t M, int32_t K, int32_
                    const float* W, const uint64_t* seeds, const float* wz,
                    const float* queries, const orc_predicate* preds, int64_t nq,
                    const int64_t* pos, int32_t P, int32_t n_neg, double tau, double lambda,
-                   double lr, float* bank_out, float* W_out, float* wz_out, int64_t* neg,
-                   double* loss) {
+                   double lr, double lr_wz, float* bank_out, float* W_out, float* wz_out,
+                   int64_t* neg, double* loss) {
     const int32_t D = M * ds, V = P + n_neg;
     const int64_t nB = B * M * r, nW = (int64_t)M * r * K * ds;
     int64_t* cand = (int64_t*)malloc(sizeof(int64_t) * (size_t)(nq > 0 ? nq : 1) * (V > 0 ? V : 1));
@@ -766,7 +769,7 @@ int orc_train_step(const uint8_t* codes, int64_t N, int32_t M, int32_t K, int32_
                                nq, cand, P, V, tau, lambda, gb, gW, gz);
         for (int64_t e = 0; e < nB; ++e) bank_out[e] = (float)((double)bank[e] - lr * gb[e]);
         for (int64_t e = 0; e < nW; ++e) W_out[e] = (float)((double)W[e] - lr * gW[e]);
-        for (int32_t d = 0; d < D; ++d) wz_out[d] = (float)((double)wz[d] - lr * gz[d]);
+        for (int32_t d = 0; d < D; ++d) wz_out[d] = (float)((double)wz[d] - lr_wz * gz[d]);
     }
     free(cand);
     free(gb);

@@ -176,15 +176,16 @@ int orc_mine_negatives(const uint8_t* codes, int64_t N, int32_t M, int32_t K, in
                        const float* queries, const orc_predicate* preds, int64_t nq,
                        const int64_t* pos, int32_t P, int32_t n_neg, int64_t* neg);
 /* One training step: mine negatives, loss and gradient, then plain SGD on
- * bank, W and w_z (new values rounded to float32 into the *_out arrays). */
+ * bank and W (step lr) and w_z (step lr_wz); new values rounded to float32
+ * into the *_out arrays. */
 int orc_train_step(const uint8_t* codes, int64_t N, int32_t M, int32_t K, int32_t ds,
                    const void* const* cols, const int32_t* types, int32_t n_attrs,
                    const float* C_pq, const float* bank, int64_t B, int32_t h, int32_t r,
                    const float* W, const uint64_t* seeds, const float* wz,
                    const float* queries, const orc_predicate* preds, int64_t nq,
                    const int64_t* pos, int32_t P, int32_t n_neg, double tau, double lambda,
-                   double lr, float* bank_out, float* W_out, float* wz_out, int64_t* neg,
-                   double* loss);
+                   double lr, double lr_wz, float* bank_out, float* W_out, float* wz_out,
+                   int64_t* neg, double* loss);
 
 #ifdef __cplusplus
 }

@@ -453,7 +453,8 @@ int train_check(ifvs_index* ix, const ifvs_train_params* tp, int64_t nq, bool st
         return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", tp->flags);
     if (!(tp->tau > 0.f) || !std::isfinite(tp->tau)) return set_err(IFVS_ERR_ARG, "tau must be finite and > 0");
     if (!(tp->lambda >= 0.f) || !std::isfinite(tp->lambda)) return set_err(IFVS_ERR_ARG, "lambda must be finite and >= 0");
-    if (step && (!(tp->lr >= 0.f) || !std::isfinite(tp->lr))) return set_err(IFVS_ERR_ARG, "lr must be finite and >= 0");
+    if (step && (!(tp->lr >= 0.f) || !std::isfinite(tp->lr) || !(tp->lr_wz >= 0.f) || !std::isfinite(tp->lr_wz)))
+        return set_err(IFVS_ERR_ARG, "lr and lr_wz must be finite and >= 0");
     const int V = tp->n_pos + tp->n_neg;
     if (tp->n_pos < 0 || tp->n_neg < 0 || V < 1 || V > kTrainMaxV)
         return set_err(IFVS_ERR_ARG, "n_pos = %d, n_neg = %d: need n_pos, n_neg >= 0 and 1 <= n_pos + n_neg <= %d",
@@ -1320,7 +1321,7 @@ int ifvs_train_step(ifvs_index* ix, const float* queries, const ifvs_predicate* 
     }
     {
         Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
-        CUDA_TRY(st.end(launch_sgd(ix->t_wz.as<float>(), ix->t_gwz.as<float>(), ix->D, tp->lr, s)));
+        CUDA_TRY(st.end(launch_sgd(ix->t_wz.as<float>(), ix->t_gwz.as<float>(), ix->D, tp->lr_wz, s)));
     }
     TRY(copy_out(s, o.dio, wz, ix->t_wz.p, sizeof(float) * ix->D));
     if (negatives && tp->n_neg > 0)

@@ -40,8 +40,9 @@ class SearchParams(C.Structure):
 
 
 class TrainParams(C.Structure):
-    _fields_ = [("tau", C.c_float), ("lam", C.c_float), ("lr", C.c_float), ("n_pos", C.c_int32),
-                ("n_neg", C.c_int32), ("flags", C.c_uint32), ("stream", C.c_void_p)]
+    _fields_ = [("tau", C.c_float), ("lam", C.c_float), ("lr", C.c_float), ("lr_wz", C.c_float),
+                ("n_pos", C.c_int32), ("n_neg", C.c_int32), ("flags", C.c_uint32),
+                ("stream", C.c_void_p)]
 
 
 def _load():
@@ -292,9 +293,10 @@ def ifvs_pq_train(X, C_init, iters, device=0, C_out=None, objective=None, flags=
     return C_out, (objective[:iters] if objective is not None else None)
 
 
-def _train_params(tau, lam, lr, n_pos, n_neg, flags, stream):
+def _train_params(tau, lam, lr, n_pos, n_neg, flags, stream, lr_wz=None):
     tp = TrainParams()
     tp.tau, tp.lam, tp.lr = float(tau), float(lam), float(lr)
+    tp.lr_wz = float(lr if lr_wz is None else lr_wz)
     tp.n_pos, tp.n_neg = int(n_pos), int(n_neg)
     tp.flags = flags
     tp.stream = stream
@@ -323,9 +325,10 @@ def ifvs_train_grad(ix, queries, preds, wz, cand, n_pos, tau, lam, B, Mr, W_shap
 
 
 def ifvs_train_step(ix, queries, preds, wz, positives, n_neg, tau, lam, lr, flags=0, stream=None,
-                    negatives=None):
-    """One SGD step; updates the index's bank and W and ``wz`` in place.
-    Returns (loss, negatives [nq][n_neg])."""
+                    negatives=None, lr_wz=None):
+    """One SGD step (step lr for the bank and W, lr_wz for w_z, default lr);
+    updates the index's bank and W and ``wz`` in place.  Returns (loss,
+    negatives [nq][n_neg])."""
     dio = bool(flags & IFVS_F_DEVICE_IO)
     nq, P = int(positives.shape[0]), int(positives.shape[1])
     if not dio:
@@ -335,7 +338,7 @@ def ifvs_train_step(ix, queries, preds, wz, positives, n_neg, tau, lam, lr, flag
         if not (isinstance(wz, np.ndarray) and wz.dtype == np.float32 and wz.flags.c_contiguous):
             raise ValueError("wz must be a C-contiguous float32 array (updated in place)")
         negatives = np.empty((nq, n_neg), np.int64)
-    tp = _train_params(tau, lam, lr, P, n_neg, flags, stream)
+    tp = _train_params(tau, lam, lr, P, n_neg, flags, stream, lr_wz)
     loss = C.c_double(0.0)
     _check(_lib.ifvs_train_step(ix, _ptr(queries), _ptr(preds), nq, _ptr(wz), _ptr(positives),
                                 C.byref(tp), _ptr(negatives), C.byref(loss)))

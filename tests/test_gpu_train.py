@@ -173,15 +173,43 @@ def test_initial_state_moves_only_the_bank_and_w_z(ifvs, orc):
     assert not np.array_equal(b, c.bank) and not np.array_equal(wz, c.wz)
 
 
-def test_training_lowers_the_loss(ifvs, orc):
-    """Repeated steps on one mini-batch (negatives re-mined each step) bring
-    the loss down."""
+def test_frozen_w_z_step_matches_the_oracle(ifvs, orc, case):
+    """lr_wz = 0 keeps w_f where it is while the bank and W take their step."""
+    lr = 0.5
+    g = case.index(ifvs)
+    wz = case.wz.copy()
+    g.train_step(case.qs.q, case.qs.preds, wz, case.pos, NNEG, TAU, LAM, lr, lr_wz=0.0)
+    _, b2, W2, z2, neg_o = orc.train_step(case.ix.codes, case.ix.attrs, case.ix.codebook, case.bank,
+                                          case.W, case.cond.seeds, case.wz, case.qs.q,
+                                          case.qs.preds, case.pos, NNEG, TAU, LAM, lr, lr_wz=0.0)
+    np.testing.assert_array_equal(wz, case.wz)
+    np.testing.assert_array_equal(z2, case.wz)
+    b, W = g.conditioning()
+    _, gb, gW, _ = case.oracle_loss(orc, np.concatenate([case.pos, neg_o], 1))
+    for new, ref, grad in ((b, b2, gb), (W, W2, gW)):
+        bound = lr * GRAD_TOL * np.abs(grad).max() + np.spacing(np.abs(ref).astype(np.float32))
+        assert (np.abs(new.astype(np.float64) - ref) <= bound).all()
+
+
+def test_training_raises_recall_on_its_batch(ifvs, orc):
+    """Repeated steps on one mini-batch from the paper's initial state (zero
+    bank, w_f = 1 held fixed), negatives re-mined each step: the loss falls
+    and the search ranks more of the ground truth into the top P."""
     c = Case(orc, zero_bank=True, salt=2, nq=16)
     g = c.index(ifvs)
     wz = c.wz.copy()
-    losses = [g.train_step(c.qs.q, c.qs.preds, wz, c.pos, NNEG, TAU, 0.001, 0.5)[0]
+
+    def recall():
+        ids, _, _ = g.search(c.qs.q, c.qs.preds, P, wz=np.tile(wz, (len(c.qs.q), 1)))
+        return np.mean([len(np.intersect1d(a[a >= 0], b)) / max(1, (a >= 0).sum())
+                        for a, b in zip(c.pos, ids)])
+
+    r0 = recall()
+    losses = [g.train_step(c.qs.q, c.qs.preds, wz, c.pos, NNEG, TAU, 0.001, 5.0, lr_wz=0.0)[0]
               for _ in range(30)]
+    r1 = recall()
     assert losses[-1] < 0.8 * losses[0], losses
+    assert r1 > r0 + 0.05, (r0, r1)
 
 
 def test_deterministic_and_device_io(ifvs, orc, case):

@@ -61,24 +61,26 @@ MUTATIONS = {
     "Lloyd keeps the old centroid": ("Co[(int64_t)c * ds + t] = cnt[c] > 0 ? (float)(sum[(int64_t)c * ds + t] / (double)cnt[c])",
                                      "Co[(int64_t)c * ds + t] = cnt[c] > 0 ? Ci[(int64_t)c * ds + t]"),
     "Lloyd reseeds with the nearest point": ("if (dmin[i * M + m] > dmin[far * M + m]) far = i;", "if (dmin[i * M + m] < dmin[far * M + m]) far = i;"),
-    'train: negatives pushed the wrong way': ('if (cq[n] >= 0) gam[n] -= exp(-(dist[n] - dmin) / tau) / Z / tau;',
-                                              'if (cq[n] >= 0) gam[n] += exp(-(dist[n] - dmin) / tau) / Z / tau;'),
-    'train: anchor gradient halved': ('const double gD = gC[e] + 2.0 * lambda * delta[e];',
-                                      'const double gD = gC[e] + lambda * delta[e];'),
-    'train: w_z gradient without the sigmoid': ('g_wz[d] += gw[d] * sigmoid((double)wz[d]) / (double)nq;',
-                                                'g_wz[d] += gw[d] / (double)nq;'),
-    'train: positives summed, not averaged': ('lpos /= npos;',
-                                              'lpos /= 1;'),
-    'train: mining keeps positives': ('if (!is_pos) neg[qi * n_neg + got++] = id;',
-                                      'neg[qi * n_neg + got++] = id;'),
-    'train: W gradient without alpha': ('g_W[w] += alpha[m * r + j] * gD / (double)nq;',
-                                        'g_W[w] += gD / (double)nq;'),
-    'train: codeword gradient sign': ('gC[e] += gam[v] * (-2.0 * wf[m * ds + t] * diff);',
-                                      'gC[e] += gam[v] * (2.0 * wf[m * ds + t] * diff);'),
-    'train: bank gradient to the first fetch only': ('for (int32_t i = 0; i < h; ++i)\n            for (int32_t e = 0; e < Mr; ++e) g_bank',
-                                                     'for (int32_t i = 0; i < 1; ++i)\n            for (int32_t e = 0; e < Mr; ++e) g_bank'),
-    'train: SGD ascends': ('bank_out[e] = (float)((double)bank[e] - lr * gb[e]);',
-                           'bank_out[e] = (float)((double)bank[e] + lr * gb[e]);'),
+    "train: negatives pushed the wrong way": ("if (cq[n] >= 0) gam[n] -= exp(-(dist[n] - dmin) / tau) / Z / tau;",
+                                              "if (cq[n] >= 0) gam[n] += exp(-(dist[n] - dmin) / tau) / Z / tau;"),
+    "train: anchor gradient halved": ("const double gD = gC[e] + 2.0 * lambda * delta[e];",
+                                      "const double gD = gC[e] + lambda * delta[e];"),
+    "train: w_z gradient without the sigmoid": ("g_wz[d] += gw[d] * sigmoid((double)wz[d]) / (double)nq;",
+                                                "g_wz[d] += gw[d] / (double)nq;"),
+    "train: positives summed, not averaged": ("lpos /= npos;",
+                                              "lpos /= 1;"),
+    "train: mining keeps positives": ("if (!is_pos) neg[qi * n_neg + got++] = id;",
+                                      "neg[qi * n_neg + got++] = id;"),
+    "train: W gradient without alpha": ("g_W[w] += alpha[m * r + j] * gD / (double)nq;",
+                                        "g_W[w] += gD / (double)nq;"),
+    "train: codeword gradient sign": ("gC[e] += gam[v] * (-2.0 * wf[m * ds + t] * diff);",
+                                      "gC[e] += gam[v] * (2.0 * wf[m * ds + t] * diff);"),
+    "train: bank gradient to the first fetch only": ("for (int32_t i = 0; i < h; ++i)\n            for (int32_t e = 0; e < Mr; ++e) g_bank",
+                                                     "for (int32_t i = 0; i < 1; ++i)\n            for (int32_t e = 0; e < Mr; ++e) g_bank"),
+    "train: w_z stepped with the bank's step size": ("wz_out[d] = (float)((double)wz[d] - lr_wz * gz[d]);",
+                                                     "wz_out[d] = (float)((double)wz[d] - lr * gz[d]);"),
+    "train: SGD ascends": ("bank_out[e] = (float)((double)bank[e] - lr * gb[e]);",
+                           "bank_out[e] = (float)((double)bank[e] + lr * gb[e]);"),
 }
 
 

@@ -215,3 +215,10 @@ def test_sgd_step_is_the_gradient_step_and_descends(orc):
     np.testing.assert_array_equal(z2, (t["wz"] - lr * gz).astype(np.float32))
     L2 = _loss(orc, t, cand, P, tau, lam, bank=b2, W=W2, wz=z2)
     assert L2 < L
+    # a step size of its own for w_z: 0 keeps it, bank and W move as before
+    _, b3, W3, z3, _ = orc.train_step(t["codes"], t["cols"], t["C_pq"], t["bank"], t["W"],
+                                      t["seeds"], t["wz"], t["queries"], t["preds"], pos,
+                                      n_neg, tau, lam, lr, lr_wz=0.0)
+    np.testing.assert_array_equal(z3, t["wz"])
+    np.testing.assert_array_equal(b3, b2)
+    np.testing.assert_array_equal(W3, W2)
