@@ -742,6 +742,24 @@ def run_train(args):
         cpu = {"value": nsamp / sec, "unit": "queries/s", "cores": 1, "kind": "oracle",
                "sample": "one training step on %d queries of the %g bin (full N)" % (nsamp, b.sel)}
 
+    # roofline of the dominant kernel, the mining scan: with the codes in L2
+    # its bound is the shared-memory look-up rate (one conflict-free 32-lane
+    # load per SM per cycle); look-ups per launch = passing rows x M
+    srt = np.sort(ix.attrs[0].astype(np.int64))
+    npass = [np.searchsorted(srt, b.preds["c"][:, 0]["hi"], "left") -
+             np.searchsorted(srt, b.preds["c"][:, 0]["lo"], "left") for b in batches]
+    lookups = sum(float(npass[(args.warmup + i) % nb].sum()) * w.M for i in range(args.steps))
+    scan_ms, scan_n = stages["scan"]
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    mhz = (clk or {}).get("sm_max_mhz") or 2070.0
+    peak = sms * 32 * mhz * 1e6
+    achieved = (lookups / scan_n) / (scan_ms / scan_n / 1000.0) if scan_n else None
+    roofline = {"kernel": "k_scan (mining)", "bound": "smem", "achieved": achieved, "peak": peak,
+                "unit": "look-ups/s", "frac": achieved / peak if achieved else None, "traffic": None,
+                "peak_kind": "derived: %d SMs x 32 lanes x %.0f MHz (one conflict-free shared load "
+                             "per SM per cycle)" % (sms, mhz),
+                "avg_launch_ms": scan_ms / scan_n if scan_n else None,
+                "lookups_per_launch": lookups / scan_n if scan_n else None}
     train_ms = stages["train"][0]
     line = {
         "metric": "training throughput (queries per second through ifvs_train_step)",
@@ -756,7 +774,7 @@ def run_train(args):
                    "lr": args.train_lr, "lr_wz": args.train_lr_wz, "bins": list(w.sels),
                    "parallelism": "replicas" if world > 1 else "single",
                    "l2": "codes (%.0f MB) fit in L2" % (w.N * w.M / 1e6)},
-        "stage_ms": {k: v[0] for k, v in stages.items()},
+        "roofline": roofline, "stage_ms": {k: v[0] for k, v in stages.items()},
         "train_share": train_ms / sum(v[0] for v in stages.values()),
         "gpu_launches": launches, "clocks": clk, "e2e": e2e, "cpu_baseline": cpu,
         "loss_first": losses[0], "loss_last": losses[-1],

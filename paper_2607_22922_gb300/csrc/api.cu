@@ -114,8 +114,8 @@ struct ifvs_index {
     DevBuf w_q, w_wz, w_preds, w_canon, w_err, w_bm, w_rows, w_npass, w_idx, w_alpha, w_wf,
         w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist, w_tab;
     // training workspace
-    DevBuf t_cand, t_pos, t_mined, t_mdist, t_gC, t_gw, t_loss, t_G, t_gW, t_galpha, t_gbank,
-        t_gwz, t_wz, t_neg;
+    DevBuf t_cand, t_pos, t_mined, t_mdist, t_gC, t_gw, t_loss, t_G, t_gW, t_gWpart, t_galpha,
+        t_gbank, t_gwz, t_wz, t_neg;
     // timing
     double stage_ms[IFVS_N_STAGES] = {0};
     int64_t stage_launches[IFVS_N_STAGES] = {0};
@@ -170,7 +170,7 @@ void free_index(ifvs_index* ix) {
                       &ix->w_lut, &ix->w_cifvs, &ix->w_part, &ix->w_ids, &ix->w_dists,
                       &ix->w_cand, &ix->w_cdist, &ix->w_tab, &ix->t_cand, &ix->t_pos,
                       &ix->t_mined, &ix->t_mdist, &ix->t_gC, &ix->t_gw, &ix->t_loss, &ix->t_G,
-                      &ix->t_gW, &ix->t_galpha, &ix->t_gbank, &ix->t_gwz, &ix->t_wz, &ix->t_neg};
+                      &ix->t_gW, &ix->t_gWpart, &ix->t_galpha, &ix->t_gbank, &ix->t_gwz, &ix->t_wz, &ix->t_neg};
     for (DevBuf* b : bufs) release(*b);
     for (auto& pr : ix->pending) {
         ix->ev_free.push_back(pr.second.first);
@@ -207,8 +207,8 @@ struct Stage {
             if (a) cudaEventRecord(a, s);
         }
     }
-    cudaError_t end(cudaError_t launch_err) {
-        ix->stage_launches[stage] += 1;
+    cudaError_t end(cudaError_t launch_err, int launches = 1) {
+        ix->stage_launches[stage] += launches;
         if (on && a) {
             cudaEvent_t b = ix->event();
             if (b) {
@@ -466,6 +466,9 @@ int train_check(ifvs_index* ix, const ifvs_train_params* tp, int64_t nq, bool st
     if (ix->r > kTrainMaxR) return set_err(IFVS_ERR_UNSUPPORTED, "training supports r <= %d (index: %d)", kTrainMaxR, ix->r);
     if (train_query_smem(V, ix->M * ix->r) > (size_t)ix->max_smem)
         return set_err(IFVS_ERR_UNSUPPORTED, "M r = %d with %d candidates exceeds shared memory", ix->M * ix->r, V);
+    if (train_galpha_smem(ix->r, ix->K * ix->ds) > (size_t)ix->max_smem)
+        return set_err(IFVS_ERR_UNSUPPORTED, "r K ds = %d floats of W per subspace exceed shared memory",
+                       ix->r * ix->K * ix->ds);
     o->dio = tp->flags & IFVS_F_DEVICE_IO;
     o->timing = tp->flags & IFVS_F_STAGE_TIMING;
     o->stream = reinterpret_cast<cudaStream_t>(tp->stream);
@@ -507,8 +510,10 @@ int train_gradient(ifvs_index* ix, cudaStream_t s, const Opts& o, const TrainQue
     }
     {
         Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
-        CUDA_TRY(st.end(launch_train_gW(a.alpha, a.gC, ix->d_W, a.n, ix->M, ix->r, KD, a.lambda, inv_n,
-                                        ix->t_gW.as<float>(), s)));
+        int nl = 0;
+        const cudaError_t e = launch_train_gW(a.alpha, a.gC, ix->d_W, a.n, ix->M, ix->r, KD, a.lambda,
+                                              inv_n, ix->t_gWpart.as<float>(), ix->t_gW.as<float>(), s, &nl);
+        CUDA_TRY(st.end(e, nl));
     }
     {
         Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
@@ -536,6 +541,7 @@ int train_buffers(ifvs_index* ix, int64_t n, int V) {
     TRY(ensure(ix->t_loss, sizeof(double) * n));
     TRY(ensure(ix->t_G, sizeof(float) * ix->M * ix->r * ix->r));
     TRY(ensure(ix->t_gW, sizeof(float) * ix->M * ix->r * KD));
+    TRY(ensure(ix->t_gWpart, train_gW_scratch(n, ix->M, ix->r, (int)KD)));
     TRY(ensure(ix->t_galpha, sizeof(float) * n * Mr));
     TRY(ensure(ix->t_gbank, sizeof(float) * ix->B * Mr));
     TRY(ensure(ix->t_gwz, sizeof(float) * ix->D));

@@ -202,9 +202,13 @@ size_t train_query_smem(int V, int Mr);
 cudaError_t launch_train_gram(const float* W, int M, int r, int KD, float* G, cudaStream_t s);
 // per query: candidates, distances, softmax, loss, gC (zeroed by the caller), dL/dw_f
 cudaError_t launch_train_query(const TrainQueryArgs& a, cudaStream_t s);
-// gW [M][r][K ds] of the mean loss (written, not accumulated)
+// gW [M][r][K ds] of the mean loss (written, not accumulated); scratch of
+// train_gW_scratch bytes; *launches = kernels launched
+size_t train_gW_scratch(int64_t n, int M, int r, int KD);
 cudaError_t launch_train_gW(const float* alpha, const float* gC, const float* W, int64_t n, int M, int r,
-                            int KD, float lambda, float inv_n, float* gW, cudaStream_t s);
+                            int KD, float lambda, float inv_n, float* scratch, float* gW,
+                            cudaStream_t s, int* launches);
+size_t train_galpha_smem(int r, int KD);
 // galpha [n][M r] per query (not divided by n)
 cudaError_t launch_train_galpha(const float* gC, const float* W, const float* G, const float* alpha,
                                 int64_t n, int M, int r, int KD, float lambda, float* galpha,

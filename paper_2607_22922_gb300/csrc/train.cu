@@ -77,6 +77,7 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a)
     float* alpha = reinterpret_cast<float*>(red + kTrainWarps);   // [Mr]
     const int64_t q = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nwarps = blockDim.x >> 5;
 
     if (tid == 0) {
         const int64_t* pos = a.pos + q * a.pos_stride;
@@ -140,38 +141,50 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a)
     __syncthreads();
     for (int v = tid; v < V; v += blockDim.x) {
         double s = 0.0;
-        for (int w = 0; w < kTrainWarps; ++w) s += part[v * kTrainWarps + w];
+        for (int w = 0; w < nwarps; ++w) s += part[v * kTrainWarps + w];
         dist[v] = s;
-        gam[v] = 0.0;
     }
     __syncthreads();
 
-    // softmax of each positive against the negatives (warp 0)
+    // Softmax of each positive g against the negatives N, with the shift
+    // m_g = min(dist_g, m_N), m_N = min over N:
+    //   Z_g = exp(-(d_g - m_g)/tau) + exp(-(m_N - m_g)/tau) S,  S = sum_n u_n,
+    //   u_n = exp(-(d_n - m_N)/tau),  p_n(g) = u_n exp(-(m_N - m_g)/tau) / Z_g,
+    // so each negative's exponential is shared by all positives (warp 0).
     if (warp == 0) {
+        double mN = INFINITY;
+        for (int n = a.P + lane; n < V; n += 32)
+            if (cand[n] >= 0) mN = fmin(mN, dist[n]);
+        mN = warp_min(mN);
+        double S = 0.0;
+        for (int n = a.P + lane; n < V; n += 32) {
+            const double u = cand[n] >= 0 ? exp(-(dist[n] - mN) / a.tau) : 0.0;
+            gam[n] = u;
+            S += u;
+        }
+        S = warp_sum(S);
+        double lpos = 0.0, csum = 0.0;
         int npos = 0;
-        double lpos = 0.0;
-        for (int g = 0; g < a.P; ++g) {
+        for (int g = lane; g < a.P; g += 32) {
+            gam[g] = 0.0;
             if (cand[g] < 0) continue;
             ++npos;
-            double dm = dist[g];
-            for (int n = a.P + lane; n < V; n += 32)
-                if (cand[n] >= 0) dm = fmin(dm, dist[n]);
-            dm = warp_min(dm);
-            double z = 0.0;
-            for (int n = a.P + lane; n < V; n += 32)
-                if (cand[n] >= 0) z += exp(-(dist[n] - dm) / a.tau);
-            z = warp_sum(z) + exp(-(dist[g] - dm) / a.tau);
-            lpos += dist[g] / a.tau - dm / a.tau + log(z);
-            for (int n = a.P + lane; n < V; n += 32)
-                if (cand[n] >= 0) gam[n] -= exp(-(dist[n] - dm) / a.tau) / z / a.tau;
-            if (lane == 0) gam[g] += (1.0 - exp(-(dist[g] - dm) / a.tau) / z) / a.tau;
-            __syncwarp();
+            const double mg = fmin(dist[g], mN);
+            const double eg = exp(-(dist[g] - mg) / a.tau);
+            const double en = S > 0.0 ? exp(-(mN - mg) / a.tau) : 0.0;
+            const double z = eg + en * S;
+            lpos += dist[g] / a.tau - mg / a.tau + log(z);
+            gam[g] = (1.0 - eg / z) / a.tau;
+            csum += en / z;
         }
-        if (npos > 0) {
-            for (int v = lane; v < V; v += 32) gam[v] /= npos;
-            lpos /= npos;
-        }
-        if (lane == 0) red[0] = lpos;
+        lpos = warp_sum(lpos);
+        csum = warp_sum(csum);
+        npos = __reduce_add_sync(0xFFFFFFFFu, npos);
+        __syncwarp();
+        const double inv = npos > 0 ? 1.0 / npos : 0.0;
+        for (int n = a.P + lane; n < V; n += 32) gam[n] = -gam[n] * csum / a.tau * inv;
+        for (int g = lane; g < a.P; g += 32) gam[g] *= inv;
+        if (lane == 0) red[0] = npos > 0 ? lpos * inv : 0.0;
     }
     // anchor ||Delta||^2 = sum_m alpha[m]^T G_m alpha[m]
     double an = 0.0;
@@ -189,7 +202,7 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a)
     __syncthreads();
     if (tid == 0) {
         double s = 0.0;
-        for (int w = 0; w < kTrainWarps; ++w) s += red[w];
+        for (int w = 0; w < nwarps; ++w) s += red[w];
         a.loss[q] = lpos + (double)a.lambda * s;
     }
 
@@ -211,120 +224,195 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a)
     }
 }
 
-// dL/dW[m][j][e] = inv_n (sum_q alpha_q[m][j] gC_q[m][e] + 2 lambda sum_j' A_m[j][j'] W[m][j'][e]);
-// grid (M, ceil(KD / 256)); r <= kTrainMaxR
-__global__ void __launch_bounds__(kTrainThreads) k_train_gW(const float* __restrict__ alpha,
-                                                            const float* __restrict__ gC,
-                                                            const float* __restrict__ W, int64_t n,
-                                                            int M, int r, int KD, float lambda,
-                                                            float inv_n, float* __restrict__ gW) {
-    __shared__ float A[kTrainMaxR * kTrainMaxR];
-    __shared__ float as[kTrainThreads * kTrainMaxR / 8];   // alpha of a chunk of queries
-    const int m = blockIdx.x;
-    const int e = blockIdx.y * kTrainThreads + threadIdx.x;
+// A[m][j][j'] = sum over the queries of alpha_q[m][j] alpha_q[m][j'] (one CTA per entry)
+__global__ void __launch_bounds__(kTrainThreads) k_train_acov(const float* __restrict__ alpha, int64_t n,
+                                                              int M, int r, float* __restrict__ A) {
+    __shared__ float part[kTrainWarps];
+    const int b = blockIdx.x;
+    const int m = b / (r * r), j = (b / r) % r, j2 = b % r;
     const int Mr = M * r;
-    for (int t = threadIdx.x; t < r * r; t += kTrainThreads) {
-        const int j = t / r, j2 = t % r;
-        float s = 0.f;
-        for (int64_t q = 0; q < n; ++q) s += alpha[q * Mr + m * r + j] * alpha[q * Mr + m * r + j2];
-        A[t] = s;
-    }
-    float acc[kTrainMaxR];
+    float s = 0.f;
+    for (int64_t q = threadIdx.x; q < n; q += kTrainThreads)
+        s += alpha[q * Mr + m * r + j] * alpha[q * Mr + m * r + j2];
 #pragma unroll
-    for (int j = 0; j < kTrainMaxR; ++j) acc[j] = 0.f;
-    const int qc = (kTrainThreads * kTrainMaxR / 8) / r;   // queries per staged chunk
-    for (int64_t q0 = 0; q0 < n; q0 += qc) {
-        const int nc = (int)min((int64_t)qc, n - q0);
-        __syncthreads();
-        for (int t = threadIdx.x; t < nc * r; t += kTrainThreads)
-            as[t] = alpha[(q0 + t / r) * Mr + m * r + t % r];
-        __syncthreads();
-        if (e < KD)
-            for (int i = 0; i < nc; ++i) {
-                const float g = gC[((q0 + i) * M + m) * (int64_t)KD + e];
-#pragma unroll
-                for (int j = 0; j < kTrainMaxR; ++j)
-                    if (j < r) acc[j] += as[i * r + j] * g;
-            }
-    }
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+    if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = s;
     __syncthreads();
-    if (e >= KD) return;
-#pragma unroll
-    for (int j = 0; j < kTrainMaxR; ++j) {
-        if (j >= r) break;
-        float an = 0.f;
-        for (int j2 = 0; j2 < r; ++j2) an += A[j * r + j2] * W[((int64_t)m * r + j2) * KD + e];
-        gW[((int64_t)m * r + j) * KD + e] = (acc[j] + 2.f * lambda * an) * inv_n;
+    if (threadIdx.x == 0) {
+        float t = 0.f;
+        for (int w = 0; w < kTrainWarps; ++w) t += part[w];
+        A[b] = t;
     }
 }
 
-// dL/dalpha_q[m][j] = <gC_q[m], W[m][j]> + 2 lambda sum_j' G_m[j][j'] alpha_q[m][j'];
-// grid (n, M)
+// Partial sums of alpha_q[m][j] gC_q[m][e] over one slice of kGWQueries
+// queries: grid (M, ceil(KD / 256), slices); part [slices][M][r][KD]
+constexpr int kGWQueries = 64;
+__global__ void __launch_bounds__(kTrainThreads) k_train_gW_part(const float* __restrict__ alpha,
+                                                                 const float* __restrict__ gC, int64_t n,
+                                                                 int M, int r, int KD,
+                                                                 float* __restrict__ part) {
+    __shared__ float as[kGWQueries * kTrainMaxR];
+    const int m = blockIdx.x;
+    const int e = blockIdx.y * kTrainThreads + threadIdx.x;
+    const int64_t q0 = (int64_t)blockIdx.z * kGWQueries;
+    const int nc = (int)min((int64_t)kGWQueries, n - q0);
+    const int Mr = M * r;
+    for (int t = threadIdx.x; t < nc * r; t += kTrainThreads)
+        as[t] = alpha[(q0 + t / r) * Mr + m * r + t % r];
+    __syncthreads();
+    if (e >= KD) return;
+    float acc[kTrainMaxR];
+#pragma unroll
+    for (int j = 0; j < kTrainMaxR; ++j) acc[j] = 0.f;
+    for (int i = 0; i < nc; ++i) {
+        const float g = gC[((q0 + i) * M + m) * (int64_t)KD + e];
+#pragma unroll
+        for (int j = 0; j < kTrainMaxR; ++j)
+            if (j < r) acc[j] += as[i * r + j] * g;
+    }
+    float* out = part + (((int64_t)blockIdx.z * M + m) * r) * KD + e;
+#pragma unroll
+    for (int j = 0; j < kTrainMaxR; ++j)
+        if (j < r) out[(int64_t)j * KD] = acc[j];
+}
+
+// dL/dW[m][j][e] = inv_n (sum over slices of part + 2 lambda sum_j' A_m[j][j'] W[m][j'][e]),
+// slices summed in order
+__global__ void k_train_gW_sum(const float* __restrict__ part, int slices, const float* __restrict__ A,
+                               const float* __restrict__ W, int M, int r, int KD, float lambda,
+                               float inv_n, float* __restrict__ gW) {
+    const int64_t total = (int64_t)M * r * KD;
+    const int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (x >= total) return;
+    const int e = (int)(x % KD);
+    const int j = (int)((x / KD) % r);
+    const int m = (int)(x / ((int64_t)KD * r));
+    float s = 0.f;
+    for (int z = 0; z < slices; ++z) s += part[(int64_t)z * total + x];
+    float an = 0.f;
+    for (int j2 = 0; j2 < r; ++j2)
+        an += A[((int64_t)m * r + j) * r + j2] * W[((int64_t)m * r + j2) * KD + e];
+    gW[x] = (s + 2.f * lambda * an) * inv_n;
+}
+
+// dL/dalpha_q[m][j] = <gC_q[m], W[m][j]> + 2 lambda sum_j' G_m[j][j'] alpha_q[m][j'].
+// grid (M, ceil(n / kGAQueries)); W[m] staged in shared memory once per CTA,
+// one warp per query at a time.
+constexpr int kGAQueries = 32;
 __global__ void __launch_bounds__(kTrainThreads) k_train_galpha(const float* __restrict__ gC,
                                                                 const float* __restrict__ W,
                                                                 const float* __restrict__ G,
                                                                 const float* __restrict__ alpha,
-                                                                int M, int r, int KD, float lambda,
-                                                                float* __restrict__ galpha) {
-    __shared__ float part[kTrainWarps][kTrainMaxR];
-    const int64_t q = blockIdx.x;
-    const int m = blockIdx.y;
+                                                                int64_t n, int M, int r, int KD,
+                                                                float lambda, float* __restrict__ galpha) {
+    extern __shared__ __align__(16) float Ws[];     // [r][KD]
+    const int m = blockIdx.x;
+    const int64_t q0 = (int64_t)blockIdx.y * kGAQueries;
     const int Mr = M * r;
-    const float* g = gC + (q * M + m) * (int64_t)KD;
-    float acc[kTrainMaxR];
-#pragma unroll
-    for (int j = 0; j < kTrainMaxR; ++j) acc[j] = 0.f;
-    for (int e = threadIdx.x; e < KD; e += kTrainThreads) {
-        const float ge = g[e];
-        if (ge == 0.f) continue;
-#pragma unroll
-        for (int j = 0; j < kTrainMaxR; ++j)
-            if (j < r) acc[j] += ge * W[((int64_t)m * r + j) * KD + e];
-    }
-#pragma unroll
-    for (int j = 0; j < kTrainMaxR; ++j) {
-        float s = acc[j];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-        if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5][j] = s;
-    }
+    const float* Wm = W + (int64_t)m * r * KD;
+    for (int t = threadIdx.x; t < r * KD; t += kTrainThreads) Ws[t] = Wm[t];
     __syncthreads();
-    if (threadIdx.x < r) {
-        const int j = threadIdx.x;
-        float s = 0.f;
-        for (int w = 0; w < kTrainWarps; ++w) s += part[w][j];
-        float an = 0.f;
-        for (int j2 = 0; j2 < r; ++j2) an += G[((int64_t)m * r + j) * r + j2] * alpha[q * Mr + m * r + j2];
-        galpha[q * Mr + m * r + j] = s + 2.f * lambda * an;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int i = warp; i < kGAQueries; i += kTrainWarps) {
+        const int64_t q = q0 + i;
+        if (q >= n) break;
+        const float* g = gC + (q * M + m) * (int64_t)KD;
+        float acc[kTrainMaxR];
+#pragma unroll
+        for (int j = 0; j < kTrainMaxR; ++j) acc[j] = 0.f;
+        for (int e = lane; e < KD; e += 32) {
+            const float ge = g[e];
+#pragma unroll
+            for (int j = 0; j < kTrainMaxR; ++j)
+                if (j < r) acc[j] += ge * Ws[j * KD + e];
+        }
+#pragma unroll
+        for (int j = 0; j < kTrainMaxR; ++j) {
+            if (j >= r) break;
+            float v = acc[j];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+            acc[j] = v;
+        }
+        if (lane < r) {
+            float mine = 0.f;
+#pragma unroll
+            for (int j = 0; j < kTrainMaxR; ++j)
+                if (j == lane) mine = acc[j];
+            float an = 0.f;
+            for (int j2 = 0; j2 < r; ++j2)
+                an += G[((int64_t)m * r + lane) * r + j2] * alpha[q * Mr + m * r + j2];
+            galpha[q * Mr + m * r + lane] = mine + 2.f * lambda * an;
+        }
     }
 }
 
-// dL/dbank: one CTA per fetch p = (q, i); the first fetch of each bank row
-// sums, in fetch order, the dL/dalpha of every fetch of that row
-__global__ void k_train_bank(const uint32_t* __restrict__ idx, int64_t n_fetch, int h, int Mr,
-                             const float* __restrict__ galpha, float inv_n, float* __restrict__ gbank) {
+// dL/dbank: one CTA per fetch p = (q, i).  The first fetch of each bank row
+// gathers, in fetch order, the fetches of that row and sums their dL/dalpha.
+constexpr int kBankList = 512;
+__global__ void __launch_bounds__(kTrainThreads) k_train_bank(const uint32_t* __restrict__ idx,
+                                                              int64_t n_fetch, int h, int Mr,
+                                                              const float* __restrict__ galpha,
+                                                              float inv_n, float* __restrict__ gbank) {
+    __shared__ int64_t list[kBankList];
+    __shared__ int wcnt[kTrainWarps];
+    __shared__ int total;
     const int64_t p = blockIdx.x;
     const uint32_t b = idx[p];
-    for (int64_t p2 = 0; p2 < p; ++p2)
-        if (idx[p2] == b) return;
+    int earlier = 0;
+    for (int64_t p2 = threadIdx.x; p2 < p; p2 += blockDim.x) earlier |= idx[p2] == b;
+    if (__syncthreads_or(earlier)) return;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    if (threadIdx.x == 0) total = 0;
+    __syncthreads();
+    for (int64_t c0 = p; c0 < n_fetch; c0 += blockDim.x) {
+        const int64_t p2 = c0 + threadIdx.x;
+        const bool f = p2 < n_fetch && idx[p2] == b;
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, f);
+        if (lane == 0) wcnt[warp] = __popc(bal);
+        __syncthreads();
+        int off = total;
+        for (int w = 0; w < warp; ++w) off += wcnt[w];
+        off += __popc(bal & ((1u << lane) - 1u));
+        if (f && off < kBankList) list[off] = p2;
+        __syncthreads();
+        if (threadIdx.x == 0)
+            for (int w = 0; w < nw; ++w) total += wcnt[w];
+        __syncthreads();
+    }
+    const int cnt = total;
     for (int e = threadIdx.x; e < Mr; e += blockDim.x) {
         float s = 0.f;
-        for (int64_t p2 = p; p2 < n_fetch; ++p2)
-            if (idx[p2] == b) s += galpha[(p2 / h) * Mr + e];
+        if (cnt <= kBankList) {
+            for (int i = 0; i < cnt; ++i) s += galpha[(list[i] / h) * Mr + e];
+        } else {
+            for (int64_t p2 = p; p2 < n_fetch; ++p2)
+                if (idx[p2] == b) s += galpha[(p2 / h) * Mr + e];
+        }
         gbank[(int64_t)b * Mr + e] = s * inv_n;
     }
 }
 
-// dL/dw_z[d] = inv_n sum_q dL/dw_f[q][d] sigmoid(w_z[d])
-__global__ void k_train_wz(const float* __restrict__ gw, int64_t n, int D, const float* __restrict__ wz,
-                           float inv_n, float* __restrict__ gwz) {
-    const int d = blockIdx.x * blockDim.x + threadIdx.x;
-    if (d >= D) return;
+// dL/dw_z[d] = inv_n sum_q dL/dw_f[q][d] sigmoid(w_z[d]); block (32 dims, 32
+// query lanes), lane y sums the queries q = y (mod 32) in order, then the 32
+// lanes are added in order
+__global__ void __launch_bounds__(1024) k_train_wz(const float* __restrict__ gw, int64_t n, int D,
+                                                   const float* __restrict__ wz, float inv_n,
+                                                   float* __restrict__ gwz) {
+    __shared__ double part[32][33];
+    const int d = blockIdx.x * 32 + threadIdx.x;
     double s = 0.0;
-    for (int64_t q = 0; q < n; ++q) s += (double)gw[q * D + d];
+    if (d < D)
+        for (int64_t q = threadIdx.y; q < n; q += 32) s += (double)gw[q * D + d];
+    part[threadIdx.y][threadIdx.x] = s;
+    __syncthreads();
+    if (threadIdx.y != 0 || d >= D) return;
+    double t = 0.0;
+    for (int y = 0; y < 32; ++y) t += part[y][threadIdx.x];
     const float x = wz[d];
     const float sg = x >= 0.f ? 1.f / (1.f + expf(-x)) : expf(x) / (1.f + expf(x));
-    gwz[d] = (float)s * sg * inv_n;
+    gwz[d] = (float)t * sg * inv_n;
 }
 
 // theta <- theta - lr * g
@@ -347,35 +435,59 @@ cudaError_t launch_train_query(const TrainQueryArgs& a, cudaStream_t s) {
     const size_t smem = train_query_smem(a.P + a.n_neg, a.M * a.r);
     cudaError_t e = cudaFuncSetAttribute(k_train_query, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k_train_query<<<(unsigned)a.n, kTrainThreads, smem, s>>>(a);
+    // threads own dimensions: no more threads than (32-rounded) dimensions
+    const int threads = a.D >= kTrainThreads ? kTrainThreads : ((a.D + 31) / 32) * 32;
+    k_train_query<<<(unsigned)a.n, threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
+size_t train_gW_scratch(int64_t n, int M, int r, int KD) {
+    const int64_t slices = (n + kGWQueries - 1) / kGWQueries;
+    return sizeof(float) * (size_t)(slices * M * r * KD + M * r * r);
+}
+
 cudaError_t launch_train_gW(const float* alpha, const float* gC, const float* W, int64_t n, int M, int r,
-                            int KD, float lambda, float inv_n, float* gW, cudaStream_t s) {
-    dim3 grid((unsigned)M, (unsigned)((KD + kTrainThreads - 1) / kTrainThreads));
-    k_train_gW<<<grid, kTrainThreads, 0, s>>>(alpha, gC, W, n, M, r, KD, lambda, inv_n, gW);
+                            int KD, float lambda, float inv_n, float* scratch, float* gW,
+                            cudaStream_t s, int* launches) {
+    const int slices = (int)((n + kGWQueries - 1) / kGWQueries);
+    float* A = scratch;
+    float* part = scratch + M * r * r;
+    k_train_acov<<<(unsigned)(M * r * r), kTrainThreads, 0, s>>>(alpha, n, M, r, A);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)M, (unsigned)((KD + kTrainThreads - 1) / kTrainThreads), (unsigned)slices);
+    k_train_gW_part<<<grid, kTrainThreads, 0, s>>>(alpha, gC, n, M, r, KD, part);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const int64_t total = (int64_t)M * r * KD;
+    k_train_gW_sum<<<(unsigned)((total + 255) / 256), 256, 0, s>>>(part, slices, A, W, M, r, KD, lambda,
+                                                                    inv_n, gW);
+    if (launches) *launches = 3;
     return cudaGetLastError();
 }
 
 cudaError_t launch_train_galpha(const float* gC, const float* W, const float* G, const float* alpha,
                                 int64_t n, int M, int r, int KD, float lambda, float* galpha,
                                 cudaStream_t s) {
-    dim3 grid((unsigned)n, (unsigned)M);
-    k_train_galpha<<<grid, kTrainThreads, 0, s>>>(gC, W, G, alpha, M, r, KD, lambda, galpha);
+    const size_t smem = sizeof(float) * (size_t)r * KD;
+    cudaError_t e = cudaFuncSetAttribute(k_train_galpha, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)M, (unsigned)((n + kGAQueries - 1) / kGAQueries));
+    k_train_galpha<<<grid, kTrainThreads, smem, s>>>(gC, W, G, alpha, n, M, r, KD, lambda, galpha);
     return cudaGetLastError();
 }
 
+size_t train_galpha_smem(int r, int KD) { return sizeof(float) * (size_t)r * KD; }
+
 cudaError_t launch_train_bank(const uint32_t* idx, int64_t n, int h, int Mr, const float* galpha,
                               float inv_n, float* gbank, cudaStream_t s) {
-    const int threads = Mr < 256 ? ((Mr + 31) / 32) * 32 : 256;
+    const int threads = Mr < kTrainThreads ? ((Mr + 31) / 32) * 32 : kTrainThreads;
     k_train_bank<<<(unsigned)(n * h), threads, 0, s>>>(idx, n * h, h, Mr, galpha, inv_n, gbank);
     return cudaGetLastError();
 }
 
 cudaError_t launch_train_wz(const float* gw, int64_t n, int D, const float* wz, float inv_n, float* gwz,
                             cudaStream_t s) {
-    k_train_wz<<<(unsigned)((D + 127) / 128), 128, 0, s>>>(gw, n, D, wz, inv_n, gwz);
+    k_train_wz<<<(unsigned)((D + 31) / 32), dim3(32, 32), 0, s>>>(gw, n, D, wz, inv_n, gwz);
     return cudaGetLastError();
 }
 
