@@ -464,11 +464,9 @@ int train_check(ifvs_index* ix, const ifvs_train_params* tp, int64_t nq, bool st
     if (step) TRY(check_scan_fits(ix, V));
     if (nq < 0 || nq > 1024) return set_err(IFVS_ERR_ARG, "nq = %lld outside 0..1024 (one mini-batch per call)", (long long)nq);
     if (ix->r > kTrainMaxR) return set_err(IFVS_ERR_UNSUPPORTED, "training supports r <= %d (index: %d)", kTrainMaxR, ix->r);
-    if (train_query_smem(V, ix->M * ix->r) > (size_t)ix->max_smem)
-        return set_err(IFVS_ERR_UNSUPPORTED, "M r = %d with %d candidates exceeds shared memory", ix->M * ix->r, V);
-    if (train_galpha_smem(ix->r, ix->K * ix->ds) > (size_t)ix->max_smem)
-        return set_err(IFVS_ERR_UNSUPPORTED, "r K ds = %d floats of W per subspace exceed shared memory",
-                       ix->r * ix->K * ix->ds);
+    if (train_query_smem(V, ix->M * ix->r, ix->D, ix->r) > (size_t)ix->max_smem)
+        return set_err(IFVS_ERR_UNSUPPORTED, "D = %d, M r = %d with %d candidates exceed shared memory",
+                       ix->D, ix->M * ix->r, V);
     o->dio = tp->flags & IFVS_F_DEVICE_IO;
     o->timing = tp->flags & IFVS_F_STAGE_TIMING;
     o->stream = reinterpret_cast<cudaStream_t>(tp->stream);
@@ -514,11 +512,6 @@ int train_gradient(ifvs_index* ix, cudaStream_t s, const Opts& o, const TrainQue
         const cudaError_t e = launch_train_gW(a.alpha, a.gC, ix->d_W, a.n, ix->M, ix->r, KD, a.lambda,
                                               inv_n, ix->t_gWpart.as<float>(), ix->t_gW.as<float>(), s, &nl);
         CUDA_TRY(st.end(e, nl));
-    }
-    {
-        Stage st(ix, s, o.timing, IFVS_STAGE_TRAIN);
-        CUDA_TRY(st.end(launch_train_galpha(a.gC, ix->d_W, ix->t_G.as<float>(), a.alpha, a.n, ix->M,
-                                            ix->r, KD, a.lambda, ix->t_galpha.as<float>(), s)));
     }
     CUDA_TRY(cudaMemsetAsync(ix->t_gbank.p, 0, sizeof(float) * (size_t)ix->B * Mr, s));
     {
@@ -576,6 +569,7 @@ TrainQueryArgs train_args(ifvs_index* ix, const ifvs_train_params* tp, int64_t n
     a.err = ix->w_err.as<int>();
     a.gC = ix->t_gC.as<float>();
     a.gw = ix->t_gw.as<float>();
+    a.galpha = ix->t_galpha.as<float>();
     a.loss = ix->t_loss.as<double>();
     return a;
 }

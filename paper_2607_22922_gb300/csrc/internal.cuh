@@ -195,12 +195,13 @@ struct TrainQueryArgs {
     int64_t* neg_out;              // [n][n_neg] or null
     float* gC;                     // [n][M][K][ds] scratch
     float* gw;                     // [n][D] scratch: dL/dw_f per query
+    float* galpha;                 // [n][M r] dL/dalpha per query (not divided by n)
     double* loss;                  // [n]
 };
-size_t train_query_smem(int V, int Mr);
+size_t train_query_smem(int V, int Mr, int D, int r);
 // G [M][r][r] = W[m] W[m]^T
 cudaError_t launch_train_gram(const float* W, int M, int r, int KD, float* G, cudaStream_t s);
-// per query: candidates, distances, softmax, loss, gC (zeroed by the caller), dL/dw_f
+// per query: candidates, distances, softmax, loss, gC (zeroed by the caller), dL/dw_f, dL/dalpha
 cudaError_t launch_train_query(const TrainQueryArgs& a, cudaStream_t s);
 // gW [M][r][K ds] of the mean loss (written, not accumulated); scratch of
 // train_gW_scratch bytes; *launches = kernels launched
@@ -208,11 +209,7 @@ size_t train_gW_scratch(int64_t n, int M, int r, int KD);
 cudaError_t launch_train_gW(const float* alpha, const float* gC, const float* W, int64_t n, int M, int r,
                             int KD, float lambda, float inv_n, float* scratch, float* gW,
                             cudaStream_t s, int* launches);
-size_t train_galpha_smem(int r, int KD);
-// galpha [n][M r] per query (not divided by n)
-cudaError_t launch_train_galpha(const float* gC, const float* W, const float* G, const float* alpha,
-                                int64_t n, int M, int r, int KD, float lambda, float* galpha,
-                                cudaStream_t s);
+
 // gbank rows fetched by the batch (other rows must be zeroed by the caller)
 cudaError_t launch_train_bank(const uint32_t* idx, int64_t n, int h, int Mr, const float* galpha,
                               float inv_n, float* gbank, cudaStream_t s);

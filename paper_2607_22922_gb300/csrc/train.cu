@@ -10,7 +10,8 @@
 //   dL/dW[m][j]         = sum_q alpha_q[m][j] gC_q[m] + 2 lambda sum_j' A_m[j][j'] W[m][j']
 //                         with A_m = sum_q alpha_q[m] alpha_q[m]^T
 //   dL/dalpha_q[m][j]   = <gC_q[m], W[m][j]> + 2 lambda sum_j' G_m[j][j'] alpha_q[m][j']
-//                         with the Gram matrix G_m = W[m] W[m]^T
+//                         with the Gram matrix G_m = W[m] W[m]^T, formed per candidate
+//                         while gC is scattered (the W values are already loaded)
 //   dL/dbank[b]         = sum over the fetches (q, i) with idx_i(q) = b of dL/dalpha_q
 //   dL/dw_z             = dL/dw_f sigmoid(w_z)
 // (each divided by the number of queries).  Every sum runs in a fixed order
@@ -75,6 +76,7 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a)
     double* gam = dist + V;                                   // [V]
     double* red = gam + V;                                    // [warps]
     float* alpha = reinterpret_cast<float*>(red + kTrainWarps);   // [Mr]
+    float* gas = alpha + Mr;                                      // [D][r]: dL/dalpha per dimension
     const int64_t q = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int nwarps = blockDim.x >> 5;
@@ -206,21 +208,43 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a)
         a.loss[q] = lpos + (double)a.lambda * s;
     }
 
-    // pass 2: gC scatter and dL/dw_f
+    // pass 2: gC scatter, dL/dw_f, and dL/dalpha through the same W values:
+    // dL/dalpha[m][j] = sum over (v, t) of gC contribution x W[m][j][c_v][t]
     float* gC = a.gC + q * (int64_t)a.M * KD;
     for (int d = tid; d < a.D; d += blockDim.x) {
         const int m = d / a.ds, t = d - m * a.ds;
         double gw = 0.0;
+        float ga[kTrainMaxR];
+#pragma unroll
+        for (int j = 0; j < kTrainMaxR; ++j) ga[j] = 0.f;
         for (int v = 0; v < V; ++v) {
             const int64_t id = cand[v];
             if (id < 0) continue;
             int c;
             const float df = diff_of(id, d, &c);
-            const float gv = (float)gam[v];
-            gC[(int64_t)m * KD + (int64_t)c * a.ds + t] += gv * (-2.f * wf[d] * df);
+            const float ge = (float)gam[v] * (-2.f * wf[d] * df);
+            const int64_t e = (int64_t)c * a.ds + t;
+            gC[(int64_t)m * KD + e] += ge;
             gw += gam[v] * (double)(df * df);
+            const float* Wc = a.W + (int64_t)m * a.r * KD + e;
+#pragma unroll
+            for (int j = 0; j < kTrainMaxR; ++j)
+                if (j < a.r) ga[j] += ge * Wc[(int64_t)j * KD];
         }
         a.gw[q * a.D + d] = (float)gw;
+#pragma unroll
+        for (int j = 0; j < kTrainMaxR; ++j)
+            if (j < a.r) gas[d * a.r + j] = ga[j];
+    }
+    __syncthreads();
+    // sum over the subspace's dimensions in order, plus the anchor 2 lambda G_m alpha[m]
+    for (int x = tid; x < Mr; x += blockDim.x) {
+        const int m = x / a.r, j = x - m * a.r;
+        float sg = 0.f;
+        for (int t = 0; t < a.ds; ++t) sg += gas[(m * a.ds + t) * a.r + j];
+        float an = 0.f;
+        for (int j2 = 0; j2 < a.r; ++j2) an += a.G[((int64_t)m * a.r + j) * a.r + j2] * alpha[m * a.r + j2];
+        a.galpha[q * Mr + x] = sg + 2.f * a.lambda * an;
     }
 }
 
@@ -265,6 +289,7 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_gW_part(const float* __
     float acc[kTrainMaxR];
 #pragma unroll
     for (int j = 0; j < kTrainMaxR; ++j) acc[j] = 0.f;
+#pragma unroll 8
     for (int i = 0; i < nc; ++i) {
         const float g = gC[((q0 + i) * M + m) * (int64_t)KD + e];
 #pragma unroll
@@ -294,58 +319,6 @@ __global__ void k_train_gW_sum(const float* __restrict__ part, int slices, const
     for (int j2 = 0; j2 < r; ++j2)
         an += A[((int64_t)m * r + j) * r + j2] * W[((int64_t)m * r + j2) * KD + e];
     gW[x] = (s + 2.f * lambda * an) * inv_n;
-}
-
-// dL/dalpha_q[m][j] = <gC_q[m], W[m][j]> + 2 lambda sum_j' G_m[j][j'] alpha_q[m][j'].
-// grid (M, ceil(n / kGAQueries)); W[m] staged in shared memory once per CTA,
-// one warp per query at a time.
-constexpr int kGAQueries = 32;
-__global__ void __launch_bounds__(kTrainThreads) k_train_galpha(const float* __restrict__ gC,
-                                                                const float* __restrict__ W,
-                                                                const float* __restrict__ G,
-                                                                const float* __restrict__ alpha,
-                                                                int64_t n, int M, int r, int KD,
-                                                                float lambda, float* __restrict__ galpha) {
-    extern __shared__ __align__(16) float Ws[];     // [r][KD]
-    const int m = blockIdx.x;
-    const int64_t q0 = (int64_t)blockIdx.y * kGAQueries;
-    const int Mr = M * r;
-    const float* Wm = W + (int64_t)m * r * KD;
-    for (int t = threadIdx.x; t < r * KD; t += kTrainThreads) Ws[t] = Wm[t];
-    __syncthreads();
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int i = warp; i < kGAQueries; i += kTrainWarps) {
-        const int64_t q = q0 + i;
-        if (q >= n) break;
-        const float* g = gC + (q * M + m) * (int64_t)KD;
-        float acc[kTrainMaxR];
-#pragma unroll
-        for (int j = 0; j < kTrainMaxR; ++j) acc[j] = 0.f;
-        for (int e = lane; e < KD; e += 32) {
-            const float ge = g[e];
-#pragma unroll
-            for (int j = 0; j < kTrainMaxR; ++j)
-                if (j < r) acc[j] += ge * Ws[j * KD + e];
-        }
-#pragma unroll
-        for (int j = 0; j < kTrainMaxR; ++j) {
-            if (j >= r) break;
-            float v = acc[j];
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-            acc[j] = v;
-        }
-        if (lane < r) {
-            float mine = 0.f;
-#pragma unroll
-            for (int j = 0; j < kTrainMaxR; ++j)
-                if (j == lane) mine = acc[j];
-            float an = 0.f;
-            for (int j2 = 0; j2 < r; ++j2)
-                an += G[((int64_t)m * r + lane) * r + j2] * alpha[q * Mr + m * r + j2];
-            galpha[q * Mr + m * r + lane] = mine + 2.f * lambda * an;
-        }
-    }
 }
 
 // dL/dbank: one CTA per fetch p = (q, i).  The first fetch of each bank row
@@ -421,9 +394,9 @@ __global__ void k_sgd(float* __restrict__ theta, const float* __restrict__ g, in
     if (e < n) theta[e] = theta[e] - lr * g[e];
 }
 
-size_t train_query_smem(int V, int Mr) {
+size_t train_query_smem(int V, int Mr, int D, int r) {
     return sizeof(int64_t) * V + sizeof(double) * ((size_t)V * kTrainWarps + 2 * V + kTrainWarps) +
-           sizeof(float) * Mr;
+           sizeof(float) * (Mr + (size_t)D * r);
 }
 
 cudaError_t launch_train_gram(const float* W, int M, int r, int KD, float* G, cudaStream_t s) {
@@ -432,7 +405,7 @@ cudaError_t launch_train_gram(const float* W, int M, int r, int KD, float* G, cu
 }
 
 cudaError_t launch_train_query(const TrainQueryArgs& a, cudaStream_t s) {
-    const size_t smem = train_query_smem(a.P + a.n_neg, a.M * a.r);
+    const size_t smem = train_query_smem(a.P + a.n_neg, a.M * a.r, a.D, a.r);
     cudaError_t e = cudaFuncSetAttribute(k_train_query, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     // threads own dimensions: no more threads than (32-rounded) dimensions
@@ -464,19 +437,6 @@ cudaError_t launch_train_gW(const float* alpha, const float* gC, const float* W,
     if (launches) *launches = 3;
     return cudaGetLastError();
 }
-
-cudaError_t launch_train_galpha(const float* gC, const float* W, const float* G, const float* alpha,
-                                int64_t n, int M, int r, int KD, float lambda, float* galpha,
-                                cudaStream_t s) {
-    const size_t smem = sizeof(float) * (size_t)r * KD;
-    cudaError_t e = cudaFuncSetAttribute(k_train_galpha, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    dim3 grid((unsigned)M, (unsigned)((n + kGAQueries - 1) / kGAQueries));
-    k_train_galpha<<<grid, kTrainThreads, smem, s>>>(gC, W, G, alpha, n, M, r, KD, lambda, galpha);
-    return cudaGetLastError();
-}
-
-size_t train_galpha_smem(int r, int KD) { return sizeof(float) * (size_t)r * KD; }
 
 cudaError_t launch_train_bank(const uint32_t* idx, int64_t n, int h, int Mr, const float* galpha,
                               float inv_n, float* gbank, cudaStream_t s) {
