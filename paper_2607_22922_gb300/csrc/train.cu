@@ -66,6 +66,7 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_gram(const float* __res
 // scatter of dL/dC into the query's dense gC slice and dL/dw_f.  Each thread
 // owns the dimensions d = tid + i * blockDim, so every gC address (m, *, t)
 // is written by one thread only, in candidate order.
+template <int RMAX>
 __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a) {
     extern __shared__ __align__(16) unsigned char sm[];
     const int V = a.P + a.n_neg;
@@ -214,9 +215,9 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a)
     for (int d = tid; d < a.D; d += blockDim.x) {
         const int m = d / a.ds, t = d - m * a.ds;
         double gw = 0.0;
-        float ga[kTrainMaxR];
+        float ga[RMAX];
 #pragma unroll
-        for (int j = 0; j < kTrainMaxR; ++j) ga[j] = 0.f;
+        for (int j = 0; j < RMAX; ++j) ga[j] = 0.f;
         for (int v = 0; v < V; ++v) {
             const int64_t id = cand[v];
             if (id < 0) continue;
@@ -228,12 +229,12 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_query(TrainQueryArgs a)
             gw += gam[v] * (double)(df * df);
             const float* Wc = a.W + (int64_t)m * a.r * KD + e;
 #pragma unroll
-            for (int j = 0; j < kTrainMaxR; ++j)
+            for (int j = 0; j < RMAX; ++j)
                 if (j < a.r) ga[j] += ge * Wc[(int64_t)j * KD];
         }
         a.gw[q * a.D + d] = (float)gw;
 #pragma unroll
-        for (int j = 0; j < kTrainMaxR; ++j)
+        for (int j = 0; j < RMAX; ++j)
             if (j < a.r) gas[d * a.r + j] = ga[j];
     }
     __syncthreads();
@@ -272,6 +273,7 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_acov(const float* __res
 // Partial sums of alpha_q[m][j] gC_q[m][e] over one slice of kGWQueries
 // queries: grid (M, ceil(KD / 256), slices); part [slices][M][r][KD]
 constexpr int kGWQueries = 64;
+template <int RMAX>
 __global__ void __launch_bounds__(kTrainThreads) k_train_gW_part(const float* __restrict__ alpha,
                                                                  const float* __restrict__ gC, int64_t n,
                                                                  int M, int r, int KD,
@@ -286,19 +288,19 @@ __global__ void __launch_bounds__(kTrainThreads) k_train_gW_part(const float* __
         as[t] = alpha[(q0 + t / r) * Mr + m * r + t % r];
     __syncthreads();
     if (e >= KD) return;
-    float acc[kTrainMaxR];
+    float acc[RMAX];
 #pragma unroll
-    for (int j = 0; j < kTrainMaxR; ++j) acc[j] = 0.f;
+    for (int j = 0; j < RMAX; ++j) acc[j] = 0.f;
 #pragma unroll 8
     for (int i = 0; i < nc; ++i) {
         const float g = gC[((q0 + i) * M + m) * (int64_t)KD + e];
 #pragma unroll
-        for (int j = 0; j < kTrainMaxR; ++j)
+        for (int j = 0; j < RMAX; ++j)
             if (j < r) acc[j] += as[i * r + j] * g;
     }
     float* out = part + (((int64_t)blockIdx.z * M + m) * r) * KD + e;
 #pragma unroll
-    for (int j = 0; j < kTrainMaxR; ++j)
+    for (int j = 0; j < RMAX; ++j)
         if (j < r) out[(int64_t)j * KD] = acc[j];
 }
 
@@ -406,11 +408,12 @@ cudaError_t launch_train_gram(const float* W, int M, int r, int KD, float* G, cu
 
 cudaError_t launch_train_query(const TrainQueryArgs& a, cudaStream_t s) {
     const size_t smem = train_query_smem(a.P + a.n_neg, a.M * a.r, a.D, a.r);
-    cudaError_t e = cudaFuncSetAttribute(k_train_query, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
     // threads own dimensions: no more threads than (32-rounded) dimensions
     const int threads = a.D >= kTrainThreads ? kTrainThreads : ((a.D + 31) / 32) * 32;
-    k_train_query<<<(unsigned)a.n, threads, smem, s>>>(a);
+    auto kern = a.r <= 8 ? k_train_query<8> : k_train_query<kTrainMaxR>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<(unsigned)a.n, threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -429,7 +432,10 @@ cudaError_t launch_train_gW(const float* alpha, const float* gC, const float* W,
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)M, (unsigned)((KD + kTrainThreads - 1) / kTrainThreads), (unsigned)slices);
-    k_train_gW_part<<<grid, kTrainThreads, 0, s>>>(alpha, gC, n, M, r, KD, part);
+    if (r <= 8)
+        k_train_gW_part<8><<<grid, kTrainThreads, 0, s>>>(alpha, gC, n, M, r, KD, part);
+    else
+        k_train_gW_part<kTrainMaxR><<<grid, kTrainThreads, 0, s>>>(alpha, gC, n, M, r, KD, part);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const int64_t total = (int64_t)M * r * KD;
     k_train_gW_sum<<<(unsigned)((total + 255) / 256), 256, 0, s>>>(part, slices, A, W, M, r, KD, lambda,

@@ -31,8 +31,10 @@ def ifvs():
 
 
 class Case:
-    def __init__(self, orc, n=5000, nq=8, sel=0.1, zero_bank=False, salt=0):
+    def __init__(self, orc, n=5000, nq=8, sel=0.1, zero_bank=False, salt=0, r=None):
         w = synth.scaled(synth.WORKLOADS["gmm10k-d128-m16"], N=n)
+        if r is not None:
+            w = synth.scaled(w, r=r)
         self.w = w
         self.ix = synth.make_index(w)
         self.cond = synth.make_conditioning(self.ix)
@@ -101,6 +103,20 @@ def test_gradients_across_temperatures(ifvs, orc, case, tau, lam):
     _close(gbg, gb, tol)
     _close(gWg, gW, tol)
     _close(gzg, gz, tol)
+
+
+@pytest.mark.parametrize("r", [1, 12, 32])
+def test_gradients_for_other_ranks(ifvs, orc, r):
+    """r = 1 and r > 8 run the kernels' wide-accumulator variants."""
+    c = Case(orc, n=3000, nq=6, salt=4, r=r)
+    cand = np.concatenate([c.pos, c.oracle_negatives(orc)], 1)
+    L, gb, gW, gz = c.oracle_loss(orc, cand)
+    g = c.index(ifvs)
+    Lg, gbg, gWg, gzg = g.train_grad(c.qs.q, c.qs.preds, c.wz, cand, P, TAU, LAM)
+    assert abs(Lg - L) <= 1e-6 * abs(L)
+    _close(gbg, gb)
+    _close(gWg, gW)
+    _close(gzg, gz)
 
 
 def _oracle_pool_dists(orc, case, i, bank, W, wz):
