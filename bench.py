@@ -37,6 +37,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 WORKLOAD = "gmm100m-d128-m16"
+LIST_DEFAULT_PPM = 20000     # the library's default row-list threshold (2 % of N)
 TRAIN_WORKLOAD = "sift1m-d128-m16"
 CPU_SAMPLE_ROWS = 10_000_000
 
@@ -54,6 +55,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--chunk-blocks", type=int, default=0, help="scan chunk size in 1024-row blocks (0 = auto)")
+    ap.add_argument("--list-max-ppm", type=int, default=0,
+                    help="row-list scan for one-column pools up to this many rows per million "
+                         "(0 = library default, -1 = never)")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
     ap.add_argument("--mode", default="search", choices=["search", "pq", "train"],
                     help="search: the query path; pq: PQ encoding + Lloyd training of the index; "
@@ -333,7 +337,8 @@ def run_ifvs(args):
         q, p, wz = dev_in[b]
         oi, od, on = dev_out[b]
         ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on,
-                               flags=flags, stream=sptr, chunk_blocks=args.chunk_blocks)
+                               flags=flags, stream=sptr, chunk_blocks=args.chunk_blocks,
+                               list_max_ppm=args.list_max_ppm)
 
     for i in range(args.warmup):
         step(i)
@@ -365,25 +370,34 @@ def run_ifvs(args):
     stages = g.stage_times(reset=True)
     launches = sum(v[1] for v in stages.values())
 
-    # per-bin figures and the scan roofline (algorithmic bytes: passing rows'
-    # codes + the bin's lane-major bitmap, per query)
+    # per-bin figures and the scan-stage roofline.  Algorithmic bytes per
+    # query: the passing rows' codes, plus the lane-major bitmap on the bitmap
+    # path or the passing rows' 4-byte ids on the row-list path (one-column
+    # predicates whose pool is within the list threshold)
     per_bin = {}
     n_blocks = (w.N + 1023) // 1024
+    ppm = args.list_max_ppm if args.list_max_ppm != 0 else LIST_DEFAULT_PPM
+    list_rows = -1 if ppm < 0 else w.N * ppm // 1000000
     scan_bytes = 0.0
     for b, qs in enumerate(batches):
         ms_b = [step_ms[i] for i in range(args.steps) if (args.warmup + i) % nb == b]
-        npass = dev_out[b][2].cpu().numpy()
+        npass = dev_out[b][2].cpu().numpy().astype(np.float64)
         nsteps_b = len(ms_b)
-        scan_bytes += nsteps_b * float((npass * w.M).sum() + len(npass) * n_blocks * 128)
+        one_col = (qs.preds["n_clauses"] == 1) if not w.conjunctive else np.zeros(len(npass), bool)
+        on_list = one_col & (npass <= list_rows)
+        per_q = npass * w.M + np.where(on_list, npass * 4, n_blocks * 128)
+        scan_bytes += nsteps_b * float(per_q.sum())
         per_bin[str(qs.sel)] = {
             "qps": (len(qs.q) * nsteps_b) / (sum(ms_b) / 1000.0) if ms_b else None,
             "ms_per_batch": float(np.mean(ms_b)) if ms_b else None,
-            "mean_selectivity": float(npass.mean() / w.N)}
+            "mean_selectivity": float(npass.mean() / w.N),
+            "row_list_share": float(on_list.mean())}
     scan_ms, scan_n = stages["scan"]
     hbm_peak, peak_kind = measured_peaks()
     achieved = (scan_bytes / scan_n) / (scan_ms / scan_n / 1000.0) / 1e9 if scan_n else None
     traffic = scan_traffic()
-    roofline = {"kernel": "k_scan", "bound": "hbm", "achieved": achieved, "peak": hbm_peak,
+    roofline = {"kernel": "scan stage (k_scan + k_scan_list)", "bound": "hbm", "achieved": achieved,
+                "peak": hbm_peak,
                 "unit": "GB/s", "frac": achieved / hbm_peak if achieved else None,
                 "traffic": traffic, "peak_kind": peak_kind + " (hbm copy, burst)",
                 "avg_launch_ms": scan_ms / scan_n if scan_n else None,
@@ -410,7 +424,7 @@ def run_ifvs(args):
             q, p, wz, _ = host_in[b]
             oi, od, on, _ = host_out[b]
             ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr,
-                                   chunk_blocks=args.chunk_blocks)
+                                   chunk_blocks=args.chunk_blocks, list_max_ppm=args.list_max_ppm)
 
         for i in range(args.warmup):
             hstep(i)

@@ -100,6 +100,9 @@ struct ifvs_index {
     int n_attrs = 0;
     int32_t types[IFVS_MAX_ATTRS] = {0, 0, 0, 0};
     void* d_attr[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
+    // per column: row ids sorted by (value, row) and the values in that order
+    uint32_t* d_srt_rows[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
+    int32_t* d_srt_vals[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
     uint8_t* d_codes = nullptr;
     float* d_vec = nullptr;
     bool has_cb = false;
@@ -112,7 +115,7 @@ struct ifvs_index {
     size_t bytes = 0;
     // workspace
     DevBuf w_q, w_wz, w_preds, w_canon, w_err, w_bm, w_rows, w_npass, w_idx, w_alpha, w_wf,
-        w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist, w_tab;
+        w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist, w_tab, w_plan;
     // training workspace
     DevBuf t_cand, t_pos, t_mined, t_mdist, t_gC, t_gw, t_loss, t_G, t_gW, t_gWpart, t_galpha,
         t_gbank, t_gwz, t_wz, t_neg;
@@ -122,6 +125,15 @@ struct ifvs_index {
     std::vector<cudaEvent_t> ev_free;
     std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> pending;
 
+    SortedCols sorted() const {
+        SortedCols c;
+        for (int i = 0; i < IFVS_MAX_ATTRS; ++i) {
+            c.rows[i] = d_srt_rows[i];
+            c.vals[i] = d_srt_vals[i];
+        }
+        c.n = n_attrs;
+        return c;
+    }
     AttrCols cols() const {
         AttrCols c;
         for (int i = 0; i < IFVS_MAX_ATTRS; ++i) {
@@ -160,15 +172,18 @@ void free_index(ifvs_index* ix) {
     if (!ix) return;
     DeviceGuard g(ix->device);
     if (ix->stream) cudaStreamSynchronize(ix->stream);
-    for (int i = 0; i < IFVS_MAX_ATTRS; ++i)
+    for (int i = 0; i < IFVS_MAX_ATTRS; ++i) {
         if (ix->d_attr[i]) cudaFree(ix->d_attr[i]);
+        if (ix->d_srt_rows[i]) cudaFree(ix->d_srt_rows[i]);
+        if (ix->d_srt_vals[i]) cudaFree(ix->d_srt_vals[i]);
+    }
     void* ptrs[] = {ix->d_codes, ix->d_vec, ix->d_cpq, ix->d_bank, ix->d_W, ix->d_seeds};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     DevBuf* bufs[] = {&ix->w_q, &ix->w_wz, &ix->w_preds, &ix->w_canon, &ix->w_err, &ix->w_bm,
                       &ix->w_rows, &ix->w_npass, &ix->w_idx, &ix->w_alpha, &ix->w_wf,
                       &ix->w_lut, &ix->w_cifvs, &ix->w_part, &ix->w_ids, &ix->w_dists,
-                      &ix->w_cand, &ix->w_cdist, &ix->w_tab, &ix->t_cand, &ix->t_pos,
+                      &ix->w_cand, &ix->w_cdist, &ix->w_tab, &ix->w_plan, &ix->t_cand, &ix->t_pos,
                       &ix->t_mined, &ix->t_mdist, &ix->t_gC, &ix->t_gw, &ix->t_loss, &ix->t_G,
                       &ix->t_gW, &ix->t_gWpart, &ix->t_galpha, &ix->t_gbank, &ix->t_gwz, &ix->t_wz, &ix->t_neg};
     for (DevBuf* b : bufs) release(*b);
@@ -190,6 +205,60 @@ int dev_alloc(ifvs_index* ix, void** p, size_t bytes) {
         return set_err(IFVS_ERR_OOM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
     }
     ix->bytes += bytes;
+    return 0;
+}
+
+// Row ids of one attribute column sorted by (value, row), and the values in
+// that order, uploaded to the device: a stable LSD radix sort on the host
+// (two 16-bit digit passes over (key, row) pairs; key = value bits with the
+// sign flipped, so unsigned order is signed order).
+int build_sorted_column(ifvs_index* ix, int c, const void* col, int32_t type, bool dio) {
+    const int64_t N = ix->N;
+    std::vector<uint32_t> key((size_t)N), row((size_t)N), key2((size_t)N), row2((size_t)N);
+    {
+        const size_t es = type == IFVS_ATTR_I16 ? 2 : 4;
+        std::vector<uint8_t> raw;
+        const uint8_t* src = (const uint8_t*)col;
+        if (dio) {
+            raw.resize((size_t)N * es);
+            CUDA_TRY(cudaMemcpy(raw.data(), col, (size_t)N * es, cudaMemcpyDeviceToHost));
+            src = raw.data();
+        }
+        for (int64_t i = 0; i < N; ++i) {
+            int32_t v;
+            if (type == IFVS_ATTR_I16) {
+                int16_t h;
+                memcpy(&h, src + i * 2, 2);
+                v = h;
+            } else {
+                memcpy(&v, src + i * 4, 4);
+            }
+            key[(size_t)i] = (uint32_t)v ^ 0x80000000u;
+            row[(size_t)i] = (uint32_t)i;
+        }
+    }
+    std::vector<int64_t> cnt(65537);
+    for (int pass = 0; pass < 2; ++pass) {
+        const int sh = 16 * pass;
+        std::fill(cnt.begin(), cnt.end(), 0);
+        for (int64_t i = 0; i < N; ++i) ++cnt[((key[(size_t)i] >> sh) & 0xFFFFu) + 1];
+        for (int d = 0; d < 65536; ++d) cnt[d + 1] += cnt[d];
+        for (int64_t i = 0; i < N; ++i) {
+            const int64_t at = cnt[(key[(size_t)i] >> sh) & 0xFFFFu]++;
+            key2[(size_t)at] = key[(size_t)i];
+            row2[(size_t)at] = row[(size_t)i];
+        }
+        key.swap(key2);
+        row.swap(row2);
+    }
+    for (int64_t i = 0; i < N; ++i) key[(size_t)i] ^= 0x80000000u;   // back to the signed value bits
+    void* p = nullptr;
+    TRY(dev_alloc(ix, &p, sizeof(uint32_t) * (size_t)N));
+    ix->d_srt_rows[c] = (uint32_t*)p;
+    CUDA_TRY(cudaMemcpy(p, row.data(), sizeof(uint32_t) * (size_t)N, cudaMemcpyHostToDevice));
+    TRY(dev_alloc(ix, &p, sizeof(int32_t) * (size_t)N));
+    ix->d_srt_vals[c] = (int32_t*)p;
+    CUDA_TRY(cudaMemcpy(p, key.data(), sizeof(int32_t) * (size_t)N, cudaMemcpyHostToDevice));
     return 0;
 }
 
@@ -227,8 +296,13 @@ struct Opts {
     int R = 0;
     int64_t sub_batch = 0;
     int64_t chunk_blocks = 0;
+    int32_t list_max_ppm = 0;
     cudaStream_t stream = nullptr;
 };
+
+// pools of at most 2 % of the rows take the row-list scan unless the caller
+// says otherwise (measured crossover on 10^8 rows: see the design notes)
+constexpr int32_t kListDefaultPpm = 20000;
 
 int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (!p) return 0;
@@ -238,12 +312,15 @@ int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (p->rerank < 0 || p->rerank > IFVS_MAX_K)
         return set_err(IFVS_ERR_ARG, "rerank depth %d outside 0..%d", p->rerank, IFVS_MAX_K);
     if (p->sub_batch < 0) return set_err(IFVS_ERR_ARG, "sub_batch must be >= 0");
+    if (p->list_max_ppm < -1 || p->list_max_ppm > 1000000)
+        return set_err(IFVS_ERR_ARG, "list_max_ppm = %d outside -1..1000000", p->list_max_ppm);
     o->dio = p->flags & IFVS_F_DEVICE_IO;
     o->timing = p->flags & IFVS_F_STAGE_TIMING;
     o->plain = p->flags & IFVS_F_PLAIN_PQ;
     o->R = p->rerank;
     o->sub_batch = p->sub_batch;
     o->chunk_blocks = p->chunk_blocks;
+    o->list_max_ppm = p->list_max_ppm;
     o->stream = reinterpret_cast<cudaStream_t>(p->stream);
     return 0;
 }
@@ -316,10 +393,21 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
         CUDA_TRY(st.end(launch_canonicalize(dp, n, ix->cols(), ix->w_canon.as<CanonPred>(),
                                             ix->w_err.as<int>(), s)));
     }
+    // one-column predicates with small pools take the row-list scan
+    const ScanPlan* plan = nullptr;
+    if (o.list_max_ppm >= 0 && ix->n_attrs > 0) {
+        const int64_t ppm = o.list_max_ppm > 0 ? o.list_max_ppm : kListDefaultPpm;
+        const int64_t max_rows = ppm >= 1000000 ? ix->N : ix->N * ppm / 1000000;
+        TRY(ensure(ix->w_plan, sizeof(ScanPlan) * n));
+        Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);
+        CUDA_TRY(st.end(launch_plan(ix->w_canon.as<CanonPred>(), n, ix->sorted(), ix->N, max_rows,
+                                    ix->w_plan.as<ScanPlan>(), npass_u64, s)));
+        plan = ix->w_plan.as<ScanPlan>();
+    }
     {
         Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);
         CUDA_TRY(st.end(launch_filter(ix->cols(), ix->N, ix->n_blocks, ix->w_canon.as<CanonPred>(),
-                                      n, ix->w_bm.as<uint32_t>(), npass_u64, ix->num_sms, s)));
+                                      plan, n, ix->w_bm.as<uint32_t>(), npass_u64, ix->num_sms, s)));
     }
     {
         Stage st(ix, s, o.timing, IFVS_STAGE_CONDITION);
@@ -341,8 +429,13 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
     }
     {
         Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
-        CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_tab.as<float>(), ix->w_bm.as<uint32_t>(), n,
-                                    kk, sh, ix->w_part.as<uint64_t>(), s)));
+        CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_tab.as<float>(), ix->w_bm.as<uint32_t>(), plan,
+                                    n, kk, sh, ix->w_part.as<uint64_t>(), s)));
+    }
+    if (plan) {
+        Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
+        CUDA_TRY(st.end(launch_scan_list(ix->d_codes, ix->w_tab.as<float>(), ix->sorted(), plan, n, kk,
+                                         sh, ix->w_part.as<uint64_t>(), s)));
     }
     int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;
     float* m_dists = o.R > 0 ? ix->w_cdist.as<float>() : out_dists;
@@ -740,6 +833,10 @@ int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int6
             cudaMemcpyAsync(ix->d_attr[i], attr_cols[i], es * N, h2d, s) != cudaSuccess)
             return fail(cuda_fail(cudaGetLastError(), "attribute copy", __LINE__));
     }
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return fail(cuda_fail(e, "attribute upload", __LINE__));
+    for (int i = 0; i < n_attrs; ++i)
+        if ((rc = build_sorted_column(ix, i, attr_cols[i], attr_types[i], dio))) return fail(rc);
     if (vectors) {
         void* v = nullptr;
         if ((rc = dev_alloc(ix, &v, sizeof(float) * N * D))) return fail(rc);
@@ -876,9 +973,9 @@ int ifvs_filter(ifvs_index* ix, const ifvs_predicate* preds, int64_t nq, const i
         }
         {
             Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);
-            CUDA_TRY(st.end(launch_filter(ix->cols(), ix->N, ix->n_blocks, ix->w_canon.as<CanonPred>(), n,
-                                          ix->w_bm.as<uint32_t>(), ix->w_npass.as<unsigned long long>(),
-                                          ix->num_sms, s)));
+            CUDA_TRY(st.end(launch_filter(ix->cols(), ix->N, ix->n_blocks, ix->w_canon.as<CanonPred>(),
+                                          nullptr, n, ix->w_bm.as<uint32_t>(),
+                                          ix->w_npass.as<unsigned long long>(), ix->num_sms, s)));
         }
         uint32_t* rows = o.dio ? bitmaps + q0 * wrows : ix->w_rows.as<uint32_t>();
         {
@@ -1002,8 +1099,8 @@ int ifvs_scan_topk(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, in
         }
         {
             Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
-            CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_tab.as<float>(), ix->w_bm.as<uint32_t>(), n, k,
-                                        sh, ix->w_part.as<uint64_t>(), s)));
+            CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_tab.as<float>(), ix->w_bm.as<uint32_t>(), nullptr,
+                                        n, k, sh, ix->w_part.as<uint64_t>(), s)));
         }
         int64_t* oid = o.dio ? ids + q0 * k : ix->w_ids.as<int64_t>();
         float* odi = o.dio ? dists + q0 * k : ix->w_dists.as<float>();

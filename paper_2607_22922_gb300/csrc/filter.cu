@@ -32,6 +32,70 @@ cudaError_t launch_canonicalize(const ifvs_predicate* preds, int64_t nq, AttrCol
     return cudaGetLastError();
 }
 
+// Scan plan.  A predicate that constrains one column selects, for that
+// column's canonical interval [lo, lo + wm1], a contiguous segment of the
+// rows sorted by (value, row): two binary searches give it, and its length
+// is the exact pool size.  Pools up to max_rows take the row-list scan (no
+// filter pass, no bitmap); empty and malformed predicates take it with an
+// empty segment; every other query takes the bitmap path.
+__device__ __forceinline__ int64_t first_not_below(const int32_t* __restrict__ v, int64_t n, int64_t x) {
+    int64_t lo = 0, hi = n;
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if ((int64_t)v[mid] < x)
+            lo = mid + 1;
+        else
+            hi = mid;
+    }
+    return lo;
+}
+
+__global__ void k_plan(const CanonPred* __restrict__ canon, int64_t nq, SortedCols sc, int64_t N,
+                       int64_t max_rows, ScanPlan* __restrict__ plan,
+                       unsigned long long* __restrict__ npass) {
+    const int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (q >= nq) return;
+    const CanonPred cp = canon[q];
+    ScanPlan p;
+    p.a = 0;
+    p.b = 0;
+    p.col = 0;
+    p.list = 0;
+    if (cp.empty) {
+        p.list = 1;
+    } else if (__popc(cp.used) == 1) {
+        const int c = __ffs(cp.used) - 1;
+        const int32_t* vals = sc.vals_of(c);
+        if (c < sc.n && vals != nullptr) {
+            int64_t lo = 0, wm1 = 0;
+#pragma unroll
+            for (int i = 0; i < IFVS_MAX_ATTRS; ++i)
+                if (c == i) {
+                    lo = cp.lo[i];
+                    wm1 = cp.wm1[i];
+                }
+            const int64_t hi = lo + wm1;
+            const int64_t a = first_not_below(vals, N, lo);
+            const int64_t b = first_not_below(vals, N, hi + 1);
+            if (b - a <= max_rows) {
+                p.a = a;
+                p.b = b;
+                p.col = c;
+                p.list = 1;
+            }
+        }
+    }
+    plan[q] = p;
+    if (p.list) npass[q] = (unsigned long long)(p.b - p.a);
+}
+
+cudaError_t launch_plan(const CanonPred* canon, int64_t nq, SortedCols sc, int64_t N, int64_t max_rows,
+                        ScanPlan* plan, unsigned long long* npass, cudaStream_t s) {
+    if (nq <= 0) return cudaSuccess;
+    k_plan<<<(unsigned)((nq + 127) / 128), 128, 0, s>>>(canon, nq, sc, N, max_rows, plan, npass);
+    return cudaGetLastError();
+}
+
 // Fail bits of 8 rows against one interval, shifted into `fail` (row j0 + 7
 // first, so that after four calls bit j is row j).  For each row:
 // off = v - lo (mod 2^32); the carry out of off + ~wm1 is 1 exactly when
@@ -59,12 +123,16 @@ constexpr int kFilterQ = 256;   // queries staged in shared memory at a time
 template <int NA>
 __global__ void __launch_bounds__(kThreads) k_filter(AttrCols cols, int64_t N, int64_t n_blocks,
                                                      const CanonPred* __restrict__ canon,
+                                                     const ScanPlan* __restrict__ plan,
                                                      int64_t nq, int q_per_cta,
                                                      uint32_t* __restrict__ bm,
                                                      unsigned long long* __restrict__ npass) {
+    static_assert(kThreads >= kFilterQ, "one staging pass per query group");
     __shared__ int2 s_iv[kFilterQ][NA];      // (lo, ~wm1) per query and column
     __shared__ uint32_t s_keep[kFilterQ];    // 0 for a predicate no row can pass
     __shared__ uint32_t s_used[kFilterQ];
+    __shared__ int s_q[kFilterQ];            // query (offset from the group start)
+    __shared__ int s_wcnt[kWarps];
     const int lane = threadIdx.x & 31;
     const int64_t b = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
     const bool live = b < n_blocks;
@@ -96,19 +164,32 @@ __global__ void __launch_bounds__(kThreads) k_filter(AttrCols cols, int64_t N, i
     }
 
     const int64_t words = n_blocks * 32;
+    const int warp = threadIdx.x >> 5;
     for (int64_t g0 = q0; g0 < q1; g0 += kFilterQ) {
         const int ng = (int)min((int64_t)kFilterQ, q1 - g0);
         __syncthreads();
-        for (int i = threadIdx.x; i < ng; i += blockDim.x) {
-            const CanonPred cp = canon[g0 + i];
+        // stage the group's bitmap-path queries, in order (list-path queries
+        // need no bitmap and cost nothing here)
+        const int t = threadIdx.x;
+        const bool mine = t < ng && (plan == nullptr || !plan[g0 + t].list);
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, mine);
+        if (lane == 0) s_wcnt[warp] = __popc(bal);
+        __syncthreads();
+        int pos = __popc(bal & ((1u << lane) - 1u));
+        for (int w = 0; w < warp; ++w) pos += s_wcnt[w];
+        int ngd = 0;
+        for (int w = 0; w < kWarps; ++w) ngd += s_wcnt[w];
+        if (mine) {
+            const CanonPred cp = canon[g0 + t];
 #pragma unroll
-            for (int c = 0; c < NA; ++c) s_iv[i][c] = make_int2(cp.lo[c], (int32_t)~cp.wm1[c]);
-            s_keep[i] = cp.empty ? 0u : 0xFFFFFFFFu;
-            s_used[i] = cp.used;
+            for (int c = 0; c < NA; ++c) s_iv[pos][c] = make_int2(cp.lo[c], (int32_t)~cp.wm1[c]);
+            s_keep[pos] = cp.empty ? 0u : 0xFFFFFFFFu;
+            s_used[pos] = cp.used;
+            s_q[pos] = t;
         }
         __syncthreads();
         if (!live) continue;
-        for (int i = 0; i < ng; ++i) {
+        for (int i = 0; i < ngd; ++i) {
             uint32_t m = valid & s_keep[i];
             const uint32_t used = s_used[i];
 #pragma unroll
@@ -121,7 +202,7 @@ __global__ void __launch_bounds__(kThreads) k_filter(AttrCols cols, int64_t N, i
                     m &= ~fail;
                 }
             }
-            const int64_t q = g0 + i;
+            const int64_t q = g0 + s_q[i];
             bm[q * words + b * 32 + lane] = m;
             const unsigned cnt = __reduce_add_sync(0xFFFFFFFFu, (unsigned)__popc(m));
             if (lane == 0 && cnt) atomicAdd(npass + q, (unsigned long long)cnt);
@@ -130,8 +211,8 @@ __global__ void __launch_bounds__(kThreads) k_filter(AttrCols cols, int64_t N, i
 }
 
 cudaError_t launch_filter(AttrCols cols, int64_t N, int64_t n_blocks, const CanonPred* canon,
-                          int64_t nq, uint32_t* bm, unsigned long long* npass, int num_sms,
-                          cudaStream_t s) {
+                          const ScanPlan* plan, int64_t nq, uint32_t* bm, unsigned long long* npass,
+                          int num_sms, cudaStream_t s) {
     if (nq <= 0) return cudaSuccess;
     const int64_t tiles = (n_blocks + kWarps - 1) / kWarps;
     // enough CTAs to fill the GPU a few times over; each CTA walks a group
@@ -146,10 +227,10 @@ cudaError_t launch_filter(AttrCols cols, int64_t N, int64_t n_blocks, const Cano
     dim3 grid((unsigned)tiles, (unsigned)groups);
     int na = cols.n < 1 ? 1 : cols.n;
     switch (na) {
-        case 1: k_filter<1><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, nq, (int)qpc, bm, npass); break;
-        case 2: k_filter<2><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, nq, (int)qpc, bm, npass); break;
-        case 3: k_filter<3><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, nq, (int)qpc, bm, npass); break;
-        default: k_filter<4><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, nq, (int)qpc, bm, npass); break;
+        case 1: k_filter<1><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, plan, nq, (int)qpc, bm, npass); break;
+        case 2: k_filter<2><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, plan, nq, (int)qpc, bm, npass); break;
+        case 3: k_filter<3><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, plan, nq, (int)qpc, bm, npass); break;
+        default: k_filter<4><<<grid, kThreads, 0, s>>>(cols, N, n_blocks, canon, plan, nq, (int)qpc, bm, npass); break;
     }
     return cudaGetLastError();
 }

@@ -100,10 +100,44 @@ struct AttrCols {
 cudaError_t launch_canonicalize(const ifvs_predicate* preds, int64_t nq, AttrCols cols,
                                 CanonPred* out, int* err, cudaStream_t s);
 
-// Filter: lane-major pass bitmaps [nq][n_blocks * 32] + popcounts (added to npass)
+// Per-query scan plan: a one-column predicate with a pool of at most
+// max_rows rows (or an empty / malformed one) takes the row-list scan over
+// rows [a, b) of column col's sorted order; the rest take the bitmap path.
+struct ScanPlan {
+    int64_t a, b;
+    int32_t col;
+    int32_t list;      // 1: row-list scan
+};
+// Row ids of each column sorted by (value, row) and the values in that order.
+struct SortedCols {
+    const uint32_t* rows[IFVS_MAX_ATTRS];
+    const int32_t* vals[IFVS_MAX_ATTRS];
+    int32_t n;
+    // column c's arrays, selected without indexing the parameter at run time
+    __host__ __device__ const uint32_t* rows_of(int c) const {
+        const uint32_t* r = rows[0];
+#pragma unroll
+        for (int i = 1; i < IFVS_MAX_ATTRS; ++i)
+            if (c == i) r = rows[i];
+        return r;
+    }
+    __host__ __device__ const int32_t* vals_of(int c) const {
+        const int32_t* v = vals[0];
+#pragma unroll
+        for (int i = 1; i < IFVS_MAX_ATTRS; ++i)
+            if (c == i) v = vals[i];
+        return v;
+    }
+};
+// plan [nq]; writes npass of the list-path queries
+cudaError_t launch_plan(const CanonPred* canon, int64_t nq, SortedCols sc, int64_t N, int64_t max_rows,
+                        ScanPlan* plan, unsigned long long* npass, cudaStream_t s);
+
+// Filter: lane-major pass bitmaps [nq][n_blocks * 32] + popcounts (added to
+// npass) for the bitmap-path queries of `plan` (all queries when plan is null)
 cudaError_t launch_filter(AttrCols cols, int64_t N, int64_t n_blocks, const CanonPred* canon,
-                          int64_t nq, uint32_t* bm, unsigned long long* npass, int num_sms,
-                          cudaStream_t s);
+                          const ScanPlan* plan, int64_t nq, uint32_t* bm, unsigned long long* npass,
+                          int num_sms, cudaStream_t s);
 
 // 32x32 bit transposes between the lane-major layout and the row-ordered
 // layout of the ABI ([nq][ceil(N/32)]).  to_rows = true: lane-major -> rows.
@@ -142,8 +176,12 @@ int scan_kp(int k);
 // Rank: per (query, chunk) CTA, the k best keys (dist bits << 32 | row) of
 // the chunk's passing rows -> partials [nq][n_chunks][k]; `tab` holds the
 // tables written by launch_tables
-cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm, int64_t nq,
-                        int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s);
+cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm,
+                        const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
+                        uint64_t* partials, cudaStream_t s);
+// the list-path queries of `plan` (same grid and partial layout as launch_scan)
+cudaError_t launch_scan_list(const uint8_t* codes, const float* tab, SortedCols sc, const ScanPlan* plan,
+                             int64_t nq, int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s);
 // Select: merge [nq][n_lists][k] partial keys -> ids / dists
 cudaError_t launch_merge(const uint64_t* partials, int64_t nq, int n_lists, int k,
                          int64_t* ids, float* dists, cudaStream_t s);

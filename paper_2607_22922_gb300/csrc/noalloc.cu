@@ -134,7 +134,7 @@ extern "C" int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uin
         sh.n_chunks = (int)((v.n_blocks + sh.blocks_per_chunk - 1) / sh.blocks_per_chunk);
         cudaError_t e = launch_bitmap_layout(bitmaps + q0 * wrows, bm, n, v.n_blocks, wrows, false, s);
         if (e == cudaSuccess) e = launch_tables(lut + q0 * lut_n, n, v.M, v.K, v.tab_words, tab, s);
-        if (e == cudaSuccess) e = launch_scan(v.codes, tab, bm, n, k, sh, part, s);
+        if (e == cudaSuccess) e = launch_scan(v.codes, tab, bm, nullptr, n, k, sh, part, s);
         if (e == cudaSuccess) e = launch_merge(part, n, sh.n_chunks, k, ids + q0 * k, dists + q0 * k, s);
         if (e != cudaSuccess) {
             cudaGetLastError();

@@ -179,10 +179,11 @@ __device__ __forceinline__ void unpack_f32x2(uint64_t v, float& a, float& b) {
 constexpr uint32_t kDynSmemBase = 0x400u;
 
 // Distances of two M = 16 rows (codes ca, cb).  One byte permute forms
-// code * 256 + 4 * lane; FAST (table at kDynSmemBase): the table base and
-// the step go into the load's immediate offset; otherwise the base is added.
+// code * 256 + 4 * w0, w0 = the row's index mod 32 (the lane that owns it in
+// the bitmap path); FAST (table at kDynSmemBase): the table base and the step
+// go into the load's immediate offset; otherwise the base is added.
 template <bool FAST>
-__device__ __forceinline__ void lookup16x2(const uint4 ca, const uint4 cb, uint32_t tb,
+__device__ __forceinline__ void lookup16x2(const uint4 ca, const uint4 cb, uint32_t tba, uint32_t tbb,
                                            uint32_t base, float& da, float& db) {
     const uint32_t wa[4] = {ca.x, ca.y, ca.z, ca.w};
     const uint32_t wb[4] = {cb.x, cb.y, cb.z, cb.w};
@@ -190,8 +191,8 @@ __device__ __forceinline__ void lookup16x2(const uint4 ca, const uint4 cb, uint3
 #pragma unroll
     for (int s = 0; s < 16; ++s) {
         const uint32_t sel = 0x5504u | ((uint32_t)(s & 3) << 4);
-        uint32_t oa = __byte_perm(wa[s >> 2], tb, sel);
-        uint32_t ob = __byte_perm(wb[s >> 2], tb, sel);
+        uint32_t oa = __byte_perm(wa[s >> 2], tba, sel);
+        uint32_t ob = __byte_perm(wb[s >> 2], tbb, sel);
         if (!FAST) {
             oa += base;
             ob += base;
@@ -216,16 +217,17 @@ __device__ __forceinline__ void lookup16x2(const uint4 ca, const uint4 cb, uint3
     unpack_f32x2(acc, da, db);
 }
 
-// Distance of one row for any M (runtime loop; row_bytes a multiple of 4).
+// Distance of one row for any M (runtime loop; row_bytes a multiple of 4);
+// w0 = the row's index mod 32.
 __device__ __forceinline__ float lookup_any(const uint8_t* rp, bool pass, int M, int S,
-                                            const float* tab, int lane) {
+                                            const float* tab, int w0) {
     float acc = 0.f;
     for (int w = 0; w * 4 < M; ++w) {
         const uint32_t wd = pass ? __ldg(reinterpret_cast<const uint32_t*>(rp) + w) : 0u;
 #pragma unroll
         for (int bb = 0; bb < 4; ++bb) {
             const int s = 4 * w + bb;
-            if (s < M) acc += tab[(int)((wd >> (8 * bb)) & 0xFFu) * S + lane + s];
+            if (s < M) acc += tab[(int)((wd >> (8 * bb)) & 0xFFu) * S + w0 + s];
         }
     }
     return acc;
@@ -295,7 +297,7 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                     for (int u = 0; u < kU; ++u) c[u] = ldg_nc_v4(codes + (size_t)row[u] * 16, keep);
                     float d[kU];
 #pragma unroll
-                    for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, base, d[u], d[u + 1]);
+                    for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
                     uint64_t key[kU];
                     bool want = false;
 #pragma unroll
@@ -347,7 +349,7 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                 c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)row[u] * 16, keep) : make_uint4(0, 0, 0, 0);
             float d[kU];
 #pragma unroll
-            for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, base, d[u], d[u + 1]);
+            for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
             uint64_t key[kU];
             bool want = false;
 #pragma unroll
@@ -374,8 +376,8 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
 template <int KP, bool M16, int MINB>
 __global__ void __launch_bounds__(kScanThreads, MINB)
 k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
-       const uint32_t* __restrict__ bm, int64_t nq, int k, ScanShape sh,
-       uint64_t* __restrict__ partials) {
+       const uint32_t* __restrict__ bm, const ScanPlan* __restrict__ plan, int64_t nq, int k,
+       ScanShape sh, uint64_t* __restrict__ partials) {
     extern __shared__ __align__(256) uint8_t smem[];
     const int S = M16 ? 64 : sh.tab_words;
     float* tab = reinterpret_cast<float*>(smem);
@@ -385,6 +387,7 @@ k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t q = blockIdx.x;
     const int chunk = blockIdx.y;
+    if (plan != nullptr && plan[q].list) return;   // k_scan_list covers this query
 
     // 1) the query's table, replicated and rotated (see the file comment),
     //    as written by k_tables: a straight 16-byte-wide copy
@@ -434,20 +437,20 @@ k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
 
 template <int KP, bool M16, int MINB>
 static cudaError_t launch_one(const uint8_t* codes, const float* tab, const uint32_t* bm,
-                              int64_t nq, int k, const ScanShape& sh, uint64_t* partials,
-                              size_t smem, cudaStream_t s) {
+                              const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
+                              uint64_t* partials, size_t smem, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(k_scan<KP, M16, MINB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
-    k_scan<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(codes, tab, bm, nq, k, sh, partials);
+    k_scan<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(codes, tab, bm, plan, nq, k, sh, partials);
     return cudaGetLastError();
 }
 
 template <int KP>
 static cudaError_t launch_scan_kp(const uint8_t* codes, const float* tab, const uint32_t* bm,
-                                  int64_t nq, int k, const ScanShape& sh, uint64_t* partials,
-                                  cudaStream_t s) {
+                                  const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
+                                  uint64_t* partials, cudaStream_t s) {
     const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
     const size_t smem = scan_smem_bytes(sh.tab_words, KP);
     if (m16) {
@@ -456,20 +459,182 @@ static cudaError_t launch_scan_kp(const uint8_t* codes, const float* tab, const 
 #else
         if (false)
 #endif
-            return launch_one<KP, true, 2>(codes, tab, bm, nq, k, sh, partials, smem, s);
-        return launch_one<KP, true, 1>(codes, tab, bm, nq, k, sh, partials, smem, s);
+            return launch_one<KP, true, 2>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
+        return launch_one<KP, true, 1>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
     }
-    return launch_one<KP, false, 1>(codes, tab, bm, nq, k, sh, partials, smem, s);
+    return launch_one<KP, false, 1>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
 }
 
-cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm, int64_t nq,
-                        int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s) {
+cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm,
+                        const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
+                        uint64_t* partials, cudaStream_t s) {
     if (nq <= 0) return cudaSuccess;
     switch (scan_kp(k)) {
-        case 32: return launch_scan_kp<32>(codes, tab, bm, nq, k, sh, partials, s);
-        case 64: return launch_scan_kp<64>(codes, tab, bm, nq, k, sh, partials, s);
-        case 128: return launch_scan_kp<128>(codes, tab, bm, nq, k, sh, partials, s);
-        default: return launch_scan_kp<256>(codes, tab, bm, nq, k, sh, partials, s);
+        case 32: return launch_scan_kp<32>(codes, tab, bm, plan, nq, k, sh, partials, s);
+        case 64: return launch_scan_kp<64>(codes, tab, bm, plan, nq, k, sh, partials, s);
+        case 128: return launch_scan_kp<128>(codes, tab, bm, plan, nq, k, sh, partials, s);
+        default: return launch_scan_kp<256>(codes, tab, bm, plan, nq, k, sh, partials, s);
+    }
+}
+
+// ---- row-list scan ------------------------------------------------------
+//
+// For a query of the list path (ScanPlan), the pool is the segment
+// rows[a, b) of one column's sorted order.  CTA (query, chunk) takes an equal
+// share of the segment; warps take 32 kU consecutive positions at a time, a
+// row per lane and position (coalesced reads of the row ids), gather the rows'
+// codes and look them up with the table word index (row mod 32) + s: the same
+// entries, summed in the same order, as the bitmap path, where row mod 32 is
+// the owning lane.  Lanes of one warp may now share (row mod 32), so the
+// look-ups are no longer conflict-free; these pools are small.  Top-k and the
+// partial lists are those of k_scan, so k_merge serves both paths.
+
+size_t scan_list_smem_bytes(int tab_words, int kp) {
+    return (size_t)256 * tab_words * 4 + (size_t)kScanWarps * 2 * kp * 8;
+}
+
+template <int KP, bool M16, bool FAST>
+__device__ __forceinline__ void scan_rows(const uint8_t* __restrict__ codes, const uint32_t* __restrict__ rows,
+                                          int64_t s0, int64_t s1, const ScanShape& sh, const float* tab,
+                                          WarpTopK<KP>& tk, int lane, int warp) {
+    const int M = M16 ? 16 : sh.M;
+    const int S = M16 ? 64 : sh.tab_words;
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
+    const uint64_t once = policy_evict_first();
+    for (int64_t g = s0 + (int64_t)warp * 32 * kU; g < s1; g += (int64_t)kScanWarps * 32 * kU) {
+        uint32_t row[kU];
+        unsigned valid = 0u;
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            const int64_t p = g + 32 * u + lane;
+            const bool ok = p < s1;
+            row[u] = ok ? __ldg(rows + p) : 0u;
+            valid |= (unsigned)ok << u;
+        }
+        if constexpr (M16) {
+            uint4 c[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u)
+                c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)row[u] * 16, once) : make_uint4(0, 0, 0, 0);
+            float d[kU];
+#pragma unroll
+            for (int u = 0; u < kU; u += 2)
+                lookup16x2<FAST>(c[u], c[u + 1], 4u * (row[u] & 31u), 4u * (row[u + 1] & 31u), base,
+                                 d[u], d[u + 1]);
+            uint64_t key[kU];
+            bool want = false;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                key[u] = ((uint64_t)__float_as_uint(d[u]) << 32) | row[u];
+                want |= (valid >> u & 1u) && key[u] < tk.thr;
+            }
+            if (__any_sync(0xFFFFFFFFu, want)) {
+#pragma unroll
+                for (int u = 0; u < kU; ++u) tk.offer(key[u], (valid >> u & 1u) && key[u] < tk.thr, lane);
+            }
+        } else {
+#pragma unroll 1
+            for (int u = 0; u < kU; ++u) {
+                const bool pass = valid >> u & 1u;
+                const float d = lookup_any(codes + (size_t)row[u] * sh.row_bytes, pass, M, S, tab,
+                                           (int)(row[u] & 31u));
+                const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | row[u];
+                tk.offer(key, pass && key < tk.thr, lane);
+            }
+        }
+    }
+}
+
+template <int KP, bool M16, int MINB>
+__global__ void __launch_bounds__(kScanThreads, MINB)
+k_scan_list(const uint8_t* __restrict__ codes, const float* __restrict__ tables, SortedCols sc,
+            const ScanPlan* __restrict__ plan, int64_t nq, int k, ScanShape sh,
+            uint64_t* __restrict__ partials) {
+    extern __shared__ __align__(256) uint8_t smem[];
+    const int S = M16 ? 64 : sh.tab_words;
+    float* tab = reinterpret_cast<float*>(smem);
+    uint64_t* tkbuf = reinterpret_cast<uint64_t*>(smem + (size_t)256 * S * 4);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t q = blockIdx.x;
+    const int chunk = blockIdx.y;
+    const ScanPlan p = plan[q];
+    if (!p.list) return;   // k_scan covers this query
+    const int64_t len = p.b - p.a;
+    const int64_t per = (len + sh.n_chunks - 1) / sh.n_chunks;
+    const int64_t s0 = p.a + min(len, (int64_t)chunk * per);
+    const int64_t s1 = p.a + min(len, (int64_t)(chunk + 1) * per);
+    uint64_t* out = partials + (q * sh.n_chunks + chunk) * (int64_t)k;
+    if (s0 >= s1) {
+        for (int i = threadIdx.x; i < k; i += kScanThreads) out[i] = ~0ull;
+        return;
+    }
+    {
+        const float4* src = reinterpret_cast<const float4*>(tables + q * (int64_t)256 * S);
+        float4* dst = reinterpret_cast<float4*>(tab);
+        for (int i = threadIdx.x; i < 64 * S; i += kScanThreads) dst[i] = __ldg(src + i);
+    }
+    WarpTopK<KP> tk;
+    tk.init(tkbuf + warp * 2 * KP, k, lane);
+    __syncthreads();
+    const uint32_t* rows = sc.rows_of(p.col);
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
+    if constexpr (M16) {
+        if (base == kDynSmemBase)
+            scan_rows<KP, true, true>(codes, rows, s0, s1, sh, tab, tk, lane, warp);
+        else
+            scan_rows<KP, true, false>(codes, rows, s0, s1, sh, tab, tk, lane, warp);
+    } else {
+        scan_rows<KP, false, false>(codes, rows, s0, s1, sh, tab, tk, lane, warp);
+    }
+    tk.flush(lane);
+#pragma unroll 1
+    for (int step = 1; step < kScanWarps; step <<= 1) {
+        __syncthreads();
+        if ((warp & (2 * step - 1)) == 0) {
+            const uint64_t* other = tkbuf + (warp + step) * 2 * KP;
+            for (int i = lane; i < k; i += 32) tk.buf[KP + i] = other[i];
+            __syncwarp();
+            tk.flush(lane);
+        }
+    }
+    if (warp == 0)
+        for (int i = lane; i < k; i += 32) out[i] = tk.buf[i];
+}
+
+template <int KP, bool M16, int MINB>
+static cudaError_t launch_list_one(const uint8_t* codes, const float* tab, SortedCols sc,
+                                   const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
+                                   uint64_t* partials, size_t smem, cudaStream_t s) {
+    cudaError_t e = cudaFuncSetAttribute(k_scan_list<KP, M16, MINB>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
+    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(codes, tab, sc, plan, nq, k, sh, partials);
+    return cudaGetLastError();
+}
+
+template <int KP>
+static cudaError_t launch_list_kp(const uint8_t* codes, const float* tab, SortedCols sc,
+                                  const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
+                                  uint64_t* partials, cudaStream_t s) {
+    const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
+    const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
+    if (m16) {
+        if ((size_t)233472 / (smem + 1024) >= 2)
+            return launch_list_one<KP, true, 2>(codes, tab, sc, plan, nq, k, sh, partials, smem, s);
+        return launch_list_one<KP, true, 1>(codes, tab, sc, plan, nq, k, sh, partials, smem, s);
+    }
+    return launch_list_one<KP, false, 1>(codes, tab, sc, plan, nq, k, sh, partials, smem, s);
+}
+
+cudaError_t launch_scan_list(const uint8_t* codes, const float* tab, SortedCols sc, const ScanPlan* plan,
+                             int64_t nq, int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s) {
+    if (nq <= 0) return cudaSuccess;
+    switch (scan_kp(k)) {
+        case 32: return launch_list_kp<32>(codes, tab, sc, plan, nq, k, sh, partials, s);
+        case 64: return launch_list_kp<64>(codes, tab, sc, plan, nq, k, sh, partials, s);
+        case 128: return launch_list_kp<128>(codes, tab, sc, plan, nq, k, sh, partials, s);
+        default: return launch_list_kp<256>(codes, tab, sc, plan, nq, k, sh, partials, s);
     }
 }
 

@@ -49,7 +49,39 @@ def test_version_and_error_string(lib):
 
 def test_predicate_records_match_the_abi(lib):
     assert lib.PREDICATE_DTYPE.itemsize == 104 == synth.PREDICATE_DTYPE.itemsize
-    assert ctypes.sizeof(lib.SearchParams) == 24
+
+
+def test_parameter_structs_match_the_header(lib, tmp_path):
+    """sizeof / offsetof of the header's structs, compiled by gcc, against
+    the binding's ctypes layouts."""
+    import subprocess
+    structs = {"ifvs_search_params": (lib.SearchParams,
+                                      ["flags", "rerank", "sub_batch", "chunk_blocks",
+                                       "list_max_ppm", "stream"]),
+               "ifvs_train_params": (lib.TrainParams,
+                                     ["tau", "lambda", "lr", "lr_wz", "n_pos", "n_neg", "flags",
+                                      "stream"])}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "ifvs.h"', "int main(void) {"]
+    for name, (_, fields) in structs.items():
+        lines.append('printf("%%zu\\n", sizeof(%s));' % name)
+        for f in fields:
+            lines.append('printf("%%zu\\n", offsetof(%s, %s));' % (name, f))
+    lines += ['printf("%zu\\n", sizeof(ifvs_predicate));', "return 0; }"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.check_call(["gcc", "-std=c99", "-I", inc, "-o", str(exe), str(src)])
+    got = [int(x) for x in subprocess.check_output([str(exe)], text=True).split()]
+    want = []
+    for name, (cls, fields) in structs.items():
+        want.append(ctypes.sizeof(cls))
+        names = [f[0] for f in cls._fields_]
+        for f in fields:
+            want.append(getattr(cls, "lam" if f == "lambda" else f).offset)
+        assert len(names) == len(fields)
+    want.append(lib.PREDICATE_DTYPE.itemsize)
+    assert got == want
 
 
 def _pred(*clauses):

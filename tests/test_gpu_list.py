@@ -1,0 +1,149 @@
+"""The row-list scan (a one-column predicate's pool read from the rows sorted
+by that column) against the bitmap path and the oracle.
+
+Both paths sum the same table entries in the same order, so forcing one or
+the other (list_max_ppm = 1000000 / -1) must give bit-identical ids,
+distances and pass counts; each is also checked against the oracle with the
+tie rule of the other parity tests."""
+import numpy as np
+import pytest
+
+from paper_2607_22922_gb300 import synth
+from parity_util import check_topk
+
+pytestmark = pytest.mark.gpu
+
+ALWAYS, NEVER = 1000000, -1
+
+
+@pytest.fixture(scope="module")
+def ifvs():
+    from paper_2607_22922_gb300 import build
+    build.build()
+    from paper_2607_22922_gb300 import ifvs as mod
+    return mod
+
+
+def _index(ifvs, N, M=16, K=256, ds=2, seed=0, i16=True, device_io=False):
+    rng = np.random.default_rng(seed)
+    codes = rng.integers(0, K, size=(N, M)).astype(np.uint8)
+    codes[1::3] = codes[0::3][: len(codes[1::3])]       # exact ties in distance
+    attrs = [rng.integers(-500, 500, N).astype(np.int32)]
+    if i16:
+        attrs.append(rng.integers(-20, 20, N).astype(np.int16))
+    Cpq = rng.standard_normal((M, K, ds)).astype(np.float32)
+    if device_io:
+        import torch
+        dev = torch.device("cuda", 0)
+        g = ifvs.Index(torch.from_numpy(codes).to(dev), [torch.from_numpy(a).to(dev) for a in attrs],
+                       D=M * ds, K=K, device_io=True)
+    else:
+        g = ifvs.Index(codes, attrs, D=M * ds, K=K)
+    g.load_codebooks(Cpq)
+    return g, codes, attrs, Cpq
+
+
+def _preds():
+    """One-column predicates of every operator and width, on both columns,
+    plus empty, all-pass and two-column ones (the latter take the bitmap path)."""
+    rows = []
+    for lo, hi in ((0, 1), (-3, 2), (-500, -490), (100, 160), (-200, 300), (-500, 500),
+                   (499, 500), (600, 700), (7, 7)):
+        rows.append([(0, synth.OP_RANGE, lo, hi)])
+    for op, v in ((synth.OP_EQ, 17), (synth.OP_GE, 480), (synth.OP_LT, -470), (synth.OP_GT, 490),
+                  (synth.OP_LE, -495), (synth.OP_EQ, 10 ** 6)):
+        rows.append([(0, op, v)])
+    for op, v in ((synth.OP_EQ, 3), (synth.OP_GE, 19), (synth.OP_LT, -19), (synth.OP_EQ, -20)):
+        rows.append([(1, op, v)])
+    rows.append([(0, synth.OP_RANGE, -10, 10), (0, synth.OP_GE, -2)])      # one column, two clauses
+    rows.append([(0, synth.OP_RANGE, -100, 100), (1, synth.OP_EQ, 5)])    # two columns
+    rows.append([])                                                        # all pass
+    p = synth.empty_predicates(len(rows))
+    for i, cl in enumerate(rows):
+        p[i]["n_clauses"] = len(cl)
+        for j, c in enumerate(cl):
+            synth.set_clause(p[i], j, *c)
+    return p
+
+
+def _queries(n, D, seed=5):
+    return np.random.default_rng(seed).standard_normal((n, D)).astype(np.float32)
+
+
+def _check_oracle(orc, codes, attrs, Cpq, q, preds, k, ids, dists, npass):
+    oi, od, on = orc.search(codes, attrs, Cpq, q, preds, k)
+    np.testing.assert_array_equal(npass, on)
+    _, _, _, st = orc.search(codes, attrs, Cpq, q, preds, 1, want_stages=True)
+    for i in range(len(q)):
+        all_d = orc.adc_all(st["lut"][i], codes)
+        bm, _ = orc.filter_bitmap(attrs, preds[i])
+        passing = np.unpackbits(bm.view(np.uint8), bitorder="little")[: len(codes)].astype(bool)
+        check_topk(ids[i], dists[i], oi[i], od[i], all_d, passing)
+
+
+@pytest.mark.parametrize("N,k", [(1, 1), (1000, 10), (33333, 100), (100000, 256)])
+def test_list_path_equals_bitmap_path(ifvs, orc, N, k):
+    g, codes, attrs, Cpq = _index(ifvs, N)
+    p = _preds()
+    q = _queries(len(p), Cpq.shape[0] * Cpq.shape[2])
+    a = g.search(q, p, k, list_max_ppm=ALWAYS)
+    b = g.search(q, p, k, list_max_ppm=NEVER)
+    d = g.search(q, p, k)                      # default threshold: a mix of both
+    for x, y, z in zip(a, b, d):
+        np.testing.assert_array_equal(x, y)
+        np.testing.assert_array_equal(x, z)
+    if N <= 33333:
+        _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
+
+
+@pytest.mark.parametrize("M", [1, 8, 12, 24])
+def test_list_path_other_subspace_counts(ifvs, orc, M):
+    g, codes, attrs, Cpq = _index(ifvs, 20000, M=M, K=64, ds=3, seed=M)
+    p = _preds()
+    q = _queries(len(p), M * 3, seed=M)
+    a = g.search(q, p, 20, list_max_ppm=ALWAYS)
+    b = g.search(q, p, 20, list_max_ppm=NEVER)
+    for x, y in zip(a, b):
+        np.testing.assert_array_equal(x, y)
+    _check_oracle(orc, codes, attrs, Cpq, q, p, 20, *a)
+
+
+def test_list_path_with_conditioning_sub_batches_and_device_index(ifvs, orc):
+    w = synth.scaled(synth.WORKLOADS["gmm10k-d128-m16"], N=60000)
+    ix = synth.make_index(w)
+    cond = synth.make_conditioning(ix)
+    qs = synth.make_queries(ix, 0.01, nq=70)
+    for dio in (False, True):
+        if dio:
+            import torch
+            dev = torch.device("cuda", 0)
+            g = ifvs.Index(torch.from_numpy(ix.codes).to(dev),
+                           [torch.from_numpy(a).to(dev) for a in ix.attrs], D=w.D, K=w.K,
+                           device_io=True)
+        else:
+            g = ifvs.Index(ix.codes, ix.attrs, D=w.D, K=w.K)
+        g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
+        a = g.search(qs.q, qs.preds, 10, wz=qs.wz, list_max_ppm=ALWAYS, sub_batch=32)
+        b = g.search(qs.q, qs.preds, 10, wz=qs.wz, list_max_ppm=NEVER)
+        for x, y in zip(a, b):
+            np.testing.assert_array_equal(x, y)
+        oi, od, on = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q, qs.preds, 10,
+                                bank=cond.bank, W=cond.W, seeds=cond.seeds, wz=qs.wz)
+        np.testing.assert_array_equal(a[2], on)
+
+
+def test_threshold_and_launch_counts(ifvs):
+    g, codes, attrs, Cpq = _index(ifvs, 50000, seed=3)
+    p = _preds()
+    q = _queries(len(p), 32)
+    g.stage_times(reset=True)
+    g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING)
+    t = g.stage_times(reset=True)
+    assert t["filter"][1] == 2 and t["scan"][1] == 2          # plan + filter, bitmap + list scan
+    g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING, list_max_ppm=NEVER)
+    t = g.stage_times(reset=True)
+    assert t["filter"][1] == 1 and t["scan"][1] == 1
+    for bad in (-2, 1000001):
+        with pytest.raises(ifvs.IfvsError) as e:
+            g.search(q, p, 10, list_max_ppm=bad)
+        assert e.value.code == ifvs.IFVS_ERR_ARG
