@@ -37,7 +37,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 WORKLOAD = "gmm100m-d128-m16"
-LIST_DEFAULT_PPM = 20000     # the library's default row-list threshold (2 % of N)
+LIST_DEFAULT_PPM = 1000000   # the library's default sorted-copy threshold (always)
 TRAIN_WORKLOAD = "sift1m-d128-m16"
 CPU_SAMPLE_ROWS = 10_000_000
 
@@ -56,8 +56,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--chunk-blocks", type=int, default=0, help="scan chunk size in 1024-row blocks (0 = auto)")
     ap.add_argument("--list-max-ppm", type=int, default=0,
-                    help="row-list scan for one-column pools up to this many rows per million "
-                         "(0 = library default, -1 = never)")
+                    help="sorted-copy scan for one-column pools up to this many rows per million "
+                         "(0 = library default: always, -1 = never)")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
     ap.add_argument("--mode", default="search", choices=["search", "pq", "train"],
                     help="search: the query path; pq: PQ encoding + Lloyd training of the index; "
@@ -372,8 +372,8 @@ def run_ifvs(args):
 
     # per-bin figures and the scan-stage roofline.  Algorithmic bytes per
     # query: the passing rows' codes, plus the lane-major bitmap on the bitmap
-    # path or the passing rows' 4-byte ids on the row-list path (one-column
-    # predicates whose pool is within the list threshold)
+    # path (the sorted-copy path of one-column predicates reads no bitmap; the
+    # row ids it loads for top-k candidates only are not counted)
     per_bin = {}
     n_blocks = (w.N + 1023) // 1024
     ppm = args.list_max_ppm if args.list_max_ppm != 0 else LIST_DEFAULT_PPM
@@ -385,13 +385,13 @@ def run_ifvs(args):
         nsteps_b = len(ms_b)
         one_col = (qs.preds["n_clauses"] == 1) if not w.conjunctive else np.zeros(len(npass), bool)
         on_list = one_col & (npass <= list_rows)
-        per_q = npass * w.M + np.where(on_list, npass * 4, n_blocks * 128)
+        per_q = npass * w.M + np.where(on_list, 0.0, n_blocks * 128.0)
         scan_bytes += nsteps_b * float(per_q.sum())
         per_bin[str(qs.sel)] = {
             "qps": (len(qs.q) * nsteps_b) / (sum(ms_b) / 1000.0) if ms_b else None,
             "ms_per_batch": float(np.mean(ms_b)) if ms_b else None,
             "mean_selectivity": float(npass.mean() / w.N),
-            "row_list_share": float(on_list.mean())}
+            "sorted_path_share": float(on_list.mean())}
     scan_ms, scan_n = stages["scan"]
     hbm_peak, peak_kind = measured_peaks()
     achieved = (scan_bytes / scan_n) / (scan_ms / scan_n / 1000.0) / 1e9 if scan_n else None

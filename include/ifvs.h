@@ -101,12 +101,13 @@ typedef struct {
                            a tuning knob: CTAs of different queries that walk
                            the same chunk together share its codes in L2     */
     int32_t list_max_ppm; /* a query whose predicate constrains one column
-                           takes the row-list scan (its pool is a segment of
-                           the rows sorted by that column: no filter pass, no
-                           bitmap) when the pool holds at most this many rows
-                           per million of N.  0: default (20000, i.e. 2 %);
-                           -1: never; 1000000: always.  Results are the same
-                           on either path.                                   */
+                           takes the sorted-copy scan (its pool is a position
+                           range of the codes sorted by that column: no
+                           filter pass, no bitmap) when the pool holds at most
+                           this many rows per million of N.  0: default
+                           (1000000: always); -1: never.  The two paths sum a
+                           row's entries in different orders, so distances
+                           agree to float32 rounding.                         */
     void* stream;       /* cudaStream_t to run on; NULL: the index's stream   */
 } ifvs_search_params;
 
@@ -142,9 +143,10 @@ enum {
  * Codes are stored re-laid out for the scan (rows padded to a multiple of
  * 1024; each row's codes rotated so that a warp's 32 lanes read 32 distinct
  * shared-memory banks).  For every attribute column the library also keeps
- * the row ids sorted by (value, row) and the sorted values (8 bytes per row
- * and column, sorted on the host at load), from which a one-column
- * predicate's pool is a contiguous segment.
+ * the row ids sorted by (value, row), the sorted values and a copy of the
+ * code rows in that order (8 + row_bytes bytes per row and column; the order
+ * is sorted on the host at load), in which a one-column predicate's pool is
+ * a contiguous position range.
  */
 int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int64_t N,
                     int32_t M, int32_t K, const void* const* attr_cols,

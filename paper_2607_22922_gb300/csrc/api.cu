@@ -103,6 +103,7 @@ struct ifvs_index {
     // per column: row ids sorted by (value, row) and the values in that order
     uint32_t* d_srt_rows[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
     int32_t* d_srt_vals[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
+    uint8_t* d_srt_codes[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
     uint8_t* d_codes = nullptr;
     float* d_vec = nullptr;
     bool has_cb = false;
@@ -130,6 +131,7 @@ struct ifvs_index {
         for (int i = 0; i < IFVS_MAX_ATTRS; ++i) {
             c.rows[i] = d_srt_rows[i];
             c.vals[i] = d_srt_vals[i];
+            c.codes[i] = d_srt_codes[i];
         }
         c.n = n_attrs;
         return c;
@@ -176,6 +178,7 @@ void free_index(ifvs_index* ix) {
         if (ix->d_attr[i]) cudaFree(ix->d_attr[i]);
         if (ix->d_srt_rows[i]) cudaFree(ix->d_srt_rows[i]);
         if (ix->d_srt_vals[i]) cudaFree(ix->d_srt_vals[i]);
+        if (ix->d_srt_codes[i]) cudaFree(ix->d_srt_codes[i]);
     }
     void* ptrs[] = {ix->d_codes, ix->d_vec, ix->d_cpq, ix->d_bank, ix->d_W, ix->d_seeds};
     for (void* p : ptrs)
@@ -208,8 +211,9 @@ int dev_alloc(ifvs_index* ix, void** p, size_t bytes) {
     return 0;
 }
 
-// Row ids of one attribute column sorted by (value, row), and the values in
-// that order, uploaded to the device: a stable LSD radix sort on the host
+// Row ids of one attribute column sorted by (value, row), the values in that
+// order, and the code rows copied into that order (rotated by position), on
+// the device.  The order comes from a stable LSD radix sort on the host
 // (two 16-bit digit passes over (key, row) pairs; key = value bits with the
 // sign flipped, so unsigned order is signed order).
 int build_sorted_column(ifvs_index* ix, int c, const void* col, int32_t type, bool dio) {
@@ -259,6 +263,12 @@ int build_sorted_column(ifvs_index* ix, int c, const void* col, int32_t type, bo
     TRY(dev_alloc(ix, &p, sizeof(int32_t) * (size_t)N));
     ix->d_srt_vals[c] = (int32_t*)p;
     CUDA_TRY(cudaMemcpy(p, key.data(), sizeof(int32_t) * (size_t)N, cudaMemcpyHostToDevice));
+    // the code rows in this order, rotated by position
+    TRY(dev_alloc(ix, &p, (size_t)ix->n_rows_pad * ix->row_bytes));
+    ix->d_srt_codes[c] = (uint8_t*)p;
+    CUDA_TRY(launch_relayout_sorted(ix->d_codes, ix->d_srt_rows[c], N, ix->M, ix->row_bytes, ix->n_rows_pad,
+                                    ix->d_srt_codes[c], ix->stream));
+    CUDA_TRY(cudaStreamSynchronize(ix->stream));
     return 0;
 }
 
@@ -300,9 +310,9 @@ struct Opts {
     cudaStream_t stream = nullptr;
 };
 
-// pools of at most 2 % of the rows take the row-list scan unless the caller
-// says otherwise (measured crossover on 10^8 rows: see the design notes)
-constexpr int32_t kListDefaultPpm = 20000;
+// one-column predicates take the sorted-copy scan at any pool size unless the
+// caller sets a threshold
+constexpr int32_t kListDefaultPpm = 1000000;
 
 int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (!p) return 0;
@@ -434,8 +444,8 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
     }
     if (plan) {
         Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
-        CUDA_TRY(st.end(launch_scan_list(ix->d_codes, ix->w_tab.as<float>(), ix->sorted(), plan, n, kk,
-                                         sh, ix->w_part.as<uint64_t>(), s)));
+        CUDA_TRY(st.end(launch_scan_list(ix->w_tab.as<float>(), ix->sorted(), plan, n, kk, sh,
+                                         ix->w_part.as<uint64_t>(), s)));
     }
     int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;
     float* m_dists = o.R > 0 ? ix->w_cdist.as<float>() : out_dists;

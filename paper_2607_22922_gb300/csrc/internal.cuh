@@ -108,11 +108,21 @@ struct ScanPlan {
     int32_t col;
     int32_t list;      // 1: row-list scan
 };
-// Row ids of each column sorted by (value, row) and the values in that order.
+// Per column: row ids sorted by (value, row), the values in that order, and
+// a copy of the code rows in that order (position p holds row rows[p]'s
+// codes, rotated by (p mod 32) mod M, row_bytes apart, padded like the index).
 struct SortedCols {
     const uint32_t* rows[IFVS_MAX_ATTRS];
     const int32_t* vals[IFVS_MAX_ATTRS];
+    const uint8_t* codes[IFVS_MAX_ATTRS];
     int32_t n;
+    __host__ __device__ const uint8_t* codes_of(int c) const {
+        const uint8_t* r = codes[0];
+#pragma unroll
+        for (int i = 1; i < IFVS_MAX_ATTRS; ++i)
+            if (c == i) r = codes[i];
+        return r;
+    }
     // column c's arrays, selected without indexing the parameter at run time
     __host__ __device__ const uint32_t* rows_of(int c) const {
         const uint32_t* r = rows[0];
@@ -179,9 +189,14 @@ int scan_kp(int k);
 cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm,
                         const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
                         uint64_t* partials, cudaStream_t s);
-// the list-path queries of `plan` (same grid and partial layout as launch_scan)
-cudaError_t launch_scan_list(const uint8_t* codes, const float* tab, SortedCols sc, const ScanPlan* plan,
-                             int64_t nq, int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s);
+// the list-path queries of `plan`: their pool is the position range [a, b)
+// of a column's sorted copy (same grid and partial layout as launch_scan)
+cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
+                             const ScanShape& sh, uint64_t* partials, cudaStream_t s);
+// the sorted copy of the codes: dst position p <- row rows[p] of the index
+// layout `src`, re-rotated by (p mod 32) mod M; positions >= N are zero
+cudaError_t launch_relayout_sorted(const uint8_t* src, const uint32_t* rows, int64_t N, int M,
+                                   int row_bytes, int64_t n_rows_pad, uint8_t* dst, cudaStream_t s);
 // Select: merge [nq][n_lists][k] partial keys -> ids / dists
 cudaError_t launch_merge(const uint64_t* partials, int64_t nq, int n_lists, int k,
                          int64_t* ids, float* dists, cudaStream_t s);

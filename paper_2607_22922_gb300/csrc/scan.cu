@@ -477,69 +477,74 @@ cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* 
     }
 }
 
-// ---- row-list scan ------------------------------------------------------
+// ---- sorted-copy scan ---------------------------------------------------
 //
-// For a query of the list path (ScanPlan), the pool is the segment
-// rows[a, b) of one column's sorted order.  CTA (query, chunk) takes an equal
-// share of the segment; warps take 32 kU consecutive positions at a time, a
-// row per lane and position (coalesced reads of the row ids), gather the rows'
-// codes and look them up with the table word index (row mod 32) + s: the same
-// entries, summed in the same order, as the bitmap path, where row mod 32 is
-// the owning lane.  Lanes of one warp may now share (row mod 32), so the
-// look-ups are no longer conflict-free; these pools are small.  Top-k and the
-// partial lists are those of k_scan, so k_merge serves both paths.
+// For a query of the list path (ScanPlan) the pool is the position range
+// [a, b) of one column's sorted copy of the codes, whose position p holds
+// row rows[p]'s codes rotated by (p mod 32) mod M.  CTA (query, chunk) walks
+// the chunk's 1024-position blocks that meet [a, b) exactly as the bitmap
+// path walks dense blocks: lane l takes the positions = l (mod 32), so its
+// look-ups hit banks (l + s) mod 32 and the code loads are coalesced; blocks
+// cut by a or b mask their positions.  No bitmap, no per-row bit handling,
+// and the CTAs of one chunk share its codes in L2.  The row id, needed for
+// the key, is loaded only for positions whose distance can enter the top-k.
+// The sum order (the subspaces from (p mod 32) mod M on) differs from the
+// bitmap path's, so the two agree to float32 rounding.
 
 size_t scan_list_smem_bytes(int tab_words, int kp) {
     return (size_t)256 * tab_words * 4 + (size_t)kScanWarps * 2 * kp * 8;
 }
 
 template <int KP, bool M16, bool FAST>
-__device__ __forceinline__ void scan_rows(const uint8_t* __restrict__ codes, const uint32_t* __restrict__ rows,
-                                          int64_t s0, int64_t s1, const ScanShape& sh, const float* tab,
-                                          WarpTopK<KP>& tk, int lane, int warp) {
+__device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes, const uint32_t* __restrict__ rows,
+                                               int64_t a, int64_t b, int64_t blk0, int64_t blk1,
+                                               const ScanShape& sh, const float* tab, WarpTopK<KP>& tk,
+                                               int lane, int warp) {
     const int M = M16 ? 16 : sh.M;
     const int S = M16 ? 64 : sh.tab_words;
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
-    const uint64_t once = policy_evict_first();
-    for (int64_t g = s0 + (int64_t)warp * 32 * kU; g < s1; g += (int64_t)kScanWarps * 32 * kU) {
-        uint32_t row[kU];
-        unsigned valid = 0u;
-#pragma unroll
-        for (int u = 0; u < kU; ++u) {
-            const int64_t p = g + 32 * u + lane;
-            const bool ok = p < s1;
-            row[u] = ok ? __ldg(rows + p) : 0u;
-            valid |= (unsigned)ok << u;
-        }
-        if constexpr (M16) {
-            uint4 c[kU];
-#pragma unroll
-            for (int u = 0; u < kU; ++u)
-                c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)row[u] * 16, once) : make_uint4(0, 0, 0, 0);
-            float d[kU];
-#pragma unroll
-            for (int u = 0; u < kU; u += 2)
-                lookup16x2<FAST>(c[u], c[u + 1], 4u * (row[u] & 31u), 4u * (row[u + 1] & 31u), base,
-                                 d[u], d[u + 1]);
-            uint64_t key[kU];
-            bool want = false;
-#pragma unroll
-            for (int u = 0; u < kU; ++u) {
-                key[u] = ((uint64_t)__float_as_uint(d[u]) << 32) | row[u];
-                want |= (valid >> u & 1u) && key[u] < tk.thr;
-            }
-            if (__any_sync(0xFFFFFFFFu, want)) {
-#pragma unroll
-                for (int u = 0; u < kU; ++u) tk.offer(key[u], (valid >> u & 1u) && key[u] < tk.thr, lane);
-            }
-        } else {
+    const uint32_t tb = 4u * (uint32_t)lane;
+    const uint64_t keep = policy_evict_last();
+    // positions fit in 32 bits: N < 2^32 - 2048
+    const uint32_t a32 = (uint32_t)a, b32 = (uint32_t)b;
+    for (int64_t blk = blk0 + warp; blk < blk1; blk += kScanWarps) {
+        const uint32_t p0 = (uint32_t)(blk * kBlockRows);
+        const bool full = p0 >= a32 && p0 + kBlockRows <= b32;
 #pragma unroll 1
+        for (int j0 = 0; j0 < 32; j0 += kU) {
+            uint32_t pos[kU];
+            unsigned valid = 0u;
+#pragma unroll
             for (int u = 0; u < kU; ++u) {
-                const bool pass = valid >> u & 1u;
-                const float d = lookup_any(codes + (size_t)row[u] * sh.row_bytes, pass, M, S, tab,
-                                           (int)(row[u] & 31u));
-                const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | row[u];
-                tk.offer(key, pass && key < tk.thr, lane);
+                pos[u] = p0 + 32u * (uint32_t)(j0 + u) + (uint32_t)lane;
+                valid |= (unsigned)(full || (pos[u] >= a32 && pos[u] < b32)) << u;
+            }
+            float d[kU];
+            if constexpr (M16) {
+                uint4 c[kU];
+#pragma unroll
+                for (int u = 0; u < kU; ++u)
+                    c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)pos[u] * 16, keep) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
+            } else {
+#pragma unroll 1
+                for (int u = 0; u < kU; ++u)
+                    d[u] = lookup_any(codes + (size_t)pos[u] * sh.row_bytes, valid >> u & 1u, M, S, tab, lane);
+            }
+            // a position can enter the top-k only if its distance is at most
+            // the current k-th one; only those load their row id
+            const uint32_t thr_hi = (uint32_t)(tk.thr >> 32);
+            bool cand_any = false;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) cand_any |= (valid >> u & 1u) && __float_as_uint(d[u]) <= thr_hi;
+            if (!__any_sync(0xFFFFFFFFu, cand_any)) continue;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const bool cand = (valid >> u & 1u) && __float_as_uint(d[u]) <= thr_hi;
+                const uint32_t row = cand ? __ldg(rows + pos[u]) : 0u;
+                const uint64_t key = ((uint64_t)__float_as_uint(d[u]) << 32) | row;
+                tk.offer(key, cand && key < tk.thr, lane);
             }
         }
     }
@@ -547,9 +552,8 @@ __device__ __forceinline__ void scan_rows(const uint8_t* __restrict__ codes, con
 
 template <int KP, bool M16, int MINB>
 __global__ void __launch_bounds__(kScanThreads, MINB)
-k_scan_list(const uint8_t* __restrict__ codes, const float* __restrict__ tables, SortedCols sc,
-            const ScanPlan* __restrict__ plan, int64_t nq, int k, ScanShape sh,
-            uint64_t* __restrict__ partials) {
+k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
+            int k, ScanShape sh, uint64_t* __restrict__ partials) {
     extern __shared__ __align__(256) uint8_t smem[];
     const int S = M16 ? 64 : sh.tab_words;
     float* tab = reinterpret_cast<float*>(smem);
@@ -559,12 +563,12 @@ k_scan_list(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
     const int chunk = blockIdx.y;
     const ScanPlan p = plan[q];
     if (!p.list) return;   // k_scan covers this query
-    const int64_t len = p.b - p.a;
-    const int64_t per = (len + sh.n_chunks - 1) / sh.n_chunks;
-    const int64_t s0 = p.a + min(len, (int64_t)chunk * per);
-    const int64_t s1 = p.a + min(len, (int64_t)(chunk + 1) * per);
+    const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
+    const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
+    const int64_t blk0 = max(c0, p.a / kBlockRows);
+    const int64_t blk1 = min(c1, (p.b + kBlockRows - 1) / kBlockRows);
     uint64_t* out = partials + (q * sh.n_chunks + chunk) * (int64_t)k;
-    if (s0 >= s1) {
+    if (p.a >= p.b || blk0 >= blk1) {
         for (int i = threadIdx.x; i < k; i += kScanThreads) out[i] = ~0ull;
         return;
     }
@@ -576,15 +580,16 @@ k_scan_list(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
     WarpTopK<KP> tk;
     tk.init(tkbuf + warp * 2 * KP, k, lane);
     __syncthreads();
+    const uint8_t* codes = sc.codes_of(p.col);
     const uint32_t* rows = sc.rows_of(p.col);
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
     if constexpr (M16) {
         if (base == kDynSmemBase)
-            scan_rows<KP, true, true>(codes, rows, s0, s1, sh, tab, tk, lane, warp);
+            scan_positions<KP, true, true>(codes, rows, p.a, p.b, blk0, blk1, sh, tab, tk, lane, warp);
         else
-            scan_rows<KP, true, false>(codes, rows, s0, s1, sh, tab, tk, lane, warp);
+            scan_positions<KP, true, false>(codes, rows, p.a, p.b, blk0, blk1, sh, tab, tk, lane, warp);
     } else {
-        scan_rows<KP, false, false>(codes, rows, s0, s1, sh, tab, tk, lane, warp);
+        scan_positions<KP, false, false>(codes, rows, p.a, p.b, blk0, blk1, sh, tab, tk, lane, warp);
     }
     tk.flush(lane);
 #pragma unroll 1
@@ -602,40 +607,77 @@ k_scan_list(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
 }
 
 template <int KP, bool M16, int MINB>
-static cudaError_t launch_list_one(const uint8_t* codes, const float* tab, SortedCols sc,
-                                   const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
-                                   uint64_t* partials, size_t smem, cudaStream_t s) {
+static cudaError_t launch_list_one(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
+                                   int k, const ScanShape& sh, uint64_t* partials, size_t smem,
+                                   cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(k_scan_list<KP, M16, MINB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
-    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(codes, tab, sc, plan, nq, k, sh, partials);
+    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials);
     return cudaGetLastError();
 }
 
 template <int KP>
-static cudaError_t launch_list_kp(const uint8_t* codes, const float* tab, SortedCols sc,
-                                  const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
-                                  uint64_t* partials, cudaStream_t s) {
+static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
+                                  int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s) {
     const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
     const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
     if (m16) {
         if ((size_t)233472 / (smem + 1024) >= 2)
-            return launch_list_one<KP, true, 2>(codes, tab, sc, plan, nq, k, sh, partials, smem, s);
-        return launch_list_one<KP, true, 1>(codes, tab, sc, plan, nq, k, sh, partials, smem, s);
+            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, smem, s);
+        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, smem, s);
     }
-    return launch_list_one<KP, false, 1>(codes, tab, sc, plan, nq, k, sh, partials, smem, s);
+    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, smem, s);
 }
 
-cudaError_t launch_scan_list(const uint8_t* codes, const float* tab, SortedCols sc, const ScanPlan* plan,
-                             int64_t nq, int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s) {
+cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
+                             const ScanShape& sh, uint64_t* partials, cudaStream_t s) {
     if (nq <= 0) return cudaSuccess;
     switch (scan_kp(k)) {
-        case 32: return launch_list_kp<32>(codes, tab, sc, plan, nq, k, sh, partials, s);
-        case 64: return launch_list_kp<64>(codes, tab, sc, plan, nq, k, sh, partials, s);
-        case 128: return launch_list_kp<128>(codes, tab, sc, plan, nq, k, sh, partials, s);
-        default: return launch_list_kp<256>(codes, tab, sc, plan, nq, k, sh, partials, s);
+        case 32: return launch_list_kp<32>(tab, sc, plan, nq, k, sh, partials, s);
+        case 64: return launch_list_kp<64>(tab, sc, plan, nq, k, sh, partials, s);
+        case 128: return launch_list_kp<128>(tab, sc, plan, nq, k, sh, partials, s);
+        default: return launch_list_kp<256>(tab, sc, plan, nq, k, sh, partials, s);
     }
+}
+
+// sorted copy: position p <- row rows[p] (stored rotated by (row mod 32) mod M)
+// re-rotated by (p mod 32) mod M
+__global__ void k_relayout_sorted(const uint8_t* __restrict__ src, const uint32_t* __restrict__ rows,
+                                  int64_t N, int M, int row_bytes, int64_t n_rows_pad,
+                                  uint8_t* __restrict__ dst) {
+    const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (p >= n_rows_pad) return;
+    uint8_t* out = dst + p * row_bytes;
+    if (p >= N) {
+        for (int s = 0; s < row_bytes; ++s) out[s] = 0;
+        return;
+    }
+    const uint32_t row = rows[p];
+    const uint8_t* in = src + (int64_t)row * row_bytes;
+    const int rot_r = (int)(row & 31u) % M;
+    const int rot_p = (int)(p & 31) % M;
+    for (int s = 0; s < row_bytes; ++s) {
+        uint8_t v = 0;
+        if (s < M) {
+            // byte s must hold subspace (s + rot_p) mod M, stored in `in` at
+            // byte (s + rot_p - rot_r) mod M
+            int t = s + rot_p - rot_r;
+            t %= M;
+            if (t < 0) t += M;
+            v = in[t];
+        }
+        out[s] = v;
+    }
+}
+
+cudaError_t launch_relayout_sorted(const uint8_t* src, const uint32_t* rows, int64_t N, int M,
+                                   int row_bytes, int64_t n_rows_pad, uint8_t* dst, cudaStream_t s) {
+    const int threads = 256;
+    const int64_t blocks = (n_rows_pad + threads - 1) / threads;
+    k_relayout_sorted<<<(unsigned)blocks, threads, 0, s>>>(src, rows, N, M, row_bytes, n_rows_pad, dst);
+    return cudaGetLastError();
 }
 
 // ---- index layout -----------------------------------------------------------

@@ -1,10 +1,13 @@
-"""The row-list scan (a one-column predicate's pool read from the rows sorted
-by that column) against the bitmap path and the oracle.
+"""The sorted-copy scan (a one-column predicate's pool read as a position
+range of the codes sorted by that column) against the bitmap path and the
+oracle.
 
-Both paths sum the same table entries in the same order, so forcing one or
-the other (list_max_ppm = 1000000 / -1) must give bit-identical ids,
-distances and pass counts; each is also checked against the oracle with the
-tie rule of the other parity tests."""
+Forcing one path or the other (list_max_ppm = 1000000 / -1) must give the
+same pass counts exactly; each path's ids and distances are checked against
+the oracle with the tie rule of the other parity tests, and against each
+other: the paths add a row's M table entries in different orders, so their
+distances agree to float32 rounding (1e-5 relative) and ids may differ only
+among distances tied to that precision."""
 import numpy as np
 import pytest
 
@@ -81,19 +84,40 @@ def _check_oracle(orc, codes, attrs, Cpq, q, preds, k, ids, dists, npass):
         check_topk(ids[i], dists[i], oi[i], od[i], all_d, passing)
 
 
+def _same_up_to_rounding(a, b, rel=1e-5):
+    """Two searches' (ids, dists, npass): equal counts and padding, distances
+    rank by rank within rel, ids equal except among distances tied to 2 rel
+    with the k-th."""
+    ia, da, na = a
+    ib, db, nb = b
+    np.testing.assert_array_equal(na, nb)
+    np.testing.assert_array_equal(ia < 0, ib < 0)
+    for x, y, dx, dy in zip(ia, ib, da, db):
+        nv = int((x >= 0).sum())
+        if nv == 0:
+            continue
+        assert np.all(np.abs(dx[:nv].astype(np.float64) - dy[:nv]) <= rel * np.maximum(dy[:nv], 1e-30))
+        kth = float(dy[nv - 1])
+        dist_of = dict(zip(x[:nv].tolist(), dx[:nv].tolist()))
+        dist_of.update(zip(y[:nv].tolist(), dy[:nv].tolist()))
+        for i in set(x[:nv].tolist()) ^ set(y[:nv].tolist()):
+            assert abs(dist_of[i] - kth) <= 2 * rel * kth
+
+
 @pytest.mark.parametrize("N,k", [(1, 1), (1000, 10), (33333, 100), (100000, 256)])
-def test_list_path_equals_bitmap_path(ifvs, orc, N, k):
+def test_list_path_and_bitmap_path(ifvs, orc, N, k):
     g, codes, attrs, Cpq = _index(ifvs, N)
     p = _preds()
     q = _queries(len(p), Cpq.shape[0] * Cpq.shape[2])
     a = g.search(q, p, k, list_max_ppm=ALWAYS)
     b = g.search(q, p, k, list_max_ppm=NEVER)
-    d = g.search(q, p, k)                      # default threshold: a mix of both
-    for x, y, z in zip(a, b, d):
-        np.testing.assert_array_equal(x, y)
+    d = g.search(q, p, k)                      # the default: the sorted-copy path
+    for x, z in zip(a, d):
         np.testing.assert_array_equal(x, z)
+    _same_up_to_rounding(a, b)
     if N <= 33333:
         _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
+        _check_oracle(orc, codes, attrs, Cpq, q, p, k, *b)
 
 
 @pytest.mark.parametrize("M", [1, 8, 12, 24])
@@ -103,9 +127,19 @@ def test_list_path_other_subspace_counts(ifvs, orc, M):
     q = _queries(len(p), M * 3, seed=M)
     a = g.search(q, p, 20, list_max_ppm=ALWAYS)
     b = g.search(q, p, 20, list_max_ppm=NEVER)
-    for x, y in zip(a, b):
-        np.testing.assert_array_equal(x, y)
+    _same_up_to_rounding(a, b)
     _check_oracle(orc, codes, attrs, Cpq, q, p, 20, *a)
+
+
+def test_threshold_splits_a_batch(ifvs, orc):
+    """A threshold of 1 % sends the narrow predicates of a batch to the
+    sorted copy and the wide ones to the bitmap; results as either path."""
+    g, codes, attrs, Cpq = _index(ifvs, 40000, seed=9)
+    p = _preds()
+    q = _queries(len(p), 32, seed=9)
+    mixed = g.search(q, p, 30, list_max_ppm=10000)
+    _same_up_to_rounding(mixed, g.search(q, p, 30, list_max_ppm=NEVER))
+    _check_oracle(orc, codes, attrs, Cpq, q, p, 30, *mixed)
 
 
 def test_list_path_with_conditioning_sub_batches_and_device_index(ifvs, orc):
@@ -125,8 +159,7 @@ def test_list_path_with_conditioning_sub_batches_and_device_index(ifvs, orc):
         g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
         a = g.search(qs.q, qs.preds, 10, wz=qs.wz, list_max_ppm=ALWAYS, sub_batch=32)
         b = g.search(qs.q, qs.preds, 10, wz=qs.wz, list_max_ppm=NEVER)
-        for x, y in zip(a, b):
-            np.testing.assert_array_equal(x, y)
+        _same_up_to_rounding(a, b)
         oi, od, on = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q, qs.preds, 10,
                                 bank=cond.bank, W=cond.W, seeds=cond.seeds, wz=qs.wz)
         np.testing.assert_array_equal(a[2], on)
