@@ -348,6 +348,7 @@ int64_t pick_sub_batch(const ifvs_index* ix, const Opts& o, int64_t nq) {
 ScanShape scan_shape(const ifvs_index* ix, int64_t n, int kk, int64_t chunk_blocks) {
     ScanShape sh;
     sh.n_blocks = ix->n_blocks;
+    sh.n_rows = ix->N;
     sh.M = ix->M;
     sh.K = ix->K;
     sh.row_bytes = ix->row_bytes;
@@ -444,8 +445,10 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
     }
     if (plan) {
         Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
-        CUDA_TRY(st.end(launch_scan_list(ix->w_tab.as<float>(), ix->sorted(), plan, n, kk, sh,
-                                         ix->w_part.as<uint64_t>(), s)));
+        int nl = 0;
+        const cudaError_t e = launch_scan_list(ix->w_tab.as<float>(), ix->sorted(), plan, n, kk, sh,
+                                               ix->w_part.as<uint64_t>(), s, &nl);
+        CUDA_TRY(st.end(e, nl));
     }
     int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;
     float* m_dists = o.R > 0 ? ix->w_cdist.as<float>() : out_dists;

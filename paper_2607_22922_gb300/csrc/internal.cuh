@@ -178,6 +178,7 @@ struct ScanShape {
     int tab_words;         // LUT table stride in words per codeword
     int64_t blocks_per_chunk;
     int n_chunks;
+    int64_t n_rows;        // N (rows of the index)
 };
 size_t scan_smem_bytes(int tab_words, int kp);
 // CTAs of the scan resident per SM for this table stride and list size
@@ -191,8 +192,9 @@ cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* 
                         uint64_t* partials, cudaStream_t s);
 // the list-path queries of `plan`: their pool is the position range [a, b)
 // of a column's sorted copy (same grid and partial layout as launch_scan)
+// (*launches = kernels launched: a one-query and, for M = 16, a two-query kernel)
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
-                             const ScanShape& sh, uint64_t* partials, cudaStream_t s);
+                             const ScanShape& sh, uint64_t* partials, cudaStream_t s, int* launches);
 // the sorted copy of the codes: dst position p <- row rows[p] of the index
 // layout `src`, re-rotated by (p mod 32) mod M; positions >= N are zero
 cudaError_t launch_relayout_sorted(const uint8_t* src, const uint32_t* rows, int64_t N, int M,

@@ -126,6 +126,7 @@ extern "C" int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uin
                                                      (size_t)n * 256 * v.tab_words * sizeof(float));
         ScanShape sh;
         sh.n_blocks = v.n_blocks;
+        sh.n_rows = v.N;
         sh.M = v.M;
         sh.K = v.K;
         sh.row_bytes = v.row_bytes;

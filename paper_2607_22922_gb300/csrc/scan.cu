@@ -497,7 +497,7 @@ size_t scan_list_smem_bytes(int tab_words, int kp) {
 
 template <int KP, bool M16, bool FAST>
 __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes, const uint32_t* __restrict__ rows,
-                                               int64_t a, int64_t b, int64_t blk0, int64_t blk1,
+                                               int64_t a, int64_t b, int64_t blk0, int64_t blk1, int wstride,
                                                const ScanShape& sh, const float* tab, WarpTopK<KP>& tk,
                                                int lane, int warp) {
     const int M = M16 ? 16 : sh.M;
@@ -507,7 +507,7 @@ __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes
     const uint64_t keep = policy_evict_last();
     // positions fit in 32 bits: N < 2^32 - 2048
     const uint32_t a32 = (uint32_t)a, b32 = (uint32_t)b;
-    for (int64_t blk = blk0 + warp; blk < blk1; blk += kScanWarps) {
+    for (int64_t blk = blk0 + warp; blk < blk1; blk += wstride) {
         const uint32_t p0 = (uint32_t)(blk * kBlockRows);
         const bool full = p0 >= a32 && p0 + kBlockRows <= b32;
 #pragma unroll 1
@@ -550,10 +550,35 @@ __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes
     }
 }
 
+// Two consecutive sorted-path queries share a CTA when they read the same
+// column's copy, both ranges cover at least 3/4 of the rows and 3/4 of the
+// longer one is common to both (the dense queries); otherwise each takes a
+// CTA of its own.  Narrower pairs are left alone on purpose: the two kernels
+// run one after the other, so a few long two-query CTAs would leave the GPU
+// idle behind them.  Both scan kernels evaluate this rule, so each query is
+// served exactly once.
+__device__ __forceinline__ bool pair_ok(const ScanPlan& x, const ScanPlan& y, int64_t N) {
+    if (!x.list || !y.list || x.col != y.col) return false;
+    const int64_t lx = x.b - x.a, ly = y.b - y.a;
+    const int64_t common = min(x.b, y.b) - max(x.a, y.a);
+    const int64_t longer = max(lx, ly);
+    return 4 * lx >= 3 * N && 4 * ly >= 3 * N && longer > 0 && 4 * common >= 3 * longer;
+}
+
+// the single-query loop for M = 16 (FAST: table at the dynamic shared base)
+template <int KP, bool FAST>
+__device__ __forceinline__ void scan_positions_range(const uint8_t* __restrict__ codes,
+                                                     const uint32_t* __restrict__ rows, int64_t a, int64_t b,
+                                                     int64_t blk0, int64_t blk1, int wstride,
+                                                     const ScanShape& sh, const float* tab, WarpTopK<KP>& tk,
+                                                     int lane, int warp) {
+    scan_positions<KP, true, FAST>(codes, rows, a, b, blk0, blk1, wstride, sh, tab, tk, lane, warp);
+}
+
 template <int KP, bool M16, int MINB>
 __global__ void __launch_bounds__(kScanThreads, MINB)
 k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
-            int k, ScanShape sh, uint64_t* __restrict__ partials) {
+            int k, ScanShape sh, uint64_t* __restrict__ partials, int pairs) {
     extern __shared__ __align__(256) uint8_t smem[];
     const int S = M16 ? 64 : sh.tab_words;
     float* tab = reinterpret_cast<float*>(smem);
@@ -563,6 +588,10 @@ k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __r
     const int chunk = blockIdx.y;
     const ScanPlan p = plan[q];
     if (!p.list) return;   // k_scan covers this query
+    if (pairs) {           // k_scan_list_pair covers paired queries
+        const int64_t mate = q ^ 1;
+        if (mate < nq && pair_ok(plan[q & ~(int64_t)1], plan[q | 1], sh.n_rows)) return;
+    }
     const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
     const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
     const int64_t blk0 = max(c0, p.a / kBlockRows);
@@ -585,11 +614,11 @@ k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __r
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
     if constexpr (M16) {
         if (base == kDynSmemBase)
-            scan_positions<KP, true, true>(codes, rows, p.a, p.b, blk0, blk1, sh, tab, tk, lane, warp);
+            scan_positions<KP, true, true>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
         else
-            scan_positions<KP, true, false>(codes, rows, p.a, p.b, blk0, blk1, sh, tab, tk, lane, warp);
+            scan_positions<KP, true, false>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
     } else {
-        scan_positions<KP, false, false>(codes, rows, p.a, p.b, blk0, blk1, sh, tab, tk, lane, warp);
+        scan_positions<KP, false, false>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
     }
     tk.flush(lane);
 #pragma unroll 1
@@ -606,39 +635,258 @@ k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __r
         for (int i = lane; i < k; i += 32) out[i] = tk.buf[i];
 }
 
+// ---- two queries per CTA on the sorted copy --------------------------------
+//
+// When two consecutive queries both take the sorted copy of the same column
+// (M = 16), one CTA serves both: their tables sit back to back in shared
+// memory (B 64 KB after A, so both keep the immediate-offset addressing) and
+// each 16-byte code load and byte permute feeds a look-up in each table.
+// Blocks that meet only one query's range (and pairs that cannot share) run
+// the single-query loop.  16 warps, one CTA per SM.
+constexpr int kPairWarps = 16;
+constexpr int kPairThreads = kPairWarps * 32;
+constexpr uint32_t kTabBytes16 = 256u * 64u * 4u;   // one M = 16 table
+
+size_t scan_pair_smem_bytes(int kp) { return (size_t)2 * kTabBytes16 + (size_t)kPairWarps * 2 * 2 * kp * 8; }
+
+// Four distances: rows a, b (codes ca, cb) in tables A (at the dynamic
+// shared base) and B (kTabBytes16 above it).
+__device__ __forceinline__ void lookup16x2x2(const uint4 ca, const uint4 cb, uint32_t tb, float& aa,
+                                             float& ab, float& ba, float& bb) {
+    const uint32_t wa[4] = {ca.x, ca.y, ca.z, ca.w};
+    const uint32_t wb[4] = {cb.x, cb.y, cb.z, cb.w};
+    uint64_t accA = 0ull, accB = 0ull;
+#pragma unroll
+    for (int s = 0; s < 16; ++s) {
+        const uint32_t sel = 0x5504u | ((uint32_t)(s & 3) << 4);
+        const uint32_t oa = __byte_perm(wa[s >> 2], tb, sel);
+        const uint32_t ob = __byte_perm(wb[s >> 2], tb, sel);
+        float va, vb, wa2, wb2;
+        switch (s) {
+#define IFVS_LDS2_CASE(S)                                          \
+    case S:                                                        \
+        va = lds_imm<kDynSmemBase + 4 * S>(oa);                    \
+        vb = lds_imm<kDynSmemBase + 4 * S>(ob);                    \
+        wa2 = lds_imm<kDynSmemBase + kTabBytes16 + 4 * S>(oa);     \
+        wb2 = lds_imm<kDynSmemBase + kTabBytes16 + 4 * S>(ob);     \
+        break;
+            IFVS_LDS2_CASE(0) IFVS_LDS2_CASE(1) IFVS_LDS2_CASE(2) IFVS_LDS2_CASE(3)
+            IFVS_LDS2_CASE(4) IFVS_LDS2_CASE(5) IFVS_LDS2_CASE(6) IFVS_LDS2_CASE(7)
+            IFVS_LDS2_CASE(8) IFVS_LDS2_CASE(9) IFVS_LDS2_CASE(10) IFVS_LDS2_CASE(11)
+            IFVS_LDS2_CASE(12) IFVS_LDS2_CASE(13) IFVS_LDS2_CASE(14) IFVS_LDS2_CASE(15)
+#undef IFVS_LDS2_CASE
+            default: va = vb = wa2 = wb2 = 0.f; break;
+        }
+        accA = add_f32x2(accA, va, vb);
+        accB = add_f32x2(accB, wa2, wb2);
+    }
+    unpack_f32x2(accA, aa, ab);
+    unpack_f32x2(accB, ba, bb);
+}
+
+// kU2 rows per lane per round in the paired loop
+constexpr int kU2 = 4;
+
+template <int KP>
+__device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ codes,
+                                                    const uint32_t* __restrict__ rows, int64_t aA,
+                                                    int64_t bA, int64_t aB, int64_t bB, int64_t blk0,
+                                                    int64_t blk1, WarpTopK<KP>& tkA, WarpTopK<KP>& tkB,
+                                                    const float* tabA, const float* tabB,
+                                                    const ScanShape& sh, int lane, int warp) {
+    const uint32_t tb = 4u * (uint32_t)lane;
+    const uint64_t keep = policy_evict_last();
+    const uint32_t a1 = (uint32_t)aA, b1 = (uint32_t)bA, a2 = (uint32_t)aB, b2 = (uint32_t)bB;
+    for (int64_t blk = blk0 + warp; blk < blk1; blk += kPairWarps) {
+        const uint32_t p0 = (uint32_t)(blk * kBlockRows);
+        const uint32_t pe = p0 + kBlockRows;
+        const bool inA = p0 < b1 && pe > a1, inB = p0 < b2 && pe > a2;
+        if (!(inA && inB)) {
+            // one query only: the single-query loop on this block (table A
+            // is at the shared base; table B takes the base-add form)
+            if (inA)
+                scan_positions_range<KP, true>(codes, rows, aA, bA, blk, blk + 1, 1, sh, tabA, tkA, lane, 0);
+            else if (inB)
+                scan_positions_range<KP, false>(codes, rows, aB, bB, blk, blk + 1, 1, sh, tabB, tkB, lane, 0);
+            continue;
+        }
+        const bool fullA = p0 >= a1 && pe <= b1, fullB = p0 >= a2 && pe <= b2;
+#pragma unroll 1
+        for (int j0 = 0; j0 < 32; j0 += kU2) {
+            uint32_t pos[kU2];
+            unsigned vA = 0u, vB = 0u;
+#pragma unroll
+            for (int u = 0; u < kU2; ++u) {
+                pos[u] = p0 + 32u * (uint32_t)(j0 + u) + (uint32_t)lane;
+                vA |= (unsigned)(fullA || (pos[u] >= a1 && pos[u] < b1)) << u;
+                vB |= (unsigned)(fullB || (pos[u] >= a2 && pos[u] < b2)) << u;
+            }
+            const unsigned v = vA | vB;
+            uint4 c[kU2];
+#pragma unroll
+            for (int u = 0; u < kU2; ++u)
+                c[u] = (v >> u & 1u) ? ldg_nc_v4(codes + (size_t)pos[u] * 16, keep) : make_uint4(0, 0, 0, 0);
+            float dA[kU2], dB[kU2];
+#pragma unroll
+            for (int u = 0; u < kU2; u += 2) lookup16x2x2(c[u], c[u + 1], tb, dA[u], dA[u + 1], dB[u], dB[u + 1]);
+            const uint32_t hA = (uint32_t)(tkA.thr >> 32), hB = (uint32_t)(tkB.thr >> 32);
+            bool any = false;
+#pragma unroll
+            for (int u = 0; u < kU2; ++u)
+                any |= ((vA >> u & 1u) && __float_as_uint(dA[u]) <= hA) ||
+                       ((vB >> u & 1u) && __float_as_uint(dB[u]) <= hB);
+            if (!__any_sync(0xFFFFFFFFu, any)) continue;
+#pragma unroll
+            for (int u = 0; u < kU2; ++u) {
+                const bool cA = (vA >> u & 1u) && __float_as_uint(dA[u]) <= hA;
+                const bool cB = (vB >> u & 1u) && __float_as_uint(dB[u]) <= hB;
+                const uint32_t row = (cA || cB) ? __ldg(rows + pos[u]) : 0u;
+                const uint64_t kA = ((uint64_t)__float_as_uint(dA[u]) << 32) | row;
+                const uint64_t kB = ((uint64_t)__float_as_uint(dB[u]) << 32) | row;
+                tkA.offer(kA, cA && kA < tkA.thr, lane);
+                tkB.offer(kB, cB && kB < tkB.thr, lane);
+            }
+        }
+    }
+}
+
+// merge the warps' lists of one query pairwise; warp 0 writes k keys
+template <int KP, int WARPS>
+__device__ __forceinline__ void merge_warps(WarpTopK<KP>& tk, uint64_t* tkbuf, int k, int lane, int warp,
+                                            uint64_t* out) {
+    tk.flush(lane);
+#pragma unroll 1
+    for (int step = 1; step < WARPS; step <<= 1) {
+        __syncthreads();
+        if ((warp & (2 * step - 1)) == 0) {
+            const uint64_t* other = tkbuf + (warp + step) * 2 * KP;
+            for (int i = lane; i < k; i += 32) tk.buf[KP + i] = other[i];
+            __syncwarp();
+            tk.flush(lane);
+        }
+    }
+    if (warp == 0 && out != nullptr)
+        for (int i = lane; i < k; i += 32) out[i] = tk.buf[i];
+}
+
+template <int KP>
+__global__ void __launch_bounds__(kPairThreads, 1)
+k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan,
+                 int64_t nq, int k, ScanShape sh, uint64_t* __restrict__ partials) {
+    extern __shared__ __align__(256) uint8_t smem[];
+    float* tabA = reinterpret_cast<float*>(smem);
+    float* tabB = reinterpret_cast<float*>(smem + kTabBytes16);
+    uint64_t* tkbufA = reinterpret_cast<uint64_t*>(smem + 2 * kTabBytes16);
+    uint64_t* tkbufB = tkbufA + kPairWarps * 2 * KP;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t qA = 2 * (int64_t)blockIdx.x, qB = qA + 1;
+    const bool hasB = qB < nq;
+    const int chunk = blockIdx.y;
+    const ScanPlan pA = plan[qA];
+    if (!hasB) return;
+    const ScanPlan pB = plan[qB];
+    if (!pair_ok(pA, pB, sh.n_rows)) return;   // k_scan_list covers these queries
+    const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
+    const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
+    auto range = [&](const ScanPlan& p, int64_t& lo, int64_t& hi) {
+        lo = max(c0, p.a / kBlockRows);
+        hi = min(c1, (p.b + kBlockRows - 1) / kBlockRows);
+        if (!p.list || p.a >= p.b || lo >= hi) lo = hi = 0;
+    };
+    int64_t lA, hA, lB, hB;
+    range(pA, lA, hA);
+    range(pB, lB, hB);
+    uint64_t* outA = pA.list ? partials + (qA * sh.n_chunks + chunk) * (int64_t)k : nullptr;
+    uint64_t* outB = pB.list ? partials + (qB * sh.n_chunks + chunk) * (int64_t)k : nullptr;
+    if (lA == hA && lB == hB) {
+        for (int i = threadIdx.x; i < k; i += kPairThreads) {
+            if (outA) outA[i] = ~0ull;
+            if (outB) outB[i] = ~0ull;
+        }
+        return;
+    }
+    {
+        const float4* srcA = reinterpret_cast<const float4*>(tables + qA * (int64_t)256 * 64);
+        float4* dstA = reinterpret_cast<float4*>(tabA);
+        for (int i = threadIdx.x; i < 64 * 64; i += kPairThreads) dstA[i] = __ldg(srcA + i);
+        if (pB.list) {
+            const float4* srcB = reinterpret_cast<const float4*>(tables + qB * (int64_t)256 * 64);
+            float4* dstB = reinterpret_cast<float4*>(tabB);
+            for (int i = threadIdx.x; i < 64 * 64; i += kPairThreads) dstB[i] = __ldg(srcB + i);
+        }
+    }
+    WarpTopK<KP> tkA, tkB;
+    tkA.init(tkbufA + warp * 2 * KP, k, lane);
+    tkB.init(tkbufB + warp * 2 * KP, k, lane);
+    __syncthreads();
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tabA);
+    if (base == kDynSmemBase && pA.list && pB.list && pA.col == pB.col) {
+        const int64_t lo = (lA == hA) ? lB : ((lB == hB) ? lA : min(lA, lB));
+        const int64_t hi = max(hA, hB);
+        scan_positions_pair<KP>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, pB.a, pB.b, lo, hi,
+                                tkA, tkB, tabA, tabB, sh, lane, warp);
+    } else {
+        if (lA < hA)
+            scan_positions_range<KP, false>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, lA, hA,
+                                            kPairWarps, sh, tabA, tkA, lane, warp);
+        if (lB < hB)
+            scan_positions_range<KP, false>(sc.codes_of(pB.col), sc.rows_of(pB.col), pB.a, pB.b, lB, hB,
+                                            kPairWarps, sh, tabB, tkB, lane, warp);
+    }
+    merge_warps<KP, kPairWarps>(tkA, tkbufA, k, lane, warp, outA);
+    merge_warps<KP, kPairWarps>(tkB, tkbufB, k, lane, warp, outB);
+}
+
 template <int KP, bool M16, int MINB>
 static cudaError_t launch_list_one(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
-                                   int k, const ScanShape& sh, uint64_t* partials, size_t smem,
+                                   int k, const ScanShape& sh, uint64_t* partials, size_t smem, int pairs,
                                    cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(k_scan_list<KP, M16, MINB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
-    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials);
+    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, pairs);
     return cudaGetLastError();
 }
 
 template <int KP>
 static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
-                                  int k, const ScanShape& sh, uint64_t* partials, cudaStream_t s) {
+                                  int k, const ScanShape& sh, uint64_t* partials, int* launches,
+                                  cudaStream_t s) {
     const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
     const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
+    if (m16 && KP <= 128) {
+        // wide, overlapping pairs share a CTA; everything else runs one query per CTA
+        const size_t ps = scan_pair_smem_bytes(KP);
+        cudaError_t e = cudaFuncSetAttribute(k_scan_list_pair<KP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)ps);
+        if (e != cudaSuccess) return e;
+        dim3 grid((unsigned)((nq + 1) / 2), (unsigned)sh.n_chunks);
+        k_scan_list_pair<KP><<<grid, kPairThreads, ps, s>>>(tab, sc, plan, nq, k, sh, partials);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if (launches) *launches = 2;
+        if ((size_t)233472 / (smem + 1024) >= 2)
+            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, smem, 1, s);
+        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, smem, 1, s);
+    }
+    if (launches) *launches = 1;
     if (m16) {
         if ((size_t)233472 / (smem + 1024) >= 2)
-            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, smem, s);
-        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, smem, s);
+            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, smem, 0, s);
+        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, smem, 0, s);
     }
-    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, smem, s);
+    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, smem, 0, s);
 }
 
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
-                             const ScanShape& sh, uint64_t* partials, cudaStream_t s) {
+                             const ScanShape& sh, uint64_t* partials, cudaStream_t s, int* launches) {
+    if (launches) *launches = 0;
     if (nq <= 0) return cudaSuccess;
     switch (scan_kp(k)) {
-        case 32: return launch_list_kp<32>(tab, sc, plan, nq, k, sh, partials, s);
-        case 64: return launch_list_kp<64>(tab, sc, plan, nq, k, sh, partials, s);
-        case 128: return launch_list_kp<128>(tab, sc, plan, nq, k, sh, partials, s);
-        default: return launch_list_kp<256>(tab, sc, plan, nq, k, sh, partials, s);
+        case 32: return launch_list_kp<32>(tab, sc, plan, nq, k, sh, partials, launches, s);
+        case 64: return launch_list_kp<64>(tab, sc, plan, nq, k, sh, partials, launches, s);
+        case 128: return launch_list_kp<128>(tab, sc, plan, nq, k, sh, partials, launches, s);
+        default: return launch_list_kp<256>(tab, sc, plan, nq, k, sh, partials, launches, s);
     }
 }
 

@@ -131,6 +131,29 @@ def test_list_path_other_subspace_counts(ifvs, orc, M):
     _check_oracle(orc, codes, attrs, Cpq, q, p, 20, *a)
 
 
+@pytest.mark.parametrize("k", [10, 100])
+def test_pairs_of_wide_predicates(ifvs, orc, k):
+    """Consecutive queries whose ranges on one column both cover 3/4 of the
+    rows and overlap by 3/4 share a CTA (M = 16); narrower or shifted pairs,
+    an odd last query and a pair on different columns run one per CTA."""
+    g, codes, attrs, Cpq = _index(ifvs, 70000, seed=11)
+    rows = [(-500, 500), (-500, 500), (-450, 500), (-500, 480), (-300, 400), (-250, 420),
+            (-400, 300), (100, 200), (-480, 499)]
+    p = synth.empty_predicates(len(rows) + 2)
+    for i, (lo, hi) in enumerate(rows):
+        p[i]["n_clauses"] = 1
+        synth.set_clause(p[i], 0, 0, synth.OP_RANGE, lo, hi)
+    p[9]["n_clauses"] = 1
+    synth.set_clause(p[9], 0, 1, synth.OP_GE, -20)          # column 1 ...
+    p[10]["n_clauses"] = 1
+    synth.set_clause(p[10], 0, 0, synth.OP_GE, -500)        # ... beside column 0: no pair
+    q = _queries(len(p), 32, seed=11)
+    a = g.search(q, p, k, list_max_ppm=ALWAYS)
+    b = g.search(q, p, k, list_max_ppm=NEVER)
+    _same_up_to_rounding(a, b)
+    _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
+
+
 def test_threshold_splits_a_batch(ifvs, orc):
     """A threshold of 1 % sends the narrow predicates of a batch to the
     sorted copy and the wide ones to the bitmap; results as either path."""
@@ -172,7 +195,8 @@ def test_threshold_and_launch_counts(ifvs):
     g.stage_times(reset=True)
     g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
-    assert t["filter"][1] == 2 and t["scan"][1] == 2          # plan + filter, bitmap + list scan
+    # plan + filter; the bitmap scan and the sorted-copy scan's one- and two-query kernels
+    assert t["filter"][1] == 2 and t["scan"][1] == 3
     g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING, list_max_ppm=NEVER)
     t = g.stage_times(reset=True)
     assert t["filter"][1] == 1 and t["scan"][1] == 1
