@@ -37,7 +37,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 WORKLOAD = "gmm100m-d128-m16"
-LIST_DEFAULT_PPM = 1000000   # the library's default sorted-copy threshold (always)
+LIST_DEFAULT_PPM = 1000000   # the library's default sorted-copy threshold for M = 16 (always)
 TRAIN_WORKLOAD = "sift1m-d128-m16"
 CPU_SAMPLE_ROWS = 10_000_000
 
@@ -376,7 +376,7 @@ def run_ifvs(args):
     # row ids it loads for top-k candidates only are not counted)
     per_bin = {}
     n_blocks = (w.N + 1023) // 1024
-    ppm = args.list_max_ppm if args.list_max_ppm != 0 else LIST_DEFAULT_PPM
+    ppm = args.list_max_ppm if args.list_max_ppm != 0 else (LIST_DEFAULT_PPM if w.M == 16 else 20000)
     list_rows = -1 if ppm < 0 else w.N * ppm // 1000000
     scan_bytes = 0.0
     for b, qs in enumerate(batches):

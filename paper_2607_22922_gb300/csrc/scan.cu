@@ -310,7 +310,7 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                         for (int u = 0; u < kU; ++u) tk.offer(key[u], key[u] < tk.thr, lane);
                     }
                 } else {
-#pragma unroll 1
+#pragma unroll
                     for (int u = 0; u < kU; ++u) {
                         const float d = lookup_any(codes + (size_t)row[u] * row_bytes, true, M, S, tab, lane);
                         const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | row[u];
@@ -362,7 +362,7 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                 for (int u = 0; u < kU; ++u) tk.offer(key[u], (valid >> u & 1u) && key[u] < tk.thr, lane);
             }
         } else {
-#pragma unroll 1
+#pragma unroll
             for (int u = 0; u < kU; ++u) {
                 const bool pass = valid >> u & 1u;
                 const float d = lookup_any(codes + (size_t)row[u] * row_bytes, pass, M, S, tab, lane);
@@ -528,7 +528,8 @@ __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes
 #pragma unroll
                 for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
             } else {
-#pragma unroll 1
+                // unrolled, so that pos[] and d[] stay in registers
+#pragma unroll
                 for (int u = 0; u < kU; ++u)
                     d[u] = lookup_any(codes + (size_t)pos[u] * sh.row_bytes, valid >> u & 1u, M, S, tab, lane);
             }
@@ -855,8 +856,10 @@ static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPla
                                   cudaStream_t s) {
     const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
     const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
-    if (m16 && KP <= 128) {
-        // wide, overlapping pairs share a CTA; everything else runs one query per CTA
+    if (m16 && KP == 128) {
+        // wide, overlapping pairs share a CTA; everything else runs one query
+        // per CTA.  For k <= 64 the one-query kernel holds three CTAs (24
+        // warps) per SM against the pair kernel's 16 warps, and wins.
         const size_t ps = scan_pair_smem_bytes(KP);
         cudaError_t e = cudaFuncSetAttribute(k_scan_list_pair<KP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)ps);

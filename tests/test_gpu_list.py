@@ -195,8 +195,12 @@ def test_threshold_and_launch_counts(ifvs):
     g.stage_times(reset=True)
     g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
-    # plan + filter; the bitmap scan and the sorted-copy scan's one- and two-query kernels
-    assert t["filter"][1] == 2 and t["scan"][1] == 3
+    # plan + filter; the bitmap scan and the sorted-copy scan (k = 10: the
+    # one-query kernel only; the two-query kernel runs for 64 < k <= 128)
+    assert t["filter"][1] == 2 and t["scan"][1] == 2
+    g.search(q, p, 100, flags=ifvs.IFVS_F_STAGE_TIMING)
+    t = g.stage_times(reset=True)
+    assert t["scan"][1] == 3
     g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING, list_max_ppm=NEVER)
     t = g.stage_times(reset=True)
     assert t["filter"][1] == 1 and t["scan"][1] == 1
