@@ -55,6 +55,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--chunk-blocks", type=int, default=0, help="scan chunk size in 1024-row blocks (0 = auto)")
+    ap.add_argument("--rerank", type=int, default=0,
+                    help="exact float32 rerank of the R best ADC candidates (loads the raw vectors; 0 = off)")
     ap.add_argument("--list-max-ppm", type=int, default=0,
                     help="sorted-copy scan for one-column pools up to this many rows per million "
                          "(0 = library default: always, -1 = never)")
@@ -235,18 +237,41 @@ def cpu_baseline(w, ix, cond, batches, max_seconds=30.0):
 
 # ------------------------------------------------------------ recall
 
+def _pass_mask(attr_blocks, preds, device):
+    """[nq][n] pass mask of the predicates (every clause, every operator, in
+    int64) on one block of the attribute columns; measurement code for the
+    recall ground truth."""
+    import torch
+    nq = len(preds)
+    n = attr_blocks[0].shape[0]
+    stack = torch.stack(attr_blocks)                          # [n_attrs][n]
+    ok = torch.ones((nq, n), dtype=torch.bool, device=device)
+    nc = torch.from_numpy(preds["n_clauses"].astype(np.int64)).to(device)
+    for j in range(4):
+        cl = preds["c"][:, j]
+        col = torch.from_numpy(np.clip(cl["col"], 0, len(attr_blocks) - 1).astype(np.int64)).to(device)
+        op = torch.from_numpy(cl["op"].astype(np.int64)).to(device)[:, None]
+        lo = torch.from_numpy(cl["lo"].astype(np.int64)).to(device)[:, None]
+        hi = torch.from_numpy(cl["hi"].astype(np.int64)).to(device)[:, None]
+        a = stack[col]                                        # [nq][n]
+        cond = torch.where(op == 0, a == lo,
+               torch.where(op == 1, (a >= lo) & (a < hi),
+               torch.where(op == 2, a >= lo,
+               torch.where(op == 3, a < lo,
+               torch.where(op == 4, a > lo, a <= lo)))))
+        ok &= cond | (nc[:, None] <= j)
+    return ok
+
+
 def exact_topk_gpu(w, ix, q, preds, k, device):
     """Exact filtered top-k (§3.1) over the raw vectors (drawn on the device
-    block by block) for range predicates on attribute 0, in fp64 with torch:
-    ids [nq][k] (-1 padded), outside any timed region."""
+    block by block) in fp64 with torch: ids [nq][k] (-1 padded), outside any
+    timed region."""
     import torch
     from paper_2607_22922_gb300 import synth
     block = 1 << 22
     cb = torch.from_numpy(ix.codebook).to(device)
-    attr = ix.attrs[0]
     qs_all = torch.from_numpy(np.ascontiguousarray(q)).to(device).double()
-    lo_t = torch.from_numpy(np.ascontiguousarray(preds["c"][:, 0]["lo"])).to(device)
-    hi_t = torch.from_numpy(np.ascontiguousarray(preds["c"][:, 0]["hi"])).to(device)
     nq = qs_all.shape[0]
     best_d = torch.full((nq, k), float("inf"), dtype=torch.float64, device=device)
     best_i = torch.full((nq, k), -1, dtype=torch.int64, device=device)
@@ -255,8 +280,8 @@ def exact_topk_gpu(w, ix, q, preds, k, device):
         e = min(w.N, s + block)
         x = synth.raw_vectors_torch(ix, s, e, device, cb).double()
         d = qn + (x * x).sum(1)[None, :] - 2.0 * qs_all @ x.T
-        a = torch.from_numpy(attr[s:e].astype(np.int64)).to(device)
-        ok = (a[None, :] >= lo_t[:, None]) & (a[None, :] < hi_t[:, None])
+        cols = [torch.from_numpy(a[s:e].astype(np.int64)).to(device) for a in ix.attrs]
+        ok = _pass_mask(cols, preds, device)
         d = torch.where(ok, d, torch.full_like(d, float("inf")))
         kk = min(k, e - s)
         dv, di = torch.topk(d, kk, dim=1, largest=False)
@@ -314,7 +339,21 @@ def run_ifvs(args):
     cond = synth.make_conditioning(ix)
     batches = [synth.make_queries(ix, s, nq=w.batch, salt=rank) for s in w.sels]
     t_gen = time.time() - t0
-    g = ifvs.Index(ix.codes, ix.attrs, device=local)
+    if args.rerank > 0:
+        # the raw vectors, drawn on the device block by block, go into the
+        # index for the exact rerank (device I/O load: nothing on the host)
+        cbt = torch.from_numpy(ix.codebook).to(device)
+        vecs = torch.empty((w.N, w.D), dtype=torch.float32, device=device)
+        for s0 in range(0, w.N, 1 << 22):
+            s1 = min(w.N, s0 + (1 << 22))
+            vecs[s0:s1] = synth.raw_vectors_torch(ix, s0, s1, device, cbt)
+        g = ifvs.Index(torch.from_numpy(ix.codes).to(device),
+                       [torch.from_numpy(a).to(device) for a in ix.attrs], vectors=vecs, D=w.D,
+                       device=local, K=w.K, device_io=True)
+        del vecs, cbt
+        torch.cuda.empty_cache()
+    else:
+        g = ifvs.Index(ix.codes, ix.attrs, device=local)
     g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
 
     stream = torch.cuda.Stream(device=device)
@@ -338,7 +377,7 @@ def run_ifvs(args):
         oi, od, on = dev_out[b]
         ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on,
                                flags=flags, stream=sptr, chunk_blocks=args.chunk_blocks,
-                               list_max_ppm=args.list_max_ppm)
+                               list_max_ppm=args.list_max_ppm, rerank=args.rerank)
 
     for i in range(args.warmup):
         step(i)
@@ -428,7 +467,8 @@ def run_ifvs(args):
             q, p, wz, _ = host_in[b]
             oi, od, on, _ = host_out[b]
             ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr,
-                                   chunk_blocks=args.chunk_blocks, list_max_ppm=args.list_max_ppm)
+                                   chunk_blocks=args.chunk_blocks, list_max_ppm=args.list_max_ppm,
+                                   rerank=args.rerank)
 
         for i in range(args.warmup):
             hstep(i)
@@ -448,7 +488,7 @@ def run_ifvs(args):
 
     # recall@k (outside the timed regions)
     recall = None
-    if args.recall_queries > 0 and rank == 0 and not w.conjunctive:
+    if args.recall_queries > 0 and rank == 0:
         ids_by_bin = [dev_out[b][0].cpu().numpy()[:args.recall_queries] for b in range(nb)]
         recall = recall_at_k(w, ix, batches, ids_by_bin, args.recall_queries, device)
         for s, r in recall.items():
@@ -466,6 +506,7 @@ def run_ifvs(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "f32 (uint8 codes)",
         "data": "synthetic (seeded Gaussian-mixture PQ index; paper datasets and trained weights absent)",
         "config": {"workload": w.name, "N": w.N, "D": w.D, "M": w.M, "K": w.K, "k": w.k,
+                   "rerank": args.rerank,
                    "batch": w.batch, "bins": list(w.sels), "B": w.B, "h": w.h, "r": w.r,
                    "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2 (%.1f GB codes + %.1f GB attributes)"
