@@ -235,6 +235,61 @@ def cpu_baseline(w, ix, cond, batches, max_seconds=30.0):
                       "time scaled by N/rows" % (nq, rows, w.N)}
 
 
+def _oracle_worker(args):
+    """One oracle query in a worker process (memory-mapped sample arrays)."""
+    import oracle
+    paths, k, qi = args
+    codes = np.load(paths["codes"], mmap_mode="r")
+    attrs = [np.load(p, mmap_mode="r") for p in paths["attrs"]]
+    arr = {n: np.load(paths[n]) for n in ("codebook", "bank", "W", "seeds", "q", "preds", "wz")}
+    t0 = time.perf_counter()
+    oracle.search(np.asarray(codes), [np.asarray(a) for a in attrs], arr["codebook"], arr["q"][qi:qi + 1],
+                  arr["preds"][qi:qi + 1], k, bank=arr["bank"], W=arr["W"], seeds=arr["seeds"],
+                  wz=arr["wz"][qi:qi + 1])
+    return time.perf_counter() - t0
+
+
+def cpu_baseline_parallel(w, ix, cond, batches, queries_per_core=2):
+    """The same oracle on every host core: a spawn process pool (the GPU is
+    in use in this process) runs one query per task over memory-mapped
+    copies of the first CPU_SAMPLE_ROWS rows; throughput = queries / wall
+    time, scaled by N / rows."""
+    import multiprocessing as mp
+    import shutil
+    import tempfile
+    import oracle
+    oracle.build()
+    cores = os.cpu_count() or 1
+    rows = min(CPU_SAMPLE_ROWS, w.N)
+    d = tempfile.mkdtemp(prefix="ifvs_cpu_")
+    try:
+        paths = {"codes": os.path.join(d, "codes.npy"), "attrs": []}
+        np.save(paths["codes"], ix.codes[:rows])
+        for i, a in enumerate(ix.attrs):
+            pa = os.path.join(d, "attr%d.npy" % i)
+            np.save(pa, a[:rows])
+            paths["attrs"].append(pa)
+        nq = cores * queries_per_core
+        pick = [(b, j) for j in range(nq) for b in range(len(batches))][:nq]
+        q = np.stack([batches[b].q[j % len(batches[b].q)] for b, j in pick])
+        pr = np.stack([batches[b].preds[j % len(batches[b].q)] for b, j in pick])
+        wz = np.stack([batches[b].wz[j % len(batches[b].q)] for b, j in pick])
+        for n, v in (("codebook", ix.codebook), ("bank", cond.bank), ("W", cond.W), ("seeds", cond.seeds),
+                     ("q", q), ("preds", pr), ("wz", wz)):
+            paths[n] = os.path.join(d, n + ".npy")
+            np.save(paths[n], v)
+        with mp.get_context("spawn").Pool(cores) as pool:
+            pool.map(_oracle_worker, [(paths, w.k, 0)] * cores)          # warm: load the library
+            t0 = time.perf_counter()
+            pool.map(_oracle_worker, [(paths, w.k, i) for i in range(nq)])
+            wall = time.perf_counter() - t0
+    finally:
+        shutil.rmtree(d, ignore_errors=True)
+    return {"value": nq / (wall * (w.N / rows)), "unit": "queries/s", "cores": cores, "kind": "oracle",
+            "sample": "%d queries cycling through the bins, %d worker processes, over the first %d of %d "
+                      "rows; wall time scaled by N/rows" % (nq, cores, rows, w.N)}
+
+
 # ------------------------------------------------------------ recall
 
 def _pass_mask(attr_blocks, preds, device):
@@ -494,9 +549,10 @@ def run_ifvs(args):
         for s, r in recall.items():
             per_bin[str(s)]["recall@%d" % w.k] = r
 
-    cpu = None
+    cpu = cpu_par = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, ix, cond, batches)
+        cpu_par = cpu_baseline_parallel(w, ix, cond, batches)
 
     value = whole_job_qps(world, args.steps, w.batch, max_ms)
     line = {
@@ -512,7 +568,8 @@ def run_ifvs(args):
                    "l2": "inputs larger than L2 (%.1f GB codes + %.1f GB attributes)"
                          % (w.N * w.M / 1e9, w.N * 4 / 1e9)},
         "bins": per_bin, "roofline": roofline, "stage_ms": share, "gpu_launches": launches,
-        "clocks": clk, "e2e": e2e, "cpu_baseline": cpu, "setup_s": round(t_gen, 1),
+        "clocks": clk, "e2e": e2e, "cpu_baseline": cpu, "cpu_baseline_parallel": cpu_par,
+        "setup_s": round(t_gen, 1),
     }
     if rank == 0:
         s = json.dumps(line)
