@@ -105,8 +105,7 @@ typedef struct {
                            range of the codes sorted by that column: no
                            filter pass, no bitmap) when the pool holds at most
                            this many rows per million of N.  0: default
-                           (always for M = 16; 20000, i.e. 2 %, for other M);
-                           -1: never.  The two paths sum a row's entries in
+                           (1000000: always); -1: never.  The two paths sum a row's entries in
                            different orders, so distances agree to float32
                            rounding.                                          */
     void* stream;       /* cudaStream_t to run on; NULL: the index's stream   */

@@ -310,12 +310,11 @@ struct Opts {
     cudaStream_t stream = nullptr;
 };
 
-// one-column predicates take the sorted-copy scan at any pool size for
-// M = 16 (lockstep, 16-byte code rows), and up to 2 % of the rows for other
-// M, where the bitmap path's generic loop wins on wide pools (measured on
-// 10^6 x 120 codes), unless the caller sets a threshold
+// one-column predicates take the sorted-copy scan at any pool size unless
+// the caller sets a threshold: it read fewer bytes and ran faster than the
+// bitmap path in every measured selectivity bin, for M = 16 and for the
+// generic-M loop (10^6 x 120 codes)
 constexpr int32_t kListDefaultPpm = 1000000;
-constexpr int32_t kListDefaultPpmAnyM = 20000;
 
 int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (!p) return 0;
@@ -407,11 +406,10 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
         CUDA_TRY(st.end(launch_canonicalize(dp, n, ix->cols(), ix->w_canon.as<CanonPred>(),
                                             ix->w_err.as<int>(), s)));
     }
-    // one-column predicates with small pools take the row-list scan
+    // one-column predicates take the sorted-copy scan (up to the threshold)
     const ScanPlan* plan = nullptr;
     if (o.list_max_ppm >= 0 && ix->n_attrs > 0) {
-        const bool m16 = ix->M == 16 && ix->row_bytes == 16 && ix->tab_words == 64;
-        const int64_t ppm = o.list_max_ppm > 0 ? o.list_max_ppm : (m16 ? kListDefaultPpm : kListDefaultPpmAnyM);
+        const int64_t ppm = o.list_max_ppm > 0 ? o.list_max_ppm : kListDefaultPpm;
         const int64_t max_rows = ppm >= 1000000 ? ix->N : ix->N * ppm / 1000000;
         TRY(ensure(ix->w_plan, sizeof(ScanPlan) * n));
         Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);

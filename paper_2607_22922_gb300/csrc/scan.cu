@@ -233,6 +233,44 @@ __device__ __forceinline__ float lookup_any(const uint8_t* rp, bool pass, int M,
     return acc;
 }
 
+// Distances of NU rows for any M, all owned by one lane (so they share the
+// table word offset w0 = the lane): the rows' code words are read together
+// and their look-ups go into NU/2 packed f32x2 chains, independent of each
+// other; each row's entries are still added for s ascending, as in
+// lookup_any.  Rows whose bit in `valid` is clear read no codes.
+template <int NU>
+__device__ __forceinline__ void lookup_rows(const uint8_t* __restrict__ codes, const uint32_t (&idx)[NU],
+                                            unsigned valid, int row_bytes, int M, int S, const float* tab,
+                                            int w0, float (&d)[NU]) {
+    static_assert(NU % 2 == 0, "rows in pairs");
+    uint64_t acc[NU / 2];
+#pragma unroll
+    for (int u = 0; u < NU / 2; ++u) acc[u] = 0ull;
+    const float* tw = tab + w0;
+    for (int w = 0; w * 4 < M; ++w) {
+        uint32_t wd[NU];
+#pragma unroll
+        for (int u = 0; u < NU; ++u)
+            wd[u] = (valid >> u & 1u)
+                        ? __ldg(reinterpret_cast<const uint32_t*>(codes + (size_t)idx[u] * row_bytes) + w)
+                        : 0u;
+#pragma unroll
+        for (int bb = 0; bb < 4; ++bb) {
+            const int s = 4 * w + bb;
+            if (s < M) {
+#pragma unroll
+                for (int u = 0; u < NU; u += 2) {
+                    const float va = tw[(int)((wd[u] >> (8 * bb)) & 0xFFu) * S + s];
+                    const float vb = tw[(int)((wd[u + 1] >> (8 * bb)) & 0xFFu) * S + s];
+                    acc[u / 2] = add_f32x2(acc[u / 2], va, vb);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < NU; u += 2) unpack_f32x2(acc[u / 2], d[u], d[u + 1]);
+}
+
 template <int KP, bool M16, bool FAST>
 __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                                            const uint32_t* __restrict__ bmq, const ScanShape& sh,
@@ -310,10 +348,11 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                         for (int u = 0; u < kU; ++u) tk.offer(key[u], key[u] < tk.thr, lane);
                     }
                 } else {
+                    float d[kU];
+                    lookup_rows<kU>(codes, row, (1u << kU) - 1u, row_bytes, M, S, tab, lane, d);
 #pragma unroll
                     for (int u = 0; u < kU; ++u) {
-                        const float d = lookup_any(codes + (size_t)row[u] * row_bytes, true, M, S, tab, lane);
-                        const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | row[u];
+                        const uint64_t key = ((uint64_t)__float_as_uint(d[u]) << 32) | row[u];
                         tk.offer(key, key < tk.thr, lane);
                     }
                 }
@@ -362,11 +401,12 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                 for (int u = 0; u < kU; ++u) tk.offer(key[u], (valid >> u & 1u) && key[u] < tk.thr, lane);
             }
         } else {
+            float d[kU];
+            lookup_rows<kU>(codes, row, valid, row_bytes, M, S, tab, lane, d);
 #pragma unroll
             for (int u = 0; u < kU; ++u) {
                 const bool pass = valid >> u & 1u;
-                const float d = lookup_any(codes + (size_t)row[u] * row_bytes, pass, M, S, tab, lane);
-                const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | row[u];
+                const uint64_t key = ((uint64_t)__float_as_uint(d[u]) << 32) | row[u];
                 tk.offer(key, pass && key < tk.thr, lane);
             }
         }
@@ -528,10 +568,7 @@ __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes
 #pragma unroll
                 for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
             } else {
-                // unrolled, so that pos[] and d[] stay in registers
-#pragma unroll
-                for (int u = 0; u < kU; ++u)
-                    d[u] = lookup_any(codes + (size_t)pos[u] * sh.row_bytes, valid >> u & 1u, M, S, tab, lane);
+                lookup_rows<kU>(codes, pos, valid, sh.row_bytes, M, S, tab, lane, d);
             }
             // a position can enter the top-k only if its distance is at most
             // the current k-th one; only those load their row id

@@ -120,15 +120,18 @@ def test_list_path_and_bitmap_path(ifvs, orc, N, k):
         _check_oracle(orc, codes, attrs, Cpq, q, p, k, *b)
 
 
-@pytest.mark.parametrize("M", [1, 8, 12, 24])
+@pytest.mark.parametrize("M", [1, 8, 12, 24, 120])
 def test_list_path_other_subspace_counts(ifvs, orc, M):
     g, codes, attrs, Cpq = _index(ifvs, 20000, M=M, K=64, ds=3, seed=M)
     p = _preds()
     q = _queries(len(p), M * 3, seed=M)
     a = g.search(q, p, 20, list_max_ppm=ALWAYS)
     b = g.search(q, p, 20, list_max_ppm=NEVER)
+    for x, z in zip(a, g.search(q, p, 20)):    # the default, for every M: the sorted copy
+        np.testing.assert_array_equal(x, z)
     _same_up_to_rounding(a, b)
     _check_oracle(orc, codes, attrs, Cpq, q, p, 20, *a)
+    _check_oracle(orc, codes, attrs, Cpq, q, p, 20, *b)
 
 
 @pytest.mark.parametrize("k", [10, 100])
