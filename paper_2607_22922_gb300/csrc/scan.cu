@@ -40,6 +40,8 @@
 // The tile constants (warps per CTA, ring depth, rows per round) were chosen
 // by measurement on the 10^8-row workload; the macros below only exist to
 // rebuild variants for such sweeps.
+#include <climits>
+
 #include "internal.cuh"
 
 namespace ifvs {
@@ -603,16 +605,6 @@ __device__ __forceinline__ bool pair_ok(const ScanPlan& x, const ScanPlan& y, in
     return 4 * lx >= 3 * N && 4 * ly >= 3 * N && longer > 0 && 4 * common >= 3 * longer;
 }
 
-// the single-query loop for M = 16 (FAST: table at the dynamic shared base)
-template <int KP, bool FAST>
-__device__ __forceinline__ void scan_positions_range(const uint8_t* __restrict__ codes,
-                                                     const uint32_t* __restrict__ rows, int64_t a, int64_t b,
-                                                     int64_t blk0, int64_t blk1, int wstride,
-                                                     const ScanShape& sh, const float* tab, WarpTopK<KP>& tk,
-                                                     int lane, int warp) {
-    scan_positions<KP, true, FAST>(codes, rows, a, b, blk0, blk1, wstride, sh, tab, tk, lane, warp);
-}
-
 template <int KP, bool M16, int MINB>
 __global__ void __launch_bounds__(kScanThreads, MINB)
 k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
@@ -676,114 +668,220 @@ k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __r
 // ---- two queries per CTA on the sorted copy --------------------------------
 //
 // When two consecutive queries both take the sorted copy of the same column
-// (M = 16), one CTA serves both: their tables sit back to back in shared
-// memory (B 64 KB after A, so both keep the immediate-offset addressing) and
-// each 16-byte code load and byte permute feeds a look-up in each table.
-// Blocks that meet only one query's range (and pairs that cannot share) run
-// the single-query loop.  16 warps, one CTA per SM.
+// (M = 16), one CTA serves both, and one shared-memory load serves both
+// queries' look-ups.  A 64 KB table with the rows, replication and rotation
+// of the float32 one holds, in word w of codeword row c, the pair
+// qA[w mod 16][c] | qB[w mod 16][c] << 16 of 11-bit quantised entries,
+// q[m][c] = floor((LUT[m][c] - lo_m) * inv), lo_m the smallest entry of
+// subspace m, inv = 2047 / (the widest subspace's range).  Sixteen entries
+// sum to at most 32752, so one integer add accumulates both queries with no
+// carry between the halves (and bit 15 of each half stays free for the
+// candidate test, pack_bounds), and a row's sum S bounds its float32 distance
+// from below (quant_bound).  A row whose S exceeds the bound of its query's
+// current k-th key cannot enter that top-k and is dropped; every other row
+// gets its exact float32 distance from the query's unreplicated table,
+// added in the order of the one-query loop (subspace (p mod 32) mod 16
+// first), so the top-k receives the keys the one-query loop would give it.
+// Since the dropped rows are decided by integers, the shared-memory traffic
+// of the dense loop is half that of two float32 tables.  Blocks that meet
+// one query's range only run the same loop with the other query masked.
+// 16 warps, one CTA per SM.
 constexpr int kPairWarps = 16;
 constexpr int kPairThreads = kPairWarps * 32;
-constexpr uint32_t kTabBytes16 = 256u * 64u * 4u;   // one M = 16 table
+constexpr uint32_t kTabBytes16 = 256u * 64u * 4u;    // one replicated M = 16 table
+constexpr uint32_t kExactBytes16 = 256u * 16u * 4u;  // one unreplicated table, [c][m]
+constexpr int kQMax = 2047;                           // 16 * 2047 < 2^15
 
-size_t scan_pair_smem_bytes(int kp) { return (size_t)2 * kTabBytes16 + (size_t)kPairWarps * 2 * 2 * kp * 8; }
+size_t scan_pair_smem_bytes(int kp) {
+    return (size_t)kTabBytes16 + 2 * (size_t)kExactBytes16 + 64 * 4 + (size_t)kPairWarps * 2 * 2 * kp * 8;
+}
 
-// Four distances: rows a, b (codes ca, cb) in tables A (at the dynamic
-// shared base) and B (kTabBytes16 above it).
-__device__ __forceinline__ void lookup16x2x2(const uint4 ca, const uint4 cb, uint32_t tb, float& aa,
-                                             float& ab, float& ba, float& bb) {
+template <int IMM>
+__device__ __forceinline__ uint32_t lds_u32_imm(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1+%2];" : "=r"(v) : "r"(addr), "n"(IMM));
+    return v;
+}
+
+__device__ __forceinline__ uint32_t quant12(float L, float lo, float inv) {
+    const float y = __fmul_rn(__fsub_rn(L, lo), inv);
+    return (uint32_t)fminf((float)kQMax, fmaxf(0.f, y));   // truncation: floor of y >= 0
+}
+
+// The largest quantised sum S a row can have and still reach a top-k whose
+// k-th key is thr (INT_MAX: every row; -1: none).  With u = 2^-24 and
+// entries L >= 0 (so lo_m >= 0): the float32 distance d, sixteen rounded
+// additions from 0, is at least (sum_m L_m)(1 - 15u); each q_m is at most
+// (L_m - lo_m)(1 + u)^2 inv (two roundings, then floor); so
+// S <= (1 + u)^2 inv (d / (1 - 15u) - sum_m lo_m).  At d = dist(thr) the
+// bound below is at least that: each of its float32 steps carries a factor
+// 1 +- 2^-12 beyond its rounding, and sl, the float32 sum of the lo_m, is at
+// most (1 + 15u) sum_m lo_m.  A row with S above it has d > dist(thr).
+__device__ __forceinline__ int quant_bound(uint64_t thr, float sl, float inv) {
+    const uint32_t hi = (uint32_t)(thr >> 32);
+    if (inv == 0.f || hi >= 0x7F800000u) return INT_MAX;   // list not full, inf, NaN or -0
+    const float a = __fmul_rn(__uint_as_float(hi), 1.f + 0x1p-12f);
+    const float b = __fmul_rn(sl, 1.f - 0x1p-12f);
+    const float t = __fmul_rn(__fsub_rn(a, b), __fmul_rn(inv, 1.f + 0x1p-12f));
+    if (!(t < 1.0e9f)) return INT_MAX;
+    return t < 0.f ? -1 : (int)t;
+}
+
+// Quantised sums of two M = 16 rows (codes ca, cb), both queries at once:
+// the addresses of lookup16x2, integer loads, and the sums as multiply-adds
+// by `one` (= 1, unknown to the compiler), which run on the FMA pipe beside
+// the byte permutes on the integer pipe.
+template <bool FAST>
+__device__ __forceinline__ void lookup16x2_q(const uint4 ca, const uint4 cb, uint32_t tb, uint32_t base,
+                                             uint32_t one, uint32_t& sa, uint32_t& sb) {
     const uint32_t wa[4] = {ca.x, ca.y, ca.z, ca.w};
     const uint32_t wb[4] = {cb.x, cb.y, cb.z, cb.w};
-    uint64_t accA = 0ull, accB = 0ull;
+    uint32_t xa = 0u, xb = 0u;
 #pragma unroll
     for (int s = 0; s < 16; ++s) {
         const uint32_t sel = 0x5504u | ((uint32_t)(s & 3) << 4);
-        const uint32_t oa = __byte_perm(wa[s >> 2], tb, sel);
-        const uint32_t ob = __byte_perm(wb[s >> 2], tb, sel);
-        float va, vb, wa2, wb2;
-        switch (s) {
-#define IFVS_LDS2_CASE(S)                                          \
-    case S:                                                        \
-        va = lds_imm<kDynSmemBase + 4 * S>(oa);                    \
-        vb = lds_imm<kDynSmemBase + 4 * S>(ob);                    \
-        wa2 = lds_imm<kDynSmemBase + kTabBytes16 + 4 * S>(oa);     \
-        wb2 = lds_imm<kDynSmemBase + kTabBytes16 + 4 * S>(ob);     \
-        break;
-            IFVS_LDS2_CASE(0) IFVS_LDS2_CASE(1) IFVS_LDS2_CASE(2) IFVS_LDS2_CASE(3)
-            IFVS_LDS2_CASE(4) IFVS_LDS2_CASE(5) IFVS_LDS2_CASE(6) IFVS_LDS2_CASE(7)
-            IFVS_LDS2_CASE(8) IFVS_LDS2_CASE(9) IFVS_LDS2_CASE(10) IFVS_LDS2_CASE(11)
-            IFVS_LDS2_CASE(12) IFVS_LDS2_CASE(13) IFVS_LDS2_CASE(14) IFVS_LDS2_CASE(15)
-#undef IFVS_LDS2_CASE
-            default: va = vb = wa2 = wb2 = 0.f; break;
+        uint32_t oa = __byte_perm(wa[s >> 2], tb, sel);
+        uint32_t ob = __byte_perm(wb[s >> 2], tb, sel);
+        if (!FAST) {
+            oa += base;
+            ob += base;
         }
-        accA = add_f32x2(accA, va, vb);
-        accB = add_f32x2(accB, wa2, wb2);
+        constexpr uint32_t B0 = FAST ? kDynSmemBase : 0u;
+        uint32_t va, vb;
+        switch (s) {
+#define IFVS_LDQ_CASE(S)                      \
+    case S:                                   \
+        va = lds_u32_imm<B0 + 4 * S>(oa);     \
+        vb = lds_u32_imm<B0 + 4 * S>(ob);     \
+        break;
+            IFVS_LDQ_CASE(0) IFVS_LDQ_CASE(1) IFVS_LDQ_CASE(2) IFVS_LDQ_CASE(3)
+            IFVS_LDQ_CASE(4) IFVS_LDQ_CASE(5) IFVS_LDQ_CASE(6) IFVS_LDQ_CASE(7)
+            IFVS_LDQ_CASE(8) IFVS_LDQ_CASE(9) IFVS_LDQ_CASE(10) IFVS_LDQ_CASE(11)
+            IFVS_LDQ_CASE(12) IFVS_LDQ_CASE(13) IFVS_LDQ_CASE(14) IFVS_LDQ_CASE(15)
+#undef IFVS_LDQ_CASE
+            default: va = vb = 0u; break;
+        }
+        xa = va * one + xa;
+        xb = vb * one + xb;
     }
-    unpack_f32x2(accA, aa, ab);
-    unpack_f32x2(accB, ba, bb);
+    sa = xa;
+    sb = xb;
 }
+
+// Exact float32 distance of one M = 16 row of the sorted copy from an
+// unreplicated table ex[c * 16 + m]: byte s holds subspace (s + rot) mod 16,
+// rot = (p mod 32) mod 16, added for s ascending from 0, as lookup16x2 does.
+__device__ __forceinline__ float exact16(const uint4 c, const float* ex, int rot) {
+    const uint32_t w[4] = {c.x, c.y, c.z, c.w};
+    float d = 0.f;
+#pragma unroll
+    for (int s = 0; s < 16; ++s) {
+        const uint32_t code = (w[s >> 2] >> (8 * (s & 3))) & 0xFFu;
+        d = __fadd_rn(d, ex[code * 16u + (uint32_t)((s + rot) & 15)]);
+    }
+    return d;
+}
+
+// Both queries' bounds in one word: half h holds bound_h + 0x8000, bound_h
+// clamped to [-1, 0x7FFF].  A row's packed sums (each half <= 16 * 2047 <
+// 0x8000) are candidates where (packed bounds - sums) keeps bit 15 (query A)
+// or bit 31 (query B): no borrow crosses the halves.
+__device__ __forceinline__ uint32_t pack_bounds(int ta, int tb) {
+    ta = ta > 0x7FFF ? 0x7FFF : ta;
+    tb = tb > 0x7FFF ? 0x7FFF : tb;
+    return (uint32_t)(ta + 0x8000) | (uint32_t)(tb + 0x8000) << 16;
+}
+
+constexpr uint32_t kCandA = 0x00008000u, kCandB = 0x80000000u;
 
 // kU2 rows per lane per round in the paired loop
 constexpr int kU2 = 4;
 
-template <int KP>
+// One round of kU2 positions of a block: quantised sums of both queries,
+// candidates by the packed bounds, exact distances and top-k offers for the
+// candidates.  MASKED: the block is cut by one of the ranges (mask[] holds
+// kCandA / kCandB for the positions inside each query's range).
+template <int KP, bool FAST, bool MASKED>
+__device__ __forceinline__ void pair_round(const uint8_t* __restrict__ codes, const uint32_t* __restrict__ rows,
+                                           uint32_t pos0, const uint32_t (&mask)[kU2], WarpTopK<KP>& tkA,
+                                           WarpTopK<KP>& tkB, const float* exA, const float* exB, float slA,
+                                           float invA, float slB, float invB, uint32_t tb, uint32_t base,
+                                           uint32_t one, int rot, uint64_t keep, int lane, uint32_t& Tpk) {
+    uint4 c[kU2];
+#pragma unroll
+    for (int u = 0; u < kU2; ++u) {
+        const uint32_t pos = pos0 + 32u * (uint32_t)u;
+        c[u] = (!MASKED || mask[u] != 0u) ? ldg_nc_v4(codes + (size_t)pos * 16, keep) : make_uint4(0, 0, 0, 0);
+    }
+    uint32_t sq[kU2];
+#pragma unroll
+    for (int u = 0; u < kU2; u += 2) lookup16x2_q<FAST>(c[u], c[u + 1], tb, base, one, sq[u], sq[u + 1]);
+    uint32_t cb[kU2], any = 0u;
+#pragma unroll
+    for (int u = 0; u < kU2; ++u) {
+        cb[u] = (Tpk - sq[u]) & (MASKED ? mask[u] : (kCandA | kCandB));
+        any |= cb[u];
+    }
+    if (!__any_sync(0xFFFFFFFFu, any != 0u)) return;
+#pragma unroll
+    for (int u = 0; u < kU2; ++u) {
+        const uint32_t pos = pos0 + 32u * (uint32_t)u;
+        bool cA = (cb[u] & kCandA) != 0u;
+        bool cB = (cb[u] & kCandB) != 0u;
+        float dA = 0.f, dB = 0.f;
+        if (cA) dA = exact16(c[u], exA, rot);
+        if (cB) dB = exact16(c[u], exB, rot);
+        cA = cA && __float_as_uint(dA) <= (uint32_t)(tkA.thr >> 32);
+        cB = cB && __float_as_uint(dB) <= (uint32_t)(tkB.thr >> 32);
+        const uint32_t row = (cA || cB) ? __ldg(rows + pos) : 0u;
+        const uint64_t kA = ((uint64_t)__float_as_uint(dA) << 32) | row;
+        const uint64_t kB = ((uint64_t)__float_as_uint(dB) << 32) | row;
+        tkA.offer(kA, cA && kA < tkA.thr, lane);
+        tkB.offer(kB, cB && kB < tkB.thr, lane);
+    }
+    Tpk = pack_bounds(quant_bound(tkA.thr, slA, invA), quant_bound(tkB.thr, slB, invB));
+}
+
+template <int KP, bool FAST>
 __device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ codes,
                                                     const uint32_t* __restrict__ rows, int64_t aA,
                                                     int64_t bA, int64_t aB, int64_t bB, int64_t blk0,
                                                     int64_t blk1, WarpTopK<KP>& tkA, WarpTopK<KP>& tkB,
-                                                    const float* tabA, const float* tabB,
-                                                    const ScanShape& sh, int lane, int warp) {
+                                                    const float* exA, const float* exB, float slA, float invA,
+                                                    float slB, float invB, uint32_t base, uint32_t one,
+                                                    int lane, int warp) {
     const uint32_t tb = 4u * (uint32_t)lane;
+    const int rot = lane & 15;
     const uint64_t keep = policy_evict_last();
     const uint32_t a1 = (uint32_t)aA, b1 = (uint32_t)bA, a2 = (uint32_t)aB, b2 = (uint32_t)bB;
+    uint32_t Tpk = pack_bounds(quant_bound(tkA.thr, slA, invA), quant_bound(tkB.thr, slB, invB));
     for (int64_t blk = blk0 + warp; blk < blk1; blk += kPairWarps) {
         const uint32_t p0 = (uint32_t)(blk * kBlockRows);
         const uint32_t pe = p0 + kBlockRows;
         const bool inA = p0 < b1 && pe > a1, inB = p0 < b2 && pe > a2;
-        if (!(inA && inB)) {
-            // one query only: the single-query loop on this block (table A
-            // is at the shared base; table B takes the base-add form)
-            if (inA)
-                scan_positions_range<KP, true>(codes, rows, aA, bA, blk, blk + 1, 1, sh, tabA, tkA, lane, 0);
-            else if (inB)
-                scan_positions_range<KP, false>(codes, rows, aB, bB, blk, blk + 1, 1, sh, tabB, tkB, lane, 0);
+        if (!(inA || inB)) continue;
+        const bool fullA = inA && p0 >= a1 && pe <= b1, fullB = inB && p0 >= a2 && pe <= b2;
+        if (fullA && fullB) {
+            const uint32_t none[kU2] = {};
+#pragma unroll 1
+            for (int j0 = 0; j0 < 32; j0 += kU2)
+                pair_round<KP, FAST, false>(codes, rows, p0 + 32u * (uint32_t)j0 + (uint32_t)lane, none, tkA,
+                                            tkB, exA, exB, slA, invA, slB, invB, tb, base, one, rot, keep, lane,
+                                            Tpk);
             continue;
         }
-        const bool fullA = p0 >= a1 && pe <= b1, fullB = p0 >= a2 && pe <= b2;
 #pragma unroll 1
         for (int j0 = 0; j0 < 32; j0 += kU2) {
-            uint32_t pos[kU2];
-            unsigned vA = 0u, vB = 0u;
+            const uint32_t pos0 = p0 + 32u * (uint32_t)j0 + (uint32_t)lane;
+            uint32_t mask[kU2];
 #pragma unroll
             for (int u = 0; u < kU2; ++u) {
-                pos[u] = p0 + 32u * (uint32_t)(j0 + u) + (uint32_t)lane;
-                vA |= (unsigned)(fullA || (pos[u] >= a1 && pos[u] < b1)) << u;
-                vB |= (unsigned)(fullB || (pos[u] >= a2 && pos[u] < b2)) << u;
+                const uint32_t pos = pos0 + 32u * (uint32_t)u;
+                mask[u] = ((fullA || (inA && pos >= a1 && pos < b1)) ? kCandA : 0u) |
+                          ((fullB || (inB && pos >= a2 && pos < b2)) ? kCandB : 0u);
             }
-            const unsigned v = vA | vB;
-            uint4 c[kU2];
-#pragma unroll
-            for (int u = 0; u < kU2; ++u)
-                c[u] = (v >> u & 1u) ? ldg_nc_v4(codes + (size_t)pos[u] * 16, keep) : make_uint4(0, 0, 0, 0);
-            float dA[kU2], dB[kU2];
-#pragma unroll
-            for (int u = 0; u < kU2; u += 2) lookup16x2x2(c[u], c[u + 1], tb, dA[u], dA[u + 1], dB[u], dB[u + 1]);
-            const uint32_t hA = (uint32_t)(tkA.thr >> 32), hB = (uint32_t)(tkB.thr >> 32);
-            bool any = false;
-#pragma unroll
-            for (int u = 0; u < kU2; ++u)
-                any |= ((vA >> u & 1u) && __float_as_uint(dA[u]) <= hA) ||
-                       ((vB >> u & 1u) && __float_as_uint(dB[u]) <= hB);
-            if (!__any_sync(0xFFFFFFFFu, any)) continue;
-#pragma unroll
-            for (int u = 0; u < kU2; ++u) {
-                const bool cA = (vA >> u & 1u) && __float_as_uint(dA[u]) <= hA;
-                const bool cB = (vB >> u & 1u) && __float_as_uint(dB[u]) <= hB;
-                const uint32_t row = (cA || cB) ? __ldg(rows + pos[u]) : 0u;
-                const uint64_t kA = ((uint64_t)__float_as_uint(dA[u]) << 32) | row;
-                const uint64_t kB = ((uint64_t)__float_as_uint(dB[u]) << 32) | row;
-                tkA.offer(kA, cA && kA < tkA.thr, lane);
-                tkB.offer(kB, cB && kB < tkB.thr, lane);
-            }
+            pair_round<KP, FAST, true>(codes, rows, pos0, mask, tkA, tkB, exA, exB, slA, invA, slB, invB, tb,
+                                       base, one, rot, keep, lane, Tpk);
         }
     }
 }
@@ -807,15 +905,34 @@ __device__ __forceinline__ void merge_warps(WarpTopK<KP>& tk, uint64_t* tkbuf, i
         for (int i = lane; i < k; i += 32) out[i] = tk.buf[i];
 }
 
+// Quantisation parameters of one query from the per-subspace extremes
+// lo[16], hi[16]: inv (0 turns the test off: every row is rescored) and sl.
+__device__ __forceinline__ void quant_params(const float* lo, const float* hi, float& inv, float& sl) {
+    float r = 0.f, s = 0.f;
+    bool ok = true;
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {
+        r = fmaxf(r, __fsub_rn(hi[m], lo[m]));
+        s = __fadd_rn(s, lo[m]);
+        ok = ok && lo[m] >= 0.f;
+    }
+    inv = __fdiv_rn((float)kQMax, r);
+    if (!(ok && r > 0.f && isfinite(inv) && isfinite(s))) inv = 0.f;
+    sl = s;
+}
+
 template <int KP>
 __global__ void __launch_bounds__(kPairThreads, 1)
 k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan,
                  int64_t nq, int k, ScanShape sh, uint64_t* __restrict__ partials) {
     extern __shared__ __align__(256) uint8_t smem[];
-    float* tabA = reinterpret_cast<float*>(smem);
-    float* tabB = reinterpret_cast<float*>(smem + kTabBytes16);
-    uint64_t* tkbufA = reinterpret_cast<uint64_t*>(smem + 2 * kTabBytes16);
+    uint32_t* ptab = reinterpret_cast<uint32_t*>(smem);
+    float* exA = reinterpret_cast<float*>(smem + kTabBytes16);
+    float* exB = reinterpret_cast<float*>(smem + kTabBytes16 + kExactBytes16);
+    float* prm = reinterpret_cast<float*>(smem + kTabBytes16 + 2 * kExactBytes16);   // lo/hi of A, lo/hi of B
+    uint64_t* tkbufA = reinterpret_cast<uint64_t*>(smem + kTabBytes16 + 2 * kExactBytes16 + 64 * 4);
     uint64_t* tkbufB = tkbufA + kPairWarps * 2 * KP;
+    float* red = reinterpret_cast<float*>(tkbufA);   // [warp][4][16], before the lists are set up
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t qA = 2 * (int64_t)blockIdx.x, qB = qA + 1;
     const bool hasB = qB < nq;
@@ -829,48 +946,81 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     auto range = [&](const ScanPlan& p, int64_t& lo, int64_t& hi) {
         lo = max(c0, p.a / kBlockRows);
         hi = min(c1, (p.b + kBlockRows - 1) / kBlockRows);
-        if (!p.list || p.a >= p.b || lo >= hi) lo = hi = 0;
+        if (p.a >= p.b || lo >= hi) lo = hi = 0;
     };
     int64_t lA, hA, lB, hB;
     range(pA, lA, hA);
     range(pB, lB, hB);
-    uint64_t* outA = pA.list ? partials + (qA * sh.n_chunks + chunk) * (int64_t)k : nullptr;
-    uint64_t* outB = pB.list ? partials + (qB * sh.n_chunks + chunk) * (int64_t)k : nullptr;
+    uint64_t* outA = partials + (qA * sh.n_chunks + chunk) * (int64_t)k;
+    uint64_t* outB = partials + (qB * sh.n_chunks + chunk) * (int64_t)k;
     if (lA == hA && lB == hB) {
         for (int i = threadIdx.x; i < k; i += kPairThreads) {
-            if (outA) outA[i] = ~0ull;
-            if (outB) outB[i] = ~0ull;
+            outA[i] = ~0ull;
+            outB[i] = ~0ull;
         }
         return;
     }
+    // 1) unreplicated float32 tables ex[c * 16 + m] (from the replicated
+    //    tables of k_tables: word m < 16 of row c is LUT[m][c]) and the
+    //    extremes of each subspace; a thread keeps one subspace m
     {
-        const float4* srcA = reinterpret_cast<const float4*>(tables + qA * (int64_t)256 * 64);
-        float4* dstA = reinterpret_cast<float4*>(tabA);
-        for (int i = threadIdx.x; i < 64 * 64; i += kPairThreads) dstA[i] = __ldg(srcA + i);
-        if (pB.list) {
-            const float4* srcB = reinterpret_cast<const float4*>(tables + qB * (int64_t)256 * 64);
-            float4* dstB = reinterpret_cast<float4*>(tabB);
-            for (int i = threadIdx.x; i < 64 * 64; i += kPairThreads) dstB[i] = __ldg(srcB + i);
+        const float* srcA = tables + qA * (int64_t)256 * 64;
+        const float* srcB = tables + qB * (int64_t)256 * 64;
+        const int m = threadIdx.x & 15;
+        float loA = INFINITY, hiA = -INFINITY, loB = INFINITY, hiB = -INFINITY;
+        for (int i = threadIdx.x; i < 4096; i += kPairThreads) {
+            const int c = i >> 4;
+            const float x = __ldg(srcA + c * 64 + m), y = __ldg(srcB + c * 64 + m);
+            exA[i] = x;
+            exB[i] = y;
+            loA = fminf(loA, x);
+            hiA = fmaxf(hiA, x);
+            loB = fminf(loB, y);
+            hiB = fmaxf(hiB, y);
+        }
+        loA = fminf(loA, __shfl_xor_sync(0xFFFFFFFFu, loA, 16));
+        hiA = fmaxf(hiA, __shfl_xor_sync(0xFFFFFFFFu, hiA, 16));
+        loB = fminf(loB, __shfl_xor_sync(0xFFFFFFFFu, loB, 16));
+        hiB = fmaxf(hiB, __shfl_xor_sync(0xFFFFFFFFu, hiB, 16));
+        if (lane < 16) {
+            red[warp * 64 + m] = loA;
+            red[warp * 64 + 16 + m] = hiA;
+            red[warp * 64 + 32 + m] = loB;
+            red[warp * 64 + 48 + m] = hiB;
         }
     }
+    __syncthreads();
+    if (threadIdx.x < 64) {
+        const int j = threadIdx.x;   // 0-15 lo A, 16-31 hi A, 32-47 lo B, 48-63 hi B
+        const bool is_lo = (j & 16) == 0;
+        float v = red[j];
+        for (int w = 1; w < kPairWarps; ++w) v = is_lo ? fminf(v, red[w * 64 + j]) : fmaxf(v, red[w * 64 + j]);
+        prm[j] = v;
+    }
+    __syncthreads();
+    float invA, slA, invB, slB;
+    quant_params(prm, prm + 16, invA, slA);
+    quant_params(prm + 32, prm + 48, invB, slB);
+    // 2) the packed table: word w of row c = qA[w mod 16][c] | qB[..] << 16
+    for (int i = threadIdx.x; i < 256 * 64; i += kPairThreads) {
+        const int c = i >> 6, m = i & 15;
+        ptab[i] = quant12(exA[c * 16 + m], prm[m], invA) | quant12(exB[c * 16 + m], prm[32 + m], invB) << 16;
+    }
+    __syncthreads();   // the reduction scratch becomes the lists
     WarpTopK<KP> tkA, tkB;
     tkA.init(tkbufA + warp * 2 * KP, k, lane);
     tkB.init(tkbufB + warp * 2 * KP, k, lane);
     __syncthreads();
-    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tabA);
-    if (base == kDynSmemBase && pA.list && pB.list && pA.col == pB.col) {
-        const int64_t lo = (lA == hA) ? lB : ((lB == hB) ? lA : min(lA, lB));
-        const int64_t hi = max(hA, hB);
-        scan_positions_pair<KP>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, pB.a, pB.b, lo, hi,
-                                tkA, tkB, tabA, tabB, sh, lane, warp);
-    } else {
-        if (lA < hA)
-            scan_positions_range<KP, false>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, lA, hA,
-                                            kPairWarps, sh, tabA, tkA, lane, warp);
-        if (lB < hB)
-            scan_positions_range<KP, false>(sc.codes_of(pB.col), sc.rows_of(pB.col), pB.a, pB.b, lB, hB,
-                                            kPairWarps, sh, tabB, tkB, lane, warp);
-    }
+    const int64_t lo = (lA == hA) ? lB : ((lB == hB) ? lA : min(lA, lB));
+    const int64_t hi = max(hA, hB);
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(ptab);
+    const uint32_t one = (uint32_t)(k > 0);   // 1 (k >= 1), opaque to the compiler
+    if (base == kDynSmemBase)
+        scan_positions_pair<KP, true>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, pB.a, pB.b, lo, hi,
+                                      tkA, tkB, exA, exB, slA, invA, slB, invB, base, one, lane, warp);
+    else
+        scan_positions_pair<KP, false>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, pB.a, pB.b, lo, hi,
+                                       tkA, tkB, exA, exB, slA, invA, slB, invB, base, one, lane, warp);
     merge_warps<KP, kPairWarps>(tkA, tkbufA, k, lane, warp, outA);
     merge_warps<KP, kPairWarps>(tkB, tkbufB, k, lane, warp, outB);
 }

@@ -211,3 +211,80 @@ def test_threshold_and_launch_counts(ifvs):
         with pytest.raises(ifvs.IfvsError) as e:
             g.search(q, p, 10, list_max_ppm=bad)
         assert e.value.code == ifvs.IFVS_ERR_ARG
+
+
+def _wide_pairs():
+    """Consecutive pairs of one-column ranges that share a two-query CTA:
+    equal, shifted (blocks of one query only at either end), nested."""
+    rows = [(-500, 500), (-500, 500), (-450, 500), (-500, 480), (-500, 400), (-420, 500),
+            (-480, 490), (-490, 480), (-500, 500), (-375, 500)]
+    p = synth.empty_predicates(len(rows))
+    for i, (lo, hi) in enumerate(rows):
+        p[i]["n_clauses"] = 1
+        synth.set_clause(p[i], 0, 0, synth.OP_RANGE, lo, hi)
+    return p
+
+
+def _one_by_one(g, q, p, k, **kw):
+    out = [g.search(q[i:i + 1], p[i:i + 1], k, **kw) for i in range(len(q))]
+    return tuple(np.concatenate([o[j] for o in out]) for j in range(3))
+
+
+@pytest.mark.parametrize("case", ["normal", "one_wide_subspace", "constant", "tiny_range", "huge"])
+@pytest.mark.parametrize("k", [100, 128])
+def test_pair_kernel_equals_one_query_kernel(ifvs, orc, case, k):
+    """The two-query kernel drops rows by a quantised lower bound and
+    rescores the rest exactly in the one-query loop's order, so a batch whose
+    queries pair up must return, bit for bit, what each query returns alone
+    (one query per CTA).  Table shapes: ordinary; one subspace 1000x wider
+    than the others (a loose bound: most rows rescored); every codeword of a
+    subspace equal (a zero range: the test is off, all distances tie); a
+    range of a few ulps; entries near 1e35."""
+    N = 70001
+    g, codes, attrs, Cpq = _index(ifvs, N, seed=21)
+    rng = np.random.default_rng(22)
+    if case == "one_wide_subspace":
+        Cpq[3] *= 1000.0
+    elif case == "constant":
+        Cpq[:] = Cpq[:, :1, :]
+    elif case == "tiny_range":
+        Cpq = (1.0 + 1e-6 * rng.standard_normal(Cpq.shape)).astype(np.float32)
+    elif case == "huge":
+        Cpq = (Cpq * 1e17).astype(np.float32)
+    g.load_codebooks(Cpq)
+    p = _wide_pairs()
+    q = _queries(len(p), Cpq.shape[0] * Cpq.shape[2], seed=23)
+    if case == "huge":
+        q *= 1e17
+    if case == "tiny_range":
+        q[:] = 1.0
+    q[9] = q[8]                                    # a pair of identical vectors
+    g.stage_times(reset=True)
+    a = g.search(q, p, k, flags=ifvs.IFVS_F_STAGE_TIMING)
+    assert g.stage_times(reset=True)["scan"][1] == 3   # bitmap, one-query and two-query kernels
+    b = _one_by_one(g, q, p, k)
+    for x, y in zip(a, b):
+        np.testing.assert_array_equal(x, y)
+    if case != "huge":
+        _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
+
+
+def test_pair_kernel_with_conditioning(ifvs, orc):
+    """Wide pairs through the conditioned path (bank, W, w_z): the same
+    bit-for-bit agreement with single queries, and the oracle's top-k."""
+    w = synth.scaled(synth.WORKLOADS["gmm10k-d128-m16"], N=50001)
+    ix = synth.make_index(w)
+    cond = synth.make_conditioning(ix)
+    qs = synth.make_queries(ix, 1.0, nq=12)
+    g = ifvs.Index(ix.codes, ix.attrs, D=w.D, K=w.K)
+    g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
+    a = g.search(qs.q, qs.preds, 100, wz=qs.wz)
+    out = [g.search(qs.q[i:i + 1], qs.preds[i:i + 1], 100, wz=qs.wz[i:i + 1]) for i in range(12)]
+    for j in range(3):
+        np.testing.assert_array_equal(a[j], np.concatenate([o[j] for o in out]))
+    oi, od, on, st = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q, qs.preds, 100, bank=cond.bank,
+                                W=cond.W, seeds=cond.seeds, wz=qs.wz, want_stages=True)
+    np.testing.assert_array_equal(a[2], on)
+    for i in range(12):
+        all_d = orc.adc_all(st["lut"][i], ix.codes)
+        check_topk(a[0][i], a[1][i], oi[i], od[i], all_d, np.ones(w.N, bool))
