@@ -728,12 +728,10 @@ __device__ __forceinline__ int quant_bound(uint64_t thr, float sl, float inv) {
 }
 
 // Quantised sums of two M = 16 rows (codes ca, cb), both queries at once:
-// the addresses of lookup16x2, integer loads, and the sums as multiply-adds
-// by `one` (= 1, unknown to the compiler), which run on the FMA pipe beside
-// the byte permutes on the integer pipe.
+// the addresses of lookup16x2, integer loads and adds.
 template <bool FAST>
 __device__ __forceinline__ void lookup16x2_q(const uint4 ca, const uint4 cb, uint32_t tb, uint32_t base,
-                                             uint32_t one, uint32_t& sa, uint32_t& sb) {
+                                             uint32_t& sa, uint32_t& sb) {
     const uint32_t wa[4] = {ca.x, ca.y, ca.z, ca.w};
     const uint32_t wb[4] = {cb.x, cb.y, cb.z, cb.w};
     uint32_t xa = 0u, xb = 0u;
@@ -761,8 +759,8 @@ __device__ __forceinline__ void lookup16x2_q(const uint4 ca, const uint4 cb, uin
 #undef IFVS_LDQ_CASE
             default: va = vb = 0u; break;
         }
-        xa = va * one + xa;
-        xb = vb * one + xb;
+        xa += va;
+        xb += vb;
     }
     sa = xa;
     sb = xb;
@@ -794,28 +792,34 @@ __device__ __forceinline__ uint32_t pack_bounds(int ta, int tb) {
 
 constexpr uint32_t kCandA = 0x00008000u, kCandB = 0x80000000u;
 
-// kU2 rows per lane per round in the paired loop
+// kU2 rows per lane per round in the paired loop (measured: 2 rows, 8 rows,
+// and loading the next round's codes before this round's look-ups are all
+// slower at the 128-register cap of a 16-warp CTA)
 constexpr int kU2 = 4;
 
 // One round of kU2 positions of a block: quantised sums of both queries,
 // candidates by the packed bounds, exact distances and top-k offers for the
 // candidates.  MASKED: the block is cut by one of the ranges (mask[] holds
 // kCandA / kCandB for the positions inside each query's range).
-template <int KP, bool FAST, bool MASKED>
-__device__ __forceinline__ void pair_round(const uint8_t* __restrict__ codes, const uint32_t* __restrict__ rows,
-                                           uint32_t pos0, const uint32_t (&mask)[kU2], WarpTopK<KP>& tkA,
-                                           WarpTopK<KP>& tkB, const float* exA, const float* exB, float slA,
-                                           float invA, float slB, float invB, uint32_t tb, uint32_t base,
-                                           uint32_t one, int rot, uint64_t keep, int lane, uint32_t& Tpk) {
-    uint4 c[kU2];
+template <bool MASKED>
+__device__ __forceinline__ void pair_load(const uint8_t* __restrict__ codes, uint32_t pos0,
+                                          const uint32_t (&mask)[kU2], uint64_t keep, uint4 (&c)[kU2]) {
 #pragma unroll
     for (int u = 0; u < kU2; ++u) {
         const uint32_t pos = pos0 + 32u * (uint32_t)u;
         c[u] = (!MASKED || mask[u] != 0u) ? ldg_nc_v4(codes + (size_t)pos * 16, keep) : make_uint4(0, 0, 0, 0);
     }
+}
+
+template <int KP, bool FAST, bool MASKED>
+__device__ __forceinline__ void pair_round(const uint4 (&c)[kU2], const uint32_t* __restrict__ rows,
+                                           uint32_t pos0, const uint32_t (&mask)[kU2], WarpTopK<KP>& tkA,
+                                           WarpTopK<KP>& tkB, const float* exA, const float* exB, float slA,
+                                           float invA, float slB, float invB, uint32_t tb, uint32_t base,
+                                           int rot, int lane, uint32_t& Tpk) {
     uint32_t sq[kU2];
 #pragma unroll
-    for (int u = 0; u < kU2; u += 2) lookup16x2_q<FAST>(c[u], c[u + 1], tb, base, one, sq[u], sq[u + 1]);
+    for (int u = 0; u < kU2; u += 2) lookup16x2_q<FAST>(c[u], c[u + 1], tb, base, sq[u], sq[u + 1]);
     uint32_t cb[kU2], any = 0u;
 #pragma unroll
     for (int u = 0; u < kU2; ++u) {
@@ -848,8 +852,7 @@ __device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ 
                                                     int64_t bA, int64_t aB, int64_t bB, int64_t blk0,
                                                     int64_t blk1, WarpTopK<KP>& tkA, WarpTopK<KP>& tkB,
                                                     const float* exA, const float* exB, float slA, float invA,
-                                                    float slB, float invB, uint32_t base, uint32_t one,
-                                                    int lane, int warp) {
+                                                    float slB, float invB, uint32_t base, int lane, int warp) {
     const uint32_t tb = 4u * (uint32_t)lane;
     const int rot = lane & 15;
     const uint64_t keep = policy_evict_last();
@@ -863,11 +866,14 @@ __device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ 
         const bool fullA = inA && p0 >= a1 && pe <= b1, fullB = inB && p0 >= a2 && pe <= b2;
         if (fullA && fullB) {
             const uint32_t none[kU2] = {};
+            const uint32_t pb = p0 + (uint32_t)lane;
 #pragma unroll 1
-            for (int j0 = 0; j0 < 32; j0 += kU2)
-                pair_round<KP, FAST, false>(codes, rows, p0 + 32u * (uint32_t)j0 + (uint32_t)lane, none, tkA,
-                                            tkB, exA, exB, slA, invA, slB, invB, tb, base, one, rot, keep, lane,
-                                            Tpk);
+            for (int j0 = 0; j0 < 32; j0 += kU2) {
+                uint4 c[kU2];
+                pair_load<false>(codes, pb + 32u * (uint32_t)j0, none, keep, c);
+                pair_round<KP, FAST, false>(c, rows, pb + 32u * (uint32_t)j0, none, tkA, tkB, exA, exB, slA, invA,
+                                            slB, invB, tb, base, rot, lane, Tpk);
+            }
             continue;
         }
 #pragma unroll 1
@@ -880,8 +886,10 @@ __device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ 
                 mask[u] = ((fullA || (inA && pos >= a1 && pos < b1)) ? kCandA : 0u) |
                           ((fullB || (inB && pos >= a2 && pos < b2)) ? kCandB : 0u);
             }
-            pair_round<KP, FAST, true>(codes, rows, pos0, mask, tkA, tkB, exA, exB, slA, invA, slB, invB, tb,
-                                       base, one, rot, keep, lane, Tpk);
+            uint4 c[kU2];
+            pair_load<true>(codes, pos0, mask, keep, c);
+            pair_round<KP, FAST, true>(c, rows, pos0, mask, tkA, tkB, exA, exB, slA, invA, slB, invB, tb, base,
+                                       rot, lane, Tpk);
         }
     }
 }
@@ -1014,13 +1022,12 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     const int64_t lo = (lA == hA) ? lB : ((lB == hB) ? lA : min(lA, lB));
     const int64_t hi = max(hA, hB);
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(ptab);
-    const uint32_t one = (uint32_t)(k > 0);   // 1 (k >= 1), opaque to the compiler
     if (base == kDynSmemBase)
         scan_positions_pair<KP, true>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, pB.a, pB.b, lo, hi,
-                                      tkA, tkB, exA, exB, slA, invA, slB, invB, base, one, lane, warp);
+                                      tkA, tkB, exA, exB, slA, invA, slB, invB, base, lane, warp);
     else
         scan_positions_pair<KP, false>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, pB.a, pB.b, lo, hi,
-                                       tkA, tkB, exA, exB, slA, invA, slB, invB, base, one, lane, warp);
+                                       tkA, tkB, exA, exB, slA, invA, slB, invB, base, lane, warp);
     merge_warps<KP, kPairWarps>(tkA, tkbufA, k, lane, warp, outA);
     merge_warps<KP, kPairWarps>(tkB, tkbufB, k, lane, warp, outB);
 }
