@@ -60,6 +60,9 @@ def parse():
     ap.add_argument("--list-max-ppm", type=int, default=0,
                     help="sorted-copy scan for one-column pools up to this many rows per million "
                          "(0 = library default: always, -1 = never)")
+    ap.add_argument("--pair-min-rows", type=int, default=0,
+                    help="two-query CTAs for overlapping one-column ranges spanning at least this many "
+                         "rows (0 = library default, -1 = never)")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
     ap.add_argument("--mode", default="search", choices=["search", "pq", "train"],
                     help="search: the query path; pq: PQ encoding + Lloyd training of the index; "
@@ -434,7 +437,8 @@ def run_ifvs(args):
         oi, od, on = dev_out[b]
         ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on,
                                flags=flags, stream=sptr, chunk_blocks=args.chunk_blocks,
-                               list_max_ppm=args.list_max_ppm, rerank=args.rerank)
+                               list_max_ppm=args.list_max_ppm, rerank=args.rerank,
+                               pair_min_rows=args.pair_min_rows)
 
     for i in range(args.warmup):
         step(i)
@@ -525,7 +529,7 @@ def run_ifvs(args):
             oi, od, on, _ = host_out[b]
             ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr,
                                    chunk_blocks=args.chunk_blocks, list_max_ppm=args.list_max_ppm,
-                                   rerank=args.rerank)
+                                   rerank=args.rerank, pair_min_rows=args.pair_min_rows)
 
         for i in range(args.warmup):
             hstep(i)

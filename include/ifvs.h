@@ -108,6 +108,14 @@ typedef struct {
                            (1000000: always); -1: never.  The two paths sum a row's entries in
                            different orders, so distances agree to float32
                            rounding.                                          */
+    int32_t pair_min_rows; /* M = 16 sorted-copy scan: two queries on the same
+                           column whose ranges share 3/4 of the longer one and
+                           together span at least this many rows share a CTA
+                           and one shared-memory look-up per code byte (their
+                           tables quantised to 11 bits, every row that can
+                           reach a top-k rescored exactly, so results equal
+                           those of one query per CTA bit for bit).
+                           0: default (4194304); -1: never pair.             */
     void* stream;       /* cudaStream_t to run on; NULL: the index's stream   */
 } ifvs_search_params;
 

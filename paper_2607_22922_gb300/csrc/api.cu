@@ -116,7 +116,7 @@ struct ifvs_index {
     size_t bytes = 0;
     // workspace
     DevBuf w_q, w_wz, w_preds, w_canon, w_err, w_bm, w_rows, w_npass, w_idx, w_alpha, w_wf,
-        w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist, w_tab, w_plan;
+        w_lut, w_cifvs, w_part, w_ids, w_dists, w_cand, w_cdist, w_tab, w_plan, w_items;
     // training workspace
     DevBuf t_cand, t_pos, t_mined, t_mdist, t_gC, t_gw, t_loss, t_G, t_gW, t_gWpart, t_galpha,
         t_gbank, t_gwz, t_wz, t_neg;
@@ -186,7 +186,7 @@ void free_index(ifvs_index* ix) {
     DevBuf* bufs[] = {&ix->w_q, &ix->w_wz, &ix->w_preds, &ix->w_canon, &ix->w_err, &ix->w_bm,
                       &ix->w_rows, &ix->w_npass, &ix->w_idx, &ix->w_alpha, &ix->w_wf,
                       &ix->w_lut, &ix->w_cifvs, &ix->w_part, &ix->w_ids, &ix->w_dists,
-                      &ix->w_cand, &ix->w_cdist, &ix->w_tab, &ix->w_plan, &ix->t_cand, &ix->t_pos,
+                      &ix->w_cand, &ix->w_cdist, &ix->w_tab, &ix->w_plan, &ix->w_items, &ix->t_cand, &ix->t_pos,
                       &ix->t_mined, &ix->t_mdist, &ix->t_gC, &ix->t_gw, &ix->t_loss, &ix->t_G,
                       &ix->t_gW, &ix->t_gWpart, &ix->t_galpha, &ix->t_gbank, &ix->t_gwz, &ix->t_wz, &ix->t_neg};
     for (DevBuf* b : bufs) release(*b);
@@ -307,6 +307,7 @@ struct Opts {
     int64_t sub_batch = 0;
     int64_t chunk_blocks = 0;
     int32_t list_max_ppm = 0;
+    int32_t pair_min_rows = 0;
     cudaStream_t stream = nullptr;
 };
 
@@ -315,6 +316,12 @@ struct Opts {
 // bitmap path in every measured selectivity bin, for M = 16 and for the
 // generic-M loop (10^6 x 120 codes)
 constexpr int32_t kListDefaultPpm = 1000000;
+
+// two-query CTAs for ranges that together span at least 2^22 rows: on the
+// 10^8-row workload pairs were faster at 10 % and 100 % of the rows
+// (10^7, 10^8) and slower at 0.1 % and 1 % (10^5, 10^6) than one query per
+// CTA, which holds two or three CTAs per SM
+constexpr int64_t kPairDefaultMinRows = int64_t(1) << 22;
 
 int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (!p) return 0;
@@ -326,6 +333,7 @@ int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (p->sub_batch < 0) return set_err(IFVS_ERR_ARG, "sub_batch must be >= 0");
     if (p->list_max_ppm < -1 || p->list_max_ppm > 1000000)
         return set_err(IFVS_ERR_ARG, "list_max_ppm = %d outside -1..1000000", p->list_max_ppm);
+    if (p->pair_min_rows < -1) return set_err(IFVS_ERR_ARG, "pair_min_rows = %d below -1", p->pair_min_rows);
     o->dio = p->flags & IFVS_F_DEVICE_IO;
     o->timing = p->flags & IFVS_F_STAGE_TIMING;
     o->plain = p->flags & IFVS_F_PLAIN_PQ;
@@ -333,6 +341,7 @@ int parse_opts(const ifvs_search_params* p, Opts* o) {
     o->sub_batch = p->sub_batch;
     o->chunk_blocks = p->chunk_blocks;
     o->list_max_ppm = p->list_max_ppm;
+    o->pair_min_rows = p->pair_min_rows;
     o->stream = reinterpret_cast<cudaStream_t>(p->stream);
     return 0;
 }
@@ -412,6 +421,7 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
         const int64_t ppm = o.list_max_ppm > 0 ? o.list_max_ppm : kListDefaultPpm;
         const int64_t max_rows = ppm >= 1000000 ? ix->N : ix->N * ppm / 1000000;
         TRY(ensure(ix->w_plan, sizeof(ScanPlan) * n));
+        TRY(ensure(ix->w_items, (sizeof(PairItem) + 1) * n));   // pairs, then a pair flag per query
         Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);
         CUDA_TRY(st.end(launch_plan(ix->w_canon.as<CanonPred>(), n, ix->sorted(), ix->N, max_rows,
                                     ix->w_plan.as<ScanPlan>(), npass_u64, s)));
@@ -448,8 +458,11 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
     if (plan) {
         Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
         int nl = 0;
+        const int64_t pmin = o.pair_min_rows > 0 ? o.pair_min_rows : kPairDefaultMinRows;
         const cudaError_t e = launch_scan_list(ix->w_tab.as<float>(), ix->sorted(), plan, n, kk, sh,
-                                               ix->w_part.as<uint64_t>(), s, &nl);
+                                               ix->w_part.as<uint64_t>(),
+                                               o.pair_min_rows < 0 ? nullptr : ix->w_items.as<PairItem>(),
+                                               pmin, s, &nl);
         CUDA_TRY(st.end(e, nl));
     }
     int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;

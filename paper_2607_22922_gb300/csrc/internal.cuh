@@ -190,11 +190,21 @@ int scan_kp(int k);
 cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm,
                         const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
                         uint64_t* partials, cudaStream_t s);
+// One CTA's work in the M = 16 sorted-copy scan: queries qa and qb share
+// it (qb = -1: qa alone; qa = -1: no work).
+struct PairItem {
+    int32_t qa, qb;
+};
 // the list-path queries of `plan`: their pool is the position range [a, b)
-// of a column's sorted copy (same grid and partial layout as launch_scan)
-// (*launches = kernels launched: a one-query and, for M = 16, a two-query kernel)
+// of a column's sorted copy (same grid and partial layout as launch_scan).
+// For M = 16, `items` (workspace: nq PairItems followed by nq bytes)
+// receives the pairs of overlapping ranges that together span at least
+// pair_min_rows positions, which a two-query kernel serves; a one-query
+// kernel serves the other queries (all of them when items is null or
+// M != 16).  *launches = kernels launched.
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
-                             const ScanShape& sh, uint64_t* partials, cudaStream_t s, int* launches);
+                             const ScanShape& sh, uint64_t* partials, PairItem* items, int64_t pair_min_rows,
+                             cudaStream_t s, int* launches);
 // the sorted copy of the codes: dst position p <- row rows[p] of the index
 // layout `src`, re-rotated by (p mod 32) mod M; positions >= N are zero
 cudaError_t launch_relayout_sorted(const uint8_t* src, const uint32_t* rows, int64_t N, int M,

@@ -94,27 +94,46 @@ __device__ __forceinline__ void warp_sort(uint64_t* a, int n, int lane) {
     __syncwarp();
 }
 
+// The warps of a CTA that serve one query share a bound `cta` (shared
+// memory): the smallest k-th key any of them has published.  A warp's list
+// holds k distinct rows, so its k-th key is at least the CTA's true k-th
+// key, and a row whose key is above some warp's k-th key cannot be in the
+// CTA's top-k: each warp offers only keys below min(own k-th, cta).  The
+// warps' lists then still contain every row of the CTA's top-k, and the
+// shared bound lets every warp drop rows as early as the whole CTA could.
 template <int KP>
 struct WarpTopK {
     uint64_t* buf;   // [0, KP): sorted best keys; [KP, 2KP): candidates
+    uint64_t* cta;   // shared bound of the CTA's warps for this query, or null
     int cnt;
     int k;
-    uint64_t thr;    // current k-th best key (all ones while fewer than k)
+    uint64_t thr;    // keys below thr are offered: min(own k-th key, *cta)
 
-    __device__ __forceinline__ void init(uint64_t* b, int k_, int lane) {
+    __device__ __forceinline__ void init(uint64_t* b, int k_, int lane, uint64_t* cta_ = nullptr) {
         buf = b;
+        cta = cta_;
         k = k_;
         cnt = 0;
         thr = ~0ull;
         for (int i = lane; i < 2 * KP; i += 32) buf[i] = ~0ull;
         __syncwarp();
     }
+    // lower thr to the shared bound: every lane loads the same word in one
+    // broadcast (measured faster than a lane-0 load and a shuffle); any value
+    // a lane sees is a valid bound, so thr stays correct in every lane
+    __device__ __forceinline__ void refresh(int) {
+        if (cta == nullptr) return;
+        const uint64_t t = *reinterpret_cast<volatile uint64_t*>(cta);
+        if (t < thr) thr = t;
+    }
     __device__ __forceinline__ void flush(int lane) {
         warp_sort(buf, 2 * KP, lane);
         thr = buf[k - 1];
         for (int i = KP + lane; i < 2 * KP; i += 32) buf[i] = ~0ull;
+        if (cta != nullptr && lane == 0 && thr != ~0ull) atomicMin(reinterpret_cast<unsigned long long*>(cta), thr);
         __syncwarp();
         cnt = 0;
+        refresh(lane);
     }
     __device__ __forceinline__ void offer(uint64_t key, bool want, int lane) {
         const unsigned ball = __ballot_sync(0xFFFFFFFFu, want);
@@ -534,7 +553,7 @@ cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* 
 // bitmap path's, so the two agree to float32 rounding.
 
 size_t scan_list_smem_bytes(int tab_words, int kp) {
-    return (size_t)256 * tab_words * 4 + (size_t)kScanWarps * 2 * kp * 8;
+    return (size_t)256 * tab_words * 4 + (size_t)kScanWarps * 2 * kp * 8 + 16;
 }
 
 template <int KP, bool M16, bool FAST>
@@ -554,6 +573,7 @@ __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes
         const bool full = p0 >= a32 && p0 + kBlockRows <= b32;
 #pragma unroll 1
         for (int j0 = 0; j0 < 32; j0 += kU) {
+            tk.refresh(lane);
             uint32_t pos[kU];
             unsigned valid = 0u;
 #pragma unroll
@@ -590,25 +610,10 @@ __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes
     }
 }
 
-// Two consecutive sorted-path queries share a CTA when they read the same
-// column's copy, both ranges cover at least 3/4 of the rows and 3/4 of the
-// longer one is common to both (the dense queries); otherwise each takes a
-// CTA of its own.  Narrower pairs are left alone on purpose: the two kernels
-// run one after the other, so a few long two-query CTAs would leave the GPU
-// idle behind them.  Both scan kernels evaluate this rule, so each query is
-// served exactly once.
-__device__ __forceinline__ bool pair_ok(const ScanPlan& x, const ScanPlan& y, int64_t N) {
-    if (!x.list || !y.list || x.col != y.col) return false;
-    const int64_t lx = x.b - x.a, ly = y.b - y.a;
-    const int64_t common = min(x.b, y.b) - max(x.a, y.a);
-    const int64_t longer = max(lx, ly);
-    return 4 * lx >= 3 * N && 4 * ly >= 3 * N && longer > 0 && 4 * common >= 3 * longer;
-}
-
 template <int KP, bool M16, int MINB>
 __global__ void __launch_bounds__(kScanThreads, MINB)
 k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
-            int k, ScanShape sh, uint64_t* __restrict__ partials, int pairs) {
+            int k, ScanShape sh, uint64_t* __restrict__ partials, const uint8_t* __restrict__ paired) {
     extern __shared__ __align__(256) uint8_t smem[];
     const int S = M16 ? 64 : sh.tab_words;
     float* tab = reinterpret_cast<float*>(smem);
@@ -617,11 +622,8 @@ k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __r
     const int64_t q = blockIdx.x;
     const int chunk = blockIdx.y;
     const ScanPlan p = plan[q];
-    if (!p.list) return;   // k_scan covers this query
-    if (pairs) {           // k_scan_list_pair covers paired queries
-        const int64_t mate = q ^ 1;
-        if (mate < nq && pair_ok(plan[q & ~(int64_t)1], plan[q | 1], sh.n_rows)) return;
-    }
+    if (!p.list) return;                               // k_scan covers this query
+    if (paired != nullptr && paired[q]) return;        // k_scan_list_pair covers it
     const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
     const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
     const int64_t blk0 = max(c0, p.a / kBlockRows);
@@ -636,8 +638,10 @@ k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __r
         float4* dst = reinterpret_cast<float4*>(tab);
         for (int i = threadIdx.x; i < 64 * S; i += kScanThreads) dst[i] = __ldg(src + i);
     }
+    uint64_t* cta = tkbuf + kScanWarps * 2 * KP;
+    if (threadIdx.x == 0) *cta = ~0ull;
     WarpTopK<KP> tk;
-    tk.init(tkbuf + warp * 2 * KP, k, lane);
+    tk.init(tkbuf + warp * 2 * KP, k, lane, cta);
     __syncthreads();
     const uint8_t* codes = sc.codes_of(p.col);
     const uint32_t* rows = sc.rows_of(p.col);
@@ -692,8 +696,9 @@ constexpr uint32_t kTabBytes16 = 256u * 64u * 4u;    // one replicated M = 16 ta
 constexpr uint32_t kExactBytes16 = 256u * 16u * 4u;  // one unreplicated table, [c][m]
 constexpr int kQMax = 2047;                           // 16 * 2047 < 2^15
 
+// packed table, two exact tables, extremes + the two shared bounds, lists
 size_t scan_pair_smem_bytes(int kp) {
-    return (size_t)kTabBytes16 + 2 * (size_t)kExactBytes16 + 64 * 4 + (size_t)kPairWarps * 2 * 2 * kp * 8;
+    return (size_t)kTabBytes16 + 2 * (size_t)kExactBytes16 + 64 * 4 + 16 + (size_t)kPairWarps * 2 * 2 * kp * 8;
 }
 
 template <int IMM>
@@ -799,8 +804,9 @@ constexpr int kU2 = 4;
 
 // One round of kU2 positions of a block: quantised sums of both queries,
 // candidates by the packed bounds, exact distances and top-k offers for the
-// candidates.  MASKED: the block is cut by one of the ranges (mask[] holds
-// kCandA / kCandB for the positions inside each query's range).
+// candidates.  mask[] holds kCandA / kCandB for the positions inside each
+// query's range; MASKED: it differs between positions (a cut block), so
+// only positions inside a range load codes.
 template <bool MASKED>
 __device__ __forceinline__ void pair_load(const uint8_t* __restrict__ codes, uint32_t pos0,
                                           const uint32_t (&mask)[kU2], uint64_t keep, uint4 (&c)[kU2]) {
@@ -817,13 +823,20 @@ __device__ __forceinline__ void pair_round(const uint4 (&c)[kU2], const uint32_t
                                            WarpTopK<KP>& tkB, const float* exA, const float* exB, float slA,
                                            float invA, float slB, float invB, uint32_t tb, uint32_t base,
                                            int rot, int lane, uint32_t& Tpk) {
+    {
+        const uint64_t oa = tkA.thr, ob = tkB.thr;
+        tkA.refresh(lane);
+        tkB.refresh(lane);
+        if (tkA.thr != oa || tkB.thr != ob)
+            Tpk = pack_bounds(quant_bound(tkA.thr, slA, invA), quant_bound(tkB.thr, slB, invB));
+    }
     uint32_t sq[kU2];
 #pragma unroll
     for (int u = 0; u < kU2; u += 2) lookup16x2_q<FAST>(c[u], c[u + 1], tb, base, sq[u], sq[u + 1]);
     uint32_t cb[kU2], any = 0u;
 #pragma unroll
     for (int u = 0; u < kU2; ++u) {
-        cb[u] = (Tpk - sq[u]) & (MASKED ? mask[u] : (kCandA | kCandB));
+        cb[u] = (Tpk - sq[u]) & mask[u];
         any |= cb[u];
     }
     if (!__any_sync(0xFFFFFFFFu, any != 0u)) return;
@@ -864,14 +877,18 @@ __device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ 
         const bool inA = p0 < b1 && pe > a1, inB = p0 < b2 && pe > a2;
         if (!(inA || inB)) continue;
         const bool fullA = inA && p0 >= a1 && pe <= b1, fullB = inB && p0 >= a2 && pe <= b2;
-        if (fullA && fullB) {
-            const uint32_t none[kU2] = {};
+        if ((fullA || !inA) && (fullB || !inB)) {
+            // each query takes all or none of the block: one mask for all rows
+            const uint32_t mc = (fullA ? kCandA : 0u) | (fullB ? kCandB : 0u);
+            uint32_t mask[kU2];
+#pragma unroll
+            for (int u = 0; u < kU2; ++u) mask[u] = mc;
             const uint32_t pb = p0 + (uint32_t)lane;
 #pragma unroll 1
             for (int j0 = 0; j0 < 32; j0 += kU2) {
                 uint4 c[kU2];
-                pair_load<false>(codes, pb + 32u * (uint32_t)j0, none, keep, c);
-                pair_round<KP, FAST, false>(c, rows, pb + 32u * (uint32_t)j0, none, tkA, tkB, exA, exB, slA, invA,
+                pair_load<false>(codes, pb + 32u * (uint32_t)j0, mask, keep, c);
+                pair_round<KP, FAST, false>(c, rows, pb + 32u * (uint32_t)j0, mask, tkA, tkB, exA, exB, slA, invA,
                                             slB, invB, tb, base, rot, lane, Tpk);
             }
             continue;
@@ -929,26 +946,126 @@ __device__ __forceinline__ void quant_params(const float* lo, const float* hi, f
     sl = s;
 }
 
+// ---- pairing of the sorted-copy queries of a batch -------------------------
+//
+// Two queries are worth one CTA when they read the same column's copy, their
+// ranges mostly coincide (at least 3/4 of the longer range is common to both;
+// the rows of only one range then run with the other query masked) and the
+// two ranges together span at least min_rows positions (the caller's choice:
+// for short ranges the one-query kernel, with two or three CTAs per SM, was
+// measured faster).
+// k_pair_items sorts the list-path queries of each segment of kPairSeg by
+// (column, range start, query) and pairs sorted neighbours (2j, 2j + 1) that
+// qualify.  Pairs fill the segment's item slots in sorted order and the
+// unused slots get qa = -1, so the pair kernel's CTA x serves item x (or
+// nothing); `paired` marks the queries of the pairs, and k_scan_list serves
+// every other list-path query.
+constexpr int kPairSeg = 2048;
+static_assert(IFVS_MAX_ATTRS <= 4, "the pairing key keeps 2 bits of the column");
+constexpr int kPairSortThreads = 1024;
+
+__device__ __forceinline__ bool pairable(const ScanPlan& x, const ScanPlan& y, int64_t min_rows) {
+    if (!x.list || !y.list || x.col != y.col) return false;
+    const int64_t lx = x.b - x.a, ly = y.b - y.a;
+    if (lx <= 0 || ly <= 0) return false;
+    const int64_t common = min(x.b, y.b) - max(x.a, y.a);
+    const int64_t span = max(x.b, y.b) - min(x.a, y.a);
+    return 4 * common >= 3 * max(lx, ly) && span >= min_rows;
+}
+
+__global__ void __launch_bounds__(kPairSortThreads)
+k_pair_items(const ScanPlan* __restrict__ plan, int64_t nq, int64_t min_rows, PairItem* __restrict__ items,
+             uint8_t* __restrict__ paired) {
+    __shared__ uint64_t key[kPairSeg];
+    __shared__ int wsum[kPairSortThreads / 32];
+    const int64_t q0 = (int64_t)blockIdx.x * kPairSeg;
+    const int n = (int)min((int64_t)kPairSeg, nq - q0);
+    // key = col (2 bits) | range start (32 bits) | index in the segment (11 bits);
+    // queries of the bitmap path sort last as all ones
+    for (int i = threadIdx.x; i < kPairSeg; i += kPairSortThreads) {
+        uint64_t kk = ~0ull;
+        if (i < n) {
+            const ScanPlan p = plan[q0 + i];
+            if (p.list) kk = ((uint64_t)(p.col & 3) << 43) | ((uint64_t)(uint32_t)p.a << 11) | (uint64_t)i;
+        }
+        key[i] = kk;
+    }
+    // block bitonic sort, ascending
+    for (int size = 2; size <= kPairSeg; size <<= 1)
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            __syncthreads();
+            for (int t = threadIdx.x; t < kPairSeg / 2; t += kPairSortThreads) {
+                const int i = 2 * t - (t & (stride - 1));
+                const int j = i + stride;
+                const bool up = (i & size) == 0;
+                const uint64_t x = key[i], y = key[j];
+                if ((x > y) == up) {
+                    key[i] = y;
+                    key[j] = x;
+                }
+            }
+        }
+    __syncthreads();
+    // sorted neighbours (2j, 2j + 1) that qualify make an item; positions by
+    // a block-wide exclusive scan of the counts, in sorted order
+    static_assert(kPairSeg == 2 * kPairSortThreads, "one neighbour pair per thread");
+    const int j = threadIdx.x;
+    const uint64_t ka = key[2 * j], kb = key[2 * j + 1];
+    int qa = -1, qb = -1, cnt = 0;
+    if (ka != ~0ull && kb != ~0ull) {
+        qa = (int)(q0 + (int64_t)(ka & 2047u));
+        qb = (int)(q0 + (int64_t)(kb & 2047u));
+        cnt = pairable(plan[qa], plan[qb], min_rows) ? 1 : 0;
+    }
+    for (int i = j; i < n; i += kPairSortThreads) paired[q0 + i] = 0;
+    __syncthreads();
+    if (cnt) paired[qa] = paired[qb] = 1;
+    const int lane = j & 31, warp = j >> 5;
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += v;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    int before = 0, total = 0;
+    for (int w = 0; w < kPairSortThreads / 32; ++w) {
+        const int v = wsum[w];
+        before += w < warp ? v : 0;
+        total += v;
+    }
+    // segment s owns item slots [s * kPairSeg / 2, + ceil(n / 2)): at most
+    // one pair per two of its queries
+    PairItem* its = items + q0 / 2;
+    const int at = before + incl - cnt;
+    if (cnt) its[at] = PairItem{qa, qb};
+    for (int i = total + j; i < (n + 1) / 2; i += kPairSortThreads) its[i] = PairItem{-1, -1};
+}
+
 template <int KP>
 __global__ void __launch_bounds__(kPairThreads, 1)
 k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan,
-                 int64_t nq, int k, ScanShape sh, uint64_t* __restrict__ partials) {
+                 const PairItem* __restrict__ items, int k, ScanShape sh, uint64_t* __restrict__ partials) {
     extern __shared__ __align__(256) uint8_t smem[];
     uint32_t* ptab = reinterpret_cast<uint32_t*>(smem);
     float* exA = reinterpret_cast<float*>(smem + kTabBytes16);
     float* exB = reinterpret_cast<float*>(smem + kTabBytes16 + kExactBytes16);
     float* prm = reinterpret_cast<float*>(smem + kTabBytes16 + 2 * kExactBytes16);   // lo/hi of A, lo/hi of B
-    uint64_t* tkbufA = reinterpret_cast<uint64_t*>(smem + kTabBytes16 + 2 * kExactBytes16 + 64 * 4);
+    uint64_t* ctab = reinterpret_cast<uint64_t*>(smem + kTabBytes16 + 2 * kExactBytes16 + 64 * 4);   // A, B
+    uint64_t* tkbufA = reinterpret_cast<uint64_t*>(smem + kTabBytes16 + 2 * kExactBytes16 + 64 * 4 + 16);
     uint64_t* tkbufB = tkbufA + kPairWarps * 2 * KP;
     float* red = reinterpret_cast<float*>(tkbufA);   // [warp][4][16], before the lists are set up
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int64_t qA = 2 * (int64_t)blockIdx.x, qB = qA + 1;
-    const bool hasB = qB < nq;
+    const PairItem it = items[blockIdx.x];
+    if (it.qa < 0) return;
+    const int64_t qA = it.qa;
+    const bool hasB = it.qb >= 0;
+    const int64_t qB = hasB ? it.qb : it.qa;   // a single query: B mirrors A's table, with no range
     const int chunk = blockIdx.y;
     const ScanPlan pA = plan[qA];
-    if (!hasB) return;
-    const ScanPlan pB = plan[qB];
-    if (!pair_ok(pA, pB, sh.n_rows)) return;   // k_scan_list covers these queries
+    ScanPlan pB = plan[qB];
+    if (!hasB) pB.a = pB.b = 0;
     const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
     const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
     auto range = [&](const ScanPlan& p, int64_t& lo, int64_t& hi) {
@@ -960,11 +1077,11 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     range(pA, lA, hA);
     range(pB, lB, hB);
     uint64_t* outA = partials + (qA * sh.n_chunks + chunk) * (int64_t)k;
-    uint64_t* outB = partials + (qB * sh.n_chunks + chunk) * (int64_t)k;
+    uint64_t* outB = hasB ? partials + (qB * sh.n_chunks + chunk) * (int64_t)k : nullptr;
     if (lA == hA && lB == hB) {
         for (int i = threadIdx.x; i < k; i += kPairThreads) {
             outA[i] = ~0ull;
-            outB[i] = ~0ull;
+            if (outB) outB[i] = ~0ull;
         }
         return;
     }
@@ -1015,9 +1132,10 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
         ptab[i] = quant12(exA[c * 16 + m], prm[m], invA) | quant12(exB[c * 16 + m], prm[32 + m], invB) << 16;
     }
     __syncthreads();   // the reduction scratch becomes the lists
+    if (threadIdx.x < 2) ctab[threadIdx.x] = ~0ull;
     WarpTopK<KP> tkA, tkB;
-    tkA.init(tkbufA + warp * 2 * KP, k, lane);
-    tkB.init(tkbufB + warp * 2 * KP, k, lane);
+    tkA.init(tkbufA + warp * 2 * KP, k, lane, ctab);
+    tkB.init(tkbufB + warp * 2 * KP, k, lane, ctab + 1);
     __syncthreads();
     const int64_t lo = (lA == hA) ? lB : ((lB == hB) ? lA : min(lA, lB));
     const int64_t hi = max(hA, hB);
@@ -1034,56 +1152,68 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
 
 template <int KP, bool M16, int MINB>
 static cudaError_t launch_list_one(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
-                                   int k, const ScanShape& sh, uint64_t* partials, size_t smem, int pairs,
-                                   cudaStream_t s) {
+                                   int k, const ScanShape& sh, uint64_t* partials, const uint8_t* paired,
+                                   size_t smem, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(k_scan_list<KP, M16, MINB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
-    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, pairs);
+    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, paired);
     return cudaGetLastError();
+}
+
+static int max_smem_optin() {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return 0;
+    return v;
 }
 
 template <int KP>
 static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
-                                  int k, const ScanShape& sh, uint64_t* partials, int* launches,
-                                  cudaStream_t s) {
+                                  int k, const ScanShape& sh, uint64_t* partials, PairItem* items,
+                                  int64_t pair_min_rows, int* launches, cudaStream_t s) {
     const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
-    const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
-    if (m16 && KP == 128) {
-        // wide, overlapping pairs share a CTA; everything else runs one query
-        // per CTA.  For k <= 64 the one-query kernel holds three CTAs (24
-        // warps) per SM against the pair kernel's 16 warps, and wins.
-        const size_t ps = scan_pair_smem_bytes(KP);
-        cudaError_t e = cudaFuncSetAttribute(k_scan_list_pair<KP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)ps);
+    const size_t ps = scan_pair_smem_bytes(KP);
+    const uint8_t* paired = nullptr;
+    int nl = 0;
+    if (m16 && items != nullptr && ps <= (size_t)max_smem_optin()) {
+        // M = 16: long, overlapping ranges are paired by k_pair_items and
+        // served by the two-query kernel; the one-query kernel takes the rest
+        uint8_t* pd = reinterpret_cast<uint8_t*>(items + nq);
+        const unsigned segs = (unsigned)((nq + kPairSeg - 1) / kPairSeg);
+        k_pair_items<<<segs, kPairSortThreads, 0, s>>>(plan, nq, pair_min_rows, items, pd);
+        cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
-        dim3 grid((unsigned)((nq + 1) / 2), (unsigned)sh.n_chunks);
-        k_scan_list_pair<KP><<<grid, kPairThreads, ps, s>>>(tab, sc, plan, nq, k, sh, partials);
+        if ((e = cudaFuncSetAttribute(k_scan_list_pair<KP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)ps)) != cudaSuccess)
+            return e;
+        dim3 grid((unsigned)((nq + 1) / 2), (unsigned)sh.n_chunks);   // at most nq / 2 pairs
+        k_scan_list_pair<KP><<<grid, kPairThreads, ps, s>>>(tab, sc, plan, items, k, sh, partials);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
-        if (launches) *launches = 2;
-        if ((size_t)233472 / (smem + 1024) >= 2)
-            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, smem, 1, s);
-        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, smem, 1, s);
+        paired = pd;
+        nl = 2;
     }
-    if (launches) *launches = 1;
+    const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
+    if (launches) *launches = nl + 1;
     if (m16) {
         if ((size_t)233472 / (smem + 1024) >= 2)
-            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, smem, 0, s);
-        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, smem, 0, s);
+            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
+        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
     }
-    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, smem, 0, s);
+    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
 }
 
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
-                             const ScanShape& sh, uint64_t* partials, cudaStream_t s, int* launches) {
+                             const ScanShape& sh, uint64_t* partials, PairItem* items, int64_t pair_min_rows,
+                             cudaStream_t s, int* launches) {
     if (launches) *launches = 0;
     if (nq <= 0) return cudaSuccess;
     switch (scan_kp(k)) {
-        case 32: return launch_list_kp<32>(tab, sc, plan, nq, k, sh, partials, launches, s);
-        case 64: return launch_list_kp<64>(tab, sc, plan, nq, k, sh, partials, launches, s);
-        case 128: return launch_list_kp<128>(tab, sc, plan, nq, k, sh, partials, launches, s);
-        default: return launch_list_kp<256>(tab, sc, plan, nq, k, sh, partials, launches, s);
+        case 32: return launch_list_kp<32>(tab, sc, plan, nq, k, sh, partials, items, pair_min_rows, launches, s);
+        case 64: return launch_list_kp<64>(tab, sc, plan, nq, k, sh, partials, items, pair_min_rows, launches, s);
+        case 128: return launch_list_kp<128>(tab, sc, plan, nq, k, sh, partials, items, pair_min_rows, launches, s);
+        default: return launch_list_kp<256>(tab, sc, plan, nq, k, sh, partials, items, pair_min_rows, launches, s);
     }
 }
 

@@ -36,7 +36,8 @@ class IfvsError(RuntimeError):
 
 class SearchParams(C.Structure):
     _fields_ = [("flags", C.c_uint32), ("rerank", C.c_int32), ("sub_batch", C.c_int32),
-                ("chunk_blocks", C.c_int32), ("list_max_ppm", C.c_int32), ("stream", C.c_void_p)]
+                ("chunk_blocks", C.c_int32), ("list_max_ppm", C.c_int32), ("pair_min_rows", C.c_int32),
+                ("stream", C.c_void_p)]
 
 
 class TrainParams(C.Structure):
@@ -114,13 +115,14 @@ def _ptr(a):
     raise TypeError("expected a numpy array or a tensor, got %r" % type(a))
 
 
-def _params(flags=0, rerank=0, sub_batch=0, stream=None, chunk_blocks=0, list_max_ppm=0):
+def _params(flags=0, rerank=0, sub_batch=0, stream=None, chunk_blocks=0, list_max_ppm=0, pair_min_rows=0):
     p = SearchParams()
     p.flags = flags
     p.rerank = rerank
     p.sub_batch = sub_batch
     p.chunk_blocks = chunk_blocks
     p.list_max_ppm = list_max_ppm
+    p.pair_min_rows = pair_min_rows
     p.stream = stream
     return p
 
@@ -180,7 +182,8 @@ def ifvs_load_codebooks(ix, C_pq, bank=None, h=0, r=0, W=None, hash_seeds=None):
 
 
 def ifvs_search_batch(ix, queries, preds, k, wz=None, ids=None, dists=None, npass=None,
-                      flags=0, rerank=0, sub_batch=0, stream=None, chunk_blocks=0, list_max_ppm=0):
+                      flags=0, rerank=0, sub_batch=0, stream=None, chunk_blocks=0, list_max_ppm=0,
+                      pair_min_rows=0):
     """Host mode (default): numpy in, numpy out.  With IFVS_F_DEVICE_IO in
     ``flags`` every array (inputs and preallocated outputs) is a device tensor."""
     nq = int(queries.shape[0])
@@ -197,7 +200,7 @@ def ifvs_search_batch(ix, queries, preds, k, wz=None, ids=None, dists=None, npas
             dists = np.empty((nq, k), np.float32)
         if npass is None:
             npass = np.empty(nq, np.int64)
-    p = _params(flags, rerank, sub_batch, stream, chunk_blocks, list_max_ppm)
+    p = _params(flags, rerank, sub_batch, stream, chunk_blocks, list_max_ppm, pair_min_rows)
     _check(_lib.ifvs_search_batch(ix, _ptr(queries), _ptr(preds), nq, k, _ptr(wz), C.byref(p),
                                   _ptr(ids), _ptr(dists), _ptr(npass)))
     return ids, dists, npass

@@ -57,7 +57,7 @@ def test_parameter_structs_match_the_header(lib, tmp_path):
     import subprocess
     structs = {"ifvs_search_params": (lib.SearchParams,
                                       ["flags", "rerank", "sub_batch", "chunk_blocks",
-                                       "list_max_ppm", "stream"]),
+                                       "list_max_ppm", "pair_min_rows", "stream"]),
                "ifvs_train_params": (lib.TrainParams,
                                      ["tau", "lambda", "lr", "lr_wz", "n_pos", "n_neg", "flags",
                                       "stream"])}

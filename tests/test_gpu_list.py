@@ -136,9 +136,10 @@ def test_list_path_other_subspace_counts(ifvs, orc, M):
 
 @pytest.mark.parametrize("k", [10, 100])
 def test_pairs_of_wide_predicates(ifvs, orc, k):
-    """Consecutive queries whose ranges on one column both cover 3/4 of the
-    rows and overlap by 3/4 share a CTA (M = 16); narrower or shifted pairs,
-    an odd last query and a pair on different columns run one per CTA."""
+    """Queries whose ranges on one column overlap by 3/4 of the longer one
+    share a CTA (M = 16); shifted or narrow ranges, an odd query out and a
+    query on the other column run alone.  Results as the bitmap path and
+    the oracle."""
     g, codes, attrs, Cpq = _index(ifvs, 70000, seed=11)
     rows = [(-500, 500), (-500, 500), (-450, 500), (-500, 480), (-300, 400), (-250, 420),
             (-400, 300), (100, 200), (-480, 499)]
@@ -151,10 +152,12 @@ def test_pairs_of_wide_predicates(ifvs, orc, k):
     p[10]["n_clauses"] = 1
     synth.set_clause(p[10], 0, 0, synth.OP_GE, -500)        # ... beside column 0: no pair
     q = _queries(len(p), 32, seed=11)
-    a = g.search(q, p, k, list_max_ppm=ALWAYS)
+    a = g.search(q, p, k, list_max_ppm=ALWAYS, pair_min_rows=1)
     b = g.search(q, p, k, list_max_ppm=NEVER)
     _same_up_to_rounding(a, b)
     _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
+    for x, y in zip(a, g.search(q, p, k, pair_min_rows=-1)):   # no pairs: one query per CTA
+        np.testing.assert_array_equal(x, y)
 
 
 def test_threshold_splits_a_batch(ifvs, orc):
@@ -198,12 +201,15 @@ def test_threshold_and_launch_counts(ifvs):
     g.stage_times(reset=True)
     g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
-    # plan + filter; the bitmap scan and the sorted-copy scan (k = 10: the
-    # one-query kernel only; the two-query kernel runs for 64 < k <= 128)
-    assert t["filter"][1] == 2 and t["scan"][1] == 2
+    # plan + filter; the bitmap scan, the pairing of the sorted-copy queries,
+    # the two-query and the one-query sorted-copy scans, for every k
+    assert t["filter"][1] == 2 and t["scan"][1] == 4
     g.search(q, p, 100, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
-    assert t["scan"][1] == 3
+    assert t["scan"][1] == 4
+    g.search(q, p, 100, flags=ifvs.IFVS_F_STAGE_TIMING, pair_min_rows=-1)
+    t = g.stage_times(reset=True)
+    assert t["scan"][1] == 2
     g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING, list_max_ppm=NEVER)
     t = g.stage_times(reset=True)
     assert t["filter"][1] == 1 and t["scan"][1] == 1
@@ -211,6 +217,9 @@ def test_threshold_and_launch_counts(ifvs):
         with pytest.raises(ifvs.IfvsError) as e:
             g.search(q, p, 10, list_max_ppm=bad)
         assert e.value.code == ifvs.IFVS_ERR_ARG
+    with pytest.raises(ifvs.IfvsError) as e:
+        g.search(q, p, 10, pair_min_rows=-2)
+    assert e.value.code == ifvs.IFVS_ERR_ARG
 
 
 def _wide_pairs():
@@ -234,9 +243,10 @@ def _one_by_one(g, q, p, k, **kw):
 @pytest.mark.parametrize("k", [100, 128])
 def test_pair_kernel_equals_one_query_kernel(ifvs, orc, case, k):
     """The two-query kernel drops rows by a quantised lower bound and
-    rescores the rest exactly in the one-query loop's order, so a batch whose
-    queries pair up must return, bit for bit, what each query returns alone
-    (one query per CTA).  Table shapes: ordinary; one subspace 1000x wider
+    rescores the rest exactly in the one-query kernel's order, so a batch
+    whose queries pair up (pairing forced at this size) must return, bit for
+    bit, what each query returns alone and what the batch returns with no
+    pairs (one query per CTA, the one-query kernel).  Table shapes: ordinary; one subspace 1000x wider
     than the others (a loose bound: most rows rescored); every codeword of a
     subspace equal (a zero range: the test is off, all distances tie); a
     range of a few ulps; entries near 1e35."""
@@ -260,11 +270,11 @@ def test_pair_kernel_equals_one_query_kernel(ifvs, orc, case, k):
         q[:] = 1.0
     q[9] = q[8]                                    # a pair of identical vectors
     g.stage_times(reset=True)
-    a = g.search(q, p, k, flags=ifvs.IFVS_F_STAGE_TIMING)
-    assert g.stage_times(reset=True)["scan"][1] == 3   # bitmap, one-query and two-query kernels
-    b = _one_by_one(g, q, p, k)
-    for x, y in zip(a, b):
-        np.testing.assert_array_equal(x, y)
+    a = g.search(q, p, k, flags=ifvs.IFVS_F_STAGE_TIMING, pair_min_rows=1)
+    assert g.stage_times(reset=True)["scan"][1] == 4   # bitmap, pairing, two-query, one-query scans
+    for b in (_one_by_one(g, q, p, k, pair_min_rows=1), g.search(q, p, k, pair_min_rows=-1)):
+        for x, y in zip(a, b):
+            np.testing.assert_array_equal(x, y)
     if case != "huge":
         _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
 
@@ -278,13 +288,49 @@ def test_pair_kernel_with_conditioning(ifvs, orc):
     qs = synth.make_queries(ix, 1.0, nq=12)
     g = ifvs.Index(ix.codes, ix.attrs, D=w.D, K=w.K)
     g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
-    a = g.search(qs.q, qs.preds, 100, wz=qs.wz)
-    out = [g.search(qs.q[i:i + 1], qs.preds[i:i + 1], 100, wz=qs.wz[i:i + 1]) for i in range(12)]
+    a = g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=1)
+    b = g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=-1)
     for j in range(3):
-        np.testing.assert_array_equal(a[j], np.concatenate([o[j] for o in out]))
+        np.testing.assert_array_equal(a[j], b[j])
     oi, od, on, st = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q, qs.preds, 100, bank=cond.bank,
                                 W=cond.W, seeds=cond.seeds, wz=qs.wz, want_stages=True)
     np.testing.assert_array_equal(a[2], on)
     for i in range(12):
         all_d = orc.adc_all(st["lut"][i], ix.codes)
         check_topk(a[0][i], a[1][i], oi[i], od[i], all_d, np.ones(w.N, bool))
+
+
+@pytest.mark.parametrize("k", [10, 100, 200])
+def test_pairing_by_sorted_ranges(ifvs, orc, k):
+    """Ranges pair with the query whose range starts next to theirs
+    (queries sorted by column and range start, in segments of 2048; pairing
+    forced at this size): a batch of 2300 random windows (1 %, 10 % and 50 %
+    of the values, both columns) must give bit for bit the same per-query
+    results in a permuted order (other pairs form), with no pairs, and query
+    by query, and the oracle's top-k."""
+    N = 30011
+    g, codes, attrs, Cpq = _index(ifvs, N, seed=31)
+    rng = np.random.default_rng(32)
+    nq = 2300
+    p = synth.empty_predicates(nq)
+    for i in range(nq):
+        p[i]["n_clauses"] = 1
+        if i % 7 == 6:
+            lo = int(rng.integers(-20, 10))
+            synth.set_clause(p[i], 0, 1, synth.OP_RANGE, lo, lo + int(rng.integers(1, 12)))
+        else:
+            w = int(rng.choice([10, 100, 500]))
+            lo = int(rng.integers(-500, 500 - w + 1))
+            synth.set_clause(p[i], 0, 0, synth.OP_RANGE, lo, lo + w)
+    q = _queries(nq, Cpq.shape[0] * Cpq.shape[2], seed=33)
+    a = g.search(q, p, k, sub_batch=nq, pair_min_rows=1)
+    perm = rng.permutation(nq)
+    b = g.search(q[perm], p[perm], k, sub_batch=nq, pair_min_rows=1)
+    for x, y in zip(a, b):
+        np.testing.assert_array_equal(x[perm], y)
+    for x, y in zip(a, g.search(q, p, k, sub_batch=nq, pair_min_rows=-1)):
+        np.testing.assert_array_equal(x, y)
+    c = _one_by_one(g, q[:24], p[:24], k)
+    for x, y in zip(a, c):
+        np.testing.assert_array_equal(x[:24], y)
+    _check_oracle(orc, codes, attrs, Cpq, q[:64], p[:64], k, *(x[:64] for x in a))

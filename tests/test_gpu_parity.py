@@ -338,9 +338,9 @@ def test_stage_timing_counts_launches(ifvs):
     g.stage_times(reset=True)
     g.search(q, _preds(8, 0, 50), 10, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
-    # filter: the scan plan + the filter; scan: the bitmap kernel and the sorted
-    # copy's one-query kernel (k = 10)
-    expected = {"predicate": 1, "filter": 2, "condition": 1, "lut": 2, "scan": 2, "merge": 1}
+    # filter: the scan plan + the filter; scan: the bitmap kernel, the pairing
+    # of the sorted-copy queries, the two-query and one-query kernels (M = 16)
+    expected = {"predicate": 1, "filter": 2, "condition": 1, "lut": 2, "scan": 4, "merge": 1}
     for s, n in expected.items():
         assert t[s][1] == n and t[s][0] > 0.0
     assert t["rerank"][1] == 0
