@@ -492,18 +492,20 @@ def run_ifvs(args):
             "ms_per_batch": float(np.mean(ms_b)) if ms_b else None,
             "mean_selectivity": float(npass.mean() / w.N),
             "sorted_path_share": float(on_list.mean())}
-    # the scan stage (k_scan_list + k_scan, one launch of each per batch) is
-    # the unit: per-batch time from the stage events, per-batch bytes
+    # the scan stage (per batch: k_pair_items, k_scan_list_pair, k_scan_list
+    # and k_scan, one launch of each) is the unit: per-batch time from the
+    # stage events, per-batch bytes
     scan_ms, _ = stages["scan"]
     hbm_peak, peak_kind = measured_peaks()
     nbatch = args.steps
     achieved = (scan_bytes / nbatch) / (scan_ms / nbatch / 1000.0) / 1e9 if scan_ms > 0 else None
     traffic = scan_traffic()
-    roofline = {"kernel": "scan stage (k_scan_list + k_scan)", "bound": "hbm", "achieved": achieved,
+    roofline = {"kernel": "scan stage (k_scan_list_pair + k_scan_list + k_scan + k_pair_items)",
+                "bound": "hbm", "achieved": achieved,
                 "peak": hbm_peak,
                 "unit": "GB/s", "frac": achieved / hbm_peak if achieved else None,
                 "traffic": traffic, "peak_kind": peak_kind + " (hbm copy, burst)",
-                "launch_unit": "one batch of the scan stage (both kernels)",
+                "launch_unit": "one batch of the scan stage (its four kernels)",
                 "avg_launch_ms": scan_ms / nbatch,
                 "algorithmic_bytes_per_launch": scan_bytes / nbatch}
     share = {k: v[0] for k, v in stages.items()}
