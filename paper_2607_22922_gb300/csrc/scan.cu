@@ -671,9 +671,9 @@ k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __r
 
 // ---- two queries per CTA on the sorted copy --------------------------------
 //
-// When two consecutive queries both take the sorted copy of the same column
-// (M = 16), one CTA serves both, and one shared-memory load serves both
-// queries' look-ups.  A 64 KB table with the rows, replication and rotation
+// When k_pair_items (below) pairs two queries on the sorted copy of the same
+// column (M = 16), one CTA serves both, and one shared-memory load serves
+// both queries' look-ups.  A 64 KB table with the rows, replication and rotation
 // of the float32 one holds, in word w of codeword row c, the pair
 // qA[w mod 16][c] | qB[w mod 16][c] << 16 of 11-bit quantised entries,
 // q[m][c] = floor((LUT[m][c] - lo_m) * inv), lo_m the smallest entry of
@@ -807,11 +807,9 @@ constexpr uint32_t kCandA = 0x00008000u, kCandB = 0x80000000u;
 // slower at the 128-register cap of a 16-warp CTA)
 constexpr int kU2 = 4;
 
-// One round of kU2 positions of a block: quantised sums of both queries,
-// candidates by the packed bounds, exact distances and top-k offers for the
-// candidates.  mask[] holds kCandA / kCandB for the positions inside each
-// query's range; MASKED: it differs between positions (a cut block), so
-// only positions inside a range load codes.
+// Codes of a round's kU2 positions.  mask[] holds kCandA / kCandB for the
+// positions inside each query's range; MASKED: it differs between positions
+// (a cut block), so only positions inside a range load codes.
 template <bool MASKED>
 __device__ __forceinline__ void pair_load(const uint8_t* __restrict__ codes, uint32_t pos0,
                                           const uint32_t (&mask)[kU2], uint64_t keep, uint4 (&c)[kU2]) {
@@ -822,6 +820,9 @@ __device__ __forceinline__ void pair_load(const uint8_t* __restrict__ codes, uin
     }
 }
 
+// One round of kU2 positions of a block: the shared bounds refreshed,
+// quantised sums of both queries, candidates by the packed bounds, exact
+// distances and top-k offers for the candidates.
 template <int KP, bool FAST, bool MASKED>
 __device__ __forceinline__ void pair_round(const uint4 (&c)[kU2], const uint32_t* __restrict__ rows,
                                            uint32_t pos0, const uint32_t (&mask)[kU2], WarpTopK<KP>& tkA,
