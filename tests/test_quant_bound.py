@@ -47,16 +47,17 @@ def quantise(L, lo, inv):
     return np.floor(np.minimum(F(QMAX), np.maximum(F(0), y))).astype(np.int64)
 
 
-def quant_bound(thr, sl, inv):
-    """Vectorised over float32 thresholds; the kernel's quant_bound."""
+def quant_bound(thr, sl, inv, margin=2.0 ** -12):
+    """Vectorised over float32 thresholds; the kernel's quant_bound (margin:
+    the relative slack of each step, 2^-12 in the kernel)."""
     thr = np.asarray(thr, F)
     out = np.full(thr.shape, INT_MAX, np.int64)
     if inv == 0:
         return out
     with np.errstate(over="ignore", invalid="ignore"):
-        a = (thr * F(1 + 2.0 ** -12)).astype(F)
-        b = F(sl * F(1 - 2.0 ** -12))
-        t = ((a - b).astype(F) * F(inv * F(1 + 2.0 ** -12))).astype(F)
+        a = (thr * F(1 + margin)).astype(F)
+        b = F(sl * F(1 - margin))
+        t = ((a - b).astype(F) * F(inv * F(1 + margin))).astype(F)
     finite = thr.view(np.uint32) < 0x7F800000
     ok = finite & (t < F(1e9))
     out[ok] = np.where(t[ok] < 0, -1, np.floor(t[ok])).astype(np.int64)
@@ -159,3 +160,19 @@ def test_packed_candidate_test_equals_the_comparisons():
     diff = (tpk - sq).astype(np.uint32)     # wraps like the kernel's 32-bit subtract
     np.testing.assert_array_equal((diff & 0x8000) != 0, SA <= TA)
     np.testing.assert_array_equal((diff & 0x80000000) != 0, SB <= TB)
+
+
+def test_the_margins_are_needed():
+    """Without the 2^-12 slack the same replay drops rows that are within
+    their threshold (float32 rounding of the distance and of the
+    quantisation), so the checks above can tell a sound bound from an
+    unsound one."""
+    dropped = 0
+    for kind in ("tiny_range", "ulp_spaced"):
+        rng = np.random.default_rng(zlib.crc32(kind.encode()))
+        L = tables(kind, rng)
+        codes = rng.integers(0, 256, size=(60000, 16))
+        for rot in (0, 7, 15):
+            d, S, sl, inv = rows_of(L, codes, rot)
+            dropped += int((S > quant_bound(d, sl, inv, margin=0.0)).sum())
+    assert dropped > 0
