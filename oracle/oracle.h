@@ -35,10 +35,12 @@
  *     distance go to the smaller row id;
  *   - w_z absent means the paper's initial state w_f = 1 exactly.
  *
- * Parity status: every function here is pinned by tests/test_oracle_*.py
- * except orc_kmeans_pq's exact centroid values (parity unpinned: Lloyd's
- * iteration from a seeded start has no closed form; its objective and its
- * fixed points are pinned instead).
+ * Parity status: every function here is pinned by tests/test_oracle_*.py.
+ * orc_kmeans_pq's centroids after many iterations have no closed form from
+ * a general seeded start; they are pinned where one exists (one codeword:
+ * the mean; two well-separated groups: the group means; as many codewords
+ * as distinct points: zero error), and its objective is pinned to be
+ * non-increasing.
  */
 #ifndef IFVS_ORACLE_H
 #define IFVS_ORACLE_H

@@ -48,6 +48,10 @@ MUTATIONS = {
                                    "& 1u)) continue;\n        double s = 0.0;\n        for (int32_t d = 0; d < D; ++d) {\n            double diff = (double)q[d] - (double)X[i * D + d];\n            s += fabs(diff);"),
     "rerank distance not squared": ("if (i < 0 || i >= N) continue;\n        double s = 0.0;\n        for (int32_t d = 0; d < D; ++d) {\n            double diff = (double)q[d] - (double)X[i * D + d];\n            s += diff * diff;",
                                     "if (i < 0 || i >= N) continue;\n        double s = 0.0;\n        for (int32_t d = 0; d < D; ++d) {\n            double diff = (double)q[d] - (double)X[i * D + d];\n            s += fabs(diff);"),
+    "k-means update reads subspace 0": ("sum[(int64_t)assign[i] * ds + t] += (double)X[i * D + m * ds + t];",
+                                        "sum[(int64_t)assign[i] * ds + t] += (double)X[i * D + t];"),
+    "k-means assigns the farthest codeword": ("double d = sq_dist_sub(x, C + (int64_t)c * ds, ds);\n                    if (d < bd) {",
+                                              "double d = sq_dist_sub(x, C + (int64_t)c * ds, ds);\n                    if (d > bd) {"),
     "k-means mean off by one": ("C[(int64_t)c * ds + t] = sum[(int64_t)c * ds + t] / (double)cnt[c];",
                                 "C[(int64_t)c * ds + t] = sum[(int64_t)c * ds + t] / (double)(cnt[c] + 1);"),
     "encode ties to the larger codeword": ("            if (d < bd) {\n                    bd = d;\n                    best = c;\n                }\n            }\n            codes[i * M + m] = (uint8_t)best;\n        }\n}",

@@ -444,6 +444,45 @@ def test_kmeans_exact_when_codewords_cover_distinct_points(orc):
     assert obj[0, -1] == 0.0
 
 
+def test_kmeans_one_codeword_is_the_mean(orc):
+    """K = 1: whatever row seeds it, one Lloyd iteration moves the codeword
+    to the mean of the subspace's rows, and every later assignment costs the
+    total sum of squares about that mean (textbook closed forms)."""
+    rng = np.random.default_rng(31)
+    X = (3.0 + 2.0 * rng.standard_normal((257, 6))).astype(np.float32)
+    for seed in (0, 7, 123):
+        Cq, obj = orc.kmeans_pq(X, 3, 1, 4, seed)
+        x = X.astype(np.float64)
+        for m in range(3):
+            sub = x[:, 2 * m:2 * m + 2]
+            mean = sub.mean(axis=0)
+            np.testing.assert_allclose(Cq[m, 0], mean, rtol=1e-13, atol=0)
+            ss = ((sub - mean) ** 2).sum()
+            np.testing.assert_allclose(obj[m, 1:], ss, rtol=1e-12)
+            assert obj[m, 0] >= ss
+
+
+def test_kmeans_two_separated_groups_converge_to_the_group_means(orc):
+    """K = 2 on two groups far apart (spread 0.1, distance 100): from any
+    seeded start, including both seeds in one group, Lloyd's iteration ends
+    at the two group means, with the within-group sum of squares as its
+    objective."""
+    rng = np.random.default_rng(32)
+    a = (0.1 * rng.standard_normal((60, 2))).astype(np.float32)
+    b = (np.array([100.0, -50.0]) + 0.1 * rng.standard_normal((25, 2))).astype(np.float32)
+    X = np.concatenate([a, b])[rng.permutation(85)]
+    x = X.astype(np.float64)
+    ga = x[np.abs(x[:, 0]) < 50]
+    gb = x[np.abs(x[:, 0]) >= 50]
+    want = np.stack([ga.mean(axis=0), gb.mean(axis=0)])
+    ss = ((ga - ga.mean(axis=0)) ** 2).sum() + ((gb - gb.mean(axis=0)) ** 2).sum()
+    for seed in range(12):
+        Cq, obj = orc.kmeans_pq(X, 1, 2, 8, seed)
+        got = Cq[0][np.argsort(Cq[0][:, 0])]
+        np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-12)
+        np.testing.assert_allclose(obj[0, -1], ss, rtol=1e-12)
+
+
 def test_sdc_properties(orc):
     rng = np.random.default_rng(12)
     Cq = rng.standard_normal((3, 8, 2))
