@@ -38,6 +38,7 @@ if ROOT not in sys.path:
 
 WORKLOAD = "gmm100m-d128-m16"
 LIST_DEFAULT_PPM = 1000000   # the library's default sorted-copy threshold (always)
+PAIR_DEFAULT_ROWS = 1 << 22  # the library's default span from which ranges pair
 TRAIN_WORKLOAD = "sift1m-d128-m16"
 CPU_SAMPLE_ROWS = 10_000_000
 
@@ -51,7 +52,8 @@ def parse():
     ap.add_argument("--workload", default=None,
                     help="default: %s (search, pq), %s (train)" % (WORKLOAD, TRAIN_WORKLOAD))
     ap.add_argument("--rows", type=int, default=0, help="override N (smaller runs)")
-    ap.add_argument("--recall-queries", type=int, default=16, help="per bin; 0 = skip")
+    ap.add_argument("--sels", default="", help="override the selectivity bins, comma-separated fractions")
+    ap.add_argument("--recall-queries", type=int, default=64, help="per bin; 0 = skip")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--chunk-blocks", type=int, default=0, help="scan chunk size in 1024-row blocks (0 = auto)")
@@ -63,6 +65,8 @@ def parse():
     ap.add_argument("--pair-min-rows", type=int, default=0,
                     help="two-query CTAs for overlapping one-column ranges spanning at least this many "
                          "rows (0 = library default, -1 = never)")
+    ap.add_argument("--no-quads", action="store_true",
+                    help="group sorted-copy queries in pairs only (no four-query CTAs)")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
     ap.add_argument("--mode", default="search", choices=["search", "pq", "train"],
                     help="search: the query path; pq: PQ encoding + Lloyd training of the index; "
@@ -85,6 +89,8 @@ def workload(args):
     w = synth.WORKLOADS[name]
     if args.rows:
         w = synth.scaled(w, N=args.rows)
+    if args.sels:
+        w = synth.scaled(w, sels=tuple(float(x) for x in args.sels.split(",")))
     if w.batch <= 0:
         # workloads whose recipe names no batch size run 1024-query steps
         w = synth.scaled(w, batch=min(w.nq, 1024))
@@ -196,9 +202,9 @@ def measured_peaks():
     return 6800.0, "fallback"
 
 
-def kernel_traffic(summary, source):
-    """DRAM bytes per launch from a committed ncu summary, valid only while
-    the kernel's source file is unchanged."""
+def traffic_summary(summary, source):
+    """A committed ncu summary (profiles/), valid only while the kernel's
+    source file is unchanged; None otherwise."""
     p = os.path.join(ROOT, "profiles", summary)
     src = os.path.join(ROOT, "paper_2607_22922_gb300", "csrc", source)
     if not os.path.exists(p):
@@ -208,11 +214,76 @@ def kernel_traffic(summary, source):
     sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
     if d.get(source.replace(".", "_") + "_sha256") != sha:
         return None
-    return d.get("dram_bytes_per_launch")
+    return d
 
 
-def scan_traffic():
-    return kernel_traffic("scan_traffic.json", "scan.cu")
+def kernel_traffic(summary, source):
+    """DRAM bytes per launch from a committed ncu summary (or None)."""
+    d = traffic_summary(summary, source)
+    return None if d is None else d.get("dram_bytes_per_launch")
+
+
+def scan_dram(workload_name, hbm_peak):
+    """DRAM traffic of the scan stage per bin from the committed ncu summary
+    of this workload (bytes per batch and GB/s over the kernel time under
+    ncu, as a fraction of the measured HBM peak), or None."""
+    d = traffic_summary("scan_traffic.json", "scan.cu")
+    if d is None or d.get("workload_name") != workload_name:
+        return None
+    out = {"bytes_per_batch": d.get("dram_bytes_per_launch"), "source": "profiles/scan_traffic.json",
+           "how": d.get("how"), "bins": {}}
+    for sel, gb in d.get("per_bin_dram_GB", {}).items():
+        ms = d.get("per_bin_duration_ms_under_ncu", {}).get(sel)
+        gbs = gb / (ms / 1000.0) if ms else None
+        out["bins"][sel] = {"dram_GB": gb, "ms_under_ncu": ms, "GBps": gbs,
+                            "frac_of_hbm": gbs / hbm_peak if gbs and hbm_peak else None}
+    return out
+
+
+# ------------------------------------------------------------ index
+
+def build_index_gpu(w, device, ifvs, local):
+    """The workload's index built on the device with the library's PQ
+    kernels, in the paper's order (§1): raw vectors drawn from the stated
+    mixture block by block on the device (never on the host), a codebook
+    trained by ``w.pq_iters`` Lloyd iterations (ifvs_pq_train) on the first
+    ``w.pq_sample`` rows from synth's start codewords, and every row encoded
+    (ifvs_pq_encode).  Returns the synth.Index (host codes) and the seconds
+    spent."""
+    import torch
+    from paper_2607_22922_gb300 import synth
+    t0 = time.time()
+    dio = ifvs.IFVS_F_DEVICE_IO
+    # the library's calls run on torch's current stream, after the work that
+    # produces their inputs
+    sptr = torch.cuda.current_stream(device).cuda_stream
+    ct = torch.from_numpy(synth.mixture_centres(w)).to(device)
+    n_s = synth.pq_sample_rows(w)
+    block = 1 << 22
+    sample = torch.cat([synth.mixture_vectors_torch(w, ct, a, min(n_s, a + block), device)
+                        for a in range(0, n_s, block)])
+    C0 = torch.from_numpy(synth.pq_start_codebook(w, sample.cpu().numpy())).to(device)
+    C = torch.empty_like(C0)
+    ifvs.ifvs_pq_train(sample, C0, w.pq_iters, device=local, C_out=C, objective=None, flags=dio, stream=sptr)
+    del sample
+    codes = torch.empty((w.N, w.M), dtype=torch.uint8, device=device)
+    for a in range(0, w.N, block):
+        b = min(w.N, a + block)
+        x = synth.mixture_vectors_torch(w, ct, a, b, device)
+        ifvs.ifvs_pq_encode(x, C, device=local, codes=codes[a:b], flags=dio, stream=sptr)
+    torch.cuda.synchronize(device)
+    ix = synth.mixture_index(w, C.cpu().numpy(), codes.cpu().numpy(), source="mixture-torch")
+    del codes, ct
+    torch.cuda.empty_cache()
+    return ix, time.time() - t0
+
+
+def device_vectors(w, ix, a, b, device, centres_t=None):
+    """Raw vectors of rows [a, b) of a device-built index (one 2^22 block)."""
+    import torch
+    from paper_2607_22922_gb300 import synth
+    ct = centres_t if centres_t is not None else torch.from_numpy(ix.centres).to(device)
+    return synth.mixture_vectors_torch(w, ct, a, b, device)
 
 
 # ------------------------------------------------------------ CPU baseline
@@ -328,7 +399,7 @@ def exact_topk_gpu(w, ix, q, preds, k, device):
     import torch
     from paper_2607_22922_gb300 import synth
     block = 1 << 22
-    cb = torch.from_numpy(ix.codebook).to(device)
+    ct = torch.from_numpy(ix.centres).to(device)
     qs_all = torch.from_numpy(np.ascontiguousarray(q)).to(device).double()
     nq = qs_all.shape[0]
     best_d = torch.full((nq, k), float("inf"), dtype=torch.float64, device=device)
@@ -336,7 +407,7 @@ def exact_topk_gpu(w, ix, q, preds, k, device):
     qn = (qs_all * qs_all).sum(1, keepdim=True)
     for s in range(0, w.N, block):
         e = min(w.N, s + block)
-        x = synth.raw_vectors_torch(ix, s, e, device, cb).double()
+        x = device_vectors(w, ix, s, e, device, ct).double()
         d = qn + (x * x).sum(1)[None, :] - 2.0 * qs_all @ x.T
         cols = [torch.from_numpy(a[s:e].astype(np.int64)).to(device) for a in ix.attrs]
         ok = _pass_mask(cols, preds, device)
@@ -374,6 +445,65 @@ def recall_at_k(w, ix, batches, ids_by_bin, nsample, device):
     return out
 
 
+def scan_lookups(w, qs, sorted_vals, on_list, npass, pair_rows, quads=True, seg=2048):
+    """Shared-memory look-ups the scan stage executes for one batch, by the
+    library's grouping rule for one-column ranges of the sorted copy (M = 16;
+    sort by (column, range start, query) per 2048-query segment; an aligned
+    run of four sorted neighbours whose union spans at least pair_rows
+    positions and whose every range covers 3/4 of the union forms a
+    four-query group (k <= 128); otherwise neighbours 2j, 2j+1 pair when 3/4
+    of the longer range is common and the two span at least pair_rows): a
+    group costs the union of its ranges x M (one load serves all its
+    queries), any other query its pool x M."""
+    n = len(qs.q)
+    a = np.zeros(n, np.int64)
+    b = np.zeros(n, np.int64)
+    col = np.zeros(n, np.int64)
+    for i in range(n):
+        if on_list[i]:
+            c = qs.preds[i]["c"][0]
+            col[i] = c["col"]
+            v = sorted_vals[col[i]]
+            a[i] = np.searchsorted(v, c["lo"], "left")
+            b[i] = np.searchsorted(v, c["hi"], "left")
+    grouped = np.zeros(n, bool)
+    in_quad = np.zeros(n, bool)
+    union = 0.0
+
+    def pair_ok(x, y):
+        lx, ly = b[x] - a[x], b[y] - a[y]
+        if col[x] != col[y] or lx <= 0 or ly <= 0:
+            return False
+        common = min(b[x], b[y]) - max(a[x], a[y])
+        span = max(b[x], b[y]) - min(a[x], a[y])
+        return 4 * common >= 3 * max(lx, ly) and span >= pair_rows
+
+    def quad_ok(g):
+        if any(col[x] != col[g[0]] or b[x] <= a[x] for x in g):
+            return False
+        lo, hi = min(a[x] for x in g), max(b[x] for x in g)
+        return hi - lo >= pair_rows and all(4 * (b[x] - a[x]) >= 3 * (hi - lo) for x in g)
+
+    if w.M == 16 and pair_rows >= 0:
+        for s0 in range(0, n, seg):
+            idx = [i for i in range(s0, min(n, s0 + seg)) if on_list[i]]
+            idx.sort(key=lambda i: (col[i], a[i], i))
+            for r in range(0, len(idx), 4):
+                g = idx[r:r + 4]
+                if quads and w.k <= 128 and len(g) == 4 and quad_ok(g):
+                    grouped[g] = in_quad[g] = True
+                    union += max(b[x] for x in g) - min(a[x] for x in g)
+                    continue
+                for j in (0, 2):
+                    if j + 1 < len(g) and pair_ok(g[j], g[j + 1]):
+                        x, y = g[j], g[j + 1]
+                        grouped[x] = grouped[y] = True
+                        union += max(b[x], b[y]) - min(a[x], a[y])
+    single = float(npass[~grouped].sum())
+    return {"lookups": (single + union) * w.M, "grouped_share": float(grouped.mean()),
+            "quad_share": float(in_quad.mean())}
+
+
 # ------------------------------------------------------------ arms
 
 def run_ifvs(args):
@@ -393,7 +523,7 @@ def run_ifvs(args):
 
     w = workload(args)
     t0 = time.time()
-    ix = synth.make_index(w)
+    ix, t_pq = build_index_gpu(w, device, ifvs, local)
     cond = synth.make_conditioning(ix)
     batches = [synth.make_queries(ix, s, nq=w.batch, salt=rank) for s in w.sels]
     t_gen = time.time() - t0
@@ -401,15 +531,15 @@ def run_ifvs(args):
     if args.rerank > 0:
         # the raw vectors, drawn on the device block by block, go into the
         # index for the exact rerank (device I/O load: nothing on the host)
-        cbt = torch.from_numpy(ix.codebook).to(device)
+        ct = torch.from_numpy(ix.centres).to(device)
         vecs = torch.empty((w.N, w.D), dtype=torch.float32, device=device)
         for s0 in range(0, w.N, 1 << 22):
             s1 = min(w.N, s0 + (1 << 22))
-            vecs[s0:s1] = synth.raw_vectors_torch(ix, s0, s1, device, cbt)
+            vecs[s0:s1] = device_vectors(w, ix, s0, s1, device, ct)
         g = ifvs.Index(torch.from_numpy(ix.codes).to(device),
                        [torch.from_numpy(a).to(device) for a in ix.attrs], vectors=vecs, D=w.D,
                        device=local, K=w.K, device_io=True)
-        del vecs, cbt
+        del vecs, ct
         torch.cuda.empty_cache()
     else:
         g = ifvs.Index(ix.codes, ix.attrs, device=local)
@@ -429,7 +559,7 @@ def run_ifvs(args):
                         torch.empty((n, w.k), dtype=torch.float32, device=device),
                         torch.empty(n, dtype=torch.int64, device=device)))
     torch.cuda.synchronize()
-    flags = ifvs.IFVS_F_DEVICE_IO | ifvs.IFVS_F_STAGE_TIMING
+    flags = ifvs.IFVS_F_DEVICE_IO | ifvs.IFVS_F_STAGE_TIMING | (ifvs.IFVS_F_NO_QUADS if args.no_quads else 0)
 
     def step(i):
         b = i % nb
@@ -470,44 +600,58 @@ def run_ifvs(args):
     stages = g.stage_times(reset=True)
     launches = sum(v[1] for v in stages.values())
 
-    # per-bin figures and the scan-stage roofline.  Algorithmic bytes per
-    # query: the passing rows' codes, plus the lane-major bitmap on the bitmap
-    # path (the sorted-copy path of one-column predicates reads no bitmap; the
-    # row ids it loads for top-k candidates only are not counted)
+    # per-bin figures and the scan-stage roofline
     per_bin = {}
     n_blocks = (w.N + 1023) // 1024
     ppm = args.list_max_ppm if args.list_max_ppm != 0 else LIST_DEFAULT_PPM
     list_rows = -1 if ppm < 0 else w.N * ppm // 1000000
-    scan_bytes = 0.0
+    pair_rows = args.pair_min_rows if args.pair_min_rows != 0 else PAIR_DEFAULT_ROWS
+    lookups_total = code_bytes_total = 0.0
+    sorted_vals = [np.sort(a) for a in ix.attrs]
     for b, qs in enumerate(batches):
         ms_b = [step_ms[i] for i in range(args.steps) if (args.warmup + i) % nb == b]
         npass = dev_out[b][2].cpu().numpy().astype(np.float64)
         nsteps_b = len(ms_b)
         one_col = (qs.preds["n_clauses"] == 1) if not w.conjunctive else np.zeros(len(npass), bool)
         on_list = one_col & (npass <= list_rows)
-        per_q = npass * w.M + np.where(on_list, 0.0, n_blocks * 128.0)
-        scan_bytes += nsteps_b * float(per_q.sum())
+        lk = scan_lookups(w, qs, sorted_vals, on_list, npass, pair_rows, quads=not args.no_quads)
+        lookups_total += nsteps_b * lk["lookups"]
+        code_bytes_total += nsteps_b * float(npass.sum()) * w.M
         per_bin[str(qs.sel)] = {
             "qps": (len(qs.q) * nsteps_b) / (sum(ms_b) / 1000.0) if ms_b else None,
             "ms_per_batch": float(np.mean(ms_b)) if ms_b else None,
             "mean_selectivity": float(npass.mean() / w.N),
-            "sorted_path_share": float(on_list.mean())}
-    # the scan stage (per batch: k_pair_items, k_scan_list_pair, k_scan_list
-    # and k_scan, one launch of each) is the unit: per-batch time from the
-    # stage events, per-batch bytes
+            "sorted_path_share": float(on_list.mean()),
+            "grouped_share": lk["grouped_share"], "quad_share": lk["quad_share"]}
+    # The scan stage (per batch: k_pair_items, k_scan_list_pair, k_scan_list
+    # and k_scan, one launch of each) is the unit.  Its binding resource is
+    # the shared-memory look-up rate: one conflict-free 32-lane load per SM
+    # per cycle.  Executed look-ups per batch: passing positions x M for a
+    # query scanned alone, and for a pair of queries the positions of the
+    # union of their ranges x M (one load serves both).  Code bytes (every
+    # query's pool once) are reported beside it: DRAM carries far less,
+    # because the CTAs of a batch share the codes through L2.
     scan_ms, _ = stages["scan"]
-    hbm_peak, peak_kind = measured_peaks()
     nbatch = args.steps
-    achieved = (scan_bytes / nbatch) / (scan_ms / nbatch / 1000.0) / 1e9 if scan_ms > 0 else None
-    traffic = scan_traffic()
-    roofline = {"kernel": "scan stage (k_scan_list_pair + k_scan_list + k_scan + k_pair_items)",
-                "bound": "hbm", "achieved": achieved,
-                "peak": hbm_peak,
-                "unit": "GB/s", "frac": achieved / hbm_peak if achieved else None,
-                "traffic": traffic, "peak_kind": peak_kind + " (hbm copy, burst)",
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    mhz = (clk or {}).get("sm_mhz") or (clk or {}).get("sm_max_mhz") or 2070.0
+    peak = sms * 32 * mhz * 1e6
+    achieved = (lookups_total / nbatch) / (scan_ms / nbatch / 1000.0) if scan_ms > 0 else None
+    hbm_peak, peak_kind = measured_peaks()
+    dram = scan_dram(w.name, hbm_peak)
+    roofline = {"kernel": "scan stage (k_group_items + k_scan_list_quad + k_scan_list_pair + k_scan_list"
+                          " + k_scan)",
+                "bound": "smem", "achieved": achieved, "peak": peak, "unit": "look-ups/s",
+                "frac": achieved / peak if achieved else None,
+                "traffic": dram["bytes_per_batch"] if dram else None,
+                "peak_kind": "derived: %d SMs x 32 lanes x %.0f MHz (median SM clock under load; one "
+                             "conflict-free 32-lane shared load per SM per cycle)" % (sms, mhz),
                 "launch_unit": "one batch of the scan stage (its four kernels)",
                 "avg_launch_ms": scan_ms / nbatch,
-                "algorithmic_bytes_per_launch": scan_bytes / nbatch}
+                "lookups_per_launch": lookups_total / nbatch,
+                "code_bytes_per_launch": code_bytes_total / nbatch,
+                "code_bytes_per_s": (code_bytes_total / nbatch) / (scan_ms / nbatch / 1000.0) if scan_ms > 0 else None,
+                "dram": dram, "hbm_peak_gbs": hbm_peak, "hbm_peak_kind": peak_kind}
     share = {k: v[0] for k, v in stages.items()}
 
     # end to end through the C ABI with pinned host buffers
@@ -531,7 +675,8 @@ def run_ifvs(args):
             oi, od, on, _ = host_out[b]
             ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr,
                                    chunk_blocks=args.chunk_blocks, list_max_ppm=args.list_max_ppm,
-                                   rerank=args.rerank, pair_min_rows=args.pair_min_rows)
+                                   rerank=args.rerank, pair_min_rows=args.pair_min_rows,
+                                   flags=ifvs.IFVS_F_NO_QUADS if args.no_quads else 0)
 
         for i in range(args.warmup):
             hstep(i)
@@ -577,7 +722,7 @@ def run_ifvs(args):
                          % (w.N * w.M / 1e9, w.N * 4 / 1e9)},
         "bins": per_bin, "roofline": roofline, "stage_ms": share, "gpu_launches": launches,
         "clocks": clk, "e2e": e2e, "cpu_baseline": cpu, "cpu_baseline_parallel": cpu_par,
-        "setup_s": round(t_gen, 1), "index_load_s": round(t_load, 1),
+        "setup_s": round(t_gen, 1), "index_build_s": round(t_pq, 1), "index_load_s": round(t_load, 1),
     }
     if rank == 0:
         s = json.dumps(line)
@@ -611,19 +756,26 @@ def run_pq(args):
     w = workload(args)
     rows = min(args.pq_rows, w.N)
     t0 = time.time()
-    ix = synth.make_index(synth.scaled(w, N=rows))
-    cb = torch.from_numpy(ix.codebook).to(device)
+    # raw vectors of the workload's mixture (drawn on the device) and the
+    # codebook the workload's recipe trains on its first pq_sample rows
+    ct = torch.from_numpy(synth.mixture_centres(w)).to(device)
     block = 1 << 22
     X = torch.empty((rows, w.D), dtype=torch.float32, device=device)
     for s0 in range(0, rows, block):
         s1 = min(rows, s0 + block)
-        X[s0:s1] = synth.raw_vectors_torch(ix, s0, s1, device, cb)
+        X[s0:s1] = synth.mixture_vectors_torch(w, ct, s0, s1, device)
     codes = torch.empty((rows, w.M), dtype=torch.uint8, device=device)
-    torch.cuda.synchronize()
-    t_gen = time.time() - t0
     stream = torch.cuda.Stream(device=device)
     sptr = stream.cuda_stream
     dio = ifvs.IFVS_F_DEVICE_IO
+    n_s = min(synth.pq_sample_rows(w), rows)
+    cb = torch.empty((w.M, w.K, w.ds), dtype=torch.float32, device=device)
+    ifvs.ifvs_pq_train(X[:n_s], torch.from_numpy(synth.pq_start_codebook(w, X[:n_s].cpu().numpy())).to(device),
+                       w.pq_iters, device=local, C_out=cb, objective=None, flags=dio,
+                       stream=torch.cuda.current_stream(device).cuda_stream)
+    torch.cuda.synchronize()
+    codebook_host = cb.cpu().numpy()
+    t_gen = time.time() - t0
 
     def step():
         ifvs.ifvs_pq_encode(X, cb, device=local, codes=codes, flags=dio, stream=sptr)
@@ -692,12 +844,12 @@ def run_pq(args):
     if not args.no_e2e:
         hX = X.cpu().pin_memory()
         hXn = hX.numpy()
-        ifvs.ifvs_pq_encode(hXn, ix.codebook, device=local)
+        ifvs.ifvs_pq_encode(hXn, codebook_host, device=local)
         barrier(dist, device)
         torch.cuda.synchronize()
         t1 = time.perf_counter()
         for _ in range(args.steps):
-            ifvs.ifvs_pq_encode(hXn, ix.codebook, device=local)
+            ifvs.ifvs_pq_encode(hXn, codebook_host, device=local)
         e_ms = (time.perf_counter() - t1) * 1000.0
         barrier(dist, device)
         e_ms = reduce_max(dist, e_ms, device)
@@ -715,7 +867,7 @@ def run_pq(args):
         t1 = time.perf_counter()
         done = 0
         while time.perf_counter() - t1 < 10.0:
-            oracle.pq_encode_f32(Xs, ix.codebook)
+            oracle.pq_encode_f32(Xs, codebook_host)
             done += sample
         sec = time.perf_counter() - t1
         cpu = {"value": done / sec, "unit": "rows/s", "cores": 1, "kind": "oracle",
@@ -767,7 +919,7 @@ def run_train(args):
     w = workload(args)
     P, n_neg = w.k, args.train_neg
     t0 = time.time()
-    ix = synth.make_index(w)
+    ix, _ = build_index_gpu(w, device, ifvs, local)
     cond = synth.make_conditioning(ix)
     batches = [synth.make_queries(ix, s, nq=w.batch, salt=rank) for s in w.sels]
     gts = [exact_topk_gpu(w, ix, b.q, b.preds, P, device) for b in batches]
@@ -916,37 +1068,56 @@ def run_train(args):
 
 
 def run_reference(args):
-    """The oracle as it stands on the host cores, each step one query of the
-    next bin over the first CPU_SAMPLE_ROWS rows, time scaled by N / rows."""
+    """The oracle as it stands on the host cores, over every row of the
+    workload: each step runs one query per worker process (one worker per
+    core, a spawn pool), the queries cycling through the bins.  The index is
+    built by the oracle too (oracle.pq_index: the workload's mixture, Lloyd
+    training on its first pq_sample rows, float32 encoding of every row),
+    outside the timed region; no GPU is used."""
     world, rank, _ = dist_env()
     if rank != 0:
         return
+    import concurrent.futures as cf
+    import multiprocessing as mp
     from paper_2607_22922_gb300 import synth
     import oracle
+    from oracle import pq_index
     oracle.build()
     w = workload(args)
-    rows = min(CPU_SAMPLE_ROWS, w.N)
-    ws = synth.scaled(w, N=rows)        # the same rows as the first `rows` of the workload
-    ix = synth.make_index(ws)
+    cores = os.cpu_count() or 1
+    t0 = time.time()
+    oix = pq_index.OracleIndex(w, workers=cores)
+    t_build = time.time() - t0
+    ix = oix.ix
     cond = synth.make_conditioning(ix)
-    batches = [synth.make_queries(ix, s, nq=8) for s in w.sels]
-    scale = w.N / rows
+    nb = len(w.sels)
+    per_bin = max(1, -(-(args.steps + args.warmup) * cores // nb))
+    batches = [synth.make_queries(ix, s, nq=min(per_bin, max(w.batch, 1)), salt=rank) for s in w.sels]
 
-    def step(i):
-        qs = batches[i % len(batches)]
-        j = (i // len(batches)) % len(qs.q)
-        oracle.search(ix.codes, ix.attrs, ix.codebook, qs.q[j:j + 1], qs.preds[j:j + 1], w.k,
-                      bank=cond.bank, W=cond.W, seeds=cond.seeds, wz=qs.wz[j:j + 1])
+    def tasks(i):
+        out = []
+        for c in range(cores):
+            j = i * cores + c
+            qs = batches[j % nb]
+            r = (j // nb) % len(qs.q)
+            out.append((oix.paths, cond.bank, cond.W, cond.seeds, qs.q[r:r + 1], qs.preds[r:r + 1],
+                        qs.wz[r:r + 1], w.k, None))
+        return out
 
-    for i in range(args.warmup):
-        step(i)
-    t0 = time.perf_counter()
-    for i in range(args.steps):
-        step(args.warmup + i)
-    sec = (time.perf_counter() - t0) * scale
-    value = args.steps / sec
-    sample = ("1 query per step cycling through the %d bins, over the first %d of %d rows; "
-              "time scaled by N/rows" % (len(batches), rows, w.N))
+    try:
+        with cf.ProcessPoolExecutor(max_workers=cores, mp_context=mp.get_context("spawn")) as pool:
+            for i in range(args.warmup):
+                list(pool.map(pq_index._search_task, tasks(i)))
+            t0 = time.perf_counter()
+            for i in range(args.steps):
+                list(pool.map(pq_index._search_task, tasks(args.warmup + i)))
+            sec = time.perf_counter() - t0
+    finally:
+        oix.close()
+    value = args.steps * cores / sec
+    sample = ("%d queries per step (one per worker process, %d processes) cycling through the %d bins, "
+              "each over all %d rows; index built by the oracle in %.0f s before timing"
+              % (cores, cores, nb, w.N, t_build))
     line = {
         "impl": "reference",
         "metric": "QPS at recall@%d per selectivity bin (code-scan HBM GB/s vs peak)" % w.k,
@@ -954,8 +1125,8 @@ def run_reference(args):
         "warmup": args.warmup, "ms_per_step": sec * 1000.0 / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": {"workload": w.name, "N": w.N, "k": w.k,
-                                        "batch": 1, "bins": list(w.sels)},
-        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": 1, "kind": "oracle",
+                                        "batch": cores, "bins": list(w.sels)},
+        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": cores, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},

@@ -56,6 +56,13 @@ typedef enum {
     IFVS_ERR_UNSUPPORTED = -5   /* shape outside the supported range          */
 } ifvs_status;
 
+/* Every entry point that allocates device memory returns IFVS_ERR_OOM when
+ * an allocation fails, frees what the call had allocated, and leaves the
+ * index as it was (later calls may succeed).  For tests of that path the
+ * failure can be injected on the host: while the environment variable
+ * IFVS_FAIL_ALLOC holds a number n >= 1, the n-th device allocation since
+ * the variable took its current string fails without calling cudaMalloc. */
+
 /* Clause operators (Listing 1 uses = and >; all are intervals on integers):
  *   EQ    a == lo        RANGE lo <= a < hi     GE  a >= lo
  *   LT    a <  lo        GT    a >  lo          LE  a <= lo
@@ -88,6 +95,8 @@ typedef struct {
                                      on the launching stream (ifvs_stage_times) */
 #define IFVS_F_PLAIN_PQ     0x4u  /* ignore the memory bank: Delta = 0 (plain PQ
                                      ADC, baseline Pre_IndexPQ_ADC of §3.2)   */
+#define IFVS_F_NO_QUADS     0x8u  /* search: group sorted-copy queries in pairs
+                                     only, never in fours (pair_min_rows)     */
 
 typedef struct {
     uint32_t flags;     /* IFVS_F_*                                            */
@@ -108,14 +117,16 @@ typedef struct {
                            (1000000: always); -1: never.  The two paths sum a row's entries in
                            different orders, so distances agree to float32
                            rounding.                                          */
-    int32_t pair_min_rows; /* M = 16 sorted-copy scan: two queries on the same
-                           column whose ranges share 3/4 of the longer one and
-                           together span at least this many rows share a CTA
-                           and one shared-memory look-up per code byte (their
-                           tables quantised to 11 bits, every row that can
-                           reach a top-k rescored exactly, so results equal
-                           those of one query per CTA bit for bit).
-                           0: default (4194304); -1: never pair.             */
+    int32_t pair_min_rows; /* M = 16 sorted-copy scan: queries on the same
+                           column whose ranges together span at least this
+                           many rows share a CTA and one shared-memory look-up
+                           per code byte: four neighbours (by range start)
+                           each covering 3/4 of their union (tables quantised
+                           to 5 bits, k <= 128), else two sharing 3/4 of the
+                           longer range (11 bits); every row that can reach a
+                           top-k is rescored exactly, so results equal those
+                           of one query per CTA bit for bit.
+                           0: default (4194304); -1: never group.            */
     void* stream;       /* cudaStream_t to run on; NULL: the index's stream   */
 } ifvs_search_params;
 
@@ -247,9 +258,13 @@ int ifvs_scan_topk(ifvs_index* ix, const float* lut, const uint32_t* bitmaps, in
  * Sizes beyond it (one query's lane-major bitmap, N / 8 bytes rounded up to
  * 128-byte blocks, plus its 64 KB scan table (160 KB for M > 33) and k keys,
  * above the array) return
- * IFVS_ERR_UNSUPPORTED.  The first call on a device looks up the array's
- * device address (cudaGetSymbolAddress); make that first call before any
- * stream capture.  All calls share the array: calls whose work overlaps on
+ * IFVS_ERR_UNSUPPORTED, and so does a k whose scan needs more shared memory
+ * than the device offers (as in ifvs_scan_topk).  Every call looks up the
+ * array's device address on the index's device (cudaGetSymbolAddress, a
+ * host-side query), so a context torn down and created again
+ * (cudaDeviceReset) is followed; the first call on a device also loads the
+ * library's module there: make it before any stream capture.  All calls
+ * share the array: calls whose work overlaps on
  * the GPU (different streams, or threads without ordering) race.  No
  * cudaMalloc, cudaFree or allocating library routine is called.
  */
@@ -266,6 +281,28 @@ int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uint32_t* bitm
 int ifvs_rerank(ifvs_index* ix, const float* queries, const int64_t* cand, int64_t nq,
                 int32_t R, int32_t k, const ifvs_search_params* p, int64_t* ids,
                 float* dists);
+
+/*
+ * ifvs_merge_topk — Select (§2, stage 3) across row shards.  The paper has
+ * one device; when an index is split into G row shards (rows [r_g, r_g+1)
+ * on shard g, searched separately, ids offset by r_g), the k best of each
+ * shard are gathered and this call keeps the k smallest by (dist, id) of the
+ * G k entries of each query — the same ids and distances as one search over
+ * all rows.
+ *   dists   [G][nq][k] float32 per-shard distances (the layout of an
+ *           all-gather of each shard's [nq][k] result)
+ *   ids     [G][nq][k] int64 global row ids; -1 marks padding (sorted last)
+ *   dists_out, ids_out  [nq][k] out; padded with (+inf, -1) where the
+ *           shards return fewer than k rows in all
+ *   flags   IFVS_F_DEVICE_IO: all arrays are device pointers on `device`
+ *   stream  cudaStream_t for the work, or NULL (a stream of the call's own)
+ * Shards must hold disjoint rows.  With IFVS_F_DEVICE_IO and a non-NULL
+ * stream the call allocates nothing and only enqueues one kernel.  Errors:
+ * IFVS_ERR_ARG (NULL, nq < 0, G < 1, k outside 1..IFVS_MAX_K, unknown flag),
+ * IFVS_ERR_UNSUPPORTED (G k above 4096), IFVS_ERR_OOM, IFVS_ERR_CUDA.
+ */
+int ifvs_merge_topk(int32_t device, const float* dists, const int64_t* ids, int64_t nq, int32_t G,
+                    int32_t k, float* dists_out, int64_t* ids_out, uint32_t flags, void* stream);
 
 /*
  * ifvs_pq_encode — PQ encoding of raw vectors (the offline step before the

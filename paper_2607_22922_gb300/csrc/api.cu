@@ -5,7 +5,11 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <stdlib.h>
+
 #include <algorithm>
+#include <mutex>
+#include <string>
 #include <new>
 #include <utility>
 #include <cmath>
@@ -45,6 +49,36 @@ int cuda_fail(cudaError_t e, const char* what, int line) {
         if (rc_ != 0) return rc_; \
     } while (0)
 
+// Every device allocation of the library goes through device_malloc.
+// Failure injection for tests of the error path (no GPU fault involved):
+// while the environment variable IFVS_FAIL_ALLOC holds a number n >= 1,
+// the n-th device allocation counted since the variable took its current
+// value fails as if the device were out of memory (no cudaMalloc is called
+// for it); the count restarts whenever the variable's string changes (so
+// "1" and then "01" each fail the next allocation) or is unset.
+cudaError_t device_malloc(void** p, size_t bytes) {
+    static std::mutex mu;
+    static std::string last;
+    static long count = 0;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        const char* v = getenv("IFVS_FAIL_ALLOC");
+        const std::string cur = v ? v : "";
+        if (cur != last) {
+            last = cur;
+            count = 0;
+        }
+        if (!cur.empty()) {
+            const long n = strtol(cur.c_str(), nullptr, 10);
+            if (n >= 1 && ++count == n) {
+                *p = nullptr;
+                return cudaErrorMemoryAllocation;
+            }
+        }
+    }
+    return cudaMalloc(p, bytes);
+}
+
 struct DevBuf {
     void* p = nullptr;
     size_t cap = 0;
@@ -57,11 +91,11 @@ int ensure(DevBuf& b, size_t bytes) {
     if (b.p) cudaFree(b.p);
     b.p = nullptr;
     b.cap = 0;
-    cudaError_t e = cudaMalloc(&b.p, bytes);
+    cudaError_t e = device_malloc(&b.p, bytes);
     if (e != cudaSuccess) {
         cudaGetLastError();
         b.p = nullptr;
-        return set_err(IFVS_ERR_OOM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+        return set_err(IFVS_ERR_OOM, "device allocation of %zu bytes failed: %s", bytes, cudaGetErrorString(e));
     }
     b.cap = bytes;
     return 0;
@@ -201,11 +235,11 @@ void free_index(ifvs_index* ix) {
 }
 
 int dev_alloc(ifvs_index* ix, void** p, size_t bytes) {
-    cudaError_t e = cudaMalloc(p, bytes ? bytes : 16);
+    cudaError_t e = device_malloc(p, bytes ? bytes : 16);
     if (e != cudaSuccess) {
         cudaGetLastError();
         *p = nullptr;
-        return set_err(IFVS_ERR_OOM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+        return set_err(IFVS_ERR_OOM, "device allocation of %zu bytes failed: %s", bytes, cudaGetErrorString(e));
     }
     ix->bytes += bytes;
     return 0;
@@ -302,7 +336,7 @@ struct Stage {
 };
 
 struct Opts {
-    bool dio = false, timing = false, plain = false;
+    bool dio = false, timing = false, plain = false, no_quads = false;
     int R = 0;
     int64_t sub_batch = 0;
     int64_t chunk_blocks = 0;
@@ -325,7 +359,7 @@ constexpr int64_t kPairDefaultMinRows = int64_t(1) << 22;
 
 int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (!p) return 0;
-    if (p->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING | IFVS_F_PLAIN_PQ))
+    if (p->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING | IFVS_F_PLAIN_PQ | IFVS_F_NO_QUADS))
         return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", p->flags);
     if (p->chunk_blocks < 0) return set_err(IFVS_ERR_ARG, "chunk_blocks must be >= 0");
     if (p->rerank < 0 || p->rerank > IFVS_MAX_K)
@@ -337,6 +371,7 @@ int parse_opts(const ifvs_search_params* p, Opts* o) {
     o->dio = p->flags & IFVS_F_DEVICE_IO;
     o->timing = p->flags & IFVS_F_STAGE_TIMING;
     o->plain = p->flags & IFVS_F_PLAIN_PQ;
+    o->no_quads = p->flags & IFVS_F_NO_QUADS;
     o->R = p->rerank;
     o->sub_batch = p->sub_batch;
     o->chunk_blocks = p->chunk_blocks;
@@ -396,8 +431,16 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
     const int kk = o.R > 0 ? o.R : k;
     const int Mr = ix->M * ix->r;
     const bool cond = !o.plain && ix->d_bank != nullptr;
+    // Which queries take the bitmap path is decided on the device (k_plan),
+    // but with the sorted-copy path on for every pool size and one attribute
+    // column none can: every predicate then constrains at most that column.
+    // Such batches need no bitmap workspace (N / 8 bytes per query) and no
+    // filter or bitmap-scan launch.
+    const bool list_on = o.list_max_ppm >= 0 && ix->n_attrs > 0;
+    const int64_t ppm = o.list_max_ppm > 0 ? o.list_max_ppm : kListDefaultPpm;
+    const bool bitmaps = !(list_on && ppm >= 1000000 && ix->n_attrs == 1);
     TRY(ensure(ix->w_canon, sizeof(CanonPred) * n));
-    TRY(ensure(ix->w_bm, (size_t)n * ix->n_blocks * 32 * 4));
+    if (bitmaps) TRY(ensure(ix->w_bm, (size_t)n * ix->n_blocks * 32 * 4));
     TRY(ensure(ix->w_idx, sizeof(uint32_t) * n * (ix->h > 0 ? ix->h : 1)));
     TRY(ensure(ix->w_alpha, sizeof(float) * n * (Mr > 0 ? Mr : 1)));
     TRY(ensure(ix->w_wf, sizeof(float) * n * ix->D));
@@ -417,17 +460,16 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
     }
     // one-column predicates take the sorted-copy scan (up to the threshold)
     const ScanPlan* plan = nullptr;
-    if (o.list_max_ppm >= 0 && ix->n_attrs > 0) {
-        const int64_t ppm = o.list_max_ppm > 0 ? o.list_max_ppm : kListDefaultPpm;
+    if (list_on) {
         const int64_t max_rows = ppm >= 1000000 ? ix->N : ix->N * ppm / 1000000;
         TRY(ensure(ix->w_plan, sizeof(ScanPlan) * n));
-        TRY(ensure(ix->w_items, (sizeof(PairItem) + 1) * n));   // pairs, then a pair flag per query
+        TRY(ensure(ix->w_items, scan_list_workspace_bytes(n)));   // query groups of the sorted-copy scan
         Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);
         CUDA_TRY(st.end(launch_plan(ix->w_canon.as<CanonPred>(), n, ix->sorted(), ix->N, max_rows,
                                     ix->w_plan.as<ScanPlan>(), npass_u64, s)));
         plan = ix->w_plan.as<ScanPlan>();
     }
-    {
+    if (bitmaps) {
         Stage st(ix, s, o.timing, IFVS_STAGE_FILTER);
         CUDA_TRY(st.end(launch_filter(ix->cols(), ix->N, ix->n_blocks, ix->w_canon.as<CanonPred>(),
                                       plan, n, ix->w_bm.as<uint32_t>(), npass_u64, ix->num_sms, s)));
@@ -450,7 +492,7 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
         CUDA_TRY(st.end(launch_tables(ix->w_lut.as<float>(), n, ix->M, ix->K, ix->tab_words,
                                       ix->w_tab.as<float>(), s)));
     }
-    {
+    if (bitmaps) {
         Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
         CUDA_TRY(st.end(launch_scan(ix->d_codes, ix->w_tab.as<float>(), ix->w_bm.as<uint32_t>(), plan,
                                     n, kk, sh, ix->w_part.as<uint64_t>(), s)));
@@ -461,8 +503,8 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
         const int64_t pmin = o.pair_min_rows > 0 ? o.pair_min_rows : kPairDefaultMinRows;
         const cudaError_t e = launch_scan_list(ix->w_tab.as<float>(), ix->sorted(), plan, n, kk, sh,
                                                ix->w_part.as<uint64_t>(),
-                                               o.pair_min_rows < 0 ? nullptr : ix->w_items.as<PairItem>(),
-                                               pmin, s, &nl);
+                                               o.pair_min_rows < 0 ? nullptr : ix->w_items.as<uint8_t>(),
+                                               pmin, !o.no_quads, s, &nl);
         CUDA_TRY(st.end(e, nl));
     }
     int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;
@@ -715,6 +757,7 @@ int ifvs::index_view(const ifvs_index* ix, IndexView* out) {
     if (!ix) return set_err(IFVS_ERR_ARG, "index is NULL");
     out->device = ix->device;
     out->num_sms = ix->num_sms;
+    out->max_smem = ix->max_smem;
     out->N = ix->N;
     out->n_blocks = ix->n_blocks;
     out->M = ix->M;
@@ -1201,11 +1244,11 @@ struct PqArgs {
         if (s && own_stream) cudaStreamDestroy(s);
     }
     int alloc(void** p, size_t bytes) {
-        cudaError_t e = cudaMalloc(p, bytes ? bytes : 16);
+        cudaError_t e = device_malloc(p, bytes ? bytes : 16);
         if (e != cudaSuccess) {
             cudaGetLastError();
             *p = nullptr;
-            return set_err(IFVS_ERR_OOM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+            return set_err(IFVS_ERR_OOM, "device allocation of %zu bytes failed: %s", bytes, cudaGetErrorString(e));
         }
         owned.push_back(*p);
         return 0;
@@ -1252,6 +1295,54 @@ int pq_check(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, in
 }
 
 }  // namespace
+
+extern "C" int ifvs_merge_topk(int32_t device, const float* dists, const int64_t* ids, int64_t nq, int32_t G,
+                               int32_t k, float* dists_out, int64_t* ids_out, uint32_t flags, void* stream) {
+    if (nq < 0) return set_err(IFVS_ERR_ARG, "nq < 0");
+    if (G < 1) return set_err(IFVS_ERR_ARG, "G = %d < 1", G);
+    if (k < 1 || k > IFVS_MAX_K) return set_err(IFVS_ERR_ARG, "k = %d outside 1..%d", k, IFVS_MAX_K);
+    if ((int64_t)G * k > shard_merge_cap())
+        return set_err(IFVS_ERR_UNSUPPORTED, "G x k = %lld above %d", (long long)G * k, shard_merge_cap());
+    if (flags & ~IFVS_F_DEVICE_IO) return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", flags);
+    if (nq == 0) return IFVS_OK;
+    if (!dists || !ids || !dists_out || !ids_out) return set_err(IFVS_ERR_ARG, "an array argument is NULL");
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) {
+        cudaGetLastError();
+        return set_err(IFVS_ERR_CUDA, "no CUDA device is available");
+    }
+    if (device < 0 || device >= ndev) return set_err(IFVS_ERR_ARG, "device %d outside 0..%d", device, ndev - 1);
+    DeviceGuard g(device);
+    PqArgs a;
+    a.device = device;
+    if (stream) {
+        a.s = (cudaStream_t)stream;
+    } else {
+        CUDA_TRY(cudaStreamCreateWithFlags(&a.s, cudaStreamNonBlocking));
+        a.own_stream = true;
+    }
+    const bool dio = flags & IFVS_F_DEVICE_IO;
+    const size_t n_in = (size_t)G * nq * k, n_out = (size_t)nq * k;
+    const void *dd, *di;
+    TRY(a.input(dists, sizeof(float) * n_in, dio, &dd));
+    TRY(a.input(ids, sizeof(int64_t) * n_in, dio, &di));
+    float* od = dists_out;
+    int64_t* oi = ids_out;
+    if (!dio) {
+        void* p;
+        TRY(a.alloc(&p, sizeof(float) * n_out));
+        od = (float*)p;
+        TRY(a.alloc(&p, sizeof(int64_t) * n_out));
+        oi = (int64_t*)p;
+    }
+    CUDA_TRY(launch_merge_shards((const float*)dd, (const int64_t*)di, nq, G, k, od, oi, a.s));
+    if (!dio) {
+        CUDA_TRY(cudaMemcpyAsync(dists_out, od, sizeof(float) * n_out, cudaMemcpyDeviceToHost, a.s));
+        CUDA_TRY(cudaMemcpyAsync(ids_out, oi, sizeof(int64_t) * n_out, cudaMemcpyDeviceToHost, a.s));
+    }
+    if (a.own_stream || !dio) CUDA_TRY(cudaStreamSynchronize(a.s));
+    return IFVS_OK;
+}
 
 extern "C" int ifvs_pq_encode(int32_t device, const float* X, int64_t n, int32_t D, int32_t M,
                               int32_t K, const float* C_pq, uint8_t* codes, float* dmin,

@@ -37,7 +37,9 @@ cudaError_t launch_canonicalize(const ifvs_predicate* preds, int64_t nq, AttrCol
 // rows sorted by (value, row): two binary searches give it, and its length
 // is the exact pool size.  Pools up to max_rows take the row-list scan (no
 // filter pass, no bitmap); empty and malformed predicates take it with an
-// empty segment; every other query takes the bitmap path.
+// empty segment, and a predicate that constrains no column (every row
+// passes) takes it with all N positions of column 0's copy; every other
+// query takes the bitmap path.
 __device__ __forceinline__ int64_t first_not_below(const int32_t* __restrict__ v, int64_t n, int64_t x) {
     int64_t lo = 0, hi = n;
     while (lo < hi) {
@@ -63,6 +65,11 @@ __global__ void k_plan(const CanonPred* __restrict__ canon, int64_t nq, SortedCo
     p.list = 0;
     if (cp.empty) {
         p.list = 1;
+    } else if (cp.used == 0u) {
+        if (sc.n > 0 && sc.vals_of(0) != nullptr && N <= max_rows) {
+            p.b = N;
+            p.list = 1;
+        }
     } else if (__popc(cp.used) == 1) {
         const int c = __ffs(cp.used) - 1;
         const int32_t* vals = sc.vals_of(c);

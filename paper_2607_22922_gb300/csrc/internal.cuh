@@ -195,16 +195,21 @@ cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* 
 struct PairItem {
     int32_t qa, qb;
 };
+struct QuadItem {
+    int32_t q[4];
+};
 // the list-path queries of `plan`: their pool is the position range [a, b)
 // of a column's sorted copy (same grid and partial layout as launch_scan).
-// For M = 16, `items` (workspace: nq PairItems followed by nq bytes)
-// receives the pairs of overlapping ranges that together span at least
-// pair_min_rows positions, which a two-query kernel serves; a one-query
-// kernel serves the other queries (all of them when items is null or
-// M != 16).  *launches = kernels launched.
+// For M = 16, `work` (scan_list_workspace_bytes(nq) bytes) receives the
+// groups of overlapping ranges that together span at least pair_min_rows
+// positions: runs of four (served by a four-query kernel, when `quads`)
+// and pairs (a two-query kernel); a one-query kernel serves the other
+// queries (all of them when work is null or M != 16).  *launches = kernels
+// launched.
+size_t scan_list_workspace_bytes(int64_t nq);
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
-                             const ScanShape& sh, uint64_t* partials, PairItem* items, int64_t pair_min_rows,
-                             cudaStream_t s, int* launches);
+                             const ScanShape& sh, uint64_t* partials, uint8_t* work, int64_t pair_min_rows,
+                             bool quads, cudaStream_t s, int* launches);
 // the sorted copy of the codes: dst position p <- row rows[p] of the index
 // layout `src`, re-rotated by (p mod 32) mod M; positions >= N are zero
 cudaError_t launch_relayout_sorted(const uint8_t* src, const uint32_t* rows, int64_t N, int M,
@@ -213,6 +218,10 @@ cudaError_t launch_relayout_sorted(const uint8_t* src, const uint32_t* rows, int
 cudaError_t launch_merge(const uint64_t* partials, int64_t nq, int n_lists, int k,
                          int64_t* ids, float* dists, cudaStream_t s);
 // exact fp32 rerank of cand [nq][R] -> k best
+// Select across row shards: [G][nq][k] (dist, global id) -> [nq][k]
+int shard_merge_cap();
+cudaError_t launch_merge_shards(const float* dists, const int64_t* ids, int64_t nq, int G, int k,
+                                float* dists_out, int64_t* ids_out, cudaStream_t s);
 cudaError_t launch_rerank(const float* X, int64_t N, int D, const float* q, const int64_t* cand,
                           int64_t nq, int R, int k, int64_t* ids, float* dists, cudaStream_t s);
 // codes [N][M] -> rotated rows [n_rows_pad][row_bytes]; *bad = 1 if a code >= K
@@ -287,6 +296,7 @@ cudaError_t launch_sgd(float* theta, const float* g, int64_t n, float lr, cudaSt
 struct IndexView {
     int device;
     int num_sms;
+    int max_smem;  // opt-in shared memory per block on `device`, bytes
     int64_t N, n_blocks;
     int M, K, row_bytes, tab_words;
     const uint8_t* codes;

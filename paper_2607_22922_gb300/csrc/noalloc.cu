@@ -10,8 +10,11 @@
 // the library's kernels are loaded holds IFVS_STATIC_SCRATCH_BYTES of it
 // until the process exits.  Host code must not pass `g_scan_scratch` itself
 // to a kernel (on the host that name is only a stand-in for the symbol);
-// its device address comes from cudaGetSymbolAddress, taken once per device
-// with that device current, on the first call on that device.
+// its device address comes from cudaGetSymbolAddress with the index's
+// device current.  Every call repeats that host-side lookup instead of
+// caching it, so a context that was torn down and created again
+// (cudaDeviceReset) never leaves a stale address behind; the first call on
+// a device also loads the library's module there.
 //
 // Every call reuses the same array and leaves the last call's contents in
 // it.  Within one call every scratch byte is written before it is read (the
@@ -19,37 +22,24 @@
 // so nothing needs clearing; two calls whose work overlaps on the GPU (on
 // different streams, or from different threads without ordering) race on
 // the array.
-#include <mutex>
-
 #include "internal.cuh"
 
 namespace ifvs {
 namespace {
 
 constexpr size_t kScratchBytes = (size_t)IFVS_STATIC_SCRATCH_BYTES;
-constexpr int kMaxDevices = 64;
-
 __device__ __align__(256) unsigned char g_scan_scratch[kScratchBytes];
 
-std::mutex g_mu;
-void* g_scratch_addr[kMaxDevices] = {nullptr};
-
-// Device address of g_scan_scratch on `dev` (the current device).
-int scratch_address(int dev, unsigned char** out) {
-    std::lock_guard<std::mutex> lock(g_mu);
-    if (dev < 0 || dev >= kMaxDevices)
-        return report_error(IFVS_ERR_UNSUPPORTED, "device ordinal %d above %d", dev, kMaxDevices - 1);
-    if (g_scratch_addr[dev] == nullptr) {
-        void* p = nullptr;
-        cudaError_t e = cudaGetSymbolAddress(&p, g_scan_scratch);
-        if (e != cudaSuccess || p == nullptr) {
-            cudaGetLastError();
-            return report_error(IFVS_ERR_CUDA, "cudaGetSymbolAddress(scratch) failed: %s",
-                                cudaGetErrorString(e));
-        }
-        g_scratch_addr[dev] = p;
+// Device address of g_scan_scratch on the current device.
+int scratch_address(unsigned char** out) {
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_scan_scratch);
+    if (e != cudaSuccess || p == nullptr) {
+        cudaGetLastError();
+        return report_error(IFVS_ERR_CUDA, "cudaGetSymbolAddress(scratch) failed: %s",
+                            cudaGetErrorString(e));
     }
-    *out = static_cast<unsigned char*>(g_scratch_addr[dev]);
+    *out = static_cast<unsigned char*>(p);
     return 0;
 }
 
@@ -90,6 +80,11 @@ extern "C" int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uin
     if (rc != 0) return rc;
     if (nq < 0) return report_error(IFVS_ERR_ARG, "nq < 0");
     if (k < 1 || k > IFVS_MAX_K) return report_error(IFVS_ERR_ARG, "k = %d outside 1..%d", k, IFVS_MAX_K);
+    // the scan CTA's shared memory for this k and table stride, as in ifvs_scan_topk
+    if (scan_smem_bytes(v.tab_words, scan_kp(k)) > (size_t)v.max_smem)
+        return report_error(IFVS_ERR_UNSUPPORTED,
+                            "k = %d with M = %d needs %zu bytes of shared memory per CTA (device: %d)",
+                            k, v.M, scan_smem_bytes(v.tab_words, scan_kp(k)), v.max_smem);
     if (nq == 0) return IFVS_OK;
     if (!lut || !bitmaps || !ids || !dists) return report_error(IFVS_ERR_ARG, "an array argument is NULL");
     // one query must fit: its lane-major bitmap, its table and one list of k keys
@@ -106,18 +101,17 @@ extern "C" int ifvs_scan_topk_static(ifvs_index* ix, const float* lut, const uin
     }
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     unsigned char* base = nullptr;
-    rc = scratch_address(v.device, &base);
+    rc = scratch_address(&base);
     const int64_t wrows = (v.N + 31) / 32;
     const size_t lut_n = (size_t)v.M * v.K;
-    // largest sub-batch whose bitmaps and lists fit the scratch
+    // largest sub-batch (halving from nq) whose bitmaps, tables and lists fit
+    // the scratch with the allocating path's chunk split
     int64_t sb = nq;
     while (rc == 0 && sb > 1 && footprint(v, sb, chunks_for(v, sb, k), k) > kScratchBytes) sb = (sb + 1) / 2;
-    if (rc == 0 && footprint(v, sb, chunks_for(v, sb, k), k) > kScratchBytes) {
-        // a single query with the many-chunk split does not fit: use fewer chunks
-        sb = 1;
-    }
     for (int64_t q0 = 0; rc == 0 && q0 < nq; q0 += sb) {
         const int64_t n = sb < nq - q0 ? sb : nq - q0;
+        // where even one query's lists with that split overflow, use fewer
+        // chunks (one chunk always fits: checked above)
         int64_t chunks = chunks_for(v, n, k);
         while (chunks > 1 && footprint(v, n, chunks, k) > kScratchBytes) chunks = (chunks + 1) / 2;
         uint32_t* bm = reinterpret_cast<uint32_t*>(base);

@@ -19,7 +19,7 @@ LIB_PATH = os.path.join(_HERE, "libifvs.so")
 IFVS_OK, IFVS_ERR_ARG, IFVS_ERR_OOM, IFVS_ERR_CUDA, IFVS_ERR_STATE, IFVS_ERR_UNSUPPORTED = 0, -1, -2, -3, -4, -5
 IFVS_OP_EQ, IFVS_OP_RANGE, IFVS_OP_GE, IFVS_OP_LT, IFVS_OP_GT, IFVS_OP_LE = 0, 1, 2, 3, 4, 5
 IFVS_ATTR_I32, IFVS_ATTR_I16 = 0, 1
-IFVS_F_DEVICE_IO, IFVS_F_STAGE_TIMING, IFVS_F_PLAIN_PQ = 0x1, 0x2, 0x4
+IFVS_F_DEVICE_IO, IFVS_F_STAGE_TIMING, IFVS_F_PLAIN_PQ, IFVS_F_NO_QUADS = 0x1, 0x2, 0x4, 0x8
 IFVS_MAX_K, IFVS_MAX_M, IFVS_MAX_ATTRS, IFVS_N_STAGES = 256, 128, 4, 9
 STAGES = ("predicate", "filter", "condition", "lut", "scan", "merge", "rerank", "layout", "train")
 
@@ -62,6 +62,7 @@ def _load():
         "ifvs_rerank": (C.c_int, [P, P, P, I64, I32, I32, P, P, P]),
         "ifvs_scan_topk_static": (C.c_int, [P, P, P, I64, I32, P, P, P]),
         "ifvs_pq_encode": (C.c_int, [I32, P, I64, I32, I32, I32, P, P, P, U32, P]),
+        "ifvs_merge_topk": (C.c_int, [I32, P, P, I64, I32, I32, P, P, U32, P]),
         "ifvs_pq_train": (C.c_int, [I32, P, I64, I32, I32, I32, I32, P, P, P, U32, P]),
         "ifvs_train_grad": (C.c_int, [P, P, P, I64, P, P, P, P, P, P, P]),
         "ifvs_train_step": (C.c_int, [P, P, P, I64, P, P, P, P, P]),
@@ -253,6 +254,28 @@ def ifvs_scan_topk_static(ix, lut, bitmaps, k, ids, dists, stream=None):
     _check(_lib.ifvs_scan_topk_static(ix, _ptr(lut), _ptr(bitmaps), nq, k, stream, _ptr(ids),
                                       _ptr(dists)))
     return ids, dists
+
+
+def ifvs_merge_topk(dists, ids, k=None, device=0, dists_out=None, ids_out=None, flags=0, stream=None):
+    """Select across row shards: dists [G][nq][k] float32 and ids [G][nq][k]
+    int64 (global row ids, -1 = padding) -> the k smallest by (dist, id) per
+    query, [nq][k] each.  Host mode (default): numpy in, numpy out; with
+    IFVS_F_DEVICE_IO every array is a device tensor (outputs preallocated)."""
+    dio = bool(flags & IFVS_F_DEVICE_IO)
+    G, nq, kk = (int(v) for v in dists.shape)
+    k = kk if k is None else k
+    if k != kk or tuple(ids.shape) != (G, nq, kk):
+        raise ValueError("dists and ids must both be [G][nq][k]")
+    if not dio:
+        dists = _host(dists, np.float32)
+        ids = _host(ids, np.int64)
+        dists_out = np.empty((nq, k), np.float32)
+        ids_out = np.empty((nq, k), np.int64)
+    elif dists_out is None or ids_out is None:
+        raise ValueError("device I/O needs preallocated outputs")
+    _check(_lib.ifvs_merge_topk(device, _ptr(dists), _ptr(ids), nq, G, k, _ptr(dists_out), _ptr(ids_out),
+                                flags, stream))
+    return ids_out, dists_out
 
 
 def ifvs_pq_encode(X, C_pq, device=0, want_dmin=False, codes=None, dmin=None, flags=0,

@@ -1,20 +1,27 @@
 """Seeded synthetic workloads for the iFVS query path (inputs only).
 
-This module draws the inputs of the query path — a PQ index (codebook and
-uint8 codes), attribute columns, queries with predicates at a target
+This module draws the inputs of the query path and nothing else: raw
+vectors from the stated mixtures, the rows and start codewords of the PQ
+training sample, attribute columns, queries with predicates at a target
 selectivity, the conditioning parameters (memory bank, W, hash seeds) and
-per-query w_z — and nothing else.  It holds none of the method's arithmetic:
-no distances, no look-up tables, no filtering, no top-k.  The oracle and the
-GPU path both read what it returns.
+per-query w_z.  It holds none of the method's arithmetic: no k-means, no
+encoding, no distances, no look-up tables, no filtering, no top-k.
 
 The paper measures on SIFT1M / SIFT10M with a 16 x 8 PQ (§3.1, §3.2) and
 trained conditioning weights; neither the datasets nor the weights exist
-here, so every workload below is drawn from a seeded mixture with the same
-shapes.  The index is generated in PQ space: per-subspace codewords are drawn
-around mixture centres, every mixture component has a prototype code, a row
-keeps each prototype code with probability 1 - rho and otherwise takes a
-uniform codeword, and the row's raw vector is its reconstruction plus
-residual noise (raw vectors are only drawn when a test needs exact L2).
+here, so every workload is drawn from a seeded mixture with the stated
+shapes.  A workload index is built in the paper's order (§1, PQ
+background): raw vectors x = post(centre[c] + sigma * n) with c uniform over
+the mixture's components and n standard normal; a PQ codebook trained by
+Lloyd iterations per subspace on the first ``pq_sample`` rows, started from
+K distinct sample rows; every row encoded as the argmin codeword per
+subspace.  The two PQ steps are not done here: the test suite runs them
+with the oracle (``oracle.pq_index``), the benchmark with the library's
+own PQ kernels; ``Index`` holds the result.
+
+``pq_space_index`` is a second, cheaper generator for shape and edge-case
+tests (any M, K, N, including N < K): codes drawn directly in PQ space
+around prototype codes.  No workload measurement uses it.
 """
 from __future__ import annotations
 
@@ -57,16 +64,27 @@ class Workload:
     sels: tuple
     batch: int = 0             # queries per search call (0 = all)
     conjunctive: bool = False  # category = c AND date range
-    rho: float = 0.5           # probability that a row leaves its prototype code
+    rho: float = 0.5           # pq_space_index only: probability that a row leaves its prototype code
     B: int = 4096              # memory-bank rows
     h: int = 2                 # hash functions
     r: int = 8                 # adjustment rank
     seed: int = 0x1F5
+    pq_sample: int = 65_536    # rows of the PQ training sample (the first rows)
+    pq_iters: int = 25         # Lloyd iterations of the PQ training
 
     @property
     def ds(self) -> int:
         return self.D // self.M
 
+    @property
+    def sigma(self) -> float:
+        """Per-coordinate standard deviation of a component around its
+        centre, before post-processing (0.3 is stated for the Gaussian
+        mixture; the other kinds take a comparable spread in their units)."""
+        return SIGMA[self.kind]
+
+
+SIGMA = {"gauss": 0.3, "sift": 12.0, "gist": 0.01, "deep": 0.03}
 
 WORKLOADS = {
     "gmm10k-d128-m16": Workload(
@@ -100,21 +118,19 @@ def scaled(w: Workload, N: int | None = None, nq: int | None = None, **kw) -> Wo
     return dataclasses.replace(w, **d)
 
 
-# ------------------------------------------------------------------ index
+# ---------------------------------------------------------------- mixtures
 
-@dataclasses.dataclass
-class Index:
-    w: Workload
-    codebook: np.ndarray        # [M][K][ds] float32
-    codes: np.ndarray           # [N][M] uint8
-    attrs: list                 # list of int32 / int16 arrays of length N
-    cluster: np.ndarray         # [N] int32 mixture component of each row
-    prototypes: np.ndarray      # [clusters][M] uint8
-    centres: np.ndarray         # [clusters][D] float32
-    noise_sigma: float
+# Rows are drawn in blocks of BLOCK rows, each from its own seeded stream,
+# so that any row range can be drawn (in parallel, or on the device) without
+# drawing the rows before it.
+BLOCK = 1 << 16
 
 
-def _centres(w: Workload, rng) -> np.ndarray:
+def mixture_centres(w: Workload) -> np.ndarray:
+    """[clusters][D] float32 component centres, by kind: Gaussian N(0, 1);
+    SIFT-like non-negative values N(30, 25) clipped to [0, 255]; GIST-like
+    |N(0, 1)| scaled to unit norm; Deep-like N(0, 1) scaled to unit norm."""
+    rng = np.random.default_rng([w.seed, 10])
     if w.kind == "gauss":
         c = rng.standard_normal((w.clusters, w.D))
     elif w.kind == "sift":
@@ -130,28 +146,152 @@ def _centres(w: Workload, rng) -> np.ndarray:
     return c.astype(np.float32)
 
 
-def _spread(w: Workload) -> tuple:
-    """(codeword jitter, residual noise) per kind, in data units."""
-    return {"gauss": (0.3, 0.15), "sift": (12.0, 6.0), "gist": (0.01, 0.006),
-            "deep": (0.03, 0.015)}[w.kind]
+def mixture_clusters(w: Workload, start: int = 0, stop: int | None = None) -> np.ndarray:
+    """[stop - start] int32: the mixture component of each row (uniform)."""
+    stop = w.N if stop is None else stop
+    out = np.empty(stop - start, dtype=np.int32)
+    for b0 in range(start - start % BLOCK, stop, BLOCK):
+        rng = np.random.default_rng([w.seed, 11, b0 // BLOCK])
+        cl = rng.integers(0, w.clusters, size=BLOCK, dtype=np.int32)
+        a, b = max(b0, start), min(b0 + BLOCK, stop)
+        out[a - start:b - start] = cl[a - b0:b - b0]
+    return out
 
 
-def _post(w: Workload, x: np.ndarray) -> np.ndarray:
-    if w.kind == "sift":
+def post_process(kind: str, x: np.ndarray) -> np.ndarray:
+    """The kind's value domain: SIFT-like rounded to integers and clipped to
+    [0, 255]; GIST-like made non-negative and scaled to unit norm; Deep-like
+    scaled to unit norm; Gaussian unchanged."""
+    if kind == "sift":
         return np.clip(np.rint(x), 0.0, 255.0).astype(np.float32)
-    if w.kind == "gist":
+    if kind == "gist":
         x = np.abs(x)
         return (x / np.maximum(np.linalg.norm(x, axis=-1, keepdims=True), 1e-12)).astype(np.float32)
-    if w.kind == "deep":
+    if kind == "deep":
         return (x / np.maximum(np.linalg.norm(x, axis=-1, keepdims=True), 1e-12)).astype(np.float32)
     return x.astype(np.float32)
 
 
-def make_index(w: Workload, chunk: int = 4_000_000) -> Index:
-    """Codebook, codes, attribute columns (deterministic in ``w.seed``)."""
+def mixture_vectors(w: Workload, centres: np.ndarray, start: int = 0,
+                    stop: int | None = None) -> np.ndarray:
+    """[stop - start][D] float32 raw vectors of rows [start, stop):
+    post(centre[cluster] + sigma * n), n ~ N(0, I), drawn per BLOCK rows."""
+    stop = w.N if stop is None else stop
+    out = np.empty((stop - start, w.D), dtype=np.float32)
+    for b0 in range(start - start % BLOCK, stop, BLOCK):
+        a, b = max(b0, start), min(b0 + BLOCK, stop)
+        cl = mixture_clusters(w, a, b)
+        rng = np.random.default_rng([w.seed, 12, b0 // BLOCK])
+        n = rng.standard_normal((BLOCK, w.D), dtype=np.float32)[a - b0:b - b0]
+        out[a - start:b - start] = post_process(w.kind, centres[cl] + np.float32(w.sigma) * n)
+    return out
+
+
+def mixture_vectors_torch(w: Workload, centres_t, start: int, stop: int, device):
+    """Raw vectors of rows [start, stop) drawn on a torch device, for
+    datasets too large for the host: the same recipe as ``mixture_vectors``
+    (same components per row) with torch's generator for the noise, seeded
+    per 2^22-row block; rows must lie in one such block.  Not the same
+    numbers as ``mixture_vectors``: an index is built from one of the two."""
+    import torch
+    block = 1 << 22
+    if start // block != (stop - 1) // block:
+        raise ValueError("rows must lie in one 2^22-row block")
+    cl = torch.from_numpy(mixture_clusters(w, start, stop).astype(np.int64)).to(device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(w.seed) * 1_000_003 + 7 + start // block)
+    noise = torch.randn((block, w.D), generator=gen, device=device, dtype=torch.float32)
+    off = start % block
+    x = centres_t[cl] + float(w.sigma) * noise[off:off + (stop - start)]
+    if w.kind == "sift":
+        x = torch.clamp(torch.round(x), 0.0, 255.0)
+    elif w.kind == "gist":
+        x = x.abs()
+        x = x / x.norm(dim=1, keepdim=True).clamp_min(1e-12)
+    elif w.kind == "deep":
+        x = x / x.norm(dim=1, keepdim=True).clamp_min(1e-12)
+    return x
+
+
+def pq_sample_rows(w: Workload) -> int:
+    """Rows of the PQ training sample: the first min(N, pq_sample) rows (the
+    rows are independent draws, so these are a uniform sample)."""
+    return min(w.N, w.pq_sample)
+
+
+def pq_start_rows(w: Workload, n_sample: int) -> np.ndarray:
+    """K distinct rows of the training sample whose sub-vectors are the
+    start codewords of every subspace (seeded; n_sample >= K)."""
+    if n_sample < w.K:
+        raise ValueError("the PQ training sample needs at least K = %d rows" % w.K)
+    return np.random.default_rng([w.seed, 13]).choice(n_sample, size=w.K, replace=False)
+
+
+def pq_start_codebook(w: Workload, sample: np.ndarray) -> np.ndarray:
+    """[M][K][ds] float32 start codewords: subspace m of codeword j is
+    dimensions [m ds, (m+1) ds) of sample row pq_start_rows[j]."""
+    rows = sample[pq_start_rows(w, sample.shape[0])]
+    return np.ascontiguousarray(rows.reshape(w.K, w.M, w.ds).transpose(1, 0, 2), dtype=np.float32)
+
+
+def attributes(w: Workload, cluster: np.ndarray) -> list:
+    """The attribute columns: uniform int32, cluster-correlated int32
+    (cluster * 10 + U[0, 10)), Zipf(1.1) int16 category."""
+    attrs = []
+    for ai, spec in enumerate(w.attrs):
+        arng = np.random.default_rng([w.seed, 2, ai])
+        if spec.kind == "uniform":
+            a = arng.integers(spec.lo, spec.hi, size=w.N, dtype=np.int64)
+        elif spec.kind == "cluster10":
+            a = cluster.astype(np.int64) * 10 + arng.integers(0, 10, size=w.N)
+        elif spec.kind == "zipf":
+            p = zipf_probs(spec.hi - spec.lo, spec.zipf_s)
+            a = spec.lo + arng.choice(len(p), size=w.N, p=p)
+        else:
+            raise ValueError(spec.kind)
+        attrs.append(a.astype(np.int16 if spec.dtype == "int16" else np.int32))
+    return attrs
+
+
+def zipf_probs(n: int, s: float) -> np.ndarray:
+    """P(value v) ∝ (v + 1)^-s for v in [0, n) (value 0 is the most common)."""
+    p = 1.0 / np.arange(1, n + 1, dtype=np.float64) ** s
+    return p / p.sum()
+
+
+# ------------------------------------------------------------------ index
+
+@dataclasses.dataclass
+class Index:
+    w: Workload
+    codebook: np.ndarray        # [M][K][ds] float32
+    codes: np.ndarray           # [N][M] uint8
+    attrs: list                 # list of int32 / int16 arrays of length N
+    cluster: np.ndarray         # [N] int32 mixture component of each row
+    centres: np.ndarray         # [clusters][D] float32
+    source: str                 # "mixture" (numpy rows), "mixture-torch" (device rows), "pq_space"
+    prototypes: np.ndarray | None = None   # pq_space only: [clusters][M] uint8
+    noise_sigma: float = 0.0               # pq_space only: residual noise
+
+
+def mixture_index(w: Workload, codebook: np.ndarray, codes: np.ndarray,
+                  source: str = "mixture") -> Index:
+    """An Index of the mixture recipe from a trained codebook and the codes
+    of every row (built by the caller: the oracle in tests, the library's PQ
+    kernels in the benchmark)."""
+    cluster = mixture_clusters(w)
+    return Index(w, np.ascontiguousarray(codebook, np.float32), codes, attributes(w, cluster),
+                 cluster, mixture_centres(w), source)
+
+
+def pq_space_index(w: Workload, chunk: int = 4_000_000) -> Index:
+    """Shape and edge-case generator: codewords drawn around mixture centres,
+    every component has a prototype code, a row keeps each prototype code
+    with probability 1 - rho and otherwise takes a uniform codeword; the
+    row's raw vector is its reconstruction plus residual noise."""
     rng = np.random.default_rng(w.seed)
-    centres = _centres(w, rng)
-    jitter, noise = _spread(w)
+    centres = mixture_centres(w)
+    jitter, noise = w.sigma, 0.5 * w.sigma
     owner = rng.integers(0, w.clusters, size=(w.M, w.K))
     cb = np.empty((w.M, w.K, w.ds), dtype=np.float32)
     for m in range(w.M):
@@ -174,35 +314,20 @@ def make_index(w: Workload, chunk: int = 4_000_000) -> Index:
         rnd = crng.integers(0, w.K, size=(e - s, w.M), dtype=np.uint8)
         codes[s:e] = np.where(keep, prototypes[cl], rnd)
         cluster[s:e] = cl
-
-    attrs = []
-    for ai, spec in enumerate(w.attrs):
-        arng = np.random.default_rng([w.seed, 2, ai])
-        if spec.kind == "uniform":
-            a = arng.integers(spec.lo, spec.hi, size=w.N, dtype=np.int64)
-        elif spec.kind == "cluster10":
-            a = cluster.astype(np.int64) * 10 + arng.integers(0, 10, size=w.N)
-        elif spec.kind == "zipf":
-            p = zipf_probs(spec.hi - spec.lo, spec.zipf_s)
-            a = spec.lo + arng.choice(len(p), size=w.N, p=p)
-        else:
-            raise ValueError(spec.kind)
-        attrs.append(a.astype(np.int16 if spec.dtype == "int16" else np.int32))
-    return Index(w, cb, codes, attrs, cluster, prototypes, centres, noise)
-
-
-def zipf_probs(n: int, s: float) -> np.ndarray:
-    """P(value v) ∝ (v + 1)^-s for v in [0, n) (value 0 is the most common)."""
-    p = 1.0 / np.arange(1, n + 1, dtype=np.float64) ** s
-    return p / p.sum()
+    return Index(w, cb, codes, attributes(w, cluster), cluster, centres, "pq_space",
+                 prototypes, noise)
 
 
 def raw_vectors(ix: Index, start: int = 0, stop: int | None = None) -> np.ndarray:
-    """Raw vectors of rows [start, stop): reconstruction + residual noise."""
+    """Raw vectors of rows [start, stop) of a host-drawn index."""
     w = ix.w
     stop = w.N if stop is None else stop
+    if ix.source == "mixture":
+        return mixture_vectors(w, ix.centres, start, stop)
+    if ix.source != "pq_space":
+        raise ValueError("the rows of a %s index are drawn on the device" % ix.source)
     out = np.empty((stop - start, w.D), dtype=np.float32)
-    block = 1 << 16
+    block = BLOCK
     for s in range(start - start % block, stop, block):
         e = s + block
         rng = np.random.default_rng([w.seed, 3, s])
@@ -213,37 +338,8 @@ def raw_vectors(ix: Index, start: int = 0, stop: int | None = None) -> np.ndarra
         codes = ix.codes[a:b]
         rec = ix.codebook[np.arange(w.M)[None, :], codes]          # [n][M][ds] gather
         x = rec.reshape(b - a, w.D) + noise[a - s:b - s]
-        out[a - start:b - start] = _post(w, x)
+        out[a - start:b - start] = post_process(w.kind, x)
     return out
-
-
-def raw_vectors_torch(ix: Index, start: int, stop: int, device, codebook_t=None):
-    """Raw vectors of rows [start, stop) drawn on a torch device: the same
-    recipe as ``raw_vectors`` (reconstruction + residual noise) with torch's
-    generator, seeded per 2^22-row block, for datasets too large for the host.
-    Rows must not straddle a block boundary (callers walk whole blocks)."""
-    import torch
-    w = ix.w
-    block = 1 << 22
-    if start // block != (stop - 1) // block:
-        raise ValueError("rows must lie in one 2^22-row block")
-    cb = codebook_t if codebook_t is not None else torch.from_numpy(ix.codebook).to(device)
-    codes = torch.from_numpy(ix.codes[start:stop]).to(device).long()
-    m = torch.arange(w.M, device=device)[None, :]
-    rec = cb[m, codes].reshape(stop - start, w.D)
-    gen = torch.Generator(device=device)
-    gen.manual_seed(int(w.seed) * 1_000_003 + start // block)
-    noise = torch.randn((block, w.D), generator=gen, device=device, dtype=torch.float32)
-    off = start % block
-    x = rec + ix.noise_sigma * noise[off:off + (stop - start)]
-    if w.kind == "sift":
-        x = torch.clamp(torch.round(x), 0.0, 255.0)
-    elif w.kind == "gist":
-        x = x.abs()
-        x = x / x.norm(dim=1, keepdim=True).clamp_min(1e-12)
-    elif w.kind == "deep":
-        x = x / x.norm(dim=1, keepdim=True).clamp_min(1e-12)
-    return x
 
 
 # ---------------------------------------------------------------- queries
@@ -269,17 +365,16 @@ def set_clause(pred, i, col, op, lo, hi=0):
 
 def make_queries(ix: Index, sel: float, nq: int | None = None, salt: int = 0,
                  wz_sigma: float = 0.2) -> Queries:
-    """Queries drawn from the index's mixture, each with a predicate whose
-    target selectivity is ``sel``, plus per-query w_z around the identity."""
+    """Queries drawn from the index's mixture (a uniform component, its
+    centre plus sigma * N(0, I), post-processed like the rows), each with a
+    predicate whose target selectivity is ``sel``, plus per-query w_z
+    around the identity."""
     w = ix.w
     nq = w.nq if nq is None else nq
     rng = np.random.default_rng([w.seed, 4, int(round(sel * 1e6)), salt])
     cl = rng.integers(0, w.clusters, size=nq)
-    keep = rng.random((nq, w.M)) < (1.0 - w.rho)
-    rnd = rng.integers(0, w.K, size=(nq, w.M))
-    codes = np.where(keep, ix.prototypes[cl], rnd).astype(np.int64)
-    rec = ix.codebook[np.arange(w.M)[None, :], codes].reshape(nq, w.D)
-    q = _post(w, rec + ix.noise_sigma * rng.standard_normal((nq, w.D)))
+    q = post_process(w.kind, ix.centres[cl] + np.float32(w.sigma) *
+                     rng.standard_normal((nq, w.D), dtype=np.float32))
 
     preds = empty_predicates(nq)
     if w.conjunctive:

@@ -21,5 +21,22 @@ def orc():
 
 
 @pytest.fixture(scope="session")
+def oracle_index():
+    """Workload indexes built by the oracle (mixture vectors, Lloyd training,
+    float32 encoding; oracle.pq_index), cached per workload for the session."""
+    from oracle import pq_index
+    cache = {}
+
+    def get(w):
+        if w not in cache:
+            cache[w] = pq_index.OracleIndex(w)
+        return cache[w]
+
+    yield get
+    for oi in cache.values():
+        oi.close()
+
+
+@pytest.fixture(scope="session")
 def golden_dir():
     return os.path.join(ROOT, "tests", "golden")

@@ -1,60 +1,89 @@
-"""Parity at the benchmark's full size: 10^8 PQ-coded rows, 1024-query
-batches, k = 100, conditioning on, the launch configuration bench.py times.
-The oracle recomputes sampled queries of every selectivity bin one by one
-(it scans all 10^8 rows per query); the other queries are checked through
-properties that hold at any size."""
+"""Parity at the workloads' stated sizes: sift1m-d128-m16 (10^6 rows),
+gist1m-d960-m120 (10^6 x 120 subspaces), deep10m-d96-m12 (10^7 rows, two
+columns, conjunctive predicates on the bitmap path) and gmm100m-d128-m16
+(10^8 rows, k = 100), each built by its recipe with the oracle (mixture
+vectors, Lloyd-trained codebook, float32 encoding of every row).  Every bin
+runs one 1024-query batch with conditioning on, as bench.py does; 32
+queries per bin, spread over the batch (the paired and unpaired queries of
+the sorted-copy path among them), are recomputed by the oracle over all
+rows and compared element by element, and every query of the batch is
+checked through properties that hold at any size."""
 import numpy as np
 import pytest
 
 from paper_2607_22922_gb300 import synth
-from parity_util import bitmap_rows, check_topk
+from parity_util import check_topk_sparse
 
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
-SAMPLES = (0, 1023)   # queries of each batch recomputed by the oracle
+FULL = ["sift1m-d128-m16", "gist1m-d960-m120", "deep10m-d96-m12", "gmm100m-d128-m16"]
+BATCH = 1024
+SAMPLES = 32
 
 
-@pytest.fixture(scope="module")
-def full():
+def _passes(attrs, preds, ids):
+    """Pass flags of rows ``ids`` [nq][k] (-1 ignored) for each query's
+    predicate: every clause, every operator, int64 comparisons."""
+    ok = ids >= 0
+    safe = np.where(ok, ids, 0)
+    for j in range(4):
+        c = preds["c"][:, j]
+        on = preds["n_clauses"] > j
+        a = np.stack([attrs[col][safe[i]].astype(np.int64) for i, col in enumerate(c["col"])])
+        lo, hi, op = c["lo"][:, None], c["hi"][:, None], c["op"][:, None]
+        cond = np.select([op == 0, op == 1, op == 2, op == 3, op == 4, op == 5],
+                         [a == lo, (a >= lo) & (a < hi), a >= lo, a < lo, a > lo, a <= lo], default=False)
+        ok &= cond | ~on[:, None]
+    return ok
+
+
+@pytest.fixture(scope="module", params=FULL)
+def full(request, oracle_index):
     from paper_2607_22922_gb300 import build
     build.build()
     from paper_2607_22922_gb300 import ifvs
-    w = synth.WORKLOADS["gmm100m-d128-m16"]
-    ix = synth.make_index(w)
-    cond = synth.make_conditioning(ix)
-    g = ifvs.Index(ix.codes, ix.attrs)
-    g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
-    yield w, ix, cond, g
+    w = synth.WORKLOADS[request.param]
+    oi = oracle_index(w)
+    cond = synth.make_conditioning(oi.ix)
+    g = ifvs.Index(oi.ix.codes, oi.ix.attrs, D=w.D, K=w.K)
+    g.load_codebooks(oi.ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
+    yield w, oi, cond, g
     g.close()
 
 
-@pytest.mark.parametrize("sel", synth.WORKLOADS["gmm100m-d128-m16"].sels)
-def test_full_size_batch(full, orc, sel):
-    w, ix, cond, g = full
-    qs = synth.make_queries(ix, sel, nq=w.batch)
-    ids, d, npass = g.search(qs.q, qs.preds, w.k, wz=qs.wz)
-    # properties for every query of the batch
-    attr = ix.attrs[0]
-    lo = qs.preds["c"][:, 0]["lo"]
-    hi = qs.preds["c"][:, 0]["hi"]
-    for i in range(w.batch):
-        nv = min(w.k, int(npass[i]))
-        assert (ids[i, :nv] >= 0).all() and (ids[i, nv:] == -1).all()
-        a = attr[ids[i, :nv]]
-        assert ((a >= lo[i]) & (a < hi[i])).all(), "a returned row fails its predicate"
-        assert (np.diff(d[i, :nv].astype(np.float64)) >= 0).all()
-        assert len(np.unique(ids[i, :nv])) == nv
-    # exact pass counts for every query (the oracle's filter is a plain loop)
-    for i in SAMPLES:
-        _, n = orc.filter_bitmap(ix.attrs, qs.preds[i:i + 1])
-        assert npass[i] == n
-    # element by element for the sampled queries
-    for i in SAMPLES:
-        oi, od, on, st = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q[i:i + 1],
-                                    qs.preds[i:i + 1], w.k, bank=cond.bank, W=cond.W,
-                                    seeds=cond.seeds, wz=qs.wz[i:i + 1], want_stages=True)
-        assert on[0] == npass[i]
-        bm, _ = orc.filter_bitmap(ix.attrs, qs.preds[i:i + 1])
-        passing = bitmap_rows(bm, w.N)
-        all_d = orc.adc_all(st["lut"][0], ix.codes)
-        check_topk(ids[i], d[i], oi[0], od[0], all_d, passing)
+def test_full_size_matches_oracle(full):
+    w, oi, cond, g = full
+    ix = oi.ix
+    pick = np.unique(np.linspace(0, BATCH - 1, SAMPLES).astype(np.int64))
+    ties = compared = 0
+    for sel in w.sels:
+        qs = synth.make_queries(ix, sel, nq=BATCH)
+        ids, d, npass = g.search(qs.q, qs.preds, w.k, wz=qs.wz)
+        # every query: valid prefix, padding, passing rows, ascending, unique
+        ok = _passes(ix.attrs, qs.preds, ids)
+        for i in range(BATCH):
+            nv = min(w.k, int(npass[i]))
+            assert (ids[i, :nv] >= 0).all() and (ids[i, nv:] == -1).all(), (sel, i)
+            assert ok[i, :nv].all(), "query %d of the %g bin returned a failing row" % (i, sel)
+            assert (np.diff(d[i, :nv].astype(np.float64)) >= 0).all()
+            assert len(np.unique(ids[i, :nv])) == nv
+        # pass counts of one-column ranges by binary search on the sorted column
+        if not w.conjunctive:
+            srt = np.sort(ix.attrs[0])
+            c = qs.preds["c"][:, 0]
+            cnt = np.searchsorted(srt, c["hi"], "left") - np.searchsorted(srt, c["lo"], "left")
+            np.testing.assert_array_equal(npass, cnt)
+        # the sampled queries element by element against the oracle
+        res = oi.search(cond, qs.q[pick], qs.preds[pick], qs.wz[pick], w.k, check_ids=ids[pick])
+        for j, i in enumerate(pick):
+            r = res[j]
+            assert npass[i] == r["npass"], (sel, i)
+            ties += check_topk_sparse(ids[i], d[i], r["ids"], r["dists"], r["check_dist"], r["check_pass"])
+            compared += int((r["ids"] >= 0).sum())
+    # Every id that differs was checked to be tied with the k-th distance
+    # within the tolerance.  Such ties are common here: rows of one mixture
+    # component often share all their codes (equal distances), and the
+    # float32 sum order of a row depends on its position, so the GPU breaks
+    # those ties by the last ulp where the oracle (fp64) breaks them by id.
+    # They must stay a small share of the ids compared.
+    assert ties <= max(4, compared // 20), (ties, compared)

@@ -171,9 +171,9 @@ def test_threshold_splits_a_batch(ifvs, orc):
     _check_oracle(orc, codes, attrs, Cpq, q, p, 30, *mixed)
 
 
-def test_list_path_with_conditioning_sub_batches_and_device_index(ifvs, orc):
+def test_list_path_with_conditioning_sub_batches_and_device_index(ifvs, orc, oracle_index):
     w = synth.scaled(synth.WORKLOADS["gmm10k-d128-m16"], N=60000)
-    ix = synth.make_index(w)
+    ix = oracle_index(w).ix
     cond = synth.make_conditioning(ix)
     qs = synth.make_queries(ix, 0.01, nq=70)
     for dio in (False, True):
@@ -201,10 +201,17 @@ def test_threshold_and_launch_counts(ifvs):
     g.stage_times(reset=True)
     g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
-    # plan + filter; the bitmap scan, the pairing of the sorted-copy queries,
-    # the two-query and the one-query sorted-copy scans, for every k
-    assert t["filter"][1] == 2 and t["scan"][1] == 4
+    # plan + filter; the bitmap scan, the grouping of the sorted-copy
+    # queries, the four-, two- and one-query sorted-copy scans (four-query
+    # CTAs for k <= 128)
+    assert t["filter"][1] == 2 and t["scan"][1] == 5
     g.search(q, p, 100, flags=ifvs.IFVS_F_STAGE_TIMING)
+    t = g.stage_times(reset=True)
+    assert t["scan"][1] == 5
+    g.search(q, p, 100, flags=ifvs.IFVS_F_STAGE_TIMING | ifvs.IFVS_F_NO_QUADS)
+    t = g.stage_times(reset=True)
+    assert t["scan"][1] == 4
+    g.search(q, p, 200, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
     assert t["scan"][1] == 4
     g.search(q, p, 100, flags=ifvs.IFVS_F_STAGE_TIMING, pair_min_rows=-1)
@@ -242,7 +249,7 @@ def _one_by_one(g, q, p, k, **kw):
 @pytest.mark.parametrize("case", ["normal", "one_wide_subspace", "constant", "tiny_range", "huge"])
 @pytest.mark.parametrize("k", [100, 128])
 def test_pair_kernel_equals_one_query_kernel(ifvs, orc, case, k):
-    """The two-query kernel drops rows by a quantised lower bound and
+    """The four- and two-query kernels drop rows by a quantised lower bound and
     rescores the rest exactly in the one-query kernel's order, so a batch
     whose queries pair up (pairing forced at this size) must return, bit for
     bit, what each query returns alone and what the batch returns with no
@@ -271,27 +278,30 @@ def test_pair_kernel_equals_one_query_kernel(ifvs, orc, case, k):
     q[9] = q[8]                                    # a pair of identical vectors
     g.stage_times(reset=True)
     a = g.search(q, p, k, flags=ifvs.IFVS_F_STAGE_TIMING, pair_min_rows=1)
-    assert g.stage_times(reset=True)["scan"][1] == 4   # bitmap, pairing, two-query, one-query scans
-    for b in (_one_by_one(g, q, p, k, pair_min_rows=1), g.search(q, p, k, pair_min_rows=-1)):
+    # bitmap, grouping, four-, two- and one-query scans
+    assert g.stage_times(reset=True)["scan"][1] == 5
+    for b in (_one_by_one(g, q, p, k, pair_min_rows=1), g.search(q, p, k, pair_min_rows=-1),
+              g.search(q, p, k, pair_min_rows=1, flags=ifvs.IFVS_F_NO_QUADS)):
         for x, y in zip(a, b):
             np.testing.assert_array_equal(x, y)
     if case != "huge":
         _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
 
 
-def test_pair_kernel_with_conditioning(ifvs, orc):
+def test_pair_kernel_with_conditioning(ifvs, orc, oracle_index):
     """Wide pairs through the conditioned path (bank, W, w_z): the same
     bit-for-bit agreement with single queries, and the oracle's top-k."""
     w = synth.scaled(synth.WORKLOADS["gmm10k-d128-m16"], N=50001)
-    ix = synth.make_index(w)
+    ix = oracle_index(w).ix
     cond = synth.make_conditioning(ix)
     qs = synth.make_queries(ix, 1.0, nq=12)
     g = ifvs.Index(ix.codes, ix.attrs, D=w.D, K=w.K)
     g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
     a = g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=1)
-    b = g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=-1)
-    for j in range(3):
-        np.testing.assert_array_equal(a[j], b[j])
+    for b in (g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=-1),
+              g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=1, flags=ifvs.IFVS_F_NO_QUADS)):
+        for j in range(3):
+            np.testing.assert_array_equal(a[j], b[j])
     oi, od, on, st = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q, qs.preds, 100, bank=cond.bank,
                                 W=cond.W, seeds=cond.seeds, wz=qs.wz, want_stages=True)
     np.testing.assert_array_equal(a[2], on)
@@ -329,6 +339,8 @@ def test_pairing_by_sorted_ranges(ifvs, orc, k):
     for x, y in zip(a, b):
         np.testing.assert_array_equal(x[perm], y)
     for x, y in zip(a, g.search(q, p, k, sub_batch=nq, pair_min_rows=-1)):
+        np.testing.assert_array_equal(x, y)
+    for x, y in zip(a, g.search(q, p, k, sub_batch=nq, pair_min_rows=1, flags=ifvs.IFVS_F_NO_QUADS)):
         np.testing.assert_array_equal(x, y)
     c = _one_by_one(g, q[:24], p[:24], k)
     for x, y in zip(a, c):

@@ -1,6 +1,8 @@
 """CUDA path vs oracle, element by element, on seeded inputs of the five
 workload shapes (reduced so that the oracle finishes in seconds, with ragged
-tails), through the C ABI."""
+tails), through the C ABI.  Each index follows its workload's recipe: the
+stated mixture, a PQ codebook trained by the oracle's Lloyd iterations and
+the oracle's float32 encoding of every row."""
 import math
 
 import numpy as np
@@ -35,11 +37,11 @@ class Case:
 
 
 @pytest.fixture(scope="module", params=list(CASES))
-def case(request, ifvs, orc):
+def case(request, ifvs, orc, oracle_index):
     w, nq = CASES[request.param]
     c = Case()
     c.name, c.w = request.param, w
-    c.ix = synth.make_index(w)
+    c.ix = oracle_index(w).ix
     c.cond = synth.make_conditioning(c.ix)
     c.g = ifvs.Index(c.ix.codes, c.ix.attrs)
     c.g.load_codebooks(c.ix.codebook, bank=c.cond.bank, W=c.cond.W, hash_seeds=c.cond.seeds)
@@ -84,7 +86,7 @@ def test_conditioning_and_tables(case):
 
 
 def test_search_matches_oracle(case, orc):
-    ties = 0
+    ties = compared = 0
     for qs, oi, od, npass, st in case.bins:
         ids, d, gn = case.g.search(qs.q, qs.preds, case.w.k, wz=qs.wz)
         np.testing.assert_array_equal(gn, npass)
@@ -92,7 +94,11 @@ def test_search_matches_oracle(case, orc):
             _, passing = _passing(orc, case.ix, qs.preds[i:i + 1])
             all_d = orc.adc_all(st["lut"][i], case.ix.codes)
             ties += check_topk(ids[i], d[i], oi[i], od[i], all_d, passing)
-    assert ties <= 2
+            compared += int((oi[i] >= 0).sum())
+    # every differing id is tied with the k-th distance within the tolerance
+    # (rows that share their codes tie exactly; the float32 sum order depends
+    # on the row's position); they must stay a small share of the ids
+    assert ties <= max(2, compared // 20), (ties, compared)
 
 
 def test_scan_alone_from_oracle_tables(case, orc):
@@ -338,9 +344,11 @@ def test_stage_timing_counts_launches(ifvs):
     g.stage_times(reset=True)
     g.search(q, _preds(8, 0, 50), 10, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
-    # filter: the scan plan + the filter; scan: the bitmap kernel, the pairing
-    # of the sorted-copy queries, the two-query and one-query kernels (M = 16)
-    expected = {"predicate": 1, "filter": 2, "condition": 1, "lut": 2, "scan": 4, "merge": 1}
+    # one attribute column: every predicate takes the sorted copy, so no
+    # filter pass and no bitmap scan run.  filter: the scan plan; scan: the
+    # grouping of the sorted-copy queries, the four-, two- and one-query
+    # kernels (M = 16)
+    expected = {"predicate": 1, "filter": 1, "condition": 1, "lut": 2, "scan": 4, "merge": 1}
     for s, n in expected.items():
         assert t[s][1] == n and t[s][0] > 0.0
     assert t["rerank"][1] == 0

@@ -19,8 +19,8 @@ def ifvs():
 
 
 def _data(w, n, seed):
-    ix = synth.make_index(synth.scaled(w, N=n))
-    X = synth.raw_vectors(ix)
+    w = synth.scaled(w, N=n)
+    X = synth.mixture_vectors(w, synth.mixture_centres(w))
     rng = np.random.default_rng(seed)
     C0 = X[rng.choice(n, w.K, replace=False)].reshape(w.K, w.M, w.ds).transpose(1, 0, 2).copy()
     return X, C0

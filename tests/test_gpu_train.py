@@ -36,7 +36,7 @@ class Case:
         if r is not None:
             w = synth.scaled(w, r=r)
         self.w = w
-        self.ix = synth.make_index(w)
+        self.ix = synth.pq_space_index(w)
         self.cond = synth.make_conditioning(self.ix)
         self.qs = synth.make_queries(self.ix, sel, nq=nq, salt=salt)
         self.X = synth.raw_vectors(self.ix)

@@ -345,7 +345,7 @@ def test_reduces_to_plain_pq_adc(orc):
     """alpha = 0, w_f = 1 (the paper's initial state) is plain PQ ADC, whose
     ranking equals exact L2 to the reconstructions (Pre_IndexFlatL2_PQ)."""
     w = synth.scaled(synth.WORKLOADS["gmm10k-d128-m16"], N=3000, nq=5)
-    ix = synth.make_index(w)
+    ix = synth.pq_space_index(w)
     qs = synth.make_queries(ix, 0.5)
     ids, d, npass = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q, qs.preds, 10)
     rec = ix.codebook[np.arange(w.M)[None, :], ix.codes].reshape(w.N, w.D).astype(np.float64)
@@ -361,7 +361,7 @@ def test_reduces_to_plain_pq_adc(orc):
 
 def test_search_stage_outputs_consistent(orc):
     w = synth.scaled(synth.WORKLOADS["gmm10k-d128-m16"], N=500, nq=3)
-    ix = synth.make_index(w)
+    ix = synth.pq_space_index(w)
     cond = synth.make_conditioning(ix)
     qs = synth.make_queries(ix, 0.5)
     ids, d, npass, st = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q, qs.preds, 7,
@@ -380,7 +380,7 @@ def test_search_stage_outputs_consistent(orc):
 
 def test_exact_ground_truth_and_rerank(orc):
     w = synth.scaled(synth.WORKLOADS["gmm10k-d128-m16"], N=2000, nq=3)
-    ix = synth.make_index(w)
+    ix = synth.pq_space_index(w)
     X = synth.raw_vectors(ix)
     qs = synth.make_queries(ix, 0.1)
     for i in range(3):
