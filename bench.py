@@ -30,6 +30,15 @@ import subprocess
 import sys
 import time
 
+_T0 = time.time()
+
+
+def phase(msg):
+    """Progress of the run on stderr (seconds since start); stdout carries
+    only the JSON line."""
+    sys.stderr.write("[bench %7.1f s] %s\n" % (time.time() - _T0, msg))
+    sys.stderr.flush()
+
 import numpy as np
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -65,8 +74,6 @@ def parse():
     ap.add_argument("--pair-min-rows", type=int, default=0,
                     help="two-query CTAs for overlapping one-column ranges spanning at least this many "
                          "rows (0 = library default, -1 = never)")
-    ap.add_argument("--no-quads", action="store_true",
-                    help="group sorted-copy queries in pairs only (no four-query CTAs)")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
     ap.add_argument("--mode", default="search", choices=["search", "pq", "train"],
                     help="search: the query path; pq: PQ encoding + Lloyd training of the index; "
@@ -254,9 +261,17 @@ def build_index_gpu(w, device, ifvs, local):
     from paper_2607_22922_gb300 import synth
     t0 = time.time()
     dio = ifvs.IFVS_F_DEVICE_IO
-    # the library's calls run on torch's current stream, after the work that
-    # produces their inputs
-    sptr = torch.cuda.current_stream(device).cuda_stream
+    # every step (torch's draws and the library's calls) runs on one stream
+    # of its own, so each library call reads inputs that are already written
+    st = torch.cuda.Stream(device=device)
+    with torch.cuda.stream(st):
+        return _build_index_gpu(w, device, ifvs, local, st, dio, t0)
+
+
+def _build_index_gpu(w, device, ifvs, local, st, dio, t0):
+    import torch
+    from paper_2607_22922_gb300 import synth
+    sptr = st.cuda_stream
     ct = torch.from_numpy(synth.mixture_centres(w)).to(device)
     n_s = synth.pq_sample_rows(w)
     block = 1 << 22
@@ -271,7 +286,7 @@ def build_index_gpu(w, device, ifvs, local):
         b = min(w.N, a + block)
         x = synth.mixture_vectors_torch(w, ct, a, b, device)
         ifvs.ifvs_pq_encode(x, C, device=local, codes=codes[a:b], flags=dio, stream=sptr)
-    torch.cuda.synchronize(device)
+    st.synchronize()
     ix = synth.mixture_index(w, C.cpu().numpy(), codes.cpu().numpy(), source="mixture-torch")
     del codes, ct
     torch.cuda.empty_cache()
@@ -445,29 +460,30 @@ def recall_at_k(w, ix, batches, ids_by_bin, nsample, device):
     return out
 
 
-def scan_lookups(w, qs, sorted_vals, on_list, npass, pair_rows, quads=True, seg=2048):
+def scan_lookups(w, qs, sorted_vals, on_list, npass, pair_rows, seg=2048):
     """Shared-memory look-ups the scan stage executes for one batch, by the
-    library's grouping rule for one-column ranges of the sorted copy (M = 16;
-    sort by (column, range start, query) per 2048-query segment; an aligned
-    run of four sorted neighbours whose union spans at least pair_rows
-    positions and whose every range covers 3/4 of the union forms a
-    four-query group (k <= 128); otherwise neighbours 2j, 2j+1 pair when 3/4
-    of the longer range is common and the two span at least pair_rows): a
-    group costs the union of its ranges x M (one load serves all its
-    queries), any other query its pool x M."""
+    library's pairing rule for one-column ranges of the sorted copy (M = 16;
+    sort by (column, range start, query) per 2048-query segment; neighbours
+    2j, 2j+1 pair when 3/4 of the longer range is common and the two span at
+    least pair_rows): a pair costs the union of its ranges x M (one load
+    serves both queries), any other query its pool x M."""
     n = len(qs.q)
     a = np.zeros(n, np.int64)
     b = np.zeros(n, np.int64)
     col = np.zeros(n, np.int64)
-    for i in range(n):
-        if on_list[i]:
-            c = qs.preds[i]["c"][0]
-            col[i] = c["col"]
-            v = sorted_vals[col[i]]
-            a[i] = np.searchsorted(v, c["lo"], "left")
-            b[i] = np.searchsorted(v, c["hi"], "left")
-    grouped = np.zeros(n, bool)
-    in_quad = np.zeros(n, bool)
+    c0 = qs.preds["c"][:, 0]
+    col[on_list] = c0["col"][on_list]
+    for cc in np.unique(col[on_list]):
+        sel = on_list & (col == cc)
+        v = sorted_vals[cc]
+        # bounds clipped to the column's type, so that the search does not
+        # convert the whole column to int64
+        info = np.iinfo(v.dtype)
+        a[sel] = np.searchsorted(v, np.clip(c0["lo"][sel], info.min, info.max).astype(v.dtype), "left")
+        hi = c0["hi"][sel]
+        bb = np.searchsorted(v, np.clip(hi, info.min, info.max).astype(v.dtype), "left")
+        b[sel] = np.where(hi > info.max, len(v), bb)
+    paired = np.zeros(n, bool)
     union = 0.0
 
     def pair_ok(x, y):
@@ -478,30 +494,17 @@ def scan_lookups(w, qs, sorted_vals, on_list, npass, pair_rows, quads=True, seg=
         span = max(b[x], b[y]) - min(a[x], a[y])
         return 4 * common >= 3 * max(lx, ly) and span >= pair_rows
 
-    def quad_ok(g):
-        if any(col[x] != col[g[0]] or b[x] <= a[x] for x in g):
-            return False
-        lo, hi = min(a[x] for x in g), max(b[x] for x in g)
-        return hi - lo >= pair_rows and all(4 * (b[x] - a[x]) >= 3 * (hi - lo) for x in g)
-
     if w.M == 16 and pair_rows >= 0:
         for s0 in range(0, n, seg):
             idx = [i for i in range(s0, min(n, s0 + seg)) if on_list[i]]
             idx.sort(key=lambda i: (col[i], a[i], i))
-            for r in range(0, len(idx), 4):
-                g = idx[r:r + 4]
-                if quads and w.k <= 128 and len(g) == 4 and quad_ok(g):
-                    grouped[g] = in_quad[g] = True
-                    union += max(b[x] for x in g) - min(a[x] for x in g)
-                    continue
-                for j in (0, 2):
-                    if j + 1 < len(g) and pair_ok(g[j], g[j + 1]):
-                        x, y = g[j], g[j + 1]
-                        grouped[x] = grouped[y] = True
-                        union += max(b[x], b[y]) - min(a[x], a[y])
-    single = float(npass[~grouped].sum())
-    return {"lookups": (single + union) * w.M, "grouped_share": float(grouped.mean()),
-            "quad_share": float(in_quad.mean())}
+            for j in range(0, len(idx) - 1, 2):
+                x, y = idx[j], idx[j + 1]
+                if pair_ok(x, y):
+                    paired[x] = paired[y] = True
+                    union += max(b[x], b[y]) - min(a[x], a[y])
+    single = float(npass[~paired].sum())
+    return {"lookups": (single + union) * w.M, "paired_share": float(paired.mean())}
 
 
 # ------------------------------------------------------------ arms
@@ -524,6 +527,7 @@ def run_ifvs(args):
     w = workload(args)
     t0 = time.time()
     ix, t_pq = build_index_gpu(w, device, ifvs, local)
+    phase("index built (%.1f s)" % t_pq)
     cond = synth.make_conditioning(ix)
     batches = [synth.make_queries(ix, s, nq=w.batch, salt=rank) for s in w.sels]
     t_gen = time.time() - t0
@@ -545,6 +549,7 @@ def run_ifvs(args):
         g = ifvs.Index(ix.codes, ix.attrs, device=local)
     g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
     t_load = time.time() - t_load0
+    phase("index loaded")
 
     stream = torch.cuda.Stream(device=device)
     sptr = stream.cuda_stream
@@ -559,7 +564,7 @@ def run_ifvs(args):
                         torch.empty((n, w.k), dtype=torch.float32, device=device),
                         torch.empty(n, dtype=torch.int64, device=device)))
     torch.cuda.synchronize()
-    flags = ifvs.IFVS_F_DEVICE_IO | ifvs.IFVS_F_STAGE_TIMING | (ifvs.IFVS_F_NO_QUADS if args.no_quads else 0)
+    flags = ifvs.IFVS_F_DEVICE_IO | ifvs.IFVS_F_STAGE_TIMING
 
     def step(i):
         b = i % nb
@@ -614,7 +619,7 @@ def run_ifvs(args):
         nsteps_b = len(ms_b)
         one_col = (qs.preds["n_clauses"] == 1) if not w.conjunctive else np.zeros(len(npass), bool)
         on_list = one_col & (npass <= list_rows)
-        lk = scan_lookups(w, qs, sorted_vals, on_list, npass, pair_rows, quads=not args.no_quads)
+        lk = scan_lookups(w, qs, sorted_vals, on_list, npass, pair_rows)
         lookups_total += nsteps_b * lk["lookups"]
         code_bytes_total += nsteps_b * float(npass.sum()) * w.M
         per_bin[str(qs.sel)] = {
@@ -622,7 +627,7 @@ def run_ifvs(args):
             "ms_per_batch": float(np.mean(ms_b)) if ms_b else None,
             "mean_selectivity": float(npass.mean() / w.N),
             "sorted_path_share": float(on_list.mean()),
-            "grouped_share": lk["grouped_share"], "quad_share": lk["quad_share"]}
+            "paired_share": lk["paired_share"]}
     # The scan stage (per batch: k_pair_items, k_scan_list_pair, k_scan_list
     # and k_scan, one launch of each) is the unit.  Its binding resource is
     # the shared-memory look-up rate: one conflict-free 32-lane load per SM
@@ -639,8 +644,7 @@ def run_ifvs(args):
     achieved = (lookups_total / nbatch) / (scan_ms / nbatch / 1000.0) if scan_ms > 0 else None
     hbm_peak, peak_kind = measured_peaks()
     dram = scan_dram(w.name, hbm_peak)
-    roofline = {"kernel": "scan stage (k_group_items + k_scan_list_quad + k_scan_list_pair + k_scan_list"
-                          " + k_scan)",
+    roofline = {"kernel": "scan stage (k_pair_items + k_scan_list_pair + k_scan_list + k_scan)",
                 "bound": "smem", "achieved": achieved, "peak": peak, "unit": "look-ups/s",
                 "frac": achieved / peak if achieved else None,
                 "traffic": dram["bytes_per_batch"] if dram else None,
@@ -654,6 +658,7 @@ def run_ifvs(args):
                 "dram": dram, "hbm_peak_gbs": hbm_peak, "hbm_peak_kind": peak_kind}
     share = {k: v[0] for k, v in stages.items()}
 
+    phase("timed steps done")
     # end to end through the C ABI with pinned host buffers
     e2e = None
     if not args.no_e2e:
@@ -675,8 +680,7 @@ def run_ifvs(args):
             oi, od, on, _ = host_out[b]
             ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr,
                                    chunk_blocks=args.chunk_blocks, list_max_ppm=args.list_max_ppm,
-                                   rerank=args.rerank, pair_min_rows=args.pair_min_rows,
-                                   flags=ifvs.IFVS_F_NO_QUADS if args.no_quads else 0)
+                                   rerank=args.rerank, pair_min_rows=args.pair_min_rows)
 
         for i in range(args.warmup):
             hstep(i)
@@ -694,6 +698,7 @@ def run_ifvs(args):
                "h2d_bytes_per_step": nq_b * (w.D * 4 * 2 + 104),
                "d2h_bytes_per_step": nq_b * (w.k * 12 + 8)}
 
+    phase("e2e done")
     # recall@k (outside the timed regions)
     recall = None
     if args.recall_queries > 0 and rank == 0:
@@ -702,11 +707,13 @@ def run_ifvs(args):
         for s, r in recall.items():
             per_bin[str(s)]["recall@%d" % w.k] = r
 
+    phase("recall done")
     cpu = cpu_par = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, ix, cond, batches)
         cpu_par = cpu_baseline_parallel(w, ix, cond, batches)
 
+    phase("cpu baselines done")
     value = whole_job_qps(world, args.steps, w.batch, max_ms)
     line = {
         "metric": "QPS at recall@%d per selectivity bin (code-scan HBM GB/s vs peak)" % w.k,

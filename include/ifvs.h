@@ -23,6 +23,13 @@
  * fallback.  All calls are synchronous: they return once their outputs are
  * written.  No call keeps a pointer to caller memory after it returns.
  *
+ * Streams: where a call takes a stream, NULL selects a stream of the
+ * library's own (the index's, or one the call creates).  Those streams are
+ * blocking streams, so the call's kernels run after work the caller queued
+ * on the legacy default stream.  With device I/O, inputs that the caller
+ * produces on any other stream are only safe to read if that stream is
+ * passed (or synchronised before the call).
+ *
  * Errors: every call returns an ifvs_status.  On error the outputs are
  * unspecified and ifvs_last_error() (thread-local) describes the cause.
  * Nothing aborts the process and nothing throws across the ABI.
@@ -95,8 +102,6 @@ typedef struct {
                                      on the launching stream (ifvs_stage_times) */
 #define IFVS_F_PLAIN_PQ     0x4u  /* ignore the memory bank: Delta = 0 (plain PQ
                                      ADC, baseline Pre_IndexPQ_ADC of §3.2)   */
-#define IFVS_F_NO_QUADS     0x8u  /* search: group sorted-copy queries in pairs
-                                     only, never in fours (pair_min_rows)     */
 
 typedef struct {
     uint32_t flags;     /* IFVS_F_*                                            */
@@ -117,16 +122,14 @@ typedef struct {
                            (1000000: always); -1: never.  The two paths sum a row's entries in
                            different orders, so distances agree to float32
                            rounding.                                          */
-    int32_t pair_min_rows; /* M = 16 sorted-copy scan: queries on the same
-                           column whose ranges together span at least this
-                           many rows share a CTA and one shared-memory look-up
-                           per code byte: four neighbours (by range start)
-                           each covering 3/4 of their union (tables quantised
-                           to 5 bits, k <= 128), else two sharing 3/4 of the
-                           longer range (11 bits); every row that can reach a
-                           top-k is rescored exactly, so results equal those
-                           of one query per CTA bit for bit.
-                           0: default (4194304); -1: never group.            */
+    int32_t pair_min_rows; /* M = 16 sorted-copy scan: two queries on the same
+                           column whose ranges share 3/4 of the longer one
+                           and together span at least this many rows share a
+                           CTA and one shared-memory look-up per code byte
+                           (tables quantised to 11 bits; every row that can
+                           reach a top-k is rescored exactly, so results
+                           equal those of one query per CTA bit for bit).
+                           0: default (4194304); -1: never pair.             */
     void* stream;       /* cudaStream_t to run on; NULL: the index's stream   */
 } ifvs_search_params;
 

@@ -336,7 +336,7 @@ struct Stage {
 };
 
 struct Opts {
-    bool dio = false, timing = false, plain = false, no_quads = false;
+    bool dio = false, timing = false, plain = false;
     int R = 0;
     int64_t sub_batch = 0;
     int64_t chunk_blocks = 0;
@@ -359,7 +359,7 @@ constexpr int64_t kPairDefaultMinRows = int64_t(1) << 22;
 
 int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (!p) return 0;
-    if (p->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING | IFVS_F_PLAIN_PQ | IFVS_F_NO_QUADS))
+    if (p->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING | IFVS_F_PLAIN_PQ))
         return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", p->flags);
     if (p->chunk_blocks < 0) return set_err(IFVS_ERR_ARG, "chunk_blocks must be >= 0");
     if (p->rerank < 0 || p->rerank > IFVS_MAX_K)
@@ -371,7 +371,6 @@ int parse_opts(const ifvs_search_params* p, Opts* o) {
     o->dio = p->flags & IFVS_F_DEVICE_IO;
     o->timing = p->flags & IFVS_F_STAGE_TIMING;
     o->plain = p->flags & IFVS_F_PLAIN_PQ;
-    o->no_quads = p->flags & IFVS_F_NO_QUADS;
     o->R = p->rerank;
     o->sub_batch = p->sub_batch;
     o->chunk_blocks = p->chunk_blocks;
@@ -504,7 +503,7 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
         const cudaError_t e = launch_scan_list(ix->w_tab.as<float>(), ix->sorted(), plan, n, kk, sh,
                                                ix->w_part.as<uint64_t>(),
                                                o.pair_min_rows < 0 ? nullptr : ix->w_items.as<uint8_t>(),
-                                               pmin, !o.no_quads, s, &nl);
+                                               pmin, s, &nl);
         CUDA_TRY(st.end(e, nl));
     }
     int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;
@@ -844,7 +843,9 @@ int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int6
     if (cudaDeviceGetAttribute(&ix->num_sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess ||
         cudaDeviceGetAttribute(&ix->max_smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, device) != cudaSuccess)
         return fail(cuda_fail(cudaGetLastError(), "cudaDeviceGetAttribute", __LINE__));
-    if (cudaStreamCreateWithFlags(&ix->stream, cudaStreamNonBlocking) != cudaSuccess)
+    // a blocking stream: work the caller put on the legacy default stream
+    // (NULL) before a call is ordered before the call's kernels
+    if (cudaStreamCreateWithFlags(&ix->stream, cudaStreamDefault) != cudaSuccess)
         return fail(cuda_fail(cudaGetLastError(), "cudaStreamCreateWithFlags", __LINE__));
     ix->N = N;
     ix->M = M;
@@ -1288,7 +1289,8 @@ int pq_check(int32_t device, const float* X, int64_t n, int32_t D, int32_t M, in
     if (stream) {
         a->s = (cudaStream_t)stream;
     } else {
-        CUDA_TRY(cudaStreamCreateWithFlags(&a->s, cudaStreamNonBlocking));
+        // blocking: ordered after the caller's work on the legacy default stream
+        CUDA_TRY(cudaStreamCreateWithFlags(&a->s, cudaStreamDefault));
         a->own_stream = true;
     }
     return 0;
@@ -1318,7 +1320,7 @@ extern "C" int ifvs_merge_topk(int32_t device, const float* dists, const int64_t
     if (stream) {
         a.s = (cudaStream_t)stream;
     } else {
-        CUDA_TRY(cudaStreamCreateWithFlags(&a.s, cudaStreamNonBlocking));
+        CUDA_TRY(cudaStreamCreateWithFlags(&a.s, cudaStreamDefault));
         a.own_stream = true;
     }
     const bool dio = flags & IFVS_F_DEVICE_IO;

@@ -195,21 +195,17 @@ cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* 
 struct PairItem {
     int32_t qa, qb;
 };
-struct QuadItem {
-    int32_t q[4];
-};
 // the list-path queries of `plan`: their pool is the position range [a, b)
 // of a column's sorted copy (same grid and partial layout as launch_scan).
 // For M = 16, `work` (scan_list_workspace_bytes(nq) bytes) receives the
-// groups of overlapping ranges that together span at least pair_min_rows
-// positions: runs of four (served by a four-query kernel, when `quads`)
-// and pairs (a two-query kernel); a one-query kernel serves the other
-// queries (all of them when work is null or M != 16).  *launches = kernels
-// launched.
+// pairs of overlapping ranges that together span at least pair_min_rows
+// positions, served by a two-query kernel; a one-query kernel serves the
+// other queries (all of them when work is null or M != 16).  *launches =
+// kernels launched.
 size_t scan_list_workspace_bytes(int64_t nq);
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
                              const ScanShape& sh, uint64_t* partials, uint8_t* work, int64_t pair_min_rows,
-                             bool quads, cudaStream_t s, int* launches);
+                             cudaStream_t s, int* launches);
 // the sorted copy of the codes: dst position p <- row rows[p] of the index
 // layout `src`, re-rotated by (p mod 32) mod M; positions >= N are zero
 cudaError_t launch_relayout_sorted(const uint8_t* src, const uint32_t* rows, int64_t N, int M,

@@ -708,13 +708,9 @@ __device__ __forceinline__ uint32_t lds_u32_imm(uint32_t addr) {
     return v;
 }
 
-__device__ __forceinline__ uint32_t quant_q(float L, float lo, float inv, float qmax) {
-    const float y = __fmul_rn(__fsub_rn(L, lo), inv);
-    return (uint32_t)fminf(qmax, fmaxf(0.f, y));   // truncation: floor of y >= 0
-}
-
 __device__ __forceinline__ uint32_t quant12(float L, float lo, float inv) {
-    return quant_q(L, lo, inv, (float)kQMax);
+    const float y = __fmul_rn(__fsub_rn(L, lo), inv);
+    return (uint32_t)fminf((float)kQMax, fmaxf(0.f, y));   // truncation: floor of y >= 0
 }
 
 // The largest quantised sum S a row can have and still reach a top-k whose
@@ -942,8 +938,7 @@ __device__ __forceinline__ void merge_warps(WarpTopK<KP>& tk, uint64_t* tkbuf, i
 
 // Quantisation parameters of one query from the per-subspace extremes
 // lo[16], hi[16]: inv (0 turns the test off: every row is rescored) and sl.
-__device__ __forceinline__ void quant_params(const float* lo, const float* hi, float& inv, float& sl,
-                                             int qmax = kQMax) {
+__device__ __forceinline__ void quant_params(const float* lo, const float* hi, float& inv, float& sl) {
     float r = 0.f, s = 0.f;
     bool ok = true;
 #pragma unroll
@@ -952,29 +947,25 @@ __device__ __forceinline__ void quant_params(const float* lo, const float* hi, f
         s = __fadd_rn(s, lo[m]);
         ok = ok && lo[m] >= 0.f;
     }
-    inv = __fdiv_rn((float)qmax, r);
+    inv = __fdiv_rn((float)kQMax, r);
     if (!(ok && r > 0.f && isfinite(inv) && isfinite(s))) inv = 0.f;
     sl = s;
 }
 
-// ---- grouping of the sorted-copy queries of a batch ------------------------
+// ---- pairing of the sorted-copy queries of a batch -------------------------
 //
 // Two queries are worth one CTA when they read the same column's copy, their
 // ranges mostly coincide (at least 3/4 of the longer range is common to both;
 // the rows of only one range then run with the other query masked) and the
 // two ranges together span at least min_rows positions (the caller's choice:
 // for short ranges the one-query kernel, with two or three CTAs per SM, was
-// measured faster).  Four queries are worth one CTA of the four-query kernel
-// under the same rule, every member's range covering at least 3/4 of the
-// union of the four.
-// k_group_items sorts the list-path queries of each segment of kPairSeg by
-// (column, range start, query).  Each aligned run of four sorted neighbours
-// (4j .. 4j + 3) that qualifies becomes a quad item; in every other run the
-// neighbours (4j, 4j + 1) and (4j + 2, 4j + 3) that qualify become pair
-// items.  Items fill the segment's slots in sorted order and unused slots
-// get q[0] = -1, so CTA x of a kernel serves item x (or nothing); `grouped`
-// marks the queries of all items, and k_scan_list serves every other
-// list-path query.
+// measured faster).
+// k_pair_items sorts the list-path queries of each segment of kPairSeg by
+// (column, range start, query) and pairs sorted neighbours (2j, 2j + 1) that
+// qualify.  Pairs fill the segment's item slots in sorted order and the
+// unused slots get qa = -1, so the pair kernel's CTA x serves item x (or
+// nothing); `paired` marks the queries of the pairs, and k_scan_list serves
+// every other list-path query.
 constexpr int kPairSeg = 2048;
 static_assert(IFVS_MAX_ATTRS <= 4, "the pairing key keeps 2 bits of the column");
 constexpr int kPairSortThreads = 1024;
@@ -986,21 +977,6 @@ __device__ __forceinline__ bool pairable(const ScanPlan& x, const ScanPlan& y, i
     const int64_t common = min(x.b, y.b) - max(x.a, y.a);
     const int64_t span = max(x.b, y.b) - min(x.a, y.a);
     return 4 * common >= 3 * max(lx, ly) && span >= min_rows;
-}
-
-__device__ __forceinline__ bool quadable(const ScanPlan (&p)[4], int64_t min_rows) {
-    int64_t lo = p[0].a, hi = p[0].b;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        if (!p[i].list || p[i].col != p[0].col || p[i].b <= p[i].a) return false;
-        lo = min(lo, p[i].a);
-        hi = max(hi, p[i].b);
-    }
-    if (hi - lo < min_rows) return false;
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-        if (4 * (p[i].b - p[i].a) < 3 * (hi - lo)) return false;
-    return true;
 }
 
 // exclusive prefix of v over the block's threads (in thread order) and the
@@ -1027,10 +1003,9 @@ __device__ __forceinline__ int block_prefix(int v, int* wsum, int& total) {
 }
 
 __global__ void __launch_bounds__(kPairSortThreads)
-k_group_items(const ScanPlan* __restrict__ plan, int64_t nq, int64_t min_rows, int quads_on,
-              QuadItem* __restrict__ quads, PairItem* __restrict__ items, uint8_t* __restrict__ grouped) {
+k_pair_items(const ScanPlan* __restrict__ plan, int64_t nq, int64_t min_rows, PairItem* __restrict__ items,
+             uint8_t* __restrict__ paired) {
     __shared__ uint64_t key[kPairSeg];
-    __shared__ int quad_ok[kPairSeg / 4];
     __shared__ int wsum[kPairSortThreads / 32];
     const int64_t q0 = (int64_t)blockIdx.x * kPairSeg;
     const int n = (int)min((int64_t)kPairSeg, nq - q0);
@@ -1060,52 +1035,27 @@ k_group_items(const ScanPlan* __restrict__ plan, int64_t nq, int64_t min_rows, i
             }
         }
     __syncthreads();
+    // sorted neighbours (2j, 2j + 1) that qualify make an item; positions by
+    // a block-wide exclusive scan of the counts, in sorted order
     static_assert(kPairSeg == 2 * kPairSortThreads, "one neighbour pair per thread");
     const int j = threadIdx.x;
-    // runs of four sorted neighbours
-    int qd[4] = {-1, -1, -1, -1};
-    int qcnt = 0;
-    if (j < kPairSeg / 4) {
-        bool ok = quads_on != 0;
-        ScanPlan pl[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const uint64_t kk = key[4 * j + i];
-            ok = ok && kk != ~0ull;
-            qd[i] = kk != ~0ull ? (int)(q0 + (int64_t)(kk & 2047u)) : -1;
-            pl[i] = qd[i] >= 0 ? plan[qd[i]] : ScanPlan{0, 0, 0, 0};
-        }
-        qcnt = ok && quadable(pl, min_rows) ? 1 : 0;
-        quad_ok[j] = qcnt;
-    }
-    __syncthreads();
-    // neighbour pairs (2j, 2j + 1) outside quads
     const uint64_t ka = key[2 * j], kb = key[2 * j + 1];
     int qa = -1, qb = -1, cnt = 0;
-    if (ka != ~0ull && kb != ~0ull && !quad_ok[j >> 1]) {
+    if (ka != ~0ull && kb != ~0ull) {
         qa = (int)(q0 + (int64_t)(ka & 2047u));
         qb = (int)(q0 + (int64_t)(kb & 2047u));
         cnt = pairable(plan[qa], plan[qb], min_rows) ? 1 : 0;
     }
-    for (int i = j; i < n; i += kPairSortThreads) grouped[q0 + i] = 0;
+    for (int i = j; i < n; i += kPairSortThreads) paired[q0 + i] = 0;
     __syncthreads();
-    if (cnt) grouped[qa] = grouped[qb] = 1;
-    if (qcnt)
-        for (int i = 0; i < 4; ++i) grouped[qd[i]] = 1;
-    // slots: segment s owns pair slots [s kPairSeg / 2, + ceil(n / 2)) and
-    // quad slots [s kPairSeg / 4, + ceil(n / 4)), filled in sorted order
+    if (cnt) paired[qa] = paired[qb] = 1;
+    // segment s owns item slots [s kPairSeg / 2, + ceil(n / 2)): at most one
+    // pair per two of its queries
     int total = 0;
     const int at = block_prefix(cnt, wsum, total);
     PairItem* its = items + q0 / 2;
     if (cnt) its[at] = PairItem{qa, qb};
     for (int i = total + j; i < (n + 1) / 2; i += kPairSortThreads) its[i] = PairItem{-1, -1};
-    if (quads != nullptr) {
-        int qtotal = 0;
-        const int qat = block_prefix(qcnt, wsum, qtotal);
-        QuadItem* qits = quads + q0 / 4;
-        if (qcnt) qits[qat] = QuadItem{{qd[0], qd[1], qd[2], qd[3]}};
-        for (int i = qtotal + j; i < (n + 3) / 4; i += kPairSortThreads) qits[i] = QuadItem{{-1, -1, -1, -1}};
-    }
 }
 
 template <int KP>
@@ -1215,323 +1165,6 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     merge_warps<KP, kPairWarps>(tkB, tkbufB, k, lane, warp, outB);
 }
 
-// ---- four queries per CTA on the sorted copy -------------------------------
-//
-// The same scheme as the two-query kernel with four queries per look-up:
-// word w of codeword row c of the packed table holds, in byte j, query j's
-// entry of subspace w mod 16 quantised to 5 bits, q_j = floor((L - lo_m)
-// * inv_j) with inv_j = 31 / (the widest subspace's range of query j).
-// A lane adds the words of its row's first eight look-ups into one register
-// and the last eight into another: each byte then holds at most 8 * 31 = 248,
-// so no carry crosses the bytes.  X = (lo >> 2 & 0x3F3F3F3F) + (hi >> 2 &
-// 0x3F3F3F3F) holds in byte j floor(lo_j / 4) + floor(hi_j / 4) <= S_j / 4
-// (S_j the row's quantised sum for query j, at most 124), so a row with
-// S_j <= T_j (T_j = quant_bound of the query's k-th key) has X_j <= floor(T_j
-// / 4) = B_j: the packed bounds (B_j + 0x80 in byte j, B_j clamped to
-// [-1, 127]) minus X keep bit 7 of byte j for every such row, and no borrow
-// crosses the bytes.  Those rows are rescored exactly as in the two-query
-// kernel, so the keys offered to each query's top-k are those of the
-// one-query loop, bit for bit.  Per code byte: one byte permute, one
-// shared load and half an add serve four queries.  12 warps, one CTA per
-// SM: the packed table (64 KB), four unreplicated float32 tables (64 KB) and
-// 12 x 4 lists of 2 KP keys fit next to each other for KP <= 128.
-constexpr int kQuadWarps = 12;
-constexpr int kQuadThreads = kQuadWarps * 32;
-constexpr int kQMax4 = 31;            // 8 * 31 < 2^8
-constexpr int kU4 = 4;                // positions per lane per round
-
-size_t scan_quad_smem_bytes(int kp) {
-    return (size_t)kTabBytes16 + 4 * (size_t)kExactBytes16 + 128 * 4 + 4 * 8 + (size_t)kQuadWarps * 4 * 2 * kp * 8;
-}
-
-// Packed bounds of four queries: byte j = B_j + 0x80, B_j = floor(T_j / 4)
-// clamped to [-1, 127] (T_j = -1: no row; INT_MAX: every row).
-__device__ __forceinline__ uint32_t pack_bounds4(const int (&t)[4]) {
-    uint32_t r = 0u;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        int b = t[j] < 0 ? -1 : (t[j] >> 2);
-        b = b > 127 ? 127 : b;
-        r |= (uint32_t)(b + 0x80) << (8 * j);
-    }
-    return r;
-}
-
-constexpr uint32_t kCandBytes = 0x80808080u;
-
-// X of one M = 16 position (codes c) for the four queries at once.
-template <bool FAST>
-__device__ __forceinline__ uint32_t quad_sum(const uint4 c, uint32_t tb, uint32_t base) {
-    const uint32_t w[4] = {c.x, c.y, c.z, c.w};
-    uint32_t v[16];
-#pragma unroll
-    for (int s = 0; s < 16; ++s) {
-        const uint32_t sel = 0x5504u | ((uint32_t)(s & 3) << 4);
-        uint32_t o = __byte_perm(w[s >> 2], tb, sel);
-        if (!FAST) o += base;
-        constexpr uint32_t B0 = FAST ? kDynSmemBase : 0u;
-        switch (s) {
-#define IFVS_LD4_CASE(S)                         \
-    case S:                                      \
-        v[S] = lds_u32_imm<B0 + 4 * S>(o);       \
-        break;
-            IFVS_LD4_CASE(0) IFVS_LD4_CASE(1) IFVS_LD4_CASE(2) IFVS_LD4_CASE(3)
-            IFVS_LD4_CASE(4) IFVS_LD4_CASE(5) IFVS_LD4_CASE(6) IFVS_LD4_CASE(7)
-            IFVS_LD4_CASE(8) IFVS_LD4_CASE(9) IFVS_LD4_CASE(10) IFVS_LD4_CASE(11)
-            IFVS_LD4_CASE(12) IFVS_LD4_CASE(13) IFVS_LD4_CASE(14) IFVS_LD4_CASE(15)
-#undef IFVS_LD4_CASE
-            default: break;
-        }
-    }
-    uint32_t lo = 0u, hi = 0u;
-#pragma unroll
-    for (int s = 0; s < 8; ++s) {
-        lo += v[s];
-        hi += v[s + 8];
-    }
-    return ((lo >> 2) & 0x3F3F3F3Fu) + ((hi >> 2) & 0x3F3F3F3Fu);
-}
-
-// One round of kU4 positions of a block for four queries: the shared bounds
-// refreshed, quantised sums, candidates by the packed bounds, exact
-// distances and top-k offers for the candidates.  mask[u] holds 0x80 in
-// byte j when position u lies in query j's range.
-template <int KP, bool FAST>
-__device__ __forceinline__ void quad_round(const uint4 (&c)[kU4], const uint32_t* __restrict__ rows,
-                                           uint32_t pos0, const uint32_t (&mask)[kU4], WarpTopK<KP> (&tk)[4],
-                                           const float* ex, const float (&sl)[4], const float (&inv)[4],
-                                           uint32_t tb, uint32_t base, int rot, int lane, uint32_t& Bpk) {
-    {
-        bool changed = false;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const uint64_t o = tk[j].thr;
-            tk[j].refresh(lane);
-            changed |= tk[j].thr != o;
-        }
-        if (changed) {
-            int t[4];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) t[j] = quant_bound(tk[j].thr, sl[j], inv[j]);
-            Bpk = pack_bounds4(t);
-        }
-    }
-    uint32_t cb[kU4], any = 0u;
-#pragma unroll
-    for (int u = 0; u < kU4; ++u) {
-        cb[u] = (Bpk - quad_sum<FAST>(c[u], tb, base)) & mask[u];
-        any |= cb[u];
-    }
-    if (!__any_sync(0xFFFFFFFFu, any != 0u)) return;
-#pragma unroll
-    for (int u = 0; u < kU4; ++u) {
-        const uint32_t pos = pos0 + 32u * (uint32_t)u;
-        float d[4];
-        bool cj[4];
-        bool anyj = false;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            cj[j] = (cb[u] >> (8 * j + 7)) & 1u;
-            d[j] = cj[j] ? exact16(c[u], ex + j * 4096, rot) : 0.f;
-            cj[j] = cj[j] && __float_as_uint(d[j]) <= (uint32_t)(tk[j].thr >> 32);
-            anyj |= cj[j];
-        }
-        const uint32_t row = anyj ? __ldg(rows + pos) : 0u;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const uint64_t key = ((uint64_t)__float_as_uint(d[j]) << 32) | row;
-            tk[j].offer(key, cj[j] && key < tk[j].thr, lane);
-        }
-    }
-    int t[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) t[j] = quant_bound(tk[j].thr, sl[j], inv[j]);
-    Bpk = pack_bounds4(t);
-}
-
-template <int KP, bool FAST>
-__device__ __forceinline__ void scan_positions_quad(const uint8_t* __restrict__ codes,
-                                                    const uint32_t* __restrict__ rows, const int64_t (&ra)[4],
-                                                    const int64_t (&rb)[4], int64_t blk0, int64_t blk1,
-                                                    WarpTopK<KP> (&tk)[4], const float* ex, const float (&sl)[4],
-                                                    const float (&inv)[4], uint32_t base, int lane, int warp) {
-    const uint32_t tb = 4u * (uint32_t)lane;
-    const int rot = lane & 15;
-    const uint64_t keep = policy_evict_last();
-    uint32_t a32[4], b32[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        a32[j] = (uint32_t)ra[j];
-        b32[j] = (uint32_t)rb[j];
-    }
-    uint32_t Bpk;
-    {
-        int t[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) t[j] = quant_bound(tk[j].thr, sl[j], inv[j]);
-        Bpk = pack_bounds4(t);
-    }
-    for (int64_t blk = blk0 + warp; blk < blk1; blk += kQuadWarps) {
-        const uint32_t p0 = (uint32_t)(blk * kBlockRows);
-        const uint32_t pe = p0 + kBlockRows;
-        uint32_t full = 0u, in = 0u;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const bool i_ = p0 < b32[j] && pe > a32[j];
-            in |= (i_ ? 0x80u : 0u) << (8 * j);
-            full |= ((i_ && p0 >= a32[j] && pe <= b32[j]) ? 0x80u : 0u) << (8 * j);
-        }
-        if (in == 0u) continue;
-        if (full == in) {
-            // each query takes all or none of the block: one mask for all rows
-            uint32_t mask[kU4];
-#pragma unroll
-            for (int u = 0; u < kU4; ++u) mask[u] = full;
-            const uint32_t pb = p0 + (uint32_t)lane;
-#pragma unroll 1
-            for (int j0 = 0; j0 < 32; j0 += kU4) {
-                uint4 c[kU4];
-#pragma unroll
-                for (int u = 0; u < kU4; ++u)
-                    c[u] = ldg_nc_v4(codes + (size_t)(pb + 32u * (uint32_t)(j0 + u)) * 16, keep);
-                quad_round<KP, FAST>(c, rows, pb + 32u * (uint32_t)j0, mask, tk, ex, sl, inv, tb, base, rot, lane,
-                                     Bpk);
-            }
-            continue;
-        }
-#pragma unroll 1
-        for (int j0 = 0; j0 < 32; j0 += kU4) {
-            const uint32_t pos0 = p0 + 32u * (uint32_t)j0 + (uint32_t)lane;
-            uint32_t mask[kU4];
-            uint4 c[kU4];
-#pragma unroll
-            for (int u = 0; u < kU4; ++u) {
-                const uint32_t pos = pos0 + 32u * (uint32_t)u;
-                uint32_t m = 0u;
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    m |= ((pos >= a32[j] && pos < b32[j]) ? 0x80u : 0u) << (8 * j);
-                mask[u] = m;
-                c[u] = m != 0u ? ldg_nc_v4(codes + (size_t)pos * 16, keep) : make_uint4(0, 0, 0, 0);
-            }
-            quad_round<KP, FAST>(c, rows, pos0, mask, tk, ex, sl, inv, tb, base, rot, lane, Bpk);
-        }
-    }
-}
-
-template <int KP>
-__global__ void __launch_bounds__(kQuadThreads, 1)
-k_scan_list_quad(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan,
-                 const QuadItem* __restrict__ items, int k, ScanShape sh, uint64_t* __restrict__ partials) {
-    extern __shared__ __align__(256) uint8_t smem[];
-    uint32_t* ptab = reinterpret_cast<uint32_t*>(smem);
-    float* ex = reinterpret_cast<float*>(smem + kTabBytes16);                       // [4][256][16]
-    float* prm = reinterpret_cast<float*>(smem + kTabBytes16 + 4 * kExactBytes16);  // [4][lo 16 | hi 16]
-    uint64_t* ctab = reinterpret_cast<uint64_t*>(smem + kTabBytes16 + 4 * kExactBytes16 + 128 * 4);
-    uint64_t* tkbuf = ctab + 4;                                                     // [4][warps][2 KP]
-    float* red = reinterpret_cast<float*>(tkbuf);   // [warp][4][32], before the lists are set up
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const QuadItem it = items[blockIdx.x];
-    if (it.q[0] < 0) return;
-    const int chunk = blockIdx.y;
-    ScanPlan p[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) p[j] = plan[it.q[j]];
-    const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
-    const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
-    int64_t lo = INT64_MAX, hi = 0;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const int64_t l = max(c0, p[j].a / kBlockRows);
-        const int64_t h = min(c1, (p[j].b + kBlockRows - 1) / kBlockRows);
-        if (p[j].a < p[j].b && l < h) {
-            lo = min(lo, l);
-            hi = max(hi, h);
-        }
-    }
-    if (lo >= hi) {
-        for (int i = threadIdx.x; i < 4 * k; i += kQuadThreads) {
-            const int j = i / k;
-            partials[((int64_t)it.q[j] * sh.n_chunks + chunk) * (int64_t)k + (i - j * k)] = ~0ull;
-        }
-        return;
-    }
-    // 1) unreplicated float32 tables ex[j][c * 16 + m] and the extremes of
-    //    each subspace; a thread keeps one subspace m
-    {
-        const int m = threadIdx.x & 15;
-        float l4[4], h4[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            l4[j] = INFINITY;
-            h4[j] = -INFINITY;
-        }
-        for (int i = threadIdx.x; i < 4096; i += kQuadThreads) {
-            const int c = i >> 4;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const float x = __ldg(tables + (int64_t)it.q[j] * 256 * 64 + c * 64 + m);
-                ex[j * 4096 + i] = x;
-                l4[j] = fminf(l4[j], x);
-                h4[j] = fmaxf(h4[j], x);
-            }
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            l4[j] = fminf(l4[j], __shfl_xor_sync(0xFFFFFFFFu, l4[j], 16));
-            h4[j] = fmaxf(h4[j], __shfl_xor_sync(0xFFFFFFFFu, h4[j], 16));
-            if (lane < 16) {
-                red[warp * 128 + j * 32 + m] = l4[j];
-                red[warp * 128 + j * 32 + 16 + m] = h4[j];
-            }
-        }
-    }
-    __syncthreads();
-    if (threadIdx.x < 128) {
-        const int t = threadIdx.x;   // query t / 32; lo for (t & 16) == 0, else hi
-        const bool is_lo = (t & 16) == 0;
-        float v = red[t];
-        for (int w = 1; w < kQuadWarps; ++w) v = is_lo ? fminf(v, red[w * 128 + t]) : fmaxf(v, red[w * 128 + t]);
-        prm[t] = v;
-    }
-    __syncthreads();
-    float inv[4], sl[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) quant_params(prm + 32 * j, prm + 32 * j + 16, inv[j], sl[j], kQMax4);
-    // 2) the packed table: byte j of word w of row c = q_j[w mod 16][c]
-    for (int i = threadIdx.x; i < 256 * 64; i += kQuadThreads) {
-        const int c = i >> 6, m = i & 15;
-        uint32_t wd = 0u;
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-            wd |= quant_q(ex[j * 4096 + c * 16 + m], prm[32 * j + m], inv[j], (float)kQMax4) << (8 * j);
-        ptab[i] = wd;
-    }
-    __syncthreads();   // the reduction scratch becomes the lists
-    if (threadIdx.x < 4) ctab[threadIdx.x] = ~0ull;
-    WarpTopK<KP> tk[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) tk[j].init(tkbuf + ((int64_t)j * kQuadWarps + warp) * 2 * KP, k, lane, ctab + j);
-    __syncthreads();
-    int64_t ra[4], rb[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        ra[j] = p[j].a;
-        rb[j] = p[j].b;
-    }
-    const uint32_t base = (uint32_t)__cvta_generic_to_shared(ptab);
-    if (base == kDynSmemBase)
-        scan_positions_quad<KP, true>(sc.codes_of(p[0].col), sc.rows_of(p[0].col), ra, rb, lo, hi, tk, ex, sl, inv,
-                                      base, lane, warp);
-    else
-        scan_positions_quad<KP, false>(sc.codes_of(p[0].col), sc.rows_of(p[0].col), ra, rb, lo, hi, tk, ex, sl,
-                                       inv, base, lane, warp);
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-        merge_warps<KP, kQuadWarps>(tk[j], tkbuf + (int64_t)j * kQuadWarps * 2 * KP, k, lane, warp,
-                                    partials + ((int64_t)it.q[j] * sh.n_chunks + chunk) * (int64_t)k);
-}
-
 template <int KP, bool M16, int MINB>
 static cudaError_t launch_list_one(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
                                    int k, const ScanShape& sh, uint64_t* partials, const uint8_t* paired,
@@ -1552,73 +1185,56 @@ static int max_smem_optin() {
 }
 
 size_t scan_list_workspace_bytes(int64_t nq) {
-    // pair slots, quad slots (each segment rounds its count up), a flag per query
-    return (size_t)(nq + 2 * kPairSeg) * sizeof(PairItem) + (size_t)(nq / 4 + kPairSeg) * sizeof(QuadItem) +
-           (size_t)nq + 64;
+    // pair slots (each segment rounds its count up), a flag per query
+    return (size_t)(nq + 2 * kPairSeg) * sizeof(PairItem) + (size_t)nq + 64;
 }
 
 template <int KP>
 static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
                                   int k, const ScanShape& sh, uint64_t* partials, uint8_t* work,
-                                  int64_t pair_min_rows, bool quads, int* launches, cudaStream_t s) {
+                                  int64_t pair_min_rows, int* launches, cudaStream_t s) {
     const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
     const size_t ps = scan_pair_smem_bytes(KP);
-    const size_t qs = scan_quad_smem_bytes(KP);
-    const int optin = max_smem_optin();
-    const uint8_t* grouped = nullptr;
+    const uint8_t* paired = nullptr;
     int nl = 0;
-    if (m16 && work != nullptr && ps <= (size_t)optin) {
-        // M = 16: long, overlapping ranges are grouped by k_group_items and
-        // served by the four- and two-query kernels; the one-query kernel
-        // takes the rest
-        PairItem* pairs = reinterpret_cast<PairItem*>(work);
-        QuadItem* quad_items = reinterpret_cast<QuadItem*>(work + (size_t)(nq + 2 * kPairSeg) * sizeof(PairItem));
-        uint8_t* gd = reinterpret_cast<uint8_t*>(quad_items + (nq / 4 + kPairSeg));
-        const bool q_on = quads && qs <= (size_t)optin;
+    if (m16 && work != nullptr && ps <= (size_t)max_smem_optin()) {
+        // M = 16: long, overlapping ranges are paired by k_pair_items and
+        // served by the two-query kernel; the one-query kernel takes the rest
+        PairItem* items = reinterpret_cast<PairItem*>(work);
+        uint8_t* pd = reinterpret_cast<uint8_t*>(items + nq + 2 * kPairSeg);
         const unsigned segs = (unsigned)((nq + kPairSeg - 1) / kPairSeg);
-        k_group_items<<<segs, kPairSortThreads, 0, s>>>(plan, nq, pair_min_rows, q_on ? 1 : 0,
-                                                        q_on ? quad_items : nullptr, pairs, gd);
+        k_pair_items<<<segs, kPairSortThreads, 0, s>>>(plan, nq, pair_min_rows, items, pd);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
-        nl = 1;
-        if (q_on) {
-            if ((e = cudaFuncSetAttribute(k_scan_list_quad<KP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)qs)) != cudaSuccess)
-                return e;
-            dim3 grid((unsigned)((nq + 3) / 4), (unsigned)sh.n_chunks);   // at most nq / 4 quads
-            k_scan_list_quad<KP><<<grid, kQuadThreads, qs, s>>>(tab, sc, plan, quad_items, k, sh, partials);
-            if ((e = cudaGetLastError()) != cudaSuccess) return e;
-            ++nl;
-        }
         if ((e = cudaFuncSetAttribute(k_scan_list_pair<KP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       (int)ps)) != cudaSuccess)
             return e;
         dim3 grid((unsigned)((nq + 1) / 2), (unsigned)sh.n_chunks);   // at most nq / 2 pairs
-        k_scan_list_pair<KP><<<grid, kPairThreads, ps, s>>>(tab, sc, plan, pairs, k, sh, partials);
+        k_scan_list_pair<KP><<<grid, kPairThreads, ps, s>>>(tab, sc, plan, items, k, sh, partials);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
-        grouped = gd;
-        ++nl;
+        paired = pd;
+        nl = 2;
     }
     const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
     if (launches) *launches = nl + 1;
     if (m16) {
         if ((size_t)233472 / (smem + 1024) >= 2)
-            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, grouped, smem, s);
-        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, grouped, smem, s);
+            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
+        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
     }
-    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, grouped, smem, s);
+    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
 }
 
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
                              const ScanShape& sh, uint64_t* partials, uint8_t* work, int64_t pair_min_rows,
-                             bool quads, cudaStream_t s, int* launches) {
+                             cudaStream_t s, int* launches) {
     if (launches) *launches = 0;
     if (nq <= 0) return cudaSuccess;
     switch (scan_kp(k)) {
-        case 32: return launch_list_kp<32>(tab, sc, plan, nq, k, sh, partials, work, pair_min_rows, quads, launches, s);
-        case 64: return launch_list_kp<64>(tab, sc, plan, nq, k, sh, partials, work, pair_min_rows, quads, launches, s);
-        case 128: return launch_list_kp<128>(tab, sc, plan, nq, k, sh, partials, work, pair_min_rows, quads, launches, s);
-        default: return launch_list_kp<256>(tab, sc, plan, nq, k, sh, partials, work, pair_min_rows, quads, launches, s);
+        case 32: return launch_list_kp<32>(tab, sc, plan, nq, k, sh, partials, work, pair_min_rows, launches, s);
+        case 64: return launch_list_kp<64>(tab, sc, plan, nq, k, sh, partials, work, pair_min_rows, launches, s);
+        case 128: return launch_list_kp<128>(tab, sc, plan, nq, k, sh, partials, work, pair_min_rows, launches, s);
+        default: return launch_list_kp<256>(tab, sc, plan, nq, k, sh, partials, work, pair_min_rows, launches, s);
     }
 }
 

@@ -201,14 +201,10 @@ def test_threshold_and_launch_counts(ifvs):
     g.stage_times(reset=True)
     g.search(q, p, 10, flags=ifvs.IFVS_F_STAGE_TIMING)
     t = g.stage_times(reset=True)
-    # plan + filter; the bitmap scan, the grouping of the sorted-copy
-    # queries, the four-, two- and one-query sorted-copy scans (four-query
-    # CTAs for k <= 128)
-    assert t["filter"][1] == 2 and t["scan"][1] == 5
+    # plan + filter; the bitmap scan, the pairing of the sorted-copy queries,
+    # the two-query and the one-query sorted-copy scans, for every k
+    assert t["filter"][1] == 2 and t["scan"][1] == 4
     g.search(q, p, 100, flags=ifvs.IFVS_F_STAGE_TIMING)
-    t = g.stage_times(reset=True)
-    assert t["scan"][1] == 5
-    g.search(q, p, 100, flags=ifvs.IFVS_F_STAGE_TIMING | ifvs.IFVS_F_NO_QUADS)
     t = g.stage_times(reset=True)
     assert t["scan"][1] == 4
     g.search(q, p, 200, flags=ifvs.IFVS_F_STAGE_TIMING)
@@ -249,7 +245,7 @@ def _one_by_one(g, q, p, k, **kw):
 @pytest.mark.parametrize("case", ["normal", "one_wide_subspace", "constant", "tiny_range", "huge"])
 @pytest.mark.parametrize("k", [100, 128])
 def test_pair_kernel_equals_one_query_kernel(ifvs, orc, case, k):
-    """The four- and two-query kernels drop rows by a quantised lower bound and
+    """The two-query kernel drops rows by a quantised lower bound and
     rescores the rest exactly in the one-query kernel's order, so a batch
     whose queries pair up (pairing forced at this size) must return, bit for
     bit, what each query returns alone and what the batch returns with no
@@ -278,10 +274,8 @@ def test_pair_kernel_equals_one_query_kernel(ifvs, orc, case, k):
     q[9] = q[8]                                    # a pair of identical vectors
     g.stage_times(reset=True)
     a = g.search(q, p, k, flags=ifvs.IFVS_F_STAGE_TIMING, pair_min_rows=1)
-    # bitmap, grouping, four-, two- and one-query scans
-    assert g.stage_times(reset=True)["scan"][1] == 5
-    for b in (_one_by_one(g, q, p, k, pair_min_rows=1), g.search(q, p, k, pair_min_rows=-1),
-              g.search(q, p, k, pair_min_rows=1, flags=ifvs.IFVS_F_NO_QUADS)):
+    assert g.stage_times(reset=True)["scan"][1] == 4   # bitmap, pairing, two-query, one-query scans
+    for b in (_one_by_one(g, q, p, k, pair_min_rows=1), g.search(q, p, k, pair_min_rows=-1)):
         for x, y in zip(a, b):
             np.testing.assert_array_equal(x, y)
     if case != "huge":
@@ -298,10 +292,9 @@ def test_pair_kernel_with_conditioning(ifvs, orc, oracle_index):
     g = ifvs.Index(ix.codes, ix.attrs, D=w.D, K=w.K)
     g.load_codebooks(ix.codebook, bank=cond.bank, W=cond.W, hash_seeds=cond.seeds)
     a = g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=1)
-    for b in (g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=-1),
-              g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=1, flags=ifvs.IFVS_F_NO_QUADS)):
-        for j in range(3):
-            np.testing.assert_array_equal(a[j], b[j])
+    b = g.search(qs.q, qs.preds, 100, wz=qs.wz, pair_min_rows=-1)
+    for j in range(3):
+        np.testing.assert_array_equal(a[j], b[j])
     oi, od, on, st = orc.search(ix.codes, ix.attrs, ix.codebook, qs.q, qs.preds, 100, bank=cond.bank,
                                 W=cond.W, seeds=cond.seeds, wz=qs.wz, want_stages=True)
     np.testing.assert_array_equal(a[2], on)
@@ -339,8 +332,6 @@ def test_pairing_by_sorted_ranges(ifvs, orc, k):
     for x, y in zip(a, b):
         np.testing.assert_array_equal(x[perm], y)
     for x, y in zip(a, g.search(q, p, k, sub_batch=nq, pair_min_rows=-1)):
-        np.testing.assert_array_equal(x, y)
-    for x, y in zip(a, g.search(q, p, k, sub_batch=nq, pair_min_rows=1, flags=ifvs.IFVS_F_NO_QUADS)):
         np.testing.assert_array_equal(x, y)
     c = _one_by_one(g, q[:24], p[:24], k)
     for x, y in zip(a, c):

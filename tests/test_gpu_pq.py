@@ -110,3 +110,31 @@ def test_device_io_on_a_caller_stream(ifvs, orc):
     H1, hobj = ifvs.ifvs_pq_train(X, C0, 2)
     np.testing.assert_array_equal(C1.cpu().numpy(), H1)
     np.testing.assert_array_equal(obj.cpu().numpy(), hobj)
+
+
+def test_device_io_without_a_stream_orders_after_default_stream_work(ifvs):
+    """With device I/O and no stream, the call runs on a stream of the
+    library's own that must wait for the caller's pending work on the legacy
+    default stream: vectors computed there by torch right before the call
+    (no synchronisation in between) are encoded as if the call had waited."""
+    import torch
+    dev = torch.device("cuda", 0)
+    torch.cuda.synchronize()
+    M, K, ds, n = 16, 256, 8, 1 << 21
+    with torch.cuda.stream(torch.cuda.default_stream(dev)):
+        g = torch.Generator(device=dev)
+        g.manual_seed(11)
+        C = torch.randn((M, K, ds), generator=g, device=dev)
+        for rep in range(3):
+            torch.cuda.synchronize()
+            # long default-stream work that produces X, then the call at once
+            X = torch.randn((n, M * ds), generator=g, device=dev)
+            for _ in range(4):
+                X = torch.tanh(X * 1.5) * 2.0
+            codes = torch.empty((n, M), dtype=torch.uint8, device=dev)
+            ifvs.ifvs_pq_encode(X, C, codes=codes, flags=ifvs.IFVS_F_DEVICE_IO, stream=None)
+            torch.cuda.synchronize()
+            again = torch.empty_like(codes)
+            ifvs.ifvs_pq_encode(X, C, codes=again, flags=ifvs.IFVS_F_DEVICE_IO, stream=None)
+            torch.cuda.synchronize()
+            assert torch.equal(codes, again), "the encode read X before it was written (rep %d)" % rep
