@@ -74,6 +74,8 @@ def parse():
     ap.add_argument("--pair-min-rows", type=int, default=0,
                     help="two-query CTAs for overlapping one-column ranges spanning at least this many "
                          "rows (0 = library default, -1 = never)")
+    ap.add_argument("--plain-loads", action="store_true",
+                    help="one-query sorted-copy CTAs read code rows by vector loads, not bulk copies")
     ap.add_argument("--out", default="", help="also write the JSON line to this file")
     ap.add_argument("--mode", default="search", choices=["search", "pq", "train"],
                     help="search: the query path; pq: PQ encoding + Lloyd training of the index; "
@@ -564,7 +566,7 @@ def run_ifvs(args):
                         torch.empty((n, w.k), dtype=torch.float32, device=device),
                         torch.empty(n, dtype=torch.int64, device=device)))
     torch.cuda.synchronize()
-    flags = ifvs.IFVS_F_DEVICE_IO | ifvs.IFVS_F_STAGE_TIMING
+    flags = ifvs.IFVS_F_DEVICE_IO | ifvs.IFVS_F_STAGE_TIMING | (ifvs.IFVS_F_PLAIN_LOADS if args.plain_loads else 0)
 
     def step(i):
         b = i % nb
@@ -680,7 +682,8 @@ def run_ifvs(args):
             oi, od, on, _ = host_out[b]
             ifvs.ifvs_search_batch(g.h, q, p, w.k, wz=wz, ids=oi, dists=od, npass=on, stream=sptr,
                                    chunk_blocks=args.chunk_blocks, list_max_ppm=args.list_max_ppm,
-                                   rerank=args.rerank, pair_min_rows=args.pair_min_rows)
+                                   rerank=args.rerank, pair_min_rows=args.pair_min_rows,
+                                   flags=ifvs.IFVS_F_PLAIN_LOADS if args.plain_loads else 0)
 
         for i in range(args.warmup):
             hstep(i)

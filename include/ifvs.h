@@ -60,7 +60,9 @@ typedef enum {
     IFVS_ERR_OOM = -2,          /* device allocation failed                   */
     IFVS_ERR_CUDA = -3,         /* a CUDA runtime call or kernel failed       */
     IFVS_ERR_STATE = -4,        /* e.g. search before ifvs_load_codebooks     */
-    IFVS_ERR_UNSUPPORTED = -5   /* shape outside the supported range          */
+    IFVS_ERR_UNSUPPORTED = -5,  /* shape outside the supported range          */
+    IFVS_ERR_TIMEOUT = -6       /* a bounded wait inside a kernel ran out; the
+                                   results are incomplete, the GPU stays usable */
 } ifvs_status;
 
 /* Every entry point that allocates device memory returns IFVS_ERR_OOM when
@@ -68,7 +70,13 @@ typedef enum {
  * index as it was (later calls may succeed).  For tests of that path the
  * failure can be injected on the host: while the environment variable
  * IFVS_FAIL_ALLOC holds a number n >= 1, the n-th device allocation since
- * the variable took its current string fails without calling cudaMalloc. */
+ * the variable took its current string fails without calling cudaMalloc.
+ *
+ * Kernels never wait without a bound.  The sorted-copy scan waits for its
+ * bulk-copied code tiles for at most about half a second per tile; when a
+ * wait runs out the search returns IFVS_ERR_TIMEOUT and the device stays
+ * usable.  For tests of that path, while the environment variable
+ * IFVS_TEST_STALL_COPIES is "1" every such wait runs out. */
 
 /* Clause operators (Listing 1 uses = and >; all are intervals on integers):
  *   EQ    a == lo        RANGE lo <= a < hi     GE  a >= lo
@@ -102,6 +110,10 @@ typedef struct {
                                      on the launching stream (ifvs_stage_times) */
 #define IFVS_F_PLAIN_PQ     0x4u  /* ignore the memory bank: Delta = 0 (plain PQ
                                      ADC, baseline Pre_IndexPQ_ADC of §3.2)   */
+#define IFVS_F_PLAIN_LOADS  0x8u  /* search, M = 16 sorted-copy scan: one-query
+                                     CTAs read code rows with per-lane vector
+                                     loads instead of bulk copies (TMA) into
+                                     shared memory; same results              */
 
 typedef struct {
     uint32_t flags;     /* IFVS_F_*                                            */

@@ -79,6 +79,16 @@ cudaError_t device_malloc(void** p, size_t bytes) {
     return cudaMalloc(p, bytes);
 }
 
+// Timeout injection for tests of the scan's bounded waits (no GPU fault
+// involved): while the environment variable IFVS_TEST_STALL_COPIES is "1",
+// the bulk-copy barriers of the sorted-copy scan expect 16 bytes more than
+// their copies deliver, so every wait on them runs out after its bound and
+// the search returns IFVS_ERR_TIMEOUT with the context intact.
+bool stall_copies_for_tests() {
+    const char* v = getenv("IFVS_TEST_STALL_COPIES");
+    return v != nullptr && v[0] == '1' && v[1] == '\0';
+}
+
 struct DevBuf {
     void* p = nullptr;
     size_t cap = 0;
@@ -336,7 +346,7 @@ struct Stage {
 };
 
 struct Opts {
-    bool dio = false, timing = false, plain = false;
+    bool dio = false, timing = false, plain = false, plain_loads = false;
     int R = 0;
     int64_t sub_batch = 0;
     int64_t chunk_blocks = 0;
@@ -359,7 +369,7 @@ constexpr int64_t kPairDefaultMinRows = int64_t(1) << 22;
 
 int parse_opts(const ifvs_search_params* p, Opts* o) {
     if (!p) return 0;
-    if (p->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING | IFVS_F_PLAIN_PQ))
+    if (p->flags & ~(IFVS_F_DEVICE_IO | IFVS_F_STAGE_TIMING | IFVS_F_PLAIN_PQ | IFVS_F_PLAIN_LOADS))
         return set_err(IFVS_ERR_ARG, "unknown flag bits 0x%x", p->flags);
     if (p->chunk_blocks < 0) return set_err(IFVS_ERR_ARG, "chunk_blocks must be >= 0");
     if (p->rerank < 0 || p->rerank > IFVS_MAX_K)
@@ -371,6 +381,7 @@ int parse_opts(const ifvs_search_params* p, Opts* o) {
     o->dio = p->flags & IFVS_F_DEVICE_IO;
     o->timing = p->flags & IFVS_F_STAGE_TIMING;
     o->plain = p->flags & IFVS_F_PLAIN_PQ;
+    o->plain_loads = p->flags & IFVS_F_PLAIN_LOADS;
     o->R = p->rerank;
     o->sub_batch = p->sub_batch;
     o->chunk_blocks = p->chunk_blocks;
@@ -499,11 +510,15 @@ int run_path(ifvs_index* ix, cudaStream_t s, const Opts& o, const float* dq,
     if (plan) {
         Stage st(ix, s, o.timing, IFVS_STAGE_SCAN);
         int nl = 0;
-        const int64_t pmin = o.pair_min_rows > 0 ? o.pair_min_rows : kPairDefaultMinRows;
+        ListOpts lo;
+        lo.pair_min_rows = o.pair_min_rows > 0 ? o.pair_min_rows : kPairDefaultMinRows;
+        lo.bulk = !o.plain_loads;
+        lo.tx_extra = stall_copies_for_tests() ? 16u : 0u;
+        lo.err = ix->w_err.as<int>();
         const cudaError_t e = launch_scan_list(ix->w_tab.as<float>(), ix->sorted(), plan, n, kk, sh,
                                                ix->w_part.as<uint64_t>(),
                                                o.pair_min_rows < 0 ? nullptr : ix->w_items.as<uint8_t>(),
-                                               pmin, s, &nl);
+                                               lo, s, &nl);
         CUDA_TRY(st.end(e, nl));
     }
     int64_t* m_ids = o.R > 0 ? ix->w_cand.as<int64_t>() : out_ids;
@@ -592,6 +607,9 @@ int finish(ifvs_index* ix, cudaStream_t s, bool check_preds) {
     if (check_preds) {
         int err = 0;
         CUDA_TRY(cudaMemcpy(&err, ix->w_err.p, sizeof(int), cudaMemcpyDeviceToHost));
+        if (err & 4)
+            return set_err(IFVS_ERR_TIMEOUT, "a bounded wait of the scan for its bulk-copied code tiles ran out; "
+                                             "the results are incomplete");
         if (err & 2) return set_err(IFVS_ERR_ARG, "a candidate row id is outside -1..N-1");
         if (err) return set_err(IFVS_ERR_ARG, "a predicate is malformed (n_clauses outside 0..4, "
                                               "reserved != 0, column out of range or unknown operator)");

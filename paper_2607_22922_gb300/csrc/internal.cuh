@@ -202,9 +202,19 @@ struct PairItem {
 // positions, served by a two-query kernel; a one-query kernel serves the
 // other queries (all of them when work is null or M != 16).  *launches =
 // kernels launched.
+// M = 16 one-query CTAs bring their code rows in by bulk copies into shared
+// memory when `bulk` (else by per-lane vector loads); a bounded wait that
+// runs out sets bit 4 of *err.  tx_extra: bytes added to what each copy's
+// barrier expects (0; positive only to exercise the timeout path).
+struct ListOpts {
+    int64_t pair_min_rows;
+    bool bulk;
+    uint32_t tx_extra;
+    int* err;
+};
 size_t scan_list_workspace_bytes(int64_t nq);
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
-                             const ScanShape& sh, uint64_t* partials, uint8_t* work, int64_t pair_min_rows,
+                             const ScanShape& sh, uint64_t* partials, uint8_t* work, const ListOpts& lo,
                              cudaStream_t s, int* launches);
 // the sorted copy of the codes: dst position p <- row rows[p] of the index
 // layout `src`, re-rotated by (p mod 32) mod M; positions >= N are zero

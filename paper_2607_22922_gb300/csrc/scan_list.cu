@@ -1,0 +1,374 @@
+// Rank (§2 stage 2) over a one-column predicate's pool read as a position
+// range of that column's sorted copy of the codes: the one-query kernel
+// k_scan_list, and the launcher that first pairs overlapping ranges for the
+// two-query kernel (scan_pair.cu).  Design notes in scan_common.cuh.
+#include "scan_common.cuh"
+
+namespace ifvs {
+
+// ---- sorted-copy scan ---------------------------------------------------
+//
+// For a query of the list path (ScanPlan) the pool is the position range
+// [a, b) of one column's sorted copy of the codes, whose position p holds
+// row rows[p]'s codes rotated by (p mod 32) mod M.  CTA (query, chunk) walks
+// the chunk's 1024-position blocks that meet [a, b) exactly as the bitmap
+// path walks dense blocks: lane l takes the positions = l (mod 32), so its
+// look-ups hit banks (l + s) mod 32 and the code loads are coalesced; blocks
+// cut by a or b mask their positions.  No bitmap, no per-row bit handling,
+// and the CTAs of one chunk share its codes in L2.  The row id, needed for
+// the key, is loaded only for positions whose distance can enter the top-k.
+// The sum order (the subspaces from (p mod 32) mod M on) differs from the
+// bitmap path's, so the two agree to float32 rounding.
+
+size_t scan_list_smem_bytes(int tab_words, int kp) {
+    return (size_t)256 * tab_words * 4 + (size_t)kScanWarps * 2 * kp * 8 + 16;
+}
+
+template <int KP, bool M16, bool FAST>
+__device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes, const uint32_t* __restrict__ rows,
+                                               int64_t a, int64_t b, int64_t blk0, int64_t blk1, int wstride,
+                                               const ScanShape& sh, const float* tab, WarpTopK<KP>& tk,
+                                               int lane, int warp) {
+    const int M = M16 ? 16 : sh.M;
+    const int S = M16 ? 64 : sh.tab_words;
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
+    const uint32_t tb = 4u * (uint32_t)lane;
+    const uint64_t keep = policy_evict_last();
+    // positions fit in 32 bits: N < 2^32 - 2048
+    const uint32_t a32 = (uint32_t)a, b32 = (uint32_t)b;
+    for (int64_t blk = blk0 + warp; blk < blk1; blk += wstride) {
+        const uint32_t p0 = (uint32_t)(blk * kBlockRows);
+        const bool full = p0 >= a32 && p0 + kBlockRows <= b32;
+#pragma unroll 1
+        for (int j0 = 0; j0 < 32; j0 += kU) {
+            tk.refresh(lane);
+            uint32_t pos[kU];
+            unsigned valid = 0u;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                pos[u] = p0 + 32u * (uint32_t)(j0 + u) + (uint32_t)lane;
+                valid |= (unsigned)(full || (pos[u] >= a32 && pos[u] < b32)) << u;
+            }
+            float d[kU];
+            if constexpr (M16) {
+                uint4 c[kU];
+#pragma unroll
+                for (int u = 0; u < kU; ++u)
+                    c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)pos[u] * 16, keep) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
+            } else {
+                lookup_rows<kU>(codes, pos, valid, sh.row_bytes, M, S, tab, lane, d);
+            }
+            // a position can enter the top-k only if its distance is at most
+            // the current k-th one; only those load their row id
+            const uint32_t thr_hi = (uint32_t)(tk.thr >> 32);
+            bool cand_any = false;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) cand_any |= (valid >> u & 1u) && __float_as_uint(d[u]) <= thr_hi;
+            if (!__any_sync(0xFFFFFFFFu, cand_any)) continue;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const bool cand = (valid >> u & 1u) && __float_as_uint(d[u]) <= thr_hi;
+                const uint32_t row = cand ? __ldg(rows + pos[u]) : 0u;
+                const uint64_t key = ((uint64_t)__float_as_uint(d[u]) << 32) | row;
+                tk.offer(key, cand && key < tk.thr, lane);
+            }
+        }
+    }
+}
+
+template <int KP, bool M16, int MINB>
+__global__ void __launch_bounds__(kScanThreads, MINB)
+k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
+            int k, ScanShape sh, uint64_t* __restrict__ partials, const uint8_t* __restrict__ paired) {
+    extern __shared__ __align__(256) uint8_t smem[];
+    const int S = M16 ? 64 : sh.tab_words;
+    float* tab = reinterpret_cast<float*>(smem);
+    uint64_t* tkbuf = reinterpret_cast<uint64_t*>(smem + (size_t)256 * S * 4);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t q = blockIdx.x;
+    const int chunk = blockIdx.y;
+    const ScanPlan p = plan[q];
+    if (!p.list) return;                               // k_scan covers this query
+    if (paired != nullptr && paired[q]) return;        // k_scan_list_pair covers it
+    const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
+    const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
+    const int64_t blk0 = max(c0, p.a / kBlockRows);
+    const int64_t blk1 = min(c1, (p.b + kBlockRows - 1) / kBlockRows);
+    uint64_t* out = partials + (q * sh.n_chunks + chunk) * (int64_t)k;
+    if (p.a >= p.b || blk0 >= blk1) {
+        for (int i = threadIdx.x; i < k; i += kScanThreads) out[i] = ~0ull;
+        return;
+    }
+    {
+        const float4* src = reinterpret_cast<const float4*>(tables + q * (int64_t)256 * S);
+        float4* dst = reinterpret_cast<float4*>(tab);
+        for (int i = threadIdx.x; i < 64 * S; i += kScanThreads) dst[i] = __ldg(src + i);
+    }
+    uint64_t* cta = tkbuf + kScanWarps * 2 * KP;
+    if (threadIdx.x == 0) *cta = ~0ull;
+    WarpTopK<KP> tk;
+    tk.init(tkbuf + warp * 2 * KP, k, lane, cta);
+    __syncthreads();
+    const uint8_t* codes = sc.codes_of(p.col);
+    const uint32_t* rows = sc.rows_of(p.col);
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
+    if constexpr (M16) {
+        if (base == kDynSmemBase)
+            scan_positions<KP, true, true>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
+        else
+            scan_positions<KP, true, false>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
+    } else {
+        scan_positions<KP, false, false>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
+    }
+    tk.flush(lane);
+#pragma unroll 1
+    for (int step = 1; step < kScanWarps; step <<= 1) {
+        __syncthreads();
+        if ((warp & (2 * step - 1)) == 0) {
+            const uint64_t* other = tkbuf + (warp + step) * 2 * KP;
+            for (int i = lane; i < k; i += 32) tk.buf[KP + i] = other[i];
+            __syncwarp();
+            tk.flush(lane);
+        }
+    }
+    if (warp == 0)
+        for (int i = lane; i < k; i += 32) out[i] = tk.buf[i];
+}
+
+// ---- sorted-copy scan with bulk-copied code tiles (M = 16) ------------------
+//
+// The walk of k_scan_list with the code rows of every round brought into
+// shared memory by the bulk-copy engine (cp.async.bulk, the untiled form of
+// TMA) instead of per-lane vector loads.  A warp's round is 256 consecutive
+// positions (lane l takes positions 32u + l, u < kU = 8): 4 KB of codes, one
+// copy.  Each warp owns a ring of NST such tiles with an mbarrier each; lane
+// 0 issues the copy of round r + NST as soon as round r's rows sit in
+// registers, so a warp keeps NST rounds of codes in flight while it
+// computes, in shared memory rather than in registers.  A warp whose tile
+// has not arrived within the bounded wait sets bit 4 of *err (the search
+// returns IFVS_ERR_TIMEOUT), waits (bounded again) for its copies still in
+// flight, and stops scanning; its CTA still merges and writes its lists.
+// tx_extra (0 in normal use) is added to the bytes each barrier expects; a
+// positive value makes every wait run out, which exercises that path.
+// One tile per warp (NST = 1) keeps two 8-warp CTAs per SM; measured on the
+// 10^8-row workload it beat vector loads by 3 % (0.1 % pools) and 7 % (1 %),
+// while two or four tiles per warp (one CTA per SM) lost 38 % and 36 %.
+
+#ifndef IFVS_BULK_STAGES
+#define IFVS_BULK_STAGES 1
+#endif
+constexpr int kBulkStages = IFVS_BULK_STAGES;
+constexpr uint32_t kTileBytes = 32u * kU * 16u;    // one warp round: 256 positions x 16 bytes
+static_assert(32 % kU == 0, "whole rounds per block");
+constexpr int kRoundsPerBlock = 32 / kU;
+
+__host__ __device__ constexpr size_t bulk_ring_offset(int kp) {
+    return ((size_t)256 * 64 * 4 + (size_t)kScanWarps * 2 * kp * 8 + 16 + 127) / 128 * 128;
+}
+
+size_t scan_bulk_smem_bytes(int kp) {
+    return bulk_ring_offset(kp) + (size_t)kScanWarps * kBulkStages * (kTileBytes + 8);
+}
+
+template <int KP, bool FAST>
+__device__ __forceinline__ void scan_positions_bulk(const uint8_t* __restrict__ codes,
+                                                    const uint32_t* __restrict__ rows, int64_t a, int64_t b,
+                                                    int64_t blk0, int64_t blk1, const float* tab, uint8_t* ring,
+                                                    uint64_t* bars, uint32_t tx_extra, int* err, WarpTopK<KP>& tk,
+                                                    int lane, int warp) {
+    constexpr int NST = kBulkStages;
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
+    const uint32_t tb = 4u * (uint32_t)lane;
+    const uint64_t keep = policy_evict_last();
+    const uint32_t a32 = (uint32_t)a, b32 = (uint32_t)b;   // positions fit in 32 bits
+    const int64_t first = blk0 + warp;
+    const int nblk = first < blk1 ? (int)((blk1 - first + kScanWarps - 1) / kScanWarps) : 0;
+    const int R = kRoundsPerBlock * nblk;
+    const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
+    const uint32_t bar_s = (uint32_t)__cvta_generic_to_shared(bars);
+    // first position of round r of this warp
+    auto tile_pos = [&](int r) -> uint32_t {
+        return (uint32_t)((first + (int64_t)(r / kRoundsPerBlock) * kScanWarps) * kBlockRows) +
+               (uint32_t)(r % kRoundsPerBlock) * (32u * kU);
+    };
+    auto issue = [&](int r) {
+        const uint32_t st = (uint32_t)(r % NST);
+        mbar_arrive_expect_tx(bar_s + 8u * st, kTileBytes + tx_extra);
+        bulk_g2s(ring_s + st * kTileBytes, codes + (size_t)tile_pos(r) * 16, kTileBytes, bar_s + 8u * st, keep);
+    };
+    if (lane == 0)
+        for (int r = 0; r < NST && r < R; ++r) issue(r);
+#pragma unroll 1
+    for (int r = 0; r < R; ++r) {
+        const int st = r % NST;
+        if (!mbar_wait_warp(bar_s + 8u * (uint32_t)st, (uint32_t)(r / NST) & 1u)) {
+            if (lane == 0) atomicOr(err, 4);
+            // rounds r .. min(R, r + NST) - 1 were issued and not consumed
+            for (int q = r; q < R && q < r + NST; ++q)
+                mbar_wait_warp(bar_s + 8u * (uint32_t)(q % NST), (uint32_t)(q / NST) & 1u);
+            return;
+        }
+        tk.refresh(lane);
+        const uint32_t P = tile_pos(r);
+        const uint4* tile = reinterpret_cast<const uint4*>(ring + (size_t)st * kTileBytes);
+        uint4 c[kU];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) c[u] = tile[32 * u + lane];
+        __syncwarp();
+        if (lane == 0 && r + NST < R) {
+            fence_proxy_async_smem();
+            issue(r + NST);
+        }
+        const bool full = P >= a32 && P + 32u * kU <= b32;
+        uint32_t pos[kU];
+        unsigned valid = 0u;
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            pos[u] = P + 32u * (uint32_t)u + (uint32_t)lane;
+            valid |= (unsigned)(full || (pos[u] >= a32 && pos[u] < b32)) << u;
+        }
+        float d[kU];
+#pragma unroll
+        for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
+        // as in scan_positions: only candidates load their row id
+        const uint32_t thr_hi = (uint32_t)(tk.thr >> 32);
+        bool cand_any = false;
+#pragma unroll
+        for (int u = 0; u < kU; ++u) cand_any |= (valid >> u & 1u) && __float_as_uint(d[u]) <= thr_hi;
+        if (!__any_sync(0xFFFFFFFFu, cand_any)) continue;
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            const bool cand = (valid >> u & 1u) && __float_as_uint(d[u]) <= thr_hi;
+            const uint32_t row = cand ? __ldg(rows + pos[u]) : 0u;
+            const uint64_t key = ((uint64_t)__float_as_uint(d[u]) << 32) | row;
+            tk.offer(key, cand && key < tk.thr, lane);
+        }
+    }
+}
+
+template <int KP, int MINB>
+__global__ void __launch_bounds__(kScanThreads, MINB)
+k_scan_list_bulk(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
+                 int k, ScanShape sh, uint64_t* __restrict__ partials, const uint8_t* __restrict__ paired,
+                 uint32_t tx_extra, int* __restrict__ err) {
+    extern __shared__ __align__(256) uint8_t smem[];
+    float* tab = reinterpret_cast<float*>(smem);
+    uint64_t* tkbuf = reinterpret_cast<uint64_t*>(smem + (size_t)256 * 64 * 4);
+    uint8_t* ring_all = smem + bulk_ring_offset(KP);
+    uint64_t* bars_all = reinterpret_cast<uint64_t*>(ring_all + (size_t)kScanWarps * kBulkStages * kTileBytes);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t q = blockIdx.x;
+    const int chunk = blockIdx.y;
+    const ScanPlan p = plan[q];
+    if (!p.list) return;                               // k_scan covers this query
+    if (paired != nullptr && paired[q]) return;        // k_scan_list_pair covers it
+    const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
+    const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
+    const int64_t blk0 = max(c0, p.a / kBlockRows);
+    const int64_t blk1 = min(c1, (p.b + kBlockRows - 1) / kBlockRows);
+    uint64_t* out = partials + (q * sh.n_chunks + chunk) * (int64_t)k;
+    if (p.a >= p.b || blk0 >= blk1) {
+        for (int i = threadIdx.x; i < k; i += kScanThreads) out[i] = ~0ull;
+        return;
+    }
+    uint8_t* ring = ring_all + (size_t)warp * kBulkStages * kTileBytes;
+    uint64_t* bars = bars_all + warp * kBulkStages;
+    if (lane == 0) {
+        for (int i = 0; i < kBulkStages; ++i) mbar_init((uint32_t)__cvta_generic_to_shared(bars + i), 1u);
+        fence_mbar_init();
+    }
+    {
+        const float4* src = reinterpret_cast<const float4*>(tables + q * (int64_t)256 * 64);
+        float4* dst = reinterpret_cast<float4*>(tab);
+        for (int i = threadIdx.x; i < 64 * 64; i += kScanThreads) dst[i] = __ldg(src + i);
+    }
+    uint64_t* cta = tkbuf + kScanWarps * 2 * KP;
+    if (threadIdx.x == 0) *cta = ~0ull;
+    WarpTopK<KP> tk;
+    tk.init(tkbuf + warp * 2 * KP, k, lane, cta);
+    __syncthreads();
+    const uint8_t* codes = sc.codes_of(p.col);
+    const uint32_t* rows = sc.rows_of(p.col);
+    if ((uint32_t)__cvta_generic_to_shared(tab) == kDynSmemBase)
+        scan_positions_bulk<KP, true>(codes, rows, p.a, p.b, blk0, blk1, tab, ring, bars, tx_extra, err, tk, lane,
+                                      warp);
+    else
+        scan_positions_bulk<KP, false>(codes, rows, p.a, p.b, blk0, blk1, tab, ring, bars, tx_extra, err, tk, lane,
+                                       warp);
+    merge_warps<KP, kScanWarps>(tk, tkbuf, k, lane, warp, out);
+}
+
+template <int KP, int MINB>
+static cudaError_t launch_list_bulk(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
+                                    const ScanShape& sh, uint64_t* partials, const uint8_t* paired, size_t smem,
+                                    uint32_t tx_extra, int* err, cudaStream_t s) {
+    cudaError_t e = cudaFuncSetAttribute(k_scan_list_bulk<KP, MINB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
+    k_scan_list_bulk<KP, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, paired,
+                                                                tx_extra, err);
+    return cudaGetLastError();
+}
+
+template <int KP, bool M16, int MINB>
+static cudaError_t launch_list_one(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
+                                   int k, const ScanShape& sh, uint64_t* partials, const uint8_t* paired,
+                                   size_t smem, cudaStream_t s) {
+    cudaError_t e = cudaFuncSetAttribute(k_scan_list<KP, M16, MINB>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
+    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, paired);
+    return cudaGetLastError();
+}
+
+template <int KP>
+static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
+                                  int k, const ScanShape& sh, uint64_t* partials, uint8_t* work,
+                                  const ListOpts& lo, int* launches, cudaStream_t s) {
+    const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
+    const uint8_t* paired = nullptr;
+    int nl = 0;
+    if (m16 && work != nullptr) {
+        // M = 16: long, overlapping ranges are paired and served by the
+        // two-query kernel; the one-query kernel takes the rest
+        const cudaError_t e =
+            launch_pairs(tab, sc, plan, nq, k, sh, partials, work, lo.pair_min_rows, s, &paired, &nl);
+        if (e != cudaSuccess) return e;
+    }
+    if (launches) *launches = nl + 1;
+    if (m16 && lo.bulk) {
+        const size_t smem = scan_bulk_smem_bytes(KP);
+        if (smem <= (size_t)max_smem_optin()) {
+            if ((size_t)233472 / (smem + 1024) >= 2)
+                return launch_list_bulk<KP, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, lo.tx_extra,
+                                               lo.err, s);
+            return launch_list_bulk<KP, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, lo.tx_extra, lo.err,
+                                           s);
+        }
+    }
+    const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
+    if (m16) {
+        if ((size_t)233472 / (smem + 1024) >= 2)
+            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
+        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
+    }
+    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
+}
+
+cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
+                             const ScanShape& sh, uint64_t* partials, uint8_t* work, const ListOpts& lo,
+                             cudaStream_t s, int* launches) {
+    if (launches) *launches = 0;
+    if (nq <= 0) return cudaSuccess;
+    switch (scan_kp(k)) {
+        case 32: return launch_list_kp<32>(tab, sc, plan, nq, k, sh, partials, work, lo, launches, s);
+        case 64: return launch_list_kp<64>(tab, sc, plan, nq, k, sh, partials, work, lo, launches, s);
+        case 128: return launch_list_kp<128>(tab, sc, plan, nq, k, sh, partials, work, lo, launches, s);
+        default: return launch_list_kp<256>(tab, sc, plan, nq, k, sh, partials, work, lo, launches, s);
+    }
+}
+}  // namespace ifvs

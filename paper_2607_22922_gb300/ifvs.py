@@ -16,10 +16,11 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libifvs.so")
 
-IFVS_OK, IFVS_ERR_ARG, IFVS_ERR_OOM, IFVS_ERR_CUDA, IFVS_ERR_STATE, IFVS_ERR_UNSUPPORTED = 0, -1, -2, -3, -4, -5
+(IFVS_OK, IFVS_ERR_ARG, IFVS_ERR_OOM, IFVS_ERR_CUDA, IFVS_ERR_STATE, IFVS_ERR_UNSUPPORTED,
+ IFVS_ERR_TIMEOUT) = 0, -1, -2, -3, -4, -5, -6
 IFVS_OP_EQ, IFVS_OP_RANGE, IFVS_OP_GE, IFVS_OP_LT, IFVS_OP_GT, IFVS_OP_LE = 0, 1, 2, 3, 4, 5
 IFVS_ATTR_I32, IFVS_ATTR_I16 = 0, 1
-IFVS_F_DEVICE_IO, IFVS_F_STAGE_TIMING, IFVS_F_PLAIN_PQ = 0x1, 0x2, 0x4
+IFVS_F_DEVICE_IO, IFVS_F_STAGE_TIMING, IFVS_F_PLAIN_PQ, IFVS_F_PLAIN_LOADS = 0x1, 0x2, 0x4, 0x8
 IFVS_MAX_K, IFVS_MAX_M, IFVS_MAX_ATTRS, IFVS_N_STAGES = 256, 128, 4, 9
 STAGES = ("predicate", "filter", "condition", "lut", "scan", "merge", "rerank", "layout", "train")
 

@@ -337,3 +337,47 @@ def test_pairing_by_sorted_ranges(ifvs, orc, k):
     for x, y in zip(a, c):
         np.testing.assert_array_equal(x[:24], y)
     _check_oracle(orc, codes, attrs, Cpq, q[:64], p[:64], k, *(x[:64] for x in a))
+
+
+@pytest.mark.parametrize("k", [1, 10, 100, 200])
+def test_bulk_copied_tiles_equal_vector_loads(ifvs, orc, k):
+    """The one-query sorted-copy kernel reads each round's code rows either
+    by bulk copies (TMA) into shared memory, the default, or by per-lane
+    vector loads (IFVS_F_PLAIN_LOADS).  The rows, their sum order and the
+    top-k logic are the same, so the two must agree bit for bit: ranges cut
+    anywhere inside a block, empty and all-pass ranges, a ragged last block,
+    one and several queries per sub-batch; and both match the oracle."""
+    N = 150_001
+    g, codes, attrs, Cpq = _index(ifvs, N, seed=31)
+    p = _preds()
+    q = _queries(len(p), Cpq.shape[0] * Cpq.shape[2], seed=32)
+    a = g.search(q, p, k, pair_min_rows=-1)
+    for b in (g.search(q, p, k, pair_min_rows=-1, flags=ifvs.IFVS_F_PLAIN_LOADS),
+              g.search(q, p, k, pair_min_rows=-1, sub_batch=3),
+              _one_by_one(g, q, p, k, pair_min_rows=-1)):
+        for x, y in zip(a, b):
+            np.testing.assert_array_equal(x, y)
+    _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
+
+
+def test_bulk_copy_wait_runs_out_and_reports_timeout(ifvs, monkeypatch):
+    """Every wait of the scan for a bulk-copied tile is bounded.  With
+    IFVS_TEST_STALL_COPIES=1 the barriers expect more bytes than the copies
+    deliver, so each wait runs out: the search must return IFVS_ERR_TIMEOUT
+    (no fault, no hang), and the next search on the same index, with the
+    variable unset, must return the results of one that never timed out."""
+    g, codes, attrs, Cpq = _index(ifvs, 20_000, seed=41, i16=False)
+    p = synth.empty_predicates(2)
+    for i, (lo, hi) in enumerate(((-100, 300), (-500, 500))):
+        p[i]["n_clauses"] = 1
+        synth.set_clause(p[i], 0, 0, synth.OP_RANGE, lo, hi)
+    q = _queries(2, Cpq.shape[0] * Cpq.shape[2], seed=42)
+    ref = g.search(q, p, 10, pair_min_rows=-1)
+    monkeypatch.setenv("IFVS_TEST_STALL_COPIES", "1")
+    with pytest.raises(ifvs.IfvsError) as e:
+        g.search(q, p, 10, pair_min_rows=-1)
+    assert e.value.code == ifvs.IFVS_ERR_TIMEOUT
+    monkeypatch.delenv("IFVS_TEST_STALL_COPIES")
+    again = g.search(q, p, 10, pair_min_rows=-1)
+    for x, y in zip(ref, again):
+        np.testing.assert_array_equal(x, y)

@@ -346,9 +346,9 @@ def test_stage_timing_counts_launches(ifvs):
     t = g.stage_times(reset=True)
     # one attribute column: every predicate takes the sorted copy, so no
     # filter pass and no bitmap scan run.  filter: the scan plan; scan: the
-    # grouping of the sorted-copy queries, the four-, two- and one-query
-    # kernels (M = 16)
-    expected = {"predicate": 1, "filter": 1, "condition": 1, "lut": 2, "scan": 4, "merge": 1}
+    # pairing of the sorted-copy queries, the two- and one-query kernels
+    # (M = 16)
+    expected = {"predicate": 1, "filter": 1, "condition": 1, "lut": 2, "scan": 3, "merge": 1}
     for s, n in expected.items():
         assert t[s][1] == n and t[s][0] > 0.0
     assert t["rerank"][1] == 0
