@@ -211,24 +211,35 @@ def measured_peaks():
     return 6800.0, "fallback"
 
 
-def traffic_summary(summary, source):
-    """A committed ncu summary (profiles/), valid only while the kernel's
-    source file is unchanged; None otherwise."""
+SCAN_SOURCES = ("scan_common.cuh", "scan.cu", "scan_list.cu", "scan_pair.cu")
+
+
+def sources_sha256(sources):
+    """sha256 over the given csrc files, in order."""
+    h = hashlib.sha256()
+    for src in sources:
+        with open(os.path.join(ROOT, "paper_2607_22922_gb300", "csrc", src), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def traffic_summary(summary, sources):
+    """A committed ncu summary (profiles/), valid only while the kernels'
+    source files are unchanged (their sha256 is recorded in it); None
+    otherwise."""
     p = os.path.join(ROOT, "profiles", summary)
-    src = os.path.join(ROOT, "paper_2607_22922_gb300", "csrc", source)
     if not os.path.exists(p):
         return None
     with open(p) as f:
         d = json.load(f)
-    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
-    if d.get(source.replace(".", "_") + "_sha256") != sha:
+    if d.get("sources") != list(sources) or d.get("sources_sha256") != sources_sha256(sources):
         return None
     return d
 
 
-def kernel_traffic(summary, source):
+def kernel_traffic(summary, sources):
     """DRAM bytes per launch from a committed ncu summary (or None)."""
-    d = traffic_summary(summary, source)
+    d = traffic_summary(summary, sources)
     return None if d is None else d.get("dram_bytes_per_launch")
 
 
@@ -236,7 +247,7 @@ def scan_dram(workload_name, hbm_peak):
     """DRAM traffic of the scan stage per bin from the committed ncu summary
     of this workload (bytes per batch and GB/s over the kernel time under
     ncu, as a fraction of the measured HBM peak), or None."""
-    d = traffic_summary("scan_traffic.json", "scan.cu")
+    d = traffic_summary("scan_traffic.json", SCAN_SOURCES)
     if d is None or d.get("workload_name") != workload_name:
         return None
     out = {"bytes_per_batch": d.get("dram_bytes_per_launch"), "source": "profiles/scan_traffic.json",
@@ -823,7 +834,7 @@ def run_pq(args):
     peak = sms * 128 * mhz * 1e6 / 1e12
     roofline = {"kernel": "k_pq_assign", "bound": "alu", "achieved": achieved, "peak": peak,
                 "unit": "TFLOP/s", "frac": achieved / peak,
-                "traffic": kernel_traffic("pq_encode_traffic.json", "pq.cu"),
+                "traffic": kernel_traffic("pq_encode_traffic.json", ("pq.cu",)),
                 "peak_kind": "derived: %d SMs x 128 FP32 lanes x %.0f MHz (max SM clock)" % (sms, mhz),
                 "avg_launch_ms": launch_ms, "algorithmic_flop_per_launch": ops,
                 "algorithmic_bytes_per_launch": rows * (w.D * 4 + w.M)}

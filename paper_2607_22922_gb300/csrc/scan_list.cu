@@ -168,8 +168,9 @@ __host__ __device__ constexpr size_t bulk_ring_offset(int kp) {
     return ((size_t)256 * 64 * 4 + (size_t)kScanWarps * 2 * kp * 8 + 16 + 127) / 128 * 128;
 }
 
+// tiles, one barrier per tile, and the barrier of the table copy
 size_t scan_bulk_smem_bytes(int kp) {
-    return bulk_ring_offset(kp) + (size_t)kScanWarps * kBulkStages * (kTileBytes + 8);
+    return bulk_ring_offset(kp) + (size_t)kScanWarps * kBulkStages * (kTileBytes + 8) + 16;
 }
 
 template <int KP, bool FAST>
@@ -275,20 +276,30 @@ k_scan_list_bulk(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     }
     uint8_t* ring = ring_all + (size_t)warp * kBulkStages * kTileBytes;
     uint64_t* bars = bars_all + warp * kBulkStages;
+    const uint32_t tbar = (uint32_t)__cvta_generic_to_shared(bars_all + kScanWarps * kBulkStages);
     if (lane == 0) {
         for (int i = 0; i < kBulkStages; ++i) mbar_init((uint32_t)__cvta_generic_to_shared(bars + i), 1u);
+        if (threadIdx.x == 0) mbar_init(tbar, 1u);
         fence_mbar_init();
     }
-    {
-        const float4* src = reinterpret_cast<const float4*>(tables + q * (int64_t)256 * 64);
-        float4* dst = reinterpret_cast<float4*>(tab);
-        for (int i = threadIdx.x; i < 64 * 64; i += kScanThreads) dst[i] = __ldg(src + i);
+    // the query's 64 KB table (rows replicated and rotated, as k_tables
+    // wrote it) in one bulk copy, while the lists are set up
+    if (threadIdx.x == 0) {
+        mbar_arrive_expect_tx(tbar, 256u * 64u * 4u);
+        bulk_g2s((uint32_t)__cvta_generic_to_shared(tab), tables + q * (int64_t)256 * 64, 256u * 64u * 4u, tbar,
+                 policy_evict_first());
     }
     uint64_t* cta = tkbuf + kScanWarps * 2 * KP;
     if (threadIdx.x == 0) *cta = ~0ull;
     WarpTopK<KP> tk;
     tk.init(tkbuf + warp * 2 * KP, k, lane, cta);
     __syncthreads();
+    if (!mbar_wait_warp(tbar, 0u)) {
+        if (lane == 0) atomicOr(err, 4);
+        mbar_wait_warp(tbar, 0u);   // the copy may still be in flight
+        merge_warps<KP, kScanWarps>(tk, tkbuf, k, lane, warp, out);
+        return;
+    }
     const uint8_t* codes = sc.codes_of(p.col);
     const uint32_t* rows = sc.rows_of(p.col);
     if ((uint32_t)__cvta_generic_to_shared(tab) == kDynSmemBase)
