@@ -657,7 +657,8 @@ def run_ifvs(args):
     achieved = (lookups_total / nbatch) / (scan_ms / nbatch / 1000.0) if scan_ms > 0 else None
     hbm_peak, peak_kind = measured_peaks()
     dram = scan_dram(w.name, hbm_peak)
-    roofline = {"kernel": "scan stage (k_pair_items + k_scan_list_pair + k_scan_list + k_scan)",
+    roofline = {"kernel": "scan stage (k_pair_items + k_scan_list_pair + k_scan_list_bulk; k_scan_list and"
+                          " k_scan where a query takes them)",
                 "bound": "smem", "achieved": achieved, "peak": peak, "unit": "look-ups/s",
                 "frac": achieved / peak if achieved else None,
                 "traffic": dram["bytes_per_batch"] if dram else None,
