@@ -32,9 +32,28 @@ constexpr uint32_t kTabBytes16 = 256u * 64u * 4u;    // one replicated M = 16 ta
 constexpr uint32_t kExactBytes16 = 256u * 16u * 4u;  // one unreplicated table, [c][m]
 constexpr int kQMax = 2047;                           // 16 * 2047 < 2^15
 
-// packed table, two exact tables, extremes + the two shared bounds, lists
+// Deferred rescoring.  The rows of a round that pass a query's quantised
+// test (about 0.5 % of the rows on the dense bins, but in a third of the
+// warps' rounds) are not rescored where they are found, which ran the exact
+// sum for one or two lanes of the warp at a time; each warp appends them
+// (codes, position, query flags) to a buffer of kCandCap entries in shared
+// memory, and every 32 entries the warp rescores them with one entry per
+// lane.  The exact sums, the keys and the offers are the same as in place
+// (the offers only in another order, which the exact top-k does not see).
+// Lists of KP = 256 leave no room for the buffer: they rescore in place.
+#ifndef IFVS_PAIR_DEFER
+#define IFVS_PAIR_DEFER 1
+#endif
+constexpr int kCandCap = 64;   // a warp drains at 32: at most 31 + 32 entries are held
+constexpr size_t kCandWarpBytes = (size_t)kCandCap * (16 + 4 + 4);
+
+__host__ __device__ constexpr bool pair_defers(int kp) { return IFVS_PAIR_DEFER != 0 && kp <= 128; }
+
+// packed table, two exact tables, extremes + the two shared bounds, lists,
+// the candidate buffers
 size_t scan_pair_smem_bytes(int kp) {
-    return (size_t)kTabBytes16 + 2 * (size_t)kExactBytes16 + 64 * 4 + 16 + (size_t)kPairWarps * 2 * 2 * kp * 8;
+    return (size_t)kTabBytes16 + 2 * (size_t)kExactBytes16 + 64 * 4 + 16 + (size_t)kPairWarps * 2 * 2 * kp * 8 +
+           (pair_defers(kp) ? (size_t)kPairWarps * kCandWarpBytes : 0);
 }
 
 template <int IMM>
@@ -143,6 +162,45 @@ constexpr uint32_t kCandA = 0x00008000u, kCandB = 0x80000000u;
 // slower at the 128-register cap of a 16-warp CTA)
 constexpr int kU2 = 4;
 
+// A warp's candidate buffer (shared memory): entry i = codes[i], pos[i],
+// flags[i] (kCandA | kCandB for the queries whose test it passed).
+struct CandBuf {
+    uint4* codes;
+    uint32_t* pos;
+    uint32_t* flags;
+    int cnt;
+};
+
+// Rescoring of entries [first, first + n) (n <= 32), entry first + l by lane
+// l: the exact float32 distance of each flagged query in the one-query
+// kernel's order, the row id for those within the query's k-th key, the
+// offers (warp-collective).
+template <int KP>
+__device__ __forceinline__ void rescore_entries(const CandBuf& cbuf, int first, int n,
+                                                const uint32_t* __restrict__ rows, WarpTopK<KP>& tkA,
+                                                WarpTopK<KP>& tkB, const float* exA, const float* exB, int lane) {
+    uint4 c = make_uint4(0, 0, 0, 0);
+    uint32_t pos = 0u, f = 0u;
+    if (lane < n) {
+        c = cbuf.codes[first + lane];
+        pos = cbuf.pos[first + lane];
+        f = cbuf.flags[first + lane];
+    }
+    const int rot = (int)(pos & 15u);   // the lane that met position pos: pos mod 32
+    bool cA = (f & kCandA) != 0u;
+    bool cB = (f & kCandB) != 0u;
+    float dA = 0.f, dB = 0.f;
+    if (cA) dA = exact16(c, exA, rot);
+    if (cB) dB = exact16(c, exB, rot);
+    cA = cA && __float_as_uint(dA) <= (uint32_t)(tkA.thr >> 32);
+    cB = cB && __float_as_uint(dB) <= (uint32_t)(tkB.thr >> 32);
+    const uint32_t row = (cA || cB) ? __ldg(rows + pos) : 0u;
+    const uint64_t kA = ((uint64_t)__float_as_uint(dA) << 32) | row;
+    const uint64_t kB = ((uint64_t)__float_as_uint(dB) << 32) | row;
+    tkA.offer(kA, cA && kA < tkA.thr, lane);
+    tkB.offer(kB, cB && kB < tkB.thr, lane);
+}
+
 // Codes of a round's kU2 positions.  mask[] holds kCandA / kCandB for the
 // positions inside each query's range; MASKED: it differs between positions
 // (a cut block), so only positions inside a range load codes.
@@ -164,7 +222,7 @@ __device__ __forceinline__ void pair_round(const uint4 (&c)[kU2], const uint32_t
                                            uint32_t pos0, const uint32_t (&mask)[kU2], WarpTopK<KP>& tkA,
                                            WarpTopK<KP>& tkB, const float* exA, const float* exB, float slA,
                                            float invA, float slB, float invB, uint32_t tb, uint32_t base,
-                                           int rot, int lane, uint32_t& Tpk) {
+                                           int rot, int lane, uint32_t& Tpk, CandBuf& cbuf) {
     {
         const uint64_t oa = tkA.thr, ob = tkB.thr;
         tkA.refresh(lane);
@@ -182,6 +240,29 @@ __device__ __forceinline__ void pair_round(const uint4 (&c)[kU2], const uint32_t
         any |= cb[u];
     }
     if (!__any_sync(0xFFFFFFFFu, any != 0u)) return;
+    if constexpr (pair_defers(KP)) {
+        const unsigned lt = (1u << lane) - 1u;
+#pragma unroll
+        for (int u = 0; u < kU2; ++u) {
+            const unsigned ball = __ballot_sync(0xFFFFFFFFu, cb[u] != 0u);
+            if (ball == 0u) continue;
+            if (cb[u] != 0u) {
+                const int at = cbuf.cnt + __popc(ball & lt);
+                cbuf.codes[at] = c[u];
+                cbuf.pos[at] = pos0 + 32u * (uint32_t)u;
+                cbuf.flags[at] = cb[u];
+            }
+            cbuf.cnt += __popc(ball);
+            if (cbuf.cnt >= 32) {
+                __syncwarp();
+                cbuf.cnt -= 32;
+                rescore_entries<KP>(cbuf, cbuf.cnt, 32, rows, tkA, tkB, exA, exB, lane);
+                __syncwarp();   // the drained slots take the next entries
+                Tpk = pack_bounds(quant_bound(tkA.thr, slA, invA), quant_bound(tkB.thr, slB, invB));
+            }
+        }
+        return;
+    }
 #pragma unroll
     for (int u = 0; u < kU2; ++u) {
         const uint32_t pos = pos0 + 32u * (uint32_t)u;
@@ -207,7 +288,8 @@ __device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ 
                                                     int64_t bA, int64_t aB, int64_t bB, int64_t blk0,
                                                     int64_t blk1, WarpTopK<KP>& tkA, WarpTopK<KP>& tkB,
                                                     const float* exA, const float* exB, float slA, float invA,
-                                                    float slB, float invB, uint32_t base, int lane, int warp) {
+                                                    float slB, float invB, uint32_t base, int lane, int warp,
+                                                    CandBuf& cbuf) {
     const uint32_t tb = 4u * (uint32_t)lane;
     const int rot = lane & 15;
     const uint64_t keep = policy_evict_last();
@@ -231,7 +313,7 @@ __device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ 
                 uint4 c[kU2];
                 pair_load<false>(codes, pb + 32u * (uint32_t)j0, mask, keep, c);
                 pair_round<KP, FAST, false>(c, rows, pb + 32u * (uint32_t)j0, mask, tkA, tkB, exA, exB, slA, invA,
-                                            slB, invB, tb, base, rot, lane, Tpk);
+                                            slB, invB, tb, base, rot, lane, Tpk, cbuf);
             }
             continue;
         }
@@ -248,7 +330,14 @@ __device__ __forceinline__ void scan_positions_pair(const uint8_t* __restrict__ 
             uint4 c[kU2];
             pair_load<true>(codes, pos0, mask, keep, c);
             pair_round<KP, FAST, true>(c, rows, pos0, mask, tkA, tkB, exA, exB, slA, invA, slB, invB, tb, base,
-                                       rot, lane, Tpk);
+                                       rot, lane, Tpk, cbuf);
+        }
+    }
+    if constexpr (pair_defers(KP)) {
+        if (cbuf.cnt > 0) {   // warp-uniform
+            __syncwarp();
+            rescore_entries<KP>(cbuf, 0, cbuf.cnt, rows, tkA, tkB, exA, exB, lane);
+            cbuf.cnt = 0;
         }
     }
 }
@@ -387,6 +476,7 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     uint64_t* tkbufA = reinterpret_cast<uint64_t*>(smem + kTabBytes16 + 2 * kExactBytes16 + 64 * 4 + 16);
     uint64_t* tkbufB = tkbufA + kPairWarps * 2 * KP;
     float* red = reinterpret_cast<float*>(tkbufA);   // [warp][4][16], before the lists are set up
+    uint8_t* cand_base = reinterpret_cast<uint8_t*>(tkbufB + kPairWarps * 2 * KP);   // 16-byte aligned
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const PairItem it = items[blockIdx.x];
     if (it.qa < 0) return;
@@ -470,13 +560,21 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     __syncthreads();
     const int64_t lo = (lA == hA) ? lB : ((lB == hB) ? lA : min(lA, lB));
     const int64_t hi = max(hA, hB);
+    CandBuf cbuf;
+    {
+        uint8_t* wb = cand_base + (size_t)warp * kCandWarpBytes;
+        cbuf.codes = reinterpret_cast<uint4*>(wb);
+        cbuf.pos = reinterpret_cast<uint32_t*>(wb + kCandCap * 16);
+        cbuf.flags = reinterpret_cast<uint32_t*>(wb + kCandCap * 20);
+        cbuf.cnt = 0;
+    }
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(ptab);
     if (base == kDynSmemBase)
         scan_positions_pair<KP, true>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, pB.a, pB.b, lo, hi,
-                                      tkA, tkB, exA, exB, slA, invA, slB, invB, base, lane, warp);
+                                      tkA, tkB, exA, exB, slA, invA, slB, invB, base, lane, warp, cbuf);
     else
         scan_positions_pair<KP, false>(sc.codes_of(pA.col), sc.rows_of(pA.col), pA.a, pA.b, pB.a, pB.b, lo, hi,
-                                       tkA, tkB, exA, exB, slA, invA, slB, invB, base, lane, warp);
+                                       tkA, tkB, exA, exB, slA, invA, slB, invB, base, lane, warp, cbuf);
     merge_warps<KP, kPairWarps>(tkA, tkbufA, k, lane, warp, outA);
     merge_warps<KP, kPairWarps>(tkB, tkbufB, k, lane, warp, outB);
 }
