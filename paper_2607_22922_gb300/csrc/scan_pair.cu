@@ -157,10 +157,15 @@ __device__ __forceinline__ uint32_t pack_bounds(int ta, int tb) {
 
 constexpr uint32_t kCandA = 0x00008000u, kCandB = 0x80000000u;
 
-// kU2 rows per lane per round in the paired loop (measured: 2 rows, 8 rows,
-// and loading the next round's codes before this round's look-ups are all
-// slower at the 128-register cap of a 16-warp CTA)
-constexpr int kU2 = 4;
+// kU2 rows per lane per round in the paired loop.  Measured on the 10^8-row
+// dense bin with candidates rescored in batches: 8 rows 137.4 ms, 4 rows
+// 142.1 ms, 2 rows 200.1 ms per batch; 16 rows spill at the 128-register cap
+// of a 16-warp CTA.  (With in-place rescoring 4 rows had been the fastest.)
+#ifndef IFVS_PAIR_ROWS
+#define IFVS_PAIR_ROWS 8
+#endif
+constexpr int kU2 = IFVS_PAIR_ROWS;
+static_assert(kU2 % 2 == 0 && 32 % kU2 == 0, "rows in pairs, whole rounds per block");
 
 // A warp's candidate buffer (shared memory): entry i = codes[i], pos[i],
 // flags[i] (kCandA | kCandB for the queries whose test it passed).
