@@ -409,13 +409,19 @@ ScanShape scan_shape(const ifvs_index* ix, int64_t n, int kk, int64_t chunk_bloc
     sh.K = ix->K;
     sh.row_bytes = ix->row_bytes;
     sh.tab_words = ix->tab_words;
+    // Rows per scan CTA.  Every CTA pays a fixed cost (its table, its
+    // lists and their merge, one more partial list per query for k_merge),
+    // so a batch takes as few chunks as keep the GPU busy: about two waves
+    // of CTAs from the queries alone, and chunks of at most 65 536 blocks
+    // (6.7e7 rows), which keeps the long CTAs of 10^8-row dense bins from
+    // leaving a ragged last wave.  Measured with 1024-query batches:
+    // 10^8 rows 2 chunks 28.1k queries/s (1: 25.3k, 3: 27.2k, 4: 27.5k,
+    // 12 L2-sized chunks, the earlier rule: 25.4k); 10^6 rows 1 chunk 795k
+    // (2: 723k, 3: 693k).
     const int64_t resident = (int64_t)ix->num_sms * scan_ctas_per_sm(ix->tab_words, scan_kp(kk));
-    int64_t chunks = (resident * 8 + n - 1) / n;
-    // the CTAs that walk a chunk together share it through L2: keep a
-    // chunk's codes within about the L2 size (128 MB)
-    const int64_t l2_blocks = ((int64_t)128 << 20) / ((int64_t)kBlockRows * ix->row_bytes);
-    const int64_t by_l2 = (ix->n_blocks + l2_blocks - 1) / l2_blocks;
-    if (chunks < by_l2) chunks = by_l2;
+    int64_t chunks = (resident * 2 + n - 1) / n;
+    const int64_t by_rows = (ix->n_blocks + 65535) / 65536;
+    if (chunks < by_rows) chunks = by_rows;
     int64_t max_chunks = ix->n_blocks / 16;
     if (max_chunks < 1) max_chunks = 1;
     const int64_t key_cap = 32768 / kk;  // bounds the merge's input per query

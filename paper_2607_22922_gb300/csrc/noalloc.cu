@@ -43,15 +43,14 @@ int scratch_address(unsigned char** out) {
     return 0;
 }
 
-// Chunks per query for n queries: the allocating path's rule (fill the
-// GPU about eight times over, at least 16 blocks per chunk, at most 32768
-// keys per query for the merge).
+// Chunks per query for n queries: the allocating path's rule (about two
+// waves of CTAs from the queries alone, chunks of at most 65 536 blocks, at
+// least 16 blocks per chunk, at most 32768 keys per query for the merge).
 int64_t chunks_for(const IndexView& v, int64_t n, int k) {
     const int64_t resident = (int64_t)v.num_sms * scan_ctas_per_sm(v.tab_words, scan_kp(k));
-    int64_t c = (resident * 8 + n - 1) / n;
-    const int64_t l2_blocks = ((int64_t)128 << 20) / ((int64_t)kBlockRows * v.row_bytes);
-    const int64_t by_l2 = (v.n_blocks + l2_blocks - 1) / l2_blocks;
-    if (c < by_l2) c = by_l2;
+    int64_t c = (resident * 2 + n - 1) / n;
+    const int64_t by_rows = (v.n_blocks + 65535) / 65536;
+    if (c < by_rows) c = by_rows;
     int64_t cap = v.n_blocks / 16;
     if (cap < 1) cap = 1;
     if (cap > 32768 / k) cap = 32768 / k > 0 ? 32768 / k : 1;
