@@ -107,6 +107,36 @@ __device__ __forceinline__ void warp_merge_low(uint64_t* a, int n, int lane) {
     __syncwarp();
 }
 
+// Merges a warp's candidates [KP, 2KP) of buf into its sorted list [0, KP),
+// clears the candidates, publishes the new k-th key to the CTA's bound (if
+// any) and returns it.  For KP >= 64 the candidates are sorted and the KP
+// smallest of both runs kept by one bitonic merge (half the compare-
+// exchanges of one sort of 2 KP); for KP = 32 both take the same number of
+// steps and one sort of 64 measured faster (sift1m 693k against 599k
+// queries/s; 10^8 rows at KP = 128: 0.1 % and 1 % bins 1.51 -> 1.41 and
+// 4.33 -> 4.04 ms with the merge).  Out of line: the scan loops offer keys
+// at many sites and flush rarely, and one copy of the sort keeps their code
+// small (instruction-fetch stalls led the two-query kernel's profile).
+template <int KP>
+#ifndef IFVS_FLUSH_INLINE
+__device__ __noinline__
+#else
+__device__ __forceinline__
+#endif
+uint64_t flush_list(uint64_t* buf, int k, uint64_t* cta, int lane) {
+    if constexpr (KP <= 32) {
+        warp_sort(buf, 2 * KP, lane);
+    } else {
+        warp_sort(buf + KP, KP, lane);
+        warp_merge_low(buf, KP, lane);
+    }
+    const uint64_t thr = buf[k - 1];
+    for (int i = KP + lane; i < 2 * KP; i += 32) buf[i] = ~0ull;
+    if (cta != nullptr && lane == 0 && thr != ~0ull) atomicMin(reinterpret_cast<unsigned long long*>(cta), thr);
+    __syncwarp();
+    return thr;
+}
+
 // The warps of a CTA that serve one query share a bound `cta` (shared
 // memory): the smallest k-th key any of them has published.  A warp's list
 // holds k distinct rows, so its k-th key is at least the CTA's true k-th
@@ -140,22 +170,7 @@ struct WarpTopK {
         if (t < thr) thr = t;
     }
     __device__ __forceinline__ void flush(int lane) {
-        // the list [0, KP) is sorted: for KP >= 64 sort the candidates, then
-        // keep the KP smallest of both (half the compare-exchanges of one
-        // sort of 2 KP); for KP = 32 the two take the same number of steps
-        // and one sort of 64 measured faster (sift1m 693k against 599k
-        // queries/s; 10^8 rows at KP = 128: 0.1 % and 1 % bins 1.51 -> 1.41
-        // and 4.33 -> 4.04 ms with the merge)
-        if constexpr (KP <= 32) {
-            warp_sort(buf, 2 * KP, lane);
-        } else {
-            warp_sort(buf + KP, KP, lane);
-            warp_merge_low(buf, KP, lane);
-        }
-        thr = buf[k - 1];
-        for (int i = KP + lane; i < 2 * KP; i += 32) buf[i] = ~0ull;
-        if (cta != nullptr && lane == 0 && thr != ~0ull) atomicMin(reinterpret_cast<unsigned long long*>(cta), thr);
-        __syncwarp();
+        thr = flush_list<KP>(buf, k, cta, lane);
         cnt = 0;
         refresh(lane);
     }
