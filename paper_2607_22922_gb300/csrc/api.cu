@@ -878,7 +878,9 @@ int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int6
     ix->ds = D > 0 ? D / M : 0;
     ix->n_blocks = (N + kBlockRows - 1) / kBlockRows;
     ix->n_rows_pad = ix->n_blocks * kBlockRows;
-    ix->row_bytes = (int)round_up(M, 4);
+    // rows of 9 to 16 subspaces take 16 bytes (one vector load per row, and
+    // the scan loops compiled for M = 12 and 16); others M rounded up to 4
+    ix->row_bytes = (M > 8 && M <= 16) ? 16 : (int)round_up(M, 4);
     ix->tab_words = (int)round_up(M + 31, 32);
     if (scan_smem_bytes(ix->tab_words, scan_kp(1)) > (size_t)ix->max_smem)
         return fail(set_err(IFVS_ERR_UNSUPPORTED, "M = %d needs %zu bytes of shared memory (device: %d)",

@@ -21,13 +21,13 @@ int scan_ctas_per_sm(int tab_words, int kp) {
     return n < 1 ? 1 : n;
 }
 
-template <int KP, bool M16, bool FAST>
+template <int KP, int MM, bool FAST>
 __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                                            const uint32_t* __restrict__ bmq, const ScanShape& sh,
                                            int64_t b0, int64_t b1, const float* tab,
                                            uint32_t* ring, WarpTopK<KP>& tk, int lane, int warp) {
-    const int M = M16 ? 16 : sh.M;
-    const int S = M16 ? 64 : sh.tab_words;
+    const int M = MM > 0 ? MM : sh.M;
+    const int S = MM > 0 ? 64 : sh.tab_words;
     const int row_bytes = sh.row_bytes;
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
     const uint32_t tb = 4u * (uint32_t)lane;
@@ -79,13 +79,13 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
                 uint32_t row[kU];
 #pragma unroll
                 for (int u = 0; u < kU; ++u) row[u] = rb + 32u * (uint32_t)(j0 + u);
-                if constexpr (M16) {
+                if constexpr (MM > 0) {
                     uint4 c[kU];
 #pragma unroll
                     for (int u = 0; u < kU; ++u) c[u] = ldg_nc_v4(codes + (size_t)row[u] * 16, keep);
                     float d[kU];
 #pragma unroll
-                    for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
+                    for (int u = 0; u < kU; u += 2) lookup2<MM, FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
                     uint64_t key[kU];
                     bool want = false;
 #pragma unroll
@@ -131,14 +131,14 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
             if (F >= T) break;   // every word loaded and consumed
             continue;            // lanes wait for the next refill
         }
-        if constexpr (M16) {
+        if constexpr (MM > 0) {
             uint4 c[kU];
 #pragma unroll
             for (int u = 0; u < kU; ++u)
                 c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)row[u] * 16, keep) : make_uint4(0, 0, 0, 0);
             float d[kU];
 #pragma unroll
-            for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
+            for (int u = 0; u < kU; u += 2) lookup2<MM, FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
             uint64_t key[kU];
             bool want = false;
 #pragma unroll
@@ -163,13 +163,13 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
     }
 }
 
-template <int KP, bool M16, int MINB>
+template <int KP, int MM, int MINB>
 __global__ void __launch_bounds__(kScanThreads, MINB)
 k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
        const uint32_t* __restrict__ bm, const ScanPlan* __restrict__ plan, int64_t nq, int k,
        ScanShape sh, uint64_t* __restrict__ partials) {
     extern __shared__ __align__(256) uint8_t smem[];
-    const int S = M16 ? 64 : sh.tab_words;
+    const int S = MM > 0 ? 64 : sh.tab_words;
     float* tab = reinterpret_cast<float*>(smem);
     uint64_t* tkbuf = reinterpret_cast<uint64_t*>(smem + (size_t)256 * S * 4);
     uint32_t* ringbase = reinterpret_cast<uint32_t*>(smem + (size_t)256 * S * 4 +
@@ -197,13 +197,13 @@ k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
     uint32_t* ring = ringbase + warp * kRing * 32;
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
     const bool fast = base == kDynSmemBase;
-    if constexpr (M16) {
+    if constexpr (MM > 0) {
         if (fast)
-            scan_chunk<KP, true, true>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
+            scan_chunk<KP, MM, true>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
         else
-            scan_chunk<KP, true, false>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
+            scan_chunk<KP, MM, false>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
     } else {
-        scan_chunk<KP, false, false>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
+        scan_chunk<KP, 0, false>(codes, bmq, sh, b0, b1, tab, ring, tk, lane, warp);
     }
 
     // 3) merge the warps' lists pairwise (4 levels); warp 0 writes the
@@ -225,15 +225,15 @@ k_scan(const uint8_t* __restrict__ codes, const float* __restrict__ tables,
     }
 }
 
-template <int KP, bool M16, int MINB>
+template <int KP, int MM, int MINB>
 static cudaError_t launch_one(const uint8_t* codes, const float* tab, const uint32_t* bm,
                               const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
                               uint64_t* partials, size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(k_scan<KP, M16, MINB>,
+    cudaError_t e = cudaFuncSetAttribute(k_scan<KP, MM, MINB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
-    k_scan<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(codes, tab, bm, plan, nq, k, sh, partials);
+    k_scan<KP, MM, MINB><<<grid, kScanThreads, smem, s>>>(codes, tab, bm, plan, nq, k, sh, partials);
     return cudaGetLastError();
 }
 
@@ -241,18 +241,16 @@ template <int KP>
 static cudaError_t launch_scan_kp(const uint8_t* codes, const float* tab, const uint32_t* bm,
                                   const ScanPlan* plan, int64_t nq, int k, const ScanShape& sh,
                                   uint64_t* partials, cudaStream_t s) {
-    const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
+    const int mm = fixed_m(sh);
     const size_t smem = scan_smem_bytes(sh.tab_words, KP);
-    if (m16) {
-#ifndef IFVS_SCAN_ONE_CTA
-        if (scan_ctas_per_sm(sh.tab_words, KP) >= 2)
-#else
-        if (false)
-#endif
-            return launch_one<KP, true, 2>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
-        return launch_one<KP, true, 1>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
-    }
-    return launch_one<KP, false, 1>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
+    const bool two = scan_ctas_per_sm(sh.tab_words, KP) >= 2;
+    if (mm == 16)
+        return two ? launch_one<KP, 16, 2>(codes, tab, bm, plan, nq, k, sh, partials, smem, s)
+                   : launch_one<KP, 16, 1>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
+    if (mm == 12)
+        return two ? launch_one<KP, 12, 2>(codes, tab, bm, plan, nq, k, sh, partials, smem, s)
+                   : launch_one<KP, 12, 1>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
+    return launch_one<KP, 0, 1>(codes, tab, bm, plan, nq, k, sh, partials, smem, s);
 }
 
 cudaError_t launch_scan(const uint8_t* codes, const float* tab, const uint32_t* bm,

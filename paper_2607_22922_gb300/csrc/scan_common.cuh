@@ -238,18 +238,20 @@ __device__ __forceinline__ void unpack_f32x2(uint64_t v, float& a, float& b) {
 // architecture (after the 1 KB the hardware reserves); the kernel checks it.
 constexpr uint32_t kDynSmemBase = 0x400u;
 
-// Distances of two M = 16 rows (codes ca, cb).  One byte permute forms
-// code * 256 + 4 * w0, w0 = the row's index mod 32 (the lane that owns it in
-// the bitmap path); FAST (table at kDynSmemBase): the table base and the step
-// go into the load's immediate offset; otherwise the base is added.
-template <bool FAST>
-__device__ __forceinline__ void lookup16x2(const uint4 ca, const uint4 cb, uint32_t tba, uint32_t tbb,
-                                           uint32_t base, float& da, float& db) {
+// Distances of two rows of MM <= 16 subspaces (codes ca, cb: 16-byte rows,
+// table rows of 64 words).  One byte permute forms code * 256 + 4 * w0, w0 =
+// the row's index mod 32 (the lane that owns it in the bitmap path); FAST
+// (table at kDynSmemBase): the table base and the step go into the load's
+// immediate offset; otherwise the base is added.
+template <int MM, bool FAST>
+__device__ __forceinline__ void lookup2(const uint4 ca, const uint4 cb, uint32_t tba, uint32_t tbb,
+                                        uint32_t base, float& da, float& db) {
+    static_assert(MM >= 1 && MM <= 16, "16-byte rows");
     const uint32_t wa[4] = {ca.x, ca.y, ca.z, ca.w};
     const uint32_t wb[4] = {cb.x, cb.y, cb.z, cb.w};
     uint64_t acc = 0ull;
 #pragma unroll
-    for (int s = 0; s < 16; ++s) {
+    for (int s = 0; s < MM; ++s) {
         const uint32_t sel = 0x5504u | ((uint32_t)(s & 3) << 4);
         uint32_t oa = __byte_perm(wa[s >> 2], tba, sel);
         uint32_t ob = __byte_perm(wb[s >> 2], tbb, sel);
@@ -441,6 +443,14 @@ inline int max_smem_optin() {
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     if (cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return 0;
     return v;
+}
+
+// Subspace count the fixed-M scan loops are compiled for when the index
+// stores 16-byte rows with 64-word tables (M = 12 rows padded to 16 bytes,
+// or M = 16); 0: the generic-M loop.
+inline int fixed_m(const ScanShape& sh) {
+    if (sh.row_bytes != 16 || sh.tab_words != 64) return 0;
+    return (sh.M == 16 || sh.M == 12) ? sh.M : 0;
 }
 
 // Two-query scan of the sorted copy (scan_pair.cu): pairs the list-path

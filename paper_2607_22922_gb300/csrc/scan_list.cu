@@ -24,13 +24,13 @@ size_t scan_list_smem_bytes(int tab_words, int kp) {
     return (size_t)256 * tab_words * 4 + (size_t)kScanWarps * 2 * kp * 8 + 16;
 }
 
-template <int KP, bool M16, bool FAST>
+template <int KP, int MM, bool FAST>
 __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes, const uint32_t* __restrict__ rows,
                                                int64_t a, int64_t b, int64_t blk0, int64_t blk1, int wstride,
                                                const ScanShape& sh, const float* tab, WarpTopK<KP>& tk,
                                                int lane, int warp) {
-    const int M = M16 ? 16 : sh.M;
-    const int S = M16 ? 64 : sh.tab_words;
+    const int M = MM > 0 ? MM : sh.M;
+    const int S = MM > 0 ? 64 : sh.tab_words;
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
     const uint32_t tb = 4u * (uint32_t)lane;
     const uint64_t keep = policy_evict_last();
@@ -50,13 +50,13 @@ __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes
                 valid |= (unsigned)(full || (pos[u] >= a32 && pos[u] < b32)) << u;
             }
             float d[kU];
-            if constexpr (M16) {
+            if constexpr (MM > 0) {
                 uint4 c[kU];
 #pragma unroll
                 for (int u = 0; u < kU; ++u)
                     c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)pos[u] * 16, keep) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-                for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
+                for (int u = 0; u < kU; u += 2) lookup2<MM, FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
             } else {
                 lookup_rows<kU>(codes, pos, valid, sh.row_bytes, M, S, tab, lane, d);
             }
@@ -78,12 +78,12 @@ __device__ __forceinline__ void scan_positions(const uint8_t* __restrict__ codes
     }
 }
 
-template <int KP, bool M16, int MINB>
+template <int KP, int MM, int MINB>
 __global__ void __launch_bounds__(kScanThreads, MINB)
 k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
             int k, ScanShape sh, uint64_t* __restrict__ partials, const uint8_t* __restrict__ paired) {
     extern __shared__ __align__(256) uint8_t smem[];
-    const int S = M16 ? 64 : sh.tab_words;
+    const int S = MM > 0 ? 64 : sh.tab_words;
     float* tab = reinterpret_cast<float*>(smem);
     uint64_t* tkbuf = reinterpret_cast<uint64_t*>(smem + (size_t)256 * S * 4);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -114,13 +114,13 @@ k_scan_list(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __r
     const uint8_t* codes = sc.codes_of(p.col);
     const uint32_t* rows = sc.rows_of(p.col);
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(tab);
-    if constexpr (M16) {
+    if constexpr (MM > 0) {
         if (base == kDynSmemBase)
-            scan_positions<KP, true, true>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
+            scan_positions<KP, MM, true>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
         else
-            scan_positions<KP, true, false>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
+            scan_positions<KP, MM, false>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
     } else {
-        scan_positions<KP, false, false>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
+        scan_positions<KP, 0, false>(codes, rows, p.a, p.b, blk0, blk1, kScanWarps, sh, tab, tk, lane, warp);
     }
     tk.flush(lane);
 #pragma unroll 1
@@ -173,7 +173,7 @@ size_t scan_bulk_smem_bytes(int kp) {
     return bulk_ring_offset(kp) + (size_t)kScanWarps * kBulkStages * (kTileBytes + 8) + 16;
 }
 
-template <int KP, bool FAST>
+template <int KP, int MM, bool FAST>
 __device__ __forceinline__ void scan_positions_bulk(const uint8_t* __restrict__ codes,
                                                     const uint32_t* __restrict__ rows, int64_t a, int64_t b,
                                                     int64_t blk0, int64_t blk1, const float* tab, uint8_t* ring,
@@ -232,7 +232,7 @@ __device__ __forceinline__ void scan_positions_bulk(const uint8_t* __restrict__ 
         }
         float d[kU];
 #pragma unroll
-        for (int u = 0; u < kU; u += 2) lookup16x2<FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
+        for (int u = 0; u < kU; u += 2) lookup2<MM, FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
         // as in scan_positions: only candidates load their row id
         const uint32_t thr_hi = (uint32_t)(tk.thr >> 32);
         bool cand_any = false;
@@ -249,7 +249,7 @@ __device__ __forceinline__ void scan_positions_bulk(const uint8_t* __restrict__ 
     }
 }
 
-template <int KP, int MINB>
+template <int KP, int MM, int MINB>
 __global__ void __launch_bounds__(kScanThreads, MINB)
 k_scan_list_bulk(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
                  int k, ScanShape sh, uint64_t* __restrict__ partials, const uint8_t* __restrict__ paired,
@@ -303,36 +303,36 @@ k_scan_list_bulk(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     const uint8_t* codes = sc.codes_of(p.col);
     const uint32_t* rows = sc.rows_of(p.col);
     if ((uint32_t)__cvta_generic_to_shared(tab) == kDynSmemBase)
-        scan_positions_bulk<KP, true>(codes, rows, p.a, p.b, blk0, blk1, tab, ring, bars, tx_extra, err, tk, lane,
+        scan_positions_bulk<KP, MM, true>(codes, rows, p.a, p.b, blk0, blk1, tab, ring, bars, tx_extra, err, tk, lane,
                                       warp);
     else
-        scan_positions_bulk<KP, false>(codes, rows, p.a, p.b, blk0, blk1, tab, ring, bars, tx_extra, err, tk, lane,
+        scan_positions_bulk<KP, MM, false>(codes, rows, p.a, p.b, blk0, blk1, tab, ring, bars, tx_extra, err, tk, lane,
                                        warp);
     merge_warps<KP, kScanWarps>(tk, tkbuf, k, lane, warp, out);
 }
 
-template <int KP, int MINB>
+template <int KP, int MM, int MINB>
 static cudaError_t launch_list_bulk(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
                                     const ScanShape& sh, uint64_t* partials, const uint8_t* paired, size_t smem,
                                     uint32_t tx_extra, int* err, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(k_scan_list_bulk<KP, MINB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_scan_list_bulk<KP, MM, MINB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
-    k_scan_list_bulk<KP, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, paired,
+    k_scan_list_bulk<KP, MM, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, paired,
                                                                 tx_extra, err);
     return cudaGetLastError();
 }
 
-template <int KP, bool M16, int MINB>
+template <int KP, int MM, int MINB>
 static cudaError_t launch_list_one(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
                                    int k, const ScanShape& sh, uint64_t* partials, const uint8_t* paired,
                                    size_t smem, cudaStream_t s) {
-    cudaError_t e = cudaFuncSetAttribute(k_scan_list<KP, M16, MINB>,
+    cudaError_t e = cudaFuncSetAttribute(k_scan_list<KP, MM, MINB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
-    k_scan_list<KP, M16, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, paired);
+    k_scan_list<KP, MM, MINB><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, paired);
     return cudaGetLastError();
 }
 
@@ -340,10 +340,10 @@ template <int KP>
 static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq,
                                   int k, const ScanShape& sh, uint64_t* partials, uint8_t* work,
                                   const ListOpts& lo, int* launches, cudaStream_t s) {
-    const bool m16 = sh.M == 16 && sh.row_bytes == 16 && sh.tab_words == 64;
+    const int mm = fixed_m(sh);
     const uint8_t* paired = nullptr;
     int nl = 0;
-    if (m16 && work != nullptr) {
+    if (mm == 16 && work != nullptr) {
         // M = 16: long, overlapping ranges are paired and served by the
         // two-query kernel; the one-query kernel takes the rest
         const cudaError_t e =
@@ -351,23 +351,30 @@ static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPla
         if (e != cudaSuccess) return e;
     }
     if (launches) *launches = nl + 1;
-    if (m16 && lo.bulk) {
+    if (mm > 0 && lo.bulk) {
         const size_t smem = scan_bulk_smem_bytes(KP);
         if (smem <= (size_t)max_smem_optin()) {
-            if ((size_t)233472 / (smem + 1024) >= 2)
-                return launch_list_bulk<KP, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, lo.tx_extra,
-                                               lo.err, s);
-            return launch_list_bulk<KP, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, lo.tx_extra, lo.err,
-                                           s);
+            const bool two = (size_t)233472 / (smem + 1024) >= 2;
+            if (mm == 16)
+                return two ? launch_list_bulk<KP, 16, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem,
+                                                         lo.tx_extra, lo.err, s)
+                           : launch_list_bulk<KP, 16, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem,
+                                                         lo.tx_extra, lo.err, s);
+            return two ? launch_list_bulk<KP, 12, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, lo.tx_extra,
+                                                     lo.err, s)
+                       : launch_list_bulk<KP, 12, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, lo.tx_extra,
+                                                     lo.err, s);
         }
     }
     const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
-    if (m16) {
-        if ((size_t)233472 / (smem + 1024) >= 2)
-            return launch_list_one<KP, true, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
-        return launch_list_one<KP, true, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
-    }
-    return launch_list_one<KP, false, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
+    const bool two = (size_t)233472 / (smem + 1024) >= 2;
+    if (mm == 16)
+        return two ? launch_list_one<KP, 16, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, s)
+                   : launch_list_one<KP, 16, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
+    if (mm == 12)
+        return two ? launch_list_one<KP, 12, 2>(tab, sc, plan, nq, k, sh, partials, paired, smem, s)
+                   : launch_list_one<KP, 12, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
+    return launch_list_one<KP, 0, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, s);
 }
 
 cudaError_t launch_scan_list(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,

@@ -88,7 +88,7 @@ __device__ __forceinline__ int quant_bound(uint64_t thr, float sl, float inv) {
 }
 
 // Quantised sums of two M = 16 rows (codes ca, cb), both queries at once:
-// the addresses of lookup16x2, integer loads and adds.
+// the addresses of lookup2, integer loads and adds.
 template <bool FAST>
 __device__ __forceinline__ void lookup16x2_q(const uint4 ca, const uint4 cb, uint32_t tb, uint32_t base,
                                              uint32_t& sa, uint32_t& sb) {
@@ -131,7 +131,7 @@ __device__ __forceinline__ void lookup16x2_q(const uint4 ca, const uint4 cb, uin
 
 // Exact float32 distance of one M = 16 row of the sorted copy from an
 // unreplicated table ex[c * 16 + m]: byte s holds subspace (s + rot) mod 16,
-// rot = (p mod 32) mod 16, added for s ascending from 0, as lookup16x2 does.
+// rot = (p mod 32) mod 16, added for s ascending from 0, as lookup2 does.
 // Called for the rare candidate rows only: kept out of line, the round's
 // code is smaller (measured 1-2 % faster than inlining its eight copies).
 __device__ __noinline__ float exact16(const uint4 c, const float* ex, int rot) {
