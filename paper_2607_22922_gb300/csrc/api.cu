@@ -144,10 +144,12 @@ struct ifvs_index {
     int n_attrs = 0;
     int32_t types[IFVS_MAX_ATTRS] = {0, 0, 0, 0};
     void* d_attr[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
-    // per column: row ids sorted by (value, row) and the values in that order
-    uint32_t* d_srt_rows[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
-    int32_t* d_srt_vals[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
-    uint8_t* d_srt_codes[IFVS_MAX_ATTRS] = {nullptr, nullptr, nullptr, nullptr};
+    // sorted copies (see SortedCols): row ids in copy order, the codes in
+    // that order; the values of the one-column copies; the composite keys
+    uint32_t* d_srt_rows[kSortedCopies] = {};
+    uint8_t* d_srt_codes[kSortedCopies] = {};
+    int32_t* d_srt_vals[IFVS_MAX_ATTRS] = {};
+    uint64_t* d_ckeys[2] = {};
     uint8_t* d_codes = nullptr;
     float* d_vec = nullptr;
     bool has_cb = false;
@@ -172,11 +174,13 @@ struct ifvs_index {
 
     SortedCols sorted() const {
         SortedCols c;
-        for (int i = 0; i < IFVS_MAX_ATTRS; ++i) {
+        for (int i = 0; i < kSortedCopies; ++i) {
             c.rows[i] = d_srt_rows[i];
-            c.vals[i] = d_srt_vals[i];
             c.codes[i] = d_srt_codes[i];
         }
+        for (int i = 0; i < IFVS_MAX_ATTRS; ++i) c.vals[i] = d_srt_vals[i];
+        c.ckeys[0] = d_ckeys[0];
+        c.ckeys[1] = d_ckeys[1];
         c.n = n_attrs;
         return c;
     }
@@ -220,10 +224,14 @@ void free_index(ifvs_index* ix) {
     if (ix->stream) cudaStreamSynchronize(ix->stream);
     for (int i = 0; i < IFVS_MAX_ATTRS; ++i) {
         if (ix->d_attr[i]) cudaFree(ix->d_attr[i]);
-        if (ix->d_srt_rows[i]) cudaFree(ix->d_srt_rows[i]);
         if (ix->d_srt_vals[i]) cudaFree(ix->d_srt_vals[i]);
+    }
+    for (int i = 0; i < kSortedCopies; ++i) {
+        if (ix->d_srt_rows[i]) cudaFree(ix->d_srt_rows[i]);
         if (ix->d_srt_codes[i]) cudaFree(ix->d_srt_codes[i]);
     }
+    for (int j = 0; j < 2; ++j)
+        if (ix->d_ckeys[j]) cudaFree(ix->d_ckeys[j]);
     void* ptrs[] = {ix->d_codes, ix->d_vec, ix->d_cpq, ix->d_bank, ix->d_W, ix->d_seeds};
     for (void* p : ptrs)
         if (p) cudaFree(p);
@@ -255,65 +263,103 @@ int dev_alloc(ifvs_index* ix, void** p, size_t bytes) {
     return 0;
 }
 
-// Row ids of one attribute column sorted by (value, row), the values in that
-// order, and the code rows copied into that order (rotated by position), on
-// the device.  The order comes from a stable LSD radix sort on the host
-// (two 16-bit digit passes over (key, row) pairs; key = value bits with the
-// sign flipped, so unsigned order is signed order).
-int build_sorted_column(ifvs_index* ix, int c, const void* col, int32_t type, bool dio) {
+// A column's values as int32 on the host (device columns are copied back).
+int column_values(const void* col, int32_t type, bool dio, int64_t N, std::vector<int32_t>& out) {
+    const size_t es = type == IFVS_ATTR_I16 ? 2 : 4;
+    std::vector<uint8_t> raw;
+    const uint8_t* src = (const uint8_t*)col;
+    if (dio) {
+        raw.resize((size_t)N * es);
+        CUDA_TRY(cudaMemcpy(raw.data(), col, (size_t)N * es, cudaMemcpyDeviceToHost));
+        src = raw.data();
+    }
+    out.resize((size_t)N);
+    for (int64_t i = 0; i < N; ++i) {
+        if (type == IFVS_ATTR_I16) {
+            int16_t h;
+            memcpy(&h, src + i * 2, 2);
+            out[(size_t)i] = h;
+        } else {
+            memcpy(&out[(size_t)i], src + i * 4, 4);
+        }
+    }
+    return 0;
+}
+
+// One stable counting-sort pass of (key, row) by the 16-bit digit of key at
+// bit `shift` (least significant digit first: the passes compose into a
+// stable sort by the whole key, ties in row order).
+template <class Key>
+void radix_pass(std::vector<Key>& key, std::vector<uint32_t>& row, std::vector<Key>& key2,
+                std::vector<uint32_t>& row2, int shift, std::vector<int64_t>& cnt) {
+    const size_t n = key.size();
+    std::fill(cnt.begin(), cnt.end(), 0);
+    for (size_t i = 0; i < n; ++i) ++cnt[(size_t)((key[i] >> shift) & 0xFFFFu) + 1];
+    for (int d = 0; d < 65536; ++d) cnt[d + 1] += cnt[d];
+    for (size_t i = 0; i < n; ++i) {
+        const int64_t at = cnt[(size_t)((key[i] >> shift) & 0xFFFFu)]++;
+        key2[(size_t)at] = key[i];
+        row2[(size_t)at] = row[i];
+    }
+    key.swap(key2);
+    row.swap(row2);
+}
+
+// Uploads a sorted copy's row order and lays out its codes.
+int upload_copy(ifvs_index* ix, int c, const std::vector<uint32_t>& row) {
     const int64_t N = ix->N;
-    std::vector<uint32_t> key((size_t)N), row((size_t)N), key2((size_t)N), row2((size_t)N);
-    {
-        const size_t es = type == IFVS_ATTR_I16 ? 2 : 4;
-        std::vector<uint8_t> raw;
-        const uint8_t* src = (const uint8_t*)col;
-        if (dio) {
-            raw.resize((size_t)N * es);
-            CUDA_TRY(cudaMemcpy(raw.data(), col, (size_t)N * es, cudaMemcpyDeviceToHost));
-            src = raw.data();
-        }
-        for (int64_t i = 0; i < N; ++i) {
-            int32_t v;
-            if (type == IFVS_ATTR_I16) {
-                int16_t h;
-                memcpy(&h, src + i * 2, 2);
-                v = h;
-            } else {
-                memcpy(&v, src + i * 4, 4);
-            }
-            key[(size_t)i] = (uint32_t)v ^ 0x80000000u;
-            row[(size_t)i] = (uint32_t)i;
-        }
-    }
-    std::vector<int64_t> cnt(65537);
-    for (int pass = 0; pass < 2; ++pass) {
-        const int sh = 16 * pass;
-        std::fill(cnt.begin(), cnt.end(), 0);
-        for (int64_t i = 0; i < N; ++i) ++cnt[((key[(size_t)i] >> sh) & 0xFFFFu) + 1];
-        for (int d = 0; d < 65536; ++d) cnt[d + 1] += cnt[d];
-        for (int64_t i = 0; i < N; ++i) {
-            const int64_t at = cnt[(key[(size_t)i] >> sh) & 0xFFFFu]++;
-            key2[(size_t)at] = key[(size_t)i];
-            row2[(size_t)at] = row[(size_t)i];
-        }
-        key.swap(key2);
-        row.swap(row2);
-    }
-    for (int64_t i = 0; i < N; ++i) key[(size_t)i] ^= 0x80000000u;   // back to the signed value bits
     void* p = nullptr;
     TRY(dev_alloc(ix, &p, sizeof(uint32_t) * (size_t)N));
     ix->d_srt_rows[c] = (uint32_t*)p;
     CUDA_TRY(cudaMemcpy(p, row.data(), sizeof(uint32_t) * (size_t)N, cudaMemcpyHostToDevice));
-    TRY(dev_alloc(ix, &p, sizeof(int32_t) * (size_t)N));
-    ix->d_srt_vals[c] = (int32_t*)p;
-    CUDA_TRY(cudaMemcpy(p, key.data(), sizeof(int32_t) * (size_t)N, cudaMemcpyHostToDevice));
-    // the code rows in this order, rotated by position
     TRY(dev_alloc(ix, &p, (size_t)ix->n_rows_pad * ix->row_bytes));
     ix->d_srt_codes[c] = (uint8_t*)p;
     CUDA_TRY(launch_relayout_sorted(ix->d_codes, ix->d_srt_rows[c], N, ix->M, ix->row_bytes, ix->n_rows_pad,
                                     ix->d_srt_codes[c], ix->stream));
     CUDA_TRY(cudaStreamSynchronize(ix->stream));
     return 0;
+}
+
+// Sorted copy of column c: rows by (value, row) — a stable host radix sort
+// of the values with the sign bit flipped (unsigned order is signed order)
+// — the values in that order, and the code rows in that order.
+int build_sorted_column(ifvs_index* ix, int c, const std::vector<int32_t>& vals) {
+    const int64_t N = ix->N;
+    std::vector<uint32_t> key((size_t)N), row((size_t)N), key2((size_t)N), row2((size_t)N);
+    for (int64_t i = 0; i < N; ++i) {
+        key[(size_t)i] = (uint32_t)vals[(size_t)i] ^ 0x80000000u;
+        row[(size_t)i] = (uint32_t)i;
+    }
+    std::vector<int64_t> cnt(65537);
+    radix_pass(key, row, key2, row2, 0, cnt);
+    radix_pass(key, row, key2, row2, 16, cnt);
+    for (int64_t i = 0; i < N; ++i) key[(size_t)i] ^= 0x80000000u;   // back to the signed value bits
+    void* p = nullptr;
+    TRY(dev_alloc(ix, &p, sizeof(int32_t) * (size_t)N));
+    ix->d_srt_vals[c] = (int32_t*)p;
+    CUDA_TRY(cudaMemcpy(p, key.data(), sizeof(int32_t) * (size_t)N, cudaMemcpyHostToDevice));
+    return upload_copy(ix, c, row);
+}
+
+// Composite copy j of a two-column index: rows by (column j, column 1 - j,
+// row) — four radix passes over the 64-bit composite key — and that key of
+// each position (ckey).
+int build_composite(ifvs_index* ix, int j, const std::vector<int32_t>& primary,
+                    const std::vector<int32_t>& secondary) {
+    const int64_t N = ix->N;
+    std::vector<uint64_t> key((size_t)N), key2((size_t)N);
+    std::vector<uint32_t> row((size_t)N), row2((size_t)N);
+    for (int64_t i = 0; i < N; ++i) {
+        key[(size_t)i] = ckey(primary[(size_t)i], secondary[(size_t)i]);
+        row[(size_t)i] = (uint32_t)i;
+    }
+    std::vector<int64_t> cnt(65537);
+    for (int shift = 0; shift < 64; shift += 16) radix_pass(key, row, key2, row2, shift, cnt);
+    void* p = nullptr;
+    TRY(dev_alloc(ix, &p, sizeof(uint64_t) * (size_t)N));
+    ix->d_ckeys[j] = (uint64_t*)p;
+    CUDA_TRY(cudaMemcpy(p, key.data(), sizeof(uint64_t) * (size_t)N, cudaMemcpyHostToDevice));
+    return upload_copy(ix, kComposite + j, row);
 }
 
 // Records a CUDA event pair around one launch on the launching stream when
@@ -933,8 +979,18 @@ int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int6
     }
     e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return fail(cuda_fail(e, "attribute upload", __LINE__));
-    for (int i = 0; i < n_attrs; ++i)
-        if ((rc = build_sorted_column(ix, i, attr_cols[i], attr_types[i], dio))) return fail(rc);
+    {
+        std::vector<std::vector<int32_t>> vals((size_t)n_attrs);
+        for (int i = 0; i < n_attrs; ++i) {
+            if ((rc = column_values(attr_cols[i], attr_types[i], dio, N, vals[(size_t)i]))) return fail(rc);
+            if ((rc = build_sorted_column(ix, i, vals[(size_t)i]))) return fail(rc);
+        }
+        // two columns: both composite orders, so that a predicate fixing
+        // either column and bounding the other reads one position range
+        if (n_attrs == 2)
+            for (int jj = 0; jj < 2; ++jj)
+                if ((rc = build_composite(ix, jj, vals[(size_t)jj], vals[(size_t)(1 - jj)]))) return fail(rc);
+    }
     if (vectors) {
         void* v = nullptr;
         if ((rc = dev_alloc(ix, &v, sizeof(float) * N * D))) return fail(rc);

@@ -52,6 +52,18 @@ __device__ __forceinline__ int64_t first_not_below(const int32_t* __restrict__ v
     return lo;
 }
 
+__device__ __forceinline__ int64_t first_key_not_below(const uint64_t* __restrict__ v, int64_t n, uint64_t x) {
+    int64_t lo = 0, hi = n;
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (v[mid] < x)
+            lo = mid + 1;
+        else
+            hi = mid;
+    }
+    return lo;
+}
+
 __global__ void k_plan(const CanonPred* __restrict__ canon, int64_t nq, SortedCols sc, int64_t N,
                        int64_t max_rows, ScanPlan* __restrict__ plan,
                        unsigned long long* __restrict__ npass) {
@@ -90,6 +102,25 @@ __global__ void k_plan(const CanonPred* __restrict__ canon, int64_t nq, SortedCo
                 p.col = c;
                 p.list = 1;
             }
+        }
+    } else if (cp.used == 3u && sc.ckeys[0] != nullptr && (cp.wm1[0] == 0u || cp.wm1[1] == 0u)) {
+        // columns 0 and 1, one of them fixed to a value: a position range of
+        // the composite copy keyed by that column first
+        const int j = cp.wm1[0] == 0u ? 0 : 1;
+        const int32_t v = cp.lo[j];
+        const int32_t lo2 = cp.lo[1 - j];
+        const uint32_t w2 = cp.wm1[1 - j];
+        const uint64_t* keys = sc.ckeys_of(j);
+        const int64_t a = first_key_not_below(keys, N, ckey(v, lo2));
+        // one past (v, lo2 + w2): the next composite key (carries into the
+        // primary half when the secondary value is the largest int32)
+        const uint64_t kh = ckey(v, (int32_t)((uint32_t)lo2 + w2));
+        const int64_t b = kh == ~0ull ? N : first_key_not_below(keys, N, kh + 1ull);
+        if (b - a <= max_rows) {
+            p.a = a;
+            p.b = b;
+            p.col = kComposite + j;
+            p.list = 1;
         }
     }
     plan[q] = p;

@@ -100,34 +100,50 @@ struct AttrCols {
 cudaError_t launch_canonicalize(const ifvs_predicate* preds, int64_t nq, AttrCols cols,
                                 CanonPred* out, int* err, cudaStream_t s);
 
-// Per-query scan plan: a one-column predicate with a pool of at most
-// max_rows rows (or an empty / malformed one) takes the row-list scan over
-// rows [a, b) of column col's sorted order; the rest take the bitmap path.
+// Per-query scan plan: a predicate whose pool is one position range [a, b)
+// of a sorted copy (one constrained column; or, with composite copies, one
+// column fixed to a value and the other bounded) with at most max_rows rows,
+// or an empty / malformed one, takes the sorted-copy scan of copy `col`; the
+// rest take the bitmap path.
 struct ScanPlan {
     int64_t a, b;
     int32_t col;
     int32_t list;      // 1: row-list scan
 };
-// Per column: row ids sorted by (value, row), the values in that order, and
-// a copy of the code rows in that order (position p holds row rows[p]'s
-// codes, rotated by (p mod 32) mod M, row_bytes apart, padded like the index).
+// Sorted copies of the codes.  Copy c < IFVS_MAX_ATTRS: the rows sorted by
+// (column c's value, row); vals[c] holds the values in that order.  For an
+// index of exactly two columns, copies kComposite + j (j = 0, 1) are sorted
+// by (column j, column 1 - j, row), and ckeys[j] holds the composite key
+// ckey(v_j, v_{1-j}) of each position: a predicate fixing column j to one
+// value and bounding the other column to an interval selects one contiguous
+// position range of that copy.  Every copy: position p holds row rows[p]'s
+// codes, rotated by (p mod 32) mod M, row_bytes apart, padded like the index.
+constexpr int kComposite = IFVS_MAX_ATTRS;
+constexpr int kSortedCopies = IFVS_MAX_ATTRS + 2;
+
+// composite key: unsigned order of the pair is signed (primary, secondary) order
+__host__ __device__ inline uint64_t ckey(int32_t primary, int32_t secondary) {
+    return ((uint64_t)((uint32_t)primary ^ 0x80000000u) << 32) | (uint64_t)((uint32_t)secondary ^ 0x80000000u);
+}
+
 struct SortedCols {
-    const uint32_t* rows[IFVS_MAX_ATTRS];
+    const uint32_t* rows[kSortedCopies];
+    const uint8_t* codes[kSortedCopies];
     const int32_t* vals[IFVS_MAX_ATTRS];
-    const uint8_t* codes[IFVS_MAX_ATTRS];
+    const uint64_t* ckeys[2];
     int32_t n;
+    // copy c's arrays, selected without indexing the parameter at run time
     __host__ __device__ const uint8_t* codes_of(int c) const {
         const uint8_t* r = codes[0];
 #pragma unroll
-        for (int i = 1; i < IFVS_MAX_ATTRS; ++i)
+        for (int i = 1; i < kSortedCopies; ++i)
             if (c == i) r = codes[i];
         return r;
     }
-    // column c's arrays, selected without indexing the parameter at run time
     __host__ __device__ const uint32_t* rows_of(int c) const {
         const uint32_t* r = rows[0];
 #pragma unroll
-        for (int i = 1; i < IFVS_MAX_ATTRS; ++i)
+        for (int i = 1; i < kSortedCopies; ++i)
             if (c == i) r = rows[i];
         return r;
     }
@@ -138,6 +154,7 @@ struct SortedCols {
             if (c == i) v = vals[i];
         return v;
     }
+    __host__ __device__ const uint64_t* ckeys_of(int j) const { return j == 0 ? ckeys[0] : ckeys[1]; }
 };
 // plan [nq]; writes npass of the list-path queries
 cudaError_t launch_plan(const CanonPred* canon, int64_t nq, SortedCols sc, int64_t N, int64_t max_rows,

@@ -377,7 +377,7 @@ __device__ __forceinline__ void quant_params(const float* lo, const float* hi, f
 // nothing); `paired` marks the queries of the pairs, and k_scan_list serves
 // every other list-path query.
 constexpr int kPairSeg = 2048;
-static_assert(IFVS_MAX_ATTRS <= 4, "the pairing key keeps 2 bits of the column");
+static_assert(kSortedCopies <= 8, "the pairing key keeps 3 bits of the sorted copy");
 constexpr int kPairSortThreads = 1024;
 
 __device__ __forceinline__ bool pairable(const ScanPlan& x, const ScanPlan& y, int64_t min_rows) {
@@ -419,13 +419,13 @@ k_pair_items(const ScanPlan* __restrict__ plan, int64_t nq, int64_t min_rows, Pa
     __shared__ int wsum[kPairSortThreads / 32];
     const int64_t q0 = (int64_t)blockIdx.x * kPairSeg;
     const int n = (int)min((int64_t)kPairSeg, nq - q0);
-    // key = col (2 bits) | range start (32 bits) | index in the segment (11 bits);
+    // key = copy (3 bits) | range start (32 bits) | index in the segment (11 bits);
     // queries of the bitmap path sort last as all ones
     for (int i = threadIdx.x; i < kPairSeg; i += kPairSortThreads) {
         uint64_t kk = ~0ull;
         if (i < n) {
             const ScanPlan p = plan[q0 + i];
-            if (p.list) kk = ((uint64_t)(p.col & 3) << 43) | ((uint64_t)(uint32_t)p.a << 11) | (uint64_t)i;
+            if (p.list) kk = ((uint64_t)(p.col & 7) << 43) | ((uint64_t)(uint32_t)p.a << 11) | (uint64_t)i;
         }
         key[i] = kk;
     }

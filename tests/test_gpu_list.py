@@ -381,3 +381,61 @@ def test_bulk_copy_wait_runs_out_and_reports_timeout(ifvs, monkeypatch):
     again = g.search(q, p, 10, pair_min_rows=-1)
     for x, y in zip(ref, again):
         np.testing.assert_array_equal(x, y)
+
+
+@pytest.mark.parametrize("k", [10, 100])
+def test_composite_copies_for_two_column_predicates(ifvs, orc, k):
+    """An index of two columns keeps, besides one sorted copy per column,
+    both composite copies (rows by (column j, column 1 - j)).  A predicate
+    that fixes one column to a value and bounds the other (Listing 1's
+    `category = c AND date range`) reads one position range of the copy
+    keyed by the fixed column; pass counts must equal the oracle's and the
+    bitmap path's exactly, and top-k the oracle's with the tie rule.  Cases:
+    either column fixed, one- and two-sided bounds, both fixed, values
+    absent, empty intervals, and the largest and smallest int32 values
+    (the composite key's carry)."""
+    N = 100_003
+    rng = np.random.default_rng(51)
+    M, K, ds = 16, 256, 2
+    codes = rng.integers(0, K, size=(N, M)).astype(np.uint8)
+    a0 = rng.integers(-40, 40, N).astype(np.int32)
+    a0[::997] = np.iinfo(np.int32).max
+    a0[5::991] = np.iinfo(np.int32).min
+    a1 = rng.integers(-300, 300, N).astype(np.int16)
+    a1[7::1009] = np.iinfo(np.int16).max
+    attrs = [a0, a1]
+    Cpq = rng.standard_normal((M, K, ds)).astype(np.float32)
+    g = ifvs.Index(codes, attrs, D=M * ds, K=K)
+    g.load_codebooks(Cpq)
+    i32, i16 = np.iinfo(np.int32), np.iinfo(np.int16)
+    rows = [
+        [(0, synth.OP_EQ, 3), (1, synth.OP_RANGE, -50, 120)],
+        [(1, synth.OP_EQ, -17), (0, synth.OP_RANGE, -10, 30)],
+        [(0, synth.OP_EQ, -40), (1, synth.OP_GE, 200)],
+        [(1, synth.OP_EQ, 0), (0, synth.OP_LT, 0)],
+        [(0, synth.OP_EQ, 12), (1, synth.OP_EQ, 44)],
+        [(0, synth.OP_EQ, 1000), (1, synth.OP_RANGE, -300, 300)],     # value absent
+        [(0, synth.OP_EQ, 5), (1, synth.OP_RANGE, 10, 10)],           # empty interval
+        [(0, synth.OP_EQ, int(i32.max)), (1, synth.OP_LE, int(i16.max))],
+        [(0, synth.OP_EQ, int(i32.min)), (1, synth.OP_GE, int(i16.min))],
+        [(1, synth.OP_EQ, int(i16.max)), (0, synth.OP_GE, int(i32.min))],
+        [(0, synth.OP_RANGE, -5, 5), (1, synth.OP_RANGE, 0, 50)],     # neither fixed: bitmap path
+        [(0, synth.OP_EQ, -1), (1, synth.OP_RANGE, -300, 300), (0, synth.OP_GE, -1)],
+    ]
+    p = synth.empty_predicates(len(rows))
+    for i, cl in enumerate(rows):
+        p[i]["n_clauses"] = len(cl)
+        for j, c in enumerate(cl):
+            synth.set_clause(p[i], j, *c)
+    q = _queries(len(rows), M * ds, seed=52)
+    a = g.search(q, p, k, list_max_ppm=ALWAYS)
+    b = g.search(q, p, k, list_max_ppm=NEVER)
+    np.testing.assert_array_equal(a[2], b[2])
+    _same_up_to_rounding(a, b)
+    _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
+    # one query at a time, and the batch with pairing forced
+    for x, y in zip(a, _one_by_one(g, q, p, k)):
+        np.testing.assert_array_equal(x, y)
+    for x, y in zip(a, g.search(q, p, k, pair_min_rows=1)):
+        np.testing.assert_array_equal(x, y)
+    g.close()
