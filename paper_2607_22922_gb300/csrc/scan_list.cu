@@ -311,6 +311,158 @@ k_scan_list_bulk(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     merge_warps<KP, kScanWarps>(tk, tkbuf, k, lane, warp, out);
 }
 
+// ---- generic M: one row per lane and round from a bulk-copied tile ---------
+//
+// For M other than 12 and 16 the code rows are M rounded up to 4 bytes (120
+// for gist1m), and per-lane loads of a row's words touch one 32-byte sector
+// per lane per word: about one L1 wavefront per row and word, several times
+// the look-ups' own shared-memory wavefronts.  Here a warp's round is 32
+// consecutive positions (one per lane), 32 x row_bytes contiguous bytes (at
+// most 4 KB), brought into the warp's shared tile by one bulk copy; each lane
+// then reads its own row's words from shared memory.  A row's entries are
+// added for s ascending from its rotated first subspace, as in lookup_rows,
+// so the results equal the vector-load kernel's bit for bit.
+__host__ __device__ inline size_t bulkg_ring_offset(int tab_words, int kp) {
+    return ((size_t)256 * tab_words * 4 + (size_t)kScanWarps * 2 * kp * 8 + 16 + 127) / 128 * 128;
+}
+
+size_t scan_bulkg_smem_bytes(int tab_words, int kp, int row_bytes) {
+    return bulkg_ring_offset(tab_words, kp) + (size_t)kScanWarps * kBulkStages * (32u * row_bytes + 8) + 16;
+}
+
+template <int KP>
+__device__ __forceinline__ void scan_positions_bulkg(const uint8_t* __restrict__ codes,
+                                                     const uint32_t* __restrict__ rows, int64_t a, int64_t b,
+                                                     int64_t blk0, int64_t blk1, const ScanShape& sh,
+                                                     const float* tab, uint8_t* ring, uint64_t* bars,
+                                                     uint32_t tx_extra, int* err, WarpTopK<KP>& tk, int lane,
+                                                     int warp) {
+    constexpr int NST = kBulkStages;
+    const int M = sh.M, S = sh.tab_words, rb = sh.row_bytes, nw = sh.row_bytes / 4;
+    const uint32_t tile_bytes = 32u * (uint32_t)rb;
+    const uint64_t keep = policy_evict_last();
+    const uint32_t a32 = (uint32_t)a, b32 = (uint32_t)b;
+    const int64_t first = blk0 + warp;
+    const int nblk = first < blk1 ? (int)((blk1 - first + kScanWarps - 1) / kScanWarps) : 0;
+    const int R = 32 * nblk;   // one row per lane per round: 32 rounds per block
+    const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
+    const uint32_t bar_s = (uint32_t)__cvta_generic_to_shared(bars);
+    auto tile_pos = [&](int r) -> uint32_t {
+        return (uint32_t)((first + (int64_t)(r >> 5) * kScanWarps) * kBlockRows) + 32u * (uint32_t)(r & 31);
+    };
+    auto issue = [&](int r) {
+        const uint32_t st = (uint32_t)(r % NST);
+        mbar_arrive_expect_tx(bar_s + 8u * st, tile_bytes + tx_extra);
+        bulk_g2s(ring_s + st * tile_bytes, codes + (size_t)tile_pos(r) * rb, tile_bytes, bar_s + 8u * st, keep);
+    };
+    if (lane == 0)
+        for (int r = 0; r < NST && r < R; ++r) issue(r);
+    const float* tw = tab + lane;
+#pragma unroll 1
+    for (int r = 0; r < R; ++r) {
+        const int st = r % NST;
+        if (!mbar_wait_warp(bar_s + 8u * (uint32_t)st, (uint32_t)(r / NST) & 1u)) {
+            if (lane == 0) atomicOr(err, 4);
+            for (int q = r; q < R && q < r + NST; ++q)
+                mbar_wait_warp(bar_s + 8u * (uint32_t)(q % NST), (uint32_t)(q / NST) & 1u);
+            return;
+        }
+        tk.refresh(lane);
+        const uint32_t pos = tile_pos(r) + (uint32_t)lane;
+        const bool valid = pos >= a32 && pos < b32;
+        const uint32_t* row = reinterpret_cast<const uint32_t*>(ring + (size_t)st * tile_bytes) + lane * nw;
+        float acc = 0.f;
+#pragma unroll 2
+        for (int w = 0; w < nw; ++w) {
+            const uint32_t wd = row[w];
+#pragma unroll
+            for (int bb = 0; bb < 4; ++bb) {
+                const int s = 4 * w + bb;
+                if (s < M) acc += tw[(int)((wd >> (8 * bb)) & 0xFFu) * S + s];
+            }
+        }
+        __syncwarp();   // every lane has read its row: the tile can be refilled
+        if (lane == 0 && r + NST < R) {
+            fence_proxy_async_smem();
+            issue(r + NST);
+        }
+        const bool cand = valid && __float_as_uint(acc) <= (uint32_t)(tk.thr >> 32);
+        if (!__any_sync(0xFFFFFFFFu, cand)) continue;
+        const uint32_t id = cand ? __ldg(rows + pos) : 0u;
+        const uint64_t key = ((uint64_t)__float_as_uint(acc) << 32) | id;
+        tk.offer(key, cand && key < tk.thr, lane);
+    }
+}
+
+template <int KP>
+__global__ void __launch_bounds__(kScanThreads, 1)
+k_scan_list_bulkg(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan, int64_t nq,
+                  int k, ScanShape sh, uint64_t* __restrict__ partials, const uint8_t* __restrict__ paired,
+                  uint32_t tx_extra, int* __restrict__ err) {
+    extern __shared__ __align__(256) uint8_t smem[];
+    const int S = sh.tab_words;
+    float* tab = reinterpret_cast<float*>(smem);
+    uint64_t* tkbuf = reinterpret_cast<uint64_t*>(smem + (size_t)256 * S * 4);
+    const uint32_t tile_bytes = 32u * (uint32_t)sh.row_bytes;
+    uint8_t* ring_all = smem + bulkg_ring_offset(S, KP);
+    uint64_t* bars_all = reinterpret_cast<uint64_t*>(ring_all + (size_t)kScanWarps * kBulkStages * tile_bytes);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t q = blockIdx.x;
+    const int chunk = blockIdx.y;
+    const ScanPlan p = plan[q];
+    if (!p.list) return;
+    if (paired != nullptr && paired[q]) return;
+    const int64_t c0 = (int64_t)chunk * sh.blocks_per_chunk;
+    const int64_t c1 = min(sh.n_blocks, c0 + sh.blocks_per_chunk);
+    const int64_t blk0 = max(c0, p.a / kBlockRows);
+    const int64_t blk1 = min(c1, (p.b + kBlockRows - 1) / kBlockRows);
+    uint64_t* out = partials + (q * sh.n_chunks + chunk) * (int64_t)k;
+    if (p.a >= p.b || blk0 >= blk1) {
+        for (int i = threadIdx.x; i < k; i += kScanThreads) out[i] = ~0ull;
+        return;
+    }
+    uint8_t* ring = ring_all + (size_t)warp * kBulkStages * tile_bytes;
+    uint64_t* bars = bars_all + warp * kBulkStages;
+    const uint32_t tbar = (uint32_t)__cvta_generic_to_shared(bars_all + kScanWarps * kBulkStages);
+    if (lane == 0) {
+        for (int i = 0; i < kBulkStages; ++i) mbar_init((uint32_t)__cvta_generic_to_shared(bars + i), 1u);
+        if (threadIdx.x == 0) mbar_init(tbar, 1u);
+        fence_mbar_init();
+    }
+    if (threadIdx.x == 0) {
+        const uint32_t tb = 256u * (uint32_t)S * 4u;
+        mbar_arrive_expect_tx(tbar, tb);
+        bulk_g2s((uint32_t)__cvta_generic_to_shared(tab), tables + q * (int64_t)256 * S, tb, tbar,
+                 policy_evict_first());
+    }
+    uint64_t* cta = tkbuf + kScanWarps * 2 * KP;
+    if (threadIdx.x == 0) *cta = ~0ull;
+    WarpTopK<KP> tk;
+    tk.init(tkbuf + warp * 2 * KP, k, lane, cta);
+    __syncthreads();
+    if (!mbar_wait_warp(tbar, 0u)) {
+        if (lane == 0) atomicOr(err, 4);
+        mbar_wait_warp(tbar, 0u);
+        merge_warps<KP, kScanWarps>(tk, tkbuf, k, lane, warp, out);
+        return;
+    }
+    scan_positions_bulkg<KP>(sc.codes_of(p.col), sc.rows_of(p.col), p.a, p.b, blk0, blk1, sh, tab, ring, bars,
+                             tx_extra, err, tk, lane, warp);
+    merge_warps<KP, kScanWarps>(tk, tkbuf, k, lane, warp, out);
+}
+
+template <int KP>
+static cudaError_t launch_list_bulkg(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
+                                     const ScanShape& sh, uint64_t* partials, const uint8_t* paired, size_t smem,
+                                     uint32_t tx_extra, int* err, cudaStream_t s) {
+    cudaError_t e =
+        cudaFuncSetAttribute(k_scan_list_bulkg<KP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)nq, (unsigned)sh.n_chunks);
+    k_scan_list_bulkg<KP><<<grid, kScanThreads, smem, s>>>(tab, sc, plan, nq, k, sh, partials, paired, tx_extra, err);
+    return cudaGetLastError();
+}
+
 template <int KP, int MM, int MINB>
 static cudaError_t launch_list_bulk(const float* tab, SortedCols sc, const ScanPlan* plan, int64_t nq, int k,
                                     const ScanShape& sh, uint64_t* partials, const uint8_t* paired, size_t smem,
@@ -365,6 +517,11 @@ static cudaError_t launch_list_kp(const float* tab, SortedCols sc, const ScanPla
                        : launch_list_bulk<KP, 12, 1>(tab, sc, plan, nq, k, sh, partials, paired, smem, lo.tx_extra,
                                                      lo.err, s);
         }
+    }
+    if (mm == 0 && lo.bulk && sh.row_bytes <= 128 && sh.row_bytes % 4 == 0) {
+        const size_t smem = scan_bulkg_smem_bytes(sh.tab_words, KP, sh.row_bytes);
+        if (smem <= (size_t)max_smem_optin())
+            return launch_list_bulkg<KP>(tab, sc, plan, nq, k, sh, partials, paired, smem, lo.tx_extra, lo.err, s);
     }
     const size_t smem = scan_list_smem_bytes(sh.tab_words, KP);
     const bool two = (size_t)233472 / (smem + 1024) >= 2;

@@ -439,3 +439,20 @@ def test_composite_copies_for_two_column_predicates(ifvs, orc, k):
     for x, y in zip(a, g.search(q, p, k, pair_min_rows=1)):
         np.testing.assert_array_equal(x, y)
     g.close()
+
+
+@pytest.mark.parametrize("M,ds,k", [(8, 2, 10), (24, 1, 100), (120, 1, 10), (120, 1, 200), (5, 3, 30)])
+def test_generic_m_bulk_tiles_equal_vector_loads(ifvs, orc, M, ds, k):
+    """For M other than 12 and 16 the one-query kernel reads one row per lane
+    and round from a bulk-copied tile of 32 rows (lists of 256 keys leave no
+    room for it: the vector-load kernel runs).  Both add a row's entries in
+    the same order, so results must agree bit for bit, and with the oracle."""
+    N = 70_001
+    g, codes, attrs, Cpq = _index(ifvs, N, M=M, ds=ds, seed=61 + M)
+    p = _preds()
+    q = _queries(len(p), M * ds, seed=62)
+    a = g.search(q, p, k, pair_min_rows=-1)
+    b = g.search(q, p, k, pair_min_rows=-1, flags=ifvs.IFVS_F_PLAIN_LOADS)
+    for x, y in zip(a, b):
+        np.testing.assert_array_equal(x, y)
+    _check_oracle(orc, codes, attrs, Cpq, q, p, k, *a)
