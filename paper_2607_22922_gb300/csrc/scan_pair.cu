@@ -50,10 +50,12 @@ constexpr size_t kCandWarpBytes = (size_t)kCandCap * (16 + 4 + 4);
 __host__ __device__ constexpr bool pair_defers(int kp) { return IFVS_PAIR_DEFER != 0 && kp <= 128; }
 
 // packed table, two exact tables, extremes + the two shared bounds, lists,
-// the candidate buffers
+// the candidate buffers, the current work item (no static shared memory:
+// it would move the dynamic window off the base the look-ups' immediate
+// offsets assume)
 size_t scan_pair_smem_bytes(int kp) {
     return (size_t)kTabBytes16 + 2 * (size_t)kExactBytes16 + 64 * 4 + 16 + (size_t)kPairWarps * 2 * 2 * kp * 8 +
-           (pair_defers(kp) ? (size_t)kPairWarps * kCandWarpBytes : 0);
+           (pair_defers(kp) ? (size_t)kPairWarps * kCandWarpBytes : 0) + 16;
 }
 
 template <int IMM>
@@ -414,7 +416,8 @@ __device__ __forceinline__ int block_prefix(int v, int* wsum, int& total) {
 
 __global__ void __launch_bounds__(kPairSortThreads)
 k_pair_items(const ScanPlan* __restrict__ plan, int64_t nq, int64_t min_rows, PairItem* __restrict__ items,
-             uint8_t* __restrict__ paired) {
+             uint8_t* __restrict__ paired, unsigned* __restrict__ counter) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) *counter = 0u;   // work counter of the two-query kernel
     __shared__ uint64_t key[kPairSeg];
     __shared__ int wsum[kPairSortThreads / 32];
     const int64_t q0 = (int64_t)blockIdx.x * kPairSeg;
@@ -468,11 +471,18 @@ k_pair_items(const ScanPlan* __restrict__ plan, int64_t nq, int64_t min_rows, Pa
     for (int i = total + j; i < (n + 1) / 2; i += kPairSortThreads) its[i] = PairItem{-1, -1};
 }
 
+// Offset of the current work item in the two-query kernel's shared memory.
+__host__ __device__ constexpr size_t scan_pair_item_offset(int kp) {
+    return (size_t)kTabBytes16 + 2 * (size_t)kExactBytes16 + 64 * 4 + 16 + (size_t)kPairWarps * 2 * 2 * kp * 8 +
+           (pair_defers(kp) ? (size_t)kPairWarps * kCandWarpBytes : 0);
+}
+
+// One work item of the two-query kernel: pair slot `slot` on chunk `chunk`.
 template <int KP>
-__global__ void __launch_bounds__(kPairThreads, 1)
-k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan,
-                 const PairItem* __restrict__ items, int k, ScanShape sh, uint64_t* __restrict__ partials) {
-    extern __shared__ __align__(256) uint8_t smem[];
+__device__ __forceinline__ void pair_item(uint8_t* smem, const float* __restrict__ tables, const SortedCols& sc,
+                                          const ScanPlan* __restrict__ plan, const PairItem* __restrict__ items,
+                                          int k, const ScanShape& sh, uint64_t* __restrict__ partials, int slot,
+                                          int chunk) {
     uint32_t* ptab = reinterpret_cast<uint32_t*>(smem);
     float* exA = reinterpret_cast<float*>(smem + kTabBytes16);
     float* exB = reinterpret_cast<float*>(smem + kTabBytes16 + kExactBytes16);
@@ -483,12 +493,11 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     float* red = reinterpret_cast<float*>(tkbufA);   // [warp][4][16], before the lists are set up
     uint8_t* cand_base = reinterpret_cast<uint8_t*>(tkbufB + kPairWarps * 2 * KP);   // 16-byte aligned
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const PairItem it = items[blockIdx.x];
+    const PairItem it = items[slot];
     if (it.qa < 0) return;
     const int64_t qA = it.qa;
     const bool hasB = it.qb >= 0;
     const int64_t qB = hasB ? it.qb : it.qa;   // a single query: B mirrors A's table, with no range
-    const int chunk = blockIdx.y;
     const ScanPlan pA = plan[qA];
     ScanPlan pB = plan[qB];
     if (!hasB) pB.a = pB.b = 0;
@@ -584,8 +593,34 @@ k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan
     merge_warps<KP, kPairWarps>(tkB, tkbufB, k, lane, warp, outB);
 }
 
+// Persistent: one CTA per SM takes work items (pair slot, chunk) in the
+// order of a (slot, chunk) grid, chunk-major, from a counter that
+// k_pair_items zeroes: the CTAs that run together still walk the same chunk,
+// and no SM idles through a ragged last wave of long items (a 1024-CTA grid
+// over 152 SMs left 0.26 of its last wave empty on the dense bin).
+template <int KP>
+__global__ void __launch_bounds__(kPairThreads, 1)
+k_scan_list_pair(const float* __restrict__ tables, SortedCols sc, const ScanPlan* __restrict__ plan,
+                 const PairItem* __restrict__ items, int n_slots, unsigned* __restrict__ counter, int k,
+                 ScanShape sh, uint64_t* __restrict__ partials) {
+    extern __shared__ __align__(256) uint8_t smem[];
+    volatile unsigned* s_item = reinterpret_cast<volatile unsigned*>(smem + scan_pair_item_offset(KP));
+    const unsigned total = (unsigned)n_slots * (unsigned)sh.n_chunks;
+    for (;;) {
+        if (threadIdx.x == 0) *s_item = atomicAdd(counter, 1u);
+        __syncthreads();
+        const unsigned w = *s_item;
+        __syncthreads();   // read by all before thread 0 takes the next item
+        if (w >= total) break;
+        pair_item<KP>(smem, tables, sc, plan, items, k, sh, partials, (int)(w % (unsigned)n_slots),
+                      (int)(w / (unsigned)n_slots));
+        __syncthreads();   // the next item reuses the shared memory
+    }
+}
+
 size_t scan_list_workspace_bytes(int64_t nq) {
-    // pair slots (each segment rounds its count up), a flag per query
+    // pair slots (each segment rounds its count up), a flag per query, the
+    // two-query kernel's work counter
     return (size_t)(nq + 2 * kPairSeg) * sizeof(PairItem) + (size_t)nq + 64;
 }
 
@@ -597,15 +632,22 @@ static cudaError_t launch_pairs_kp(const float* tab, SortedCols sc, const ScanPl
     if (ps > (size_t)max_smem_optin()) return cudaSuccess;   // no pairs: one query per CTA
     PairItem* items = reinterpret_cast<PairItem*>(work);
     uint8_t* pd = reinterpret_cast<uint8_t*>(items + nq + 2 * kPairSeg);
+    unsigned* counter = reinterpret_cast<unsigned*>(work + (((size_t)(nq + 2 * kPairSeg) * sizeof(PairItem) +
+                                                             (size_t)nq + 15) / 16) * 16);
     const unsigned segs = (unsigned)((nq + kPairSeg - 1) / kPairSeg);
-    k_pair_items<<<segs, kPairSortThreads, 0, s>>>(plan, nq, pair_min_rows, items, pd);
+    k_pair_items<<<segs, kPairSortThreads, 0, s>>>(plan, nq, pair_min_rows, items, pd, counter);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if ((e = cudaFuncSetAttribute(k_scan_list_pair<KP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ps)) !=
         cudaSuccess)
         return e;
-    dim3 grid((unsigned)((nq + 1) / 2), (unsigned)sh.n_chunks);   // at most nq / 2 pairs
-    k_scan_list_pair<KP><<<grid, kPairThreads, ps, s>>>(tab, sc, plan, items, k, sh, partials);
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    const int n_slots = (int)((nq + 1) / 2);   // at most nq / 2 pairs
+    const long long items_total = (long long)n_slots * sh.n_chunks;
+    const int grid = (int)(items_total < sms ? items_total : sms);   // one CTA per SM
+    k_scan_list_pair<KP><<<grid, kPairThreads, ps, s>>>(tab, sc, plan, items, n_slots, counter, k, sh, partials);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     *paired = pd;
     *launches += 2;
