@@ -379,12 +379,7 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 
 // one arrival that also announces `bytes` of bulk-copy traffic
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
-    uint64_t state;
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 %0, [%1], %2;"
-                 : "=l"(state)
-                 : "r"(bar), "r"(bytes)
-                 : "memory");
-    (void)state;
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 
 // global -> shared copy of `bytes` (a multiple of 16, both addresses 16-byte
