@@ -392,8 +392,9 @@ def test_composite_copies_for_two_column_predicates(ifvs, orc, k):
     keyed by the fixed column; pass counts must equal the oracle's and the
     bitmap path's exactly, and top-k the oracle's with the tie rule.  Cases:
     either column fixed, one- and two-sided bounds, both fixed, values
-    absent, empty intervals, and the largest and smallest int32 values
-    (the composite key's carry)."""
+    absent, empty intervals, the largest and smallest int32 values (the
+    composite key's carry); predicates fixing neither column take the
+    bitmap path in the same batch."""
     N = 100_003
     rng = np.random.default_rng(51)
     M, K, ds = 16, 256, 2
@@ -419,7 +420,12 @@ def test_composite_copies_for_two_column_predicates(ifvs, orc, k):
         [(0, synth.OP_EQ, int(i32.max)), (1, synth.OP_LE, int(i16.max))],
         [(0, synth.OP_EQ, int(i32.min)), (1, synth.OP_GE, int(i16.min))],
         [(1, synth.OP_EQ, int(i16.max)), (0, synth.OP_GE, int(i32.min))],
-        [(0, synth.OP_RANGE, -5, 5), (1, synth.OP_RANGE, 0, 50)],     # neither fixed: bitmap path
+        # neither column fixed: bitmap path
+        [(0, synth.OP_RANGE, -5, 5), (1, synth.OP_RANGE, 0, 50)],
+        [(0, synth.OP_LE, 10), (1, synth.OP_RANGE, -300, 250)],
+        [(1, synth.OP_GE, -200), (0, synth.OP_RANGE, -40, 30)],
+        [(0, synth.OP_GE, int(i32.min)), (1, synth.OP_LT, 290)],
+        [(0, synth.OP_RANGE, -40, 40), (1, synth.OP_GE, int(i16.min))],
         [(0, synth.OP_EQ, -1), (1, synth.OP_RANGE, -300, 300), (0, synth.OP_GE, -1)],
     ]
     p = synth.empty_predicates(len(rows))
