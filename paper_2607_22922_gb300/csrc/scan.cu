@@ -37,105 +37,103 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
     const int T = first < b1 ? (int)((b1 - first + kScanWarps - 1) / kScanWarps) : 0;
     auto word_addr = [&](int t) { return bmq + (first + (int64_t)t * kScanWarps) * 32 + lane; };
 
-    // ring: words of the blocks t in [F - kRing, F) in slot t % kRing
+    // ring: words of the blocks t in [F - kRing, F) in slot t % kRing;
+    // dense: bit t % kRing set when block t has at least kDenseRows passing
+    // rows (warp-uniform)
+    uint32_t dense = 0u;
+    auto mark = [&](int t, uint32_t w) {
+        const unsigned n = __reduce_add_sync(0xFFFFFFFFu, (unsigned)__popc(w));
+        const uint32_t bit = 1u << (t % kRing);
+        dense = n >= (unsigned)kDenseRows ? (dense | bit) : (dense & ~bit);
+    };
     int F = T < kRing ? T : kRing;
 #pragma unroll
     for (int i = 0; i < kRing; ++i)
-        if (i < F) ring[i * 32 + lane] = ldg_nc_u32(word_addr(i), policy_evict_first());
+        if (i < F) {
+            const uint32_t w = ldg_nc_u32(word_addr(i), policy_evict_first());
+            ring[i * 32 + lane] = w;
+            mark(i, w);
+        }
     uint32_t pf[kHalf];
     int npf = T - F < kHalf ? T - F : kHalf;
 #pragma unroll
     for (int i = 0; i < kHalf; ++i) pf[i] = i < npf ? ldg_nc_u32(word_addr(F + i), policy_evict_first()) : 0u;
     __syncwarp();
+    // a lane stops at every dense block (held) until the whole warp has
+    // reached it, so all lanes wait at the same block
     int pos = 0;
     uint32_t cur = F > 0 ? ring[lane] : 0u;
-
-    for (;;) {
-        const int slow = (int)__reduce_min_sync(0xFFFFFFFFu, (unsigned)pos);
-        if (npf > 0 && slow >= F - kHalf) {
-#pragma unroll
-            for (int i = 0; i < kHalf; ++i)
-                if (i < npf) ring[((F + i) % kRing) * 32 + lane] = pf[i];
-            F += npf;
-            npf = T - F < kHalf ? T - F : kHalf;
-            const uint64_t once = policy_evict_first();
-#pragma unroll
-            for (int i = 0; i < kHalf; ++i) pf[i] = i < npf ? ldg_nc_u32(word_addr(F + i), once) : 0u;
-            __syncwarp();
-        }
-        // lanes whose word is used up move on before the mode is chosen
-        while (cur == 0u && pos + 1 < F) {
+    bool held = F > 0 && (dense & 1u) != 0u;
+    auto advance = [&]() {
+        while (cur == 0u && !held && pos + 1 < F) {
             ++pos;
             cur = ring[(pos % kRing) * 32 + lane];
+            held = (dense >> (pos % kRing) & 1u) != 0u;
         }
-        const bool dense = __all_sync(0xFFFFFFFFu, cur == 0xFFFFFFFFu) &&
-                           __reduce_min_sync(0xFFFFFFFFu, (unsigned)pos) ==
-                               __reduce_max_sync(0xFFFFFFFFu, (unsigned)pos);
-        if (dense) {
-            // every lane holds all 32 rows of the same block: lockstep rows
-            const uint32_t rb = (uint32_t)((first + (int64_t)pos * kScanWarps) * kBlockRows) + lane;
-#pragma unroll 1
-            for (int j0 = 0; j0 < 32; j0 += kU) {
-                uint32_t row[kU];
-#pragma unroll
-                for (int u = 0; u < kU; ++u) row[u] = rb + 32u * (uint32_t)(j0 + u);
-                if constexpr (MM > 0) {
-                    uint4 c[kU];
-#pragma unroll
-                    for (int u = 0; u < kU; ++u) c[u] = ldg_nc_v4(codes + (size_t)row[u] * 16, keep);
-                    float d[kU];
-#pragma unroll
-                    for (int u = 0; u < kU; u += 2) lookup2<MM, FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
-                    uint64_t key[kU];
-                    bool want = false;
-#pragma unroll
-                    for (int u = 0; u < kU; ++u) {
-                        key[u] = ((uint64_t)__float_as_uint(d[u]) << 32) | row[u];
-                        want |= key[u] < tk.thr;
-                    }
-                    if (__any_sync(0xFFFFFFFFu, want)) {
-#pragma unroll
-                        for (int u = 0; u < kU; ++u) tk.offer(key[u], key[u] < tk.thr, lane);
-                    }
-                } else {
-                    float d[kU];
-                    lookup_rows<kU>(codes, row, (1u << kU) - 1u, row_bytes, M, S, tab, lane, d);
-#pragma unroll
-                    for (int u = 0; u < kU; ++u) {
-                        const uint64_t key = ((uint64_t)__float_as_uint(d[u]) << 32) | row[u];
-                        tk.offer(key, key < tk.thr, lane);
-                    }
-                }
-            }
-            cur = 0u;
-            continue;
-        }
-        // up to kU passing rows of this lane
+    };
+
+    int col = -1;   // >= 0: the warp is in the dense block at pos, at this column
+    for (;;) {
         uint32_t row[kU];
         unsigned valid = 0u;
+        if (col < 0) {
+            const int slow = (int)__reduce_min_sync(0xFFFFFFFFu, (unsigned)pos);
+            if (npf > 0 && slow >= F - kHalf) {
 #pragma unroll
-        for (int u = 0; u < kU; ++u) {
-            while (cur == 0u && pos + 1 < F) {
-                ++pos;
-                cur = ring[(pos % kRing) * 32 + lane];
+                for (int i = 0; i < kHalf; ++i)
+                    if (i < npf) {
+                        ring[((F + i) % kRing) * 32 + lane] = pf[i];
+                        mark(F + i, pf[i]);
+                    }
+                F += npf;
+                npf = T - F < kHalf ? T - F : kHalf;
+                const uint64_t once = policy_evict_first();
+#pragma unroll
+                for (int i = 0; i < kHalf; ++i) pf[i] = i < npf ? ldg_nc_u32(word_addr(F + i), once) : 0u;
+                __syncwarp();
             }
-            row[u] = 0u;
-            if (cur != 0u) {
-                const int j = __ffs(cur) - 1;
-                cur &= cur - 1u;
-                row[u] = (uint32_t)((first + (int64_t)pos * kScanWarps) * kBlockRows) + 32u * (uint32_t)j + lane;
-                valid |= 1u << u;
+            // lanes whose word is used up move on before the mode is chosen
+            advance();
+            if (__all_sync(0xFFFFFFFFu, held)) col = 0;
+        }
+        if (col >= 0) {
+            // a dense block in lockstep: kU columns, 32 neighbouring rows
+            // per column, lanes whose row fails masked
+            const uint32_t rb = (uint32_t)((first + (int64_t)pos * kScanWarps) * kBlockRows) + 32u * (uint32_t)col + lane;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) row[u] = rb + 32u * (uint32_t)u;
+            valid = cur >> col & ((1u << kU) - 1u);
+            col += kU;
+            if (col == 32) {
+                col = -1;
+                cur = 0u;
+                held = false;
+            }
+        } else {
+            // up to kU passing rows of this lane
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                advance();
+                row[u] = 0u;
+                if (cur != 0u && !held) {
+                    const int j = __ffs(cur) - 1;
+                    cur &= cur - 1u;
+                    row[u] = (uint32_t)((first + (int64_t)pos * kScanWarps) * kBlockRows) + 32u * (uint32_t)j + lane;
+                    valid |= 1u << u;
+                }
+            }
+            if (__ballot_sync(0xFFFFFFFFu, valid != 0u) == 0u) {
+                // every lane is held at a dense block or out of words
+                if (F >= T && !__any_sync(0xFFFFFFFFu, held)) break;
+                continue;
             }
         }
-        if (__ballot_sync(0xFFFFFFFFu, valid != 0u) == 0u) {
-            if (F >= T) break;   // every word loaded and consumed
-            continue;            // lanes wait for the next refill
-        }
+        // rows whose bit is clear are read too, unmasked (a row of the
+        // block in lockstep, row 0 otherwise), but never offered
         if constexpr (MM > 0) {
             uint4 c[kU];
 #pragma unroll
-            for (int u = 0; u < kU; ++u)
-                c[u] = (valid >> u & 1u) ? ldg_nc_v4(codes + (size_t)row[u] * 16, keep) : make_uint4(0, 0, 0, 0);
+            for (int u = 0; u < kU; ++u) c[u] = ldg_nc_v4(codes + (size_t)row[u] * 16, keep);
             float d[kU];
 #pragma unroll
             for (int u = 0; u < kU; u += 2) lookup2<MM, FAST>(c[u], c[u + 1], tb, tb, base, d[u], d[u + 1]);
@@ -152,7 +150,7 @@ __device__ __forceinline__ void scan_chunk(const uint8_t* __restrict__ codes,
             }
         } else {
             float d[kU];
-            lookup_rows<kU>(codes, row, valid, row_bytes, M, S, tab, lane, d);
+            lookup_rows<kU>(codes, row, (1u << kU) - 1u, row_bytes, M, S, tab, lane, d);
 #pragma unroll
             for (int u = 0; u < kU; ++u) {
                 const bool pass = valid >> u & 1u;

@@ -26,9 +26,12 @@
 // bitmap words sit in a ring of 16 blocks in shared memory (lane l's word in
 // bank l); lanes advance through the ring at their own pace, eight rows per
 // round, and the ring is refilled by halves, from words prefetched into
-// registers, once every lane has left the older half.  When every lane
-// holds a full word of the same block the warp takes the block in lockstep
-// without per-row bit handling.
+// registers, once every lane has left the older half.  Lanes at different
+// blocks read rows that lie far apart, one cache line per lane; a block
+// with at least kDenseRows passing rows (of 1024) is therefore taken in
+// lockstep instead: each lane stops at it until the whole warp has arrived,
+// then the warp walks its 32 columns, 32 neighbouring rows per load, with
+// the lanes whose row fails masked.
 //
 // Top-k.  Each warp keeps a sorted list of its KP best keys and a candidate
 // area of KP slots; a key (dist bits << 32 | row) enters the area when it
@@ -56,11 +59,16 @@ namespace ifvs {
 #ifndef IFVS_SCAN_ROWS
 #define IFVS_SCAN_ROWS 8
 #endif
+#ifndef IFVS_SCAN_DENSE
+#define IFVS_SCAN_DENSE 448
+#endif
 constexpr int kScanWarps = IFVS_SCAN_WARPS;
 constexpr int kScanThreads = kScanWarps * 32;
 constexpr int kRing = IFVS_SCAN_RING;    // bitmap words per lane in the ring
 constexpr int kHalf = kRing / 2;
 constexpr int kU = IFVS_SCAN_ROWS;       // rows per lane per round (even)
+constexpr int kDenseRows = IFVS_SCAN_DENSE;   // passing rows from which a block goes in lockstep
+static_assert(kRing <= 32 && 32 % kU == 0, "one mask bit per ring slot; whole column groups");
 
 __device__ __forceinline__ void warp_sort(uint64_t* a, int n, int lane) {
     for (int size = 2; size <= n; size <<= 1)

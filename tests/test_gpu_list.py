@@ -447,6 +447,50 @@ def test_composite_copies_for_two_column_predicates(ifvs, orc, k):
     g.close()
 
 
+@pytest.mark.parametrize("M,ds,k", [(16, 2, 100), (12, 2, 10), (12, 2, 100), (8, 2, 10)])
+def test_bitmap_blocks_of_mixed_density(ifvs, orc, M, ds, k):
+    """The bitmap scan takes a 1024-row block in lockstep (all lanes on the
+    same column, failing rows masked) when enough of its rows pass, and
+    otherwise lets each lane walk its own passing rows.  Blocks here pass
+    exactly a set fraction of their rows (all, none, just above and just
+    below the switch, sparse), in an order that makes the warps cross from
+    one mode to the other many times and refill their word rings; 640
+    queries put every block of the 300-block column in a single chunk.
+    Forced onto the bitmap path, every query must give the sorted-copy
+    path's pass count exactly and its top-k up to rounding, and a sample of
+    queries must match the oracle."""
+    n_blk = 300
+    N = n_blk * 1024 + 333
+    rng = np.random.default_rng(61)
+    K = 256
+    codes = rng.integers(0, K, size=(N, M)).astype(np.uint8)
+    pattern = (1.0, 0.0, 0.5, 0.1, 0.44, 0.43, 0.9, 0.001, 0.6, 0.0, 0.45, 0.3, 1.0, 1.0, 0.05, 0.7)
+    a0 = rng.integers(100, 1000, N).astype(np.int32)          # fails every predicate below
+    for b in range(n_blk + 1):
+        r0, r1 = b * 1024, min(N, b * 1024 + 1024)
+        n_pass = int(round(pattern[(b * 7) % len(pattern)] * (r1 - r0)))
+        rows = r0 + rng.choice(r1 - r0, size=n_pass, replace=False)
+        a0[rows] = rng.integers(0, 100, n_pass)
+    attrs = [a0]
+    Cpq = rng.standard_normal((M, K, ds)).astype(np.float32)
+    g = ifvs.Index(codes, attrs, D=M * ds, K=K)
+    g.load_codebooks(Cpq)
+    nq = 640
+    widths = (100, 97, 90, 75, 50, 44, 10, 1)
+    p = synth.empty_predicates(nq)
+    for i in range(nq):
+        p[i]["n_clauses"] = 1
+        synth.set_clause(p[i], 0, 0, synth.OP_RANGE, 0, widths[i % len(widths)])
+    q = _queries(nq, M * ds, seed=62)
+    a = g.search(q, p, k, list_max_ppm=ALWAYS)
+    b = g.search(q, p, k, list_max_ppm=NEVER)
+    np.testing.assert_array_equal(a[2], b[2])
+    _same_up_to_rounding(a, b)
+    sample = np.arange(0, nq, 41)
+    _check_oracle(orc, codes, attrs, Cpq, q[sample], p[sample], k, *(x[sample] for x in b))
+    g.close()
+
+
 @pytest.mark.parametrize("M,ds,k", [(8, 2, 10), (24, 1, 100), (120, 1, 10), (120, 1, 200), (5, 3, 30)])
 def test_generic_m_bulk_tiles_equal_vector_loads(ifvs, orc, M, ds, k):
     """For M other than 12 and 16 the one-query kernel reads one row per lane
