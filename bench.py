@@ -473,30 +473,36 @@ def recall_at_k(w, ix, batches, ids_by_bin, nsample, device):
     return out
 
 
-def sorted_candidates(preds, attrs):
-    """Queries whose pool is a position range of a sorted copy, by the
-    library's rule: a predicate on one column, or, on an index of two
-    columns, one fixing a column to a single value and bounding the other
-    (the composite copy keyed by the fixed column).  Clause intervals are
-    intersected per column and clipped to the column's type."""
-    lo_of = {0: lambda c: (c["lo"], c["lo"]), 1: lambda c: (c["lo"], c["hi"] - 1),
-             2: lambda c: (c["lo"], None), 3: lambda c: (None, c["lo"] - 1),
-             4: lambda c: (c["lo"] + 1, None), 5: lambda c: (None, c["lo"])}
+def sorted_path(preds, attrs, npass, list_rows):
+    """Queries the library scans from a sorted copy, by its rule: a predicate
+    no row can pass; a predicate on no column or on one column whose pool
+    holds at most list_rows rows; on an index of two columns, one that fixes
+    a column to a single value and bounds the other, pool size likewise.
+    Clause intervals are intersected per column and clipped to the column's
+    type, as the library canonicalises them."""
+    ends = {0: lambda c: (c["lo"], c["lo"]), 1: lambda c: (c["lo"], c["hi"] - 1),
+            2: lambda c: (c["lo"], None), 3: lambda c: (None, c["lo"] - 1),
+            4: lambda c: (c["lo"] + 1, None), 5: lambda c: (None, c["lo"])}
     out = np.zeros(len(preds), bool)
     for i, p in enumerate(preds):
         iv = {}
         for c in p["c"][:int(p["n_clauses"])]:
             col = int(c["col"])
             info = np.iinfo(attrs[col].dtype)
-            lo, hi = lo_of[int(c["op"])](c)
+            lo, hi = ends[int(c["op"])](c)
             lo = info.min if lo is None else max(int(lo), info.min)
             hi = info.max if hi is None else min(int(hi), info.max)
             a, b = iv.get(col, (info.min, info.max))
             iv[col] = (max(a, lo), min(b, hi))
-        if len(iv) == 1:
+        small = npass[i] <= list_rows
+        if any(a > b for a, b in iv.values()):
             out[i] = True
-        elif len(iv) == 2 and len(attrs) == 2 and set(iv) == {0, 1}:
-            out[i] = any(a == b for a, b in iv.values())
+        elif len(iv) == 0:
+            out[i] = len(attrs) > 0 and small
+        elif len(iv) == 1:
+            out[i] = small
+        elif len(iv) == 2 and len(attrs) == 2:
+            out[i] = small and any(a == b for a, b in iv.values())
     return out
 
 
@@ -657,7 +663,7 @@ def run_ifvs(args):
         ms_b = [step_ms[i] for i in range(args.steps) if (args.warmup + i) % nb == b]
         npass = dev_out[b][2].cpu().numpy().astype(np.float64)
         nsteps_b = len(ms_b)
-        on_list = sorted_candidates(qs.preds, ix.attrs) & (npass <= list_rows)
+        on_list = sorted_path(qs.preds, ix.attrs, npass, list_rows)
         lk = scan_lookups(w, qs, sorted_vals, on_list, npass, pair_rows)
         lookups_total += nsteps_b * lk["lookups"]
         code_bytes_total += nsteps_b * float(npass.sum()) * w.M

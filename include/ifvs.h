@@ -126,14 +126,16 @@ typedef struct {
     int32_t chunk_blocks; /* rows per scan CTA in units of 1024 (0: automatic);
                            a tuning knob: CTAs of different queries that walk
                            the same chunk together share its codes in L2     */
-    int32_t list_max_ppm; /* a query whose predicate constrains one column
-                           takes the sorted-copy scan (its pool is a position
-                           range of the codes sorted by that column: no
-                           filter pass, no bitmap) when the pool holds at most
-                           this many rows per million of N.  0: default
-                           (1000000: always); -1: never.  The two paths sum a row's entries in
-                           different orders, so distances agree to float32
-                           rounding.                                          */
+    int32_t list_max_ppm; /* a query whose predicate constrains one column,
+                           or, on an index of two columns, fixes one column
+                           to a single value and bounds the other, takes the
+                           sorted-copy scan (its pool is a position range of
+                           the codes sorted by that column, or of a composite
+                           copy: no filter pass, no bitmap) when the pool
+                           holds at most this many rows per million of N.
+                           0: default (1000000: always); -1: never.  The two
+                           paths sum a row's entries in different orders, so
+                           distances agree to float32 rounding.              */
     int32_t pair_min_rows; /* M = 16 sorted-copy scan: two queries on the same
                            column whose ranges share 3/4 of the longer one
                            and together span at least this many rows share a
@@ -180,7 +182,11 @@ enum {
  * the row ids sorted by (value, row), the sorted values and a copy of the
  * code rows in that order (8 + row_bytes bytes per row and column; the order
  * is sorted on the host at load), in which a one-column predicate's pool is
- * a contiguous position range.
+ * a contiguous position range.  An index of exactly two columns also keeps
+ * two composite copies, rows by (column j, column 1 - j, row) for j = 0, 1
+ * (the 8-byte key, the row id and the code row: 12 + row_bytes bytes per
+ * row each), in which a predicate fixing column j to one value and bounding
+ * the other column is a contiguous position range.
  */
 int ifvs_load_index(ifvs_index** out, int32_t device, const uint8_t* codes, int64_t N,
                     int32_t M, int32_t K, const void* const* attr_cols,

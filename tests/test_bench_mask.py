@@ -37,3 +37,46 @@ def test_pass_mask_equals_the_oracle_filter(orc):
         rows = np.unpackbits(bm.view(np.uint8), bitorder="little")[:N].astype(bool)
         np.testing.assert_array_equal(mask[i], rows)
         assert int(mask[i].sum()) == npass
+
+
+def test_sorted_path_share_follows_the_path_rule():
+    """The benchmark reports which queries the library scans from a sorted
+    copy: a predicate no row can pass; one on no column or on one column; on
+    an index of two columns, one that fixes a column to a single value
+    (after intersecting its clauses and clipping to the column's type) and
+    bounds the other; each but the first only while its pool holds at most
+    list_rows rows.  Predicates on both columns that fix neither, and
+    predicates on several columns of a three-column index, take the bitmap
+    path."""
+    import bench
+    i32 = np.zeros(4, np.int32)
+    i16 = np.zeros(4, np.int16)
+    cases = [
+        ([(0, synth.OP_RANGE, -5, 5)], True),
+        ([(1, synth.OP_GE, 3), (1, synth.OP_LT, 9)], True),                   # one column, two clauses
+        ([], True),                                                           # every row passes
+        ([(1, synth.OP_EQ, 4), (0, synth.OP_RANGE, 0, 100)], True),
+        ([(0, synth.OP_EQ, -7), (1, synth.OP_LE, 20)], True),
+        ([(1, synth.OP_LE, 4), (0, synth.OP_RANGE, 0, 100)], False),          # neither fixed
+        ([(0, synth.OP_RANGE, 8, 9), (1, synth.OP_GT, 0)], True),             # width-one range
+        ([(0, synth.OP_GE, 3), (0, synth.OP_LE, 3), (1, synth.OP_LT, 0)], True),   # fixed by two clauses
+        ([(1, synth.OP_GE, 32767), (0, synth.OP_GT, 1)], True),               # fixed by the int16 bound
+        ([(1, synth.OP_GE, 32766), (0, synth.OP_GT, 1)], False),
+        ([(0, synth.OP_LT, -(2 ** 31) + 1), (1, synth.OP_RANGE, 0, 9)], True),   # int32 minimum only
+        ([(1, synth.OP_EQ, 40000), (0, synth.OP_GE, 0)], True),               # no int16 value: empty
+        ([(0, synth.OP_RANGE, 5, 5), (1, synth.OP_GE, 0)], True),             # empty range
+    ]
+    p = synth.empty_predicates(len(cases))
+    for i, (cl, _) in enumerate(cases):
+        p[i]["n_clauses"] = len(cl)
+        for j, c in enumerate(cl):
+            synth.set_clause(p[i], j, *c)
+    small = np.zeros(len(cases))
+    big = np.full(len(cases), 10.0)
+    want = np.array([w for _, w in cases])
+    np.testing.assert_array_equal(bench.sorted_path(p, [i32, i16], small, 5), want)
+    empty = np.array([i >= len(cases) - 2 for i in range(len(cases))])
+    np.testing.assert_array_equal(bench.sorted_path(p, [i32, i16], big, 5), empty)
+    # three columns: only predicates on fewer than two columns have a copy
+    three = np.array([len({c[0] for c in cl}) < 2 for cl, _ in cases]) | empty
+    np.testing.assert_array_equal(bench.sorted_path(p, [i32, i16, i32], small, 5), three)
