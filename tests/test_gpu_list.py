@@ -450,10 +450,10 @@ def test_composite_copies_for_two_column_predicates(ifvs, orc, k):
 @pytest.mark.parametrize("M,ds,k", [(16, 2, 100), (12, 2, 10), (12, 2, 100), (8, 2, 10)])
 def test_bitmap_blocks_of_mixed_density(ifvs, orc, M, ds, k):
     """The bitmap scan takes a 1024-row block in lockstep (all lanes on the
-    same column, failing rows masked) when enough of its rows pass, and
-    otherwise lets each lane walk its own passing rows.  Blocks here pass
-    exactly a set fraction of their rows (all, none, just above and just
-    below the switch, sparse), in an order that makes the warps cross from
+    same column, failing rows masked) when at least 448 of its 1024 rows
+    pass, and otherwise lets each lane walk its own passing rows.  Blocks
+    here pass exactly a set number of rows (all, none, 447, 448 and 449,
+    sparse), in an order that makes the warps cross from
     one mode to the other many times and refill their word rings; 640
     queries put every block of the 300-block column in a single chunk.
     Forced onto the bitmap path, every query must give the sorted-copy
@@ -464,11 +464,12 @@ def test_bitmap_blocks_of_mixed_density(ifvs, orc, M, ds, k):
     rng = np.random.default_rng(61)
     K = 256
     codes = rng.integers(0, K, size=(N, M)).astype(np.uint8)
-    pattern = (1.0, 0.0, 0.5, 0.1, 0.44, 0.43, 0.9, 0.001, 0.6, 0.0, 0.45, 0.3, 1.0, 1.0, 0.05, 0.7)
+    # passing rows per block; the lockstep threshold is 448
+    pattern = (1024, 0, 512, 102, 448, 447, 922, 1, 614, 0, 449, 307, 1024, 1024, 51, 717)
     a0 = rng.integers(100, 1000, N).astype(np.int32)          # fails every predicate below
     for b in range(n_blk + 1):
         r0, r1 = b * 1024, min(N, b * 1024 + 1024)
-        n_pass = int(round(pattern[(b * 7) % len(pattern)] * (r1 - r0)))
+        n_pass = pattern[(b * 7) % len(pattern)] * (r1 - r0) // 1024
         rows = r0 + rng.choice(r1 - r0, size=n_pass, replace=False)
         a0[rows] = rng.integers(0, 100, n_pass)
     attrs = [a0]
